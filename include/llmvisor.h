@@ -1,0 +1,223 @@
+/*
+ * llmvisor.h -- C ABI of the GB300 (sm_103a) implementation of LLMVisor's
+ * batched latency attribution.
+ *
+ * The model (Section 2, "Problem formulation", and Section 2.1, Eq. 1):
+ * a batch B of requests has latency
+ *     T_B = beta + a1*sum_i p_i + a2*sum_i c_i + a3*sum_i p_i^2 + a4*sum_i |B|
+ * with four coefficient sets, one per (phase, regime): prefill or decode, and
+ * memory-bound or compute-bound.  p_i is the number of tokens request i
+ * processes this step, c_i the number of context tokens whose KV entries it
+ * loads.  T_B splits into additive, per-request shares t_i with
+ * sum_i t_i = T_B, and shares roll up per tenant: L_u = sum_{i: u(i)=u} t_i.
+ *
+ * Readings of the paper used throughout (it leaves these open):
+ *  - sum_i |B| is taken literally: it equals n^2 for a batch of n requests.
+ *  - A batch is a prefill batch if any request in it is a prefill.
+ *  - Regime: compute-bound iff S1 = sum_i p_i >= split[phase] (tie -> compute).
+ *  - Share: t_i = beta/n + a1 p_i + a2 c_i + a3 p_i^2 + a4 n (the fixed cost and
+ *    the n^2 term are split equally; slope terms follow their request).
+ *  - Empty batch: T = 0, segment (decode, memory), no shares.
+ *  - Units: seconds, coefficients in seconds per raw feature unit.
+ *
+ * Conventions for every call:
+ *  - Every array argument is DEVICE memory owned by the caller, unless stated.
+ *    Structs (lv_arch, lv_model, lv_batches, lv_fit_report) live in HOST memory
+ *    and are copied at the call; device pointers inside lv_batches are the
+ *    caller's.  Opaque handles (lv_ctx, lv_tenant_acc) are owned by the library.
+ *  - stream is a cudaStream_t (NULL = legacy default stream).  Calls are
+ *    asynchronous with respect to the host unless stated.
+ *  - Argument errors are detected on the host and returned before anything is
+ *    launched (LV_EINVAL, LV_EOVERFLOW).  Data errors found on the device
+ *    (non-monotone offsets, negative p or c, phase not 0/1, tenant out of range,
+ *    offsets[n_batch] != n_req) never cause an out-of-bounds access: kernels
+ *    clamp and record LV_EDATA in the context's sticky status word, which
+ *    lv_ctx_status() reports.  CUDA failures return LV_ECUDA.
+ *  - Alignment: request arrays (p, c, phase, tenant) and offsets must be
+ *    16-byte aligned (they are read with bulk asynchronous copies), fp64 outputs
+ *    8-byte aligned; otherwise LV_EINVAL.
+ *  - One lv_ctx must not be used from two host threads at once.
+ */
+#ifndef LLMVISOR_H
+#define LLMVISOR_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t lv_status;
+#define LV_OK 0
+#define LV_EINVAL (-1)     /* bad argument (null/unaligned pointer, bad size, bad arch) */
+#define LV_EOVERFLOW (-2)  /* an int64 feature or constant would overflow */
+#define LV_ENODATA (-3)    /* fit group with fewer batches than coefficients */
+#define LV_ESINGULAR (-4)  /* fit group whose normal equations are singular */
+#define LV_ECUDA (-5)      /* a CUDA runtime call failed */
+#define LV_EDATA (-6)      /* invalid input data seen on the device (sticky) */
+#define LV_ENOMEM (-7)     /* device allocation failed */
+#define LV_ETIMEOUT (-8)   /* a bounded device-side wait gave up */
+
+/* Model architecture; integers only.  tp is the modelled tensor-parallel degree
+ * (an arithmetic input: constants are per rank).  kv_bytes is the KV-cache
+ * element size.  tp must divide n_q_heads, n_kv_heads and ffn_dim. */
+typedef struct {
+    int32_t n_layers, d_model, n_q_heads, n_kv_heads, head_dim, ffn_dim;
+    int32_t weight_bytes, kv_bytes, tp;
+} lv_arch;
+
+/* One coefficient set of Eq. 1, in seconds per raw unit. */
+typedef struct {
+    double beta, a1, a2, a3, a4;
+} lv_coef;
+
+/* The piecewise model: seg[phase][regime], phase 0 = decode, 1 = prefill;
+ * regime 0 = memory-bound, 1 = compute-bound (Section 2.1: two segments per
+ * phase, four coefficient sets in all).  split[phase] is the threshold on
+ * S1 = sum_i p_i at which the regime becomes compute-bound. */
+typedef struct {
+    lv_coef seg[2][2];
+    int64_t split[2];
+} lv_model;
+
+/* A set of batches in CSR form.  All pointers are DEVICE pointers.
+ *  p[n_req], c[n_req], phase[n_req] (0 decode / 1 prefill), tenant[n_req]
+ *  (0..n_tenants-1; may be NULL where no tenant roll-up is asked for),
+ *  offsets[n_batch+1] with offsets[0] = 0, non-decreasing, offsets[n_batch] = n_req.
+ *  Batch b holds requests offsets[b] .. offsets[b+1]-1. */
+typedef struct {
+    const int32_t *p, *c, *phase, *tenant;
+    const int64_t *offsets;
+    int64_t n_req, n_batch;
+    int32_t n_tenants;
+    int32_t reserved;
+} lv_batches;
+
+/* Per-group outcome of lv_fit, group g = phase*2 + regime. */
+typedef struct {
+    int64_t n[4];        /* batches in the group (empty batches excluded) */
+    int32_t status[4];   /* LV_OK, LV_ENODATA or LV_ESINGULAR */
+    int32_t dropped[4];  /* bit k set: coefficient k (0 beta .. 4 a4) not identifiable, reported as 0 */
+    double ssr[4];       /* residual sum of squares of the returned coefficients */
+    double r2[4];        /* 1 - ssr/sst */
+} lv_fit_report;
+
+typedef struct lv_ctx lv_ctx;
+typedef struct lv_tenant_acc lv_tenant_acc;
+
+/* Arithmetic used for T and shares.  AUTO picks the exact fixed-point path
+ * whenever every segment's coefficients fit it (see lv_attribute) and FP64
+ * otherwise; FP64 forces double-precision evaluation. */
+#define LV_ARITH_AUTO 0
+#define LV_ARITH_FP64 1
+
+/* Create a context on the current CUDA device.  It owns a small device scratch
+ * area and a sticky status word.  Returns LV_ECUDA/LV_ENOMEM on failure. */
+lv_status lv_ctx_create(lv_ctx **out);
+void lv_ctx_destroy(lv_ctx *ctx);
+/* Select LV_ARITH_AUTO (default) or LV_ARITH_FP64. */
+lv_status lv_ctx_set_arith(lv_ctx *ctx, int32_t mode);
+/* Synchronise `stream`, then return and clear the sticky device status
+ * (LV_OK or LV_EDATA / LV_ETIMEOUT). */
+lv_status lv_ctx_status(lv_ctx *ctx, void *stream);
+/* Static description of a status code. */
+const char *lv_status_string(lv_status s);
+/* Measurement support (no counterpart in the paper).  With timing enabled the
+ * library brackets every launch of its request-streaming kernels (the tile
+ * kernel of lv_attribute / lv_features / lv_fit, the pair kernel of lv_whatif)
+ * with CUDA events on the launching stream.  lv_ctx_kernel_time synchronises
+ * those events, returns the summed milliseconds and the number of launches
+ * since the previous query, and resets the tally.  Off by default. */
+lv_status lv_ctx_set_timing(lv_ctx *ctx, int32_t enable);
+lv_status lv_ctx_kernel_time(lv_ctx *ctx, double *ms, int64_t *launches);
+
+/* Architecture constants (Section 2.1: features proportional to FLOPs and to
+ * memory I/O).  With P_layer = d*hq*hd + 2*d*hkv*hd + hq*hd*d + 3*d*F:
+ *   phi[0] = 2*L*P_layer/tp       FLOPs per new token
+ *   phi[1] = 2*L*hkv*hd*kv_bytes/tp  KV bytes per context token
+ *   phi[2] = 2*L*hq*hd/tp         causal-attention FLOPs per p^2
+ *   *weight_bytes = L*P_layer*weight_bytes/tp   bytes of weights read per step
+ * Host only.  LV_EINVAL for non-positive fields or tp not dividing heads/FFN;
+ * LV_EOVERFLOW if a constant exceeds int64. */
+lv_status lv_arch_constants(const lv_arch *arch, int64_t phi[3], int64_t *weight_bytes);
+
+/* Per-request and per-batch features (Section 2.1 and the sums of Eq. 1).
+ *  req_feat   int64[3][n_req] (SoA) or NULL: p*phi0, c*phi1, p^2*phi2.
+ *             A product beyond int64 records LV_EDATA and stores INT64_MAX.
+ *  batch_feat int64[5][n_batch] (SoA) or NULL: S1 = sum p, S2 = sum c,
+ *             S3 = sum p^2, n, n^2.
+ *  batch_seg  uint8[n_batch] or NULL: phase*2 + regime under model->split.
+ * arch may be NULL when req_feat is NULL; model may be NULL when batch_seg is
+ * NULL.  Integer results are exact. */
+lv_status lv_features(lv_ctx *ctx, const lv_arch *arch, const lv_model *model, const lv_batches *b,
+                      int64_t *req_feat, int64_t *batch_feat, uint8_t *batch_seg, void *stream);
+
+/* Eq. 1 from precomputed aggregates: T[b] = beta + a1*S1 + a2*S2 + a3*S3 + a4*n^2
+ * with the coefficients of segment batch_seg[b]; T = 0 where n = 0.
+ * batch_feat int64[5][n_batch] as written by lv_features. */
+lv_status lv_batch_latency(lv_ctx *ctx, const lv_model *model, const int64_t *batch_feat,
+                           const uint8_t *batch_seg, int64_t n_batch, double *T, void *stream);
+
+/* The fused hot path (Eq. 1 plus the additive shares of Section 2.1): one pass
+ * over the request arrays computes every batch's sums, segment and T, each
+ * request's share t_i, and (if acc != NULL) adds every share into the tenant
+ * accumulator.  T double[n_batch] (or NULL), share double[n_req] (or NULL).
+ * b->tenant and b->n_tenants must match acc when acc is given.
+ * Arithmetic: on the default path every share is the correctly rounded value of
+ * fl(fl(beta/n) + fl(a4*n)) + a1 p + a2 c + a3 p^2 evaluated exactly in integer
+ * fixed point, and T the correctly rounded value of Eq. 1 evaluated exactly;
+ * results agree with a left-to-right double evaluation to a few ulp. */
+lv_status lv_attribute(lv_ctx *ctx, const lv_model *model, const lv_batches *b, double *T, double *share,
+                       lv_tenant_acc *acc, void *stream);
+
+/* Per-tenant accumulator (Section 2: L_u).  Every fp64 share is rounded to a
+ * multiple of 2^-72 s (exact for shares of at least 2^-20 s; the rounding error
+ * is below 1.1e-22 s otherwise) and summed EXACTLY in a 128-bit integer per
+ * tenant, so totals do not depend on summation order and are bit-identical run
+ * to run; lv_tenant_totals returns the correctly rounded fp64 value of each
+ * exact sum.  A total beyond +-2^55 s records LV_EDATA.  Accumulation
+ * continues across calls until reset. */
+lv_status lv_tenant_acc_create(lv_ctx *ctx, int32_t n_tenants, lv_tenant_acc **out);
+void lv_tenant_acc_destroy(lv_tenant_acc *acc);
+lv_status lv_tenant_acc_reset(lv_tenant_acc *acc, void *stream);
+/* Add share[i] to tenant[i]'s total for i < n_req (device arrays). */
+lv_status lv_tenant_accumulate(lv_ctx *ctx, lv_tenant_acc *acc, const double *share, const int32_t *tenant,
+                               int64_t n_req, void *stream);
+/* L double[n_tenants] (device): the current totals. */
+lv_status lv_tenant_totals(lv_ctx *ctx, lv_tenant_acc *acc, double *L, void *stream);
+/* Checkpoint / resume: the exact state is n_tenants * 16 bytes (host buffer).
+ * export synchronises the stream. */
+int64_t lv_tenant_acc_state_bytes(const lv_tenant_acc *acc);
+lv_status lv_tenant_acc_export(lv_tenant_acc *acc, void *host_state, int64_t bytes, void *stream);
+lv_status lv_tenant_acc_import(lv_tenant_acc *acc, const void *host_state, int64_t bytes, void *stream);
+
+/* Ordinary least squares of Eq. 1's coefficients per segment (Section 2.1:
+ * "fit the coefficients via ordinary least squares on profiling data").
+ * y is double[n_y][n_batch] (device): n_y latency vectors for the same batches,
+ * fitted in one pass over the requests.  inout[0..n_y-1] are HOST models: their
+ * split is read (all must be equal) and their coefficients are overwritten for
+ * every group whose status is LV_OK.  rep (host, may be NULL) receives one
+ * lv_fit_report per y vector.  Decode batches have p_i = 1, so S1 == S3: when
+ * that holds for every batch of a group the a3 column is dropped and a1
+ * carries a1 + a3.  Empty batches are skipped.  The Gram matrix is accumulated
+ * exactly in integers and X^T y exactly in fixed point; the solve runs in
+ * double-double.  Synchronous: returns after the coefficients are on the host. */
+lv_status lv_fit(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y, lv_model *inout,
+                 lv_fit_report *rep, void *stream);
+
+/* What-if (Section 1: admission control and what-if planning over alternative
+ * batch mixes).  For every pending request j (p_new, c_new, phase_new: device
+ * int32[n_pending]) and candidate batch k of `cand`:
+ *   T_new[j][k]     = Eq. 1 of the batch cand_k + {j}
+ *   share_new[j][k] = request j's share in that batch.
+ * Outputs double[n_pending][n_cand] (device, row-major, pending-major); either
+ * may be NULL. */
+lv_status lv_whatif(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, const int32_t *p_new,
+                    const int32_t *c_new, const int32_t *phase_new, int64_t n_pending, double *T_new,
+                    double *share_new, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LLMVISOR_H */

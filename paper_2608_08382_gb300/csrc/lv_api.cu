@@ -1,0 +1,633 @@
+// Host side of the C ABI declared in include/llmvisor.h: contexts, argument
+// validation, fixed-point parameter derivation and kernel launch sequences.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "llmvisor.h"
+#include "lv_fit.cuh"
+#include "lv_kernels.cuh"
+#include "lv_whatif.cuh"
+
+using namespace lv;
+
+struct lv_ctx {
+  int device = 0;
+  int sms = 0;
+  int arith = LV_ARITH_AUTO;
+  int *d_status = nullptr;
+  TilePart *d_tiles = nullptr;
+  int64_t tiles_cap = 0;
+  KEntry *d_ktab = nullptr;
+  int ktab_nk = 0;
+  bool ktab_valid = false;
+  lv_model ktab_model{};
+  int ktab_fixed = -1;
+  cudaEvent_t ev_built = nullptr;
+  cudaEvent_t ev_used = nullptr;
+  cudaStream_t ktab_stream = nullptr;
+  void *d_fit = nullptr;      // fit partials + solve output
+  size_t fit_cap = 0;
+  void *d_wi = nullptr;       // what-if per-candidate / per-pending tables
+  size_t wi_cap = 0;
+  bool timing = false;
+  std::vector<cudaEvent_t> tev;  // start/stop pairs
+  size_t tev_used = 0;
+};
+
+struct lv_tenant_acc {
+  lv_ctx *ctx = nullptr;
+  int32_t n_tenants = 0;
+  unsigned long long *d_pend = nullptr;  // [n][4]
+  i128 *d_state = nullptr;               // [n]
+};
+
+namespace {
+
+constexpr int kKTableN = 4096;
+
+#define LV_CUDA(call)                          \
+  do {                                         \
+    if ((call) != cudaSuccess) return LV_ECUDA; \
+  } while (0)
+
+bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+int lsb_exp(double x) {
+  // x = M * 2^e with M odd; returns e.  x != 0, finite.
+  int e;
+  const double f = std::frexp(std::fabs(x), &e);  // x = f * 2^e, 0.5 <= f < 1
+  uint64_t M = (uint64_t)std::ldexp(f, 53);
+  int ex = e - 53;
+  while ((M & 1ull) == 0) {
+    M >>= 1;
+    ++ex;
+  }
+  return ex;
+}
+
+int msb_exp(double x) {
+  int e;
+  std::frexp(std::fabs(x), &e);
+  return e - 1;
+}
+
+i128 host_fix_exact(double x, int E, bool *ok) {
+  bool ovf = false;
+  i128 r = double_to_fix(x, E, &ovf);
+  if (ovf) *ok = false;
+  return r;
+}
+
+// |A| as a double (for bound checks).
+double mag(i128 a) {
+  if (is_neg128(a)) a = neg128(a);
+  return std::ldexp((double)a.hi, 64) + (double)a.lo;
+}
+
+uint64_t limit_for(i128 A) {
+  const double m = mag(A);
+  if (m == 0) return (uint64_t)INT64_MAX;
+  const double lim = std::floor(std::ldexp(1.0, 124) / m);
+  if (lim >= 9.2e18) return (uint64_t)INT64_MAX;
+  return (uint64_t)lim;
+}
+
+bool finite_model(const lv_model *m) {
+  const double *c = &m->seg[0][0].beta;
+  for (int i = 0; i < 20; ++i)
+    if (!std::isfinite(c[i])) return false;
+  return true;
+}
+
+// Derives the exact fixed-point representation of every segment.  Returns
+// false when some segment's coefficients do not fit the integer path.
+bool derive_fixed(const lv_model *m, int nk, ModelP *mp) {
+  for (int s = 0; s < 4; ++s) {
+    const lv_coef &k = m->seg[s >> 1][s & 1];
+    int E = INT32_MAX;
+    const double slopes[4] = {k.a1, k.a2, k.a3, k.a4};
+    for (double v : slopes)
+      if (v != 0) E = std::min(E, lsb_exp(v));
+    if (k.beta != 0) E = std::min(E, msb_exp(k.beta) - 66);
+    if (E == INT32_MAX) E = -200;  // all-zero segment: any scale works
+    if (E < -1022 || E + 127 > 1023) return false;
+    SegFix &f = mp->fx[s];
+    std::memset(&f, 0, sizeof(f));
+    f.E = E;
+    bool ok = true;
+    f.A1 = host_fix_exact(k.a1, E, &ok);
+    f.A2 = host_fix_exact(k.a2, E, &ok);
+    f.A3 = host_fix_exact(k.a3, E, &ok);
+    f.B = host_fix_exact(k.beta, E, &ok);
+    f.A4 = host_fix_exact(k.a4, E, &ok);
+    if (!ok) return false;
+    // share path: every term below 2^124 for p <= 2^24, c < 2^31
+    if (mag(f.A1) >= std::ldexp(1.0, 100) || mag(f.A2) >= std::ldexp(1.0, 93) || mag(f.A3) >= std::ldexp(1.0, 76))
+      return false;
+    const double kmax = (std::fabs(k.beta) + std::fabs(k.a4) * nk) * 1.0000001;
+    if (std::ldexp(kmax, -E) >= std::ldexp(1.0, 123) || mag(f.B) >= std::ldexp(1.0, 124)) return false;
+    f.A13 = add128(f.A1, f.A3);
+    f.a2_narrow = (f.A2.hi == 0) ? 1 : 0;
+    f.lim[0] = limit_for(f.A1);
+    f.lim[1] = limit_for(f.A2);
+    f.lim[2] = limit_for(f.A3);
+    f.lim[3] = limit_for(f.A4);
+  }
+  return true;
+}
+
+lv_status check_model(const lv_model *m) {
+  if (!m) return LV_EINVAL;
+  if (!finite_model(m)) return LV_EINVAL;
+  return LV_OK;
+}
+
+lv_status check_batches(const lv_batches *b, bool need_tenant) {
+  if (!b) return LV_EINVAL;
+  if (b->n_req < 0 || b->n_batch < 0) return LV_EINVAL;
+  if (!b->offsets || !aligned(b->offsets, 16)) return LV_EINVAL;
+  if (b->n_req > 0) {
+    if (!b->p || !b->c || !b->phase) return LV_EINVAL;
+    if (!aligned(b->p, 16) || !aligned(b->c, 16) || !aligned(b->phase, 16)) return LV_EINVAL;
+    if (need_tenant && (!b->tenant || !aligned(b->tenant, 16))) return LV_EINVAL;
+  }
+  if (need_tenant && b->n_tenants <= 0) return LV_EINVAL;
+  if (b->n_req > (1ll << 40) || b->n_batch > (1ll << 40)) return LV_EINVAL;
+  return LV_OK;
+}
+
+lv_status ensure_tiles(lv_ctx *ctx, int64_t n) {
+  if (n <= ctx->tiles_cap) return LV_OK;
+  LV_CUDA(cudaDeviceSynchronize());
+  if (ctx->d_tiles) cudaFree(ctx->d_tiles);
+  ctx->d_tiles = nullptr;
+  int64_t cap = std::max<int64_t>(n, 1 << 16);
+  if (cudaMalloc(&ctx->d_tiles, cap * sizeof(TilePart)) != cudaSuccess) {
+    ctx->tiles_cap = 0;
+    return LV_ENOMEM;
+  }
+  ctx->tiles_cap = cap;
+  return LV_OK;
+}
+
+// Builds (or reuses) the per-model parameters and K table on `stream`.
+lv_status prepare_model(lv_ctx *ctx, const lv_model *m, cudaStream_t stream, ModelP *mp) {
+  std::memset(mp, 0, sizeof(*mp));
+  for (int s = 0; s < 4; ++s) {
+    const lv_coef &k = m->seg[s >> 1][s & 1];
+    mp->coef[s][0] = k.beta;
+    mp->coef[s][1] = k.a1;
+    mp->coef[s][2] = k.a2;
+    mp->coef[s][3] = k.a3;
+    mp->coef[s][4] = k.a4;
+  }
+  mp->split[0] = m->split[0];
+  mp->split[1] = m->split[1];
+  mp->nk = kKTableN;
+  mp->fixed = 0;
+  if (ctx->arith == LV_ARITH_AUTO) mp->fixed = derive_fixed(m, kKTableN, mp) ? 1 : 0;
+  if (!ctx->d_ktab) {
+    if (cudaMalloc(&ctx->d_ktab, sizeof(KEntry) * 4 * (kKTableN + 1)) != cudaSuccess) return LV_ENOMEM;
+  }
+  mp->ktab = ctx->d_ktab;
+  const bool same = ctx->ktab_valid && ctx->ktab_fixed == mp->fixed &&
+                    std::memcmp(&ctx->ktab_model, m, sizeof(lv_model)) == 0;
+  if (!same) {
+    // wait for earlier users of the table on any stream
+    LV_CUDA(cudaStreamWaitEvent(stream, ctx->ev_used, 0));
+    const int n = 4 * (kKTableN + 1);
+    k_ktable<<<(n + 255) / 256, 256, 0, stream>>>(*mp, ctx->d_ktab);
+    LV_CUDA(cudaGetLastError());
+    LV_CUDA(cudaEventRecord(ctx->ev_built, stream));
+    ctx->ktab_model = *m;
+    ctx->ktab_fixed = mp->fixed;
+    ctx->ktab_valid = true;
+    ctx->ktab_stream = stream;
+  } else if (stream != ctx->ktab_stream) {
+    LV_CUDA(cudaStreamWaitEvent(stream, ctx->ev_built, 0));
+  }
+  return LV_OK;
+}
+
+// Event pair around a measured launch (when timing is on).
+lv_status timing_begin(lv_ctx *ctx, cudaStream_t stream, cudaEvent_t *stop) {
+  *stop = nullptr;
+  if (!ctx->timing) return LV_OK;
+  if (ctx->tev_used + 2 > ctx->tev.size()) {
+    for (int k = 0; k < 2; ++k) {
+      cudaEvent_t e;
+      LV_CUDA(cudaEventCreate(&e));
+      ctx->tev.push_back(e);
+    }
+  }
+  cudaEvent_t start = ctx->tev[ctx->tev_used];
+  *stop = ctx->tev[ctx->tev_used + 1];
+  ctx->tev_used += 2;
+  LV_CUDA(cudaEventRecord(start, stream));
+  return LV_OK;
+}
+
+lv_status timing_end(cudaEvent_t stop, cudaStream_t stream) {
+  if (stop) LV_CUDA(cudaEventRecord(stop, stream));
+  return LV_OK;
+}
+
+template <int MODE>
+lv_status launch_tiles_mode(lv_ctx *ctx, TileArgs &a, int H, cudaStream_t stream) {
+  static bool configured = false;
+  const size_t smem = sizeof(Smem) + sizeof(uint32_t) * 4 * (size_t)H;
+  if (!configured) {
+    LV_CUDA(cudaFuncSetAttribute(k_tiles<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)(sizeof(Smem) + sizeof(uint32_t) * 4 * kHotMax)));
+    configured = true;
+  }
+  int per_sm = 0;
+  LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_tiles<MODE>, kBlock, smem));
+  if (per_sm < 1) per_sm = 1;
+  const int64_t grid = std::min<int64_t>(a.n_tiles, (int64_t)ctx->sms * per_sm);
+  if (grid <= 0) return LV_OK;
+  cudaEvent_t stop;
+  lv_status st = timing_begin(ctx, stream, &stop);
+  if (st != LV_OK) return st;
+  k_tiles<MODE><<<(unsigned)grid, kBlock, smem, stream>>>(a);
+  LV_CUDA(cudaGetLastError());
+  return timing_end(stop, stream);
+}
+
+// Partition + tile kernel for the given batches.
+lv_status run_tiles(lv_ctx *ctx, TileArgs &a, int mode, cudaStream_t stream) {
+  const int64_t units = a.n_batch + a.n_req;
+  a.n_tiles = (units + kD - 1) / kD;
+  if (a.n_batch == 0) {
+    return LV_OK;
+  }
+  lv_status st = ensure_tiles(ctx, a.n_tiles + 1);
+  if (st != LV_OK) return st;
+  a.part = ctx->d_tiles;
+  const int64_t nthreads = a.n_batch + 1;
+  const int64_t pblocks = std::min<int64_t>((nthreads + 255) / 256, (int64_t)ctx->sms * 16);
+  k_partition<<<(unsigned)pblocks, 256, 0, stream>>>(a.off, a.n_batch, a.n_req, a.n_tiles, ctx->d_tiles,
+                                                     ctx->d_status);
+  LV_CUDA(cudaGetLastError());
+  const int H = a.H;
+  switch (mode) {
+    case M_ATTR: return launch_tiles_mode<M_ATTR>(ctx, a, H, stream);
+    case M_ATTR | M_FIX: return launch_tiles_mode<M_ATTR | M_FIX>(ctx, a, H, stream);
+    case M_ATTR | M_TEN: return launch_tiles_mode<M_ATTR | M_TEN>(ctx, a, H, stream);
+    case M_ATTR | M_TEN | M_FIX: return launch_tiles_mode<M_ATTR | M_TEN | M_FIX>(ctx, a, H, stream);
+    case M_FEAT: return launch_tiles_mode<M_FEAT>(ctx, a, 0, stream);
+    default: return LV_EINVAL;
+  }
+}
+
+lv_status fold_tenants(lv_ctx *ctx, lv_tenant_acc *acc, cudaStream_t stream) {
+  const int n = acc->n_tenants;
+  k_tenant_fold<<<(n + 255) / 256, 256, 0, stream>>>(acc->d_pend, acc->d_state, n, ctx->d_status);
+  LV_CUDA(cudaGetLastError());
+  return LV_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *lv_status_string(lv_status s) {
+  switch (s) {
+    case LV_OK: return "ok";
+    case LV_EINVAL: return "invalid argument";
+    case LV_EOVERFLOW: return "int64 overflow";
+    case LV_ENODATA: return "not enough data";
+    case LV_ESINGULAR: return "singular normal equations";
+    case LV_ECUDA: return "CUDA error";
+    case LV_EDATA: return "invalid input data";
+    case LV_ENOMEM: return "out of device memory";
+    case LV_ETIMEOUT: return "device wait timed out";
+    default: return "unknown status";
+  }
+}
+
+lv_status lv_arch_constants(const lv_arch *arch, int64_t phi[3], int64_t *weight_bytes) {
+  if (!arch || !phi || !weight_bytes) return LV_EINVAL;
+  const int64_t L = arch->n_layers, d = arch->d_model, hq = arch->n_q_heads, hkv = arch->n_kv_heads;
+  const int64_t hd = arch->head_dim, F = arch->ffn_dim, wb = arch->weight_bytes, kvb = arch->kv_bytes,
+                tp = arch->tp;
+  if (L <= 0 || d <= 0 || hq <= 0 || hkv <= 0 || hd <= 0 || F <= 0 || wb <= 0 || kvb <= 0 || tp <= 0)
+    return LV_EINVAL;
+  if (hq % tp || hkv % tp || F % tp) return LV_EINVAL;
+  bool o = false;
+  auto mul = [&o](int64_t x, int64_t y) {
+    long long r;
+    o |= __builtin_mul_overflow((long long)x, (long long)y, &r);
+    return (int64_t)r;
+  };
+  auto add = [&o](int64_t x, int64_t y) {
+    long long r;
+    o |= __builtin_add_overflow((long long)x, (long long)y, &r);
+    return (int64_t)r;
+  };
+  const int64_t qw = mul(hq, hd), kvw = mul(hkv, hd);
+  int64_t P = add(add(add(mul(d, qw), mul(mul(2, d), kvw)), mul(qw, d)), mul(mul(3, d), F));
+  const int64_t phi0 = mul(mul(2, L), P) / tp;
+  const int64_t phi1 = mul(mul(mul(2, L), kvw), kvb) / tp;
+  const int64_t phi2 = mul(mul(2, L), qw) / tp;
+  const int64_t W = mul(mul(L, P), wb) / tp;
+  if (o) return LV_EOVERFLOW;
+  phi[0] = phi0;
+  phi[1] = phi1;
+  phi[2] = phi2;
+  *weight_bytes = W;
+  return LV_OK;
+}
+
+lv_status lv_ctx_create(lv_ctx **out) {
+  if (!out) return LV_EINVAL;
+  *out = nullptr;
+  lv_ctx *ctx = new (std::nothrow) lv_ctx();
+  if (!ctx) return LV_ENOMEM;
+  if (cudaGetDevice(&ctx->device) != cudaSuccess ||
+      cudaDeviceGetAttribute(&ctx->sms, cudaDevAttrMultiProcessorCount, ctx->device) != cudaSuccess) {
+    delete ctx;
+    return LV_ECUDA;
+  }
+  if (cudaMalloc(&ctx->d_status, sizeof(int)) != cudaSuccess) {
+    delete ctx;
+    return LV_ENOMEM;
+  }
+  if (cudaMemset(ctx->d_status, 0, sizeof(int)) != cudaSuccess ||
+      cudaEventCreateWithFlags(&ctx->ev_built, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&ctx->ev_used, cudaEventDisableTiming) != cudaSuccess) {
+    lv_ctx_destroy(ctx);
+    return LV_ECUDA;
+  }
+  *out = ctx;
+  return LV_OK;
+}
+
+void lv_ctx_destroy(lv_ctx *ctx) {
+  if (!ctx) return;
+  cudaDeviceSynchronize();
+  if (ctx->d_status) cudaFree(ctx->d_status);
+  if (ctx->d_tiles) cudaFree(ctx->d_tiles);
+  if (ctx->d_ktab) cudaFree(ctx->d_ktab);
+  if (ctx->d_fit) cudaFree(ctx->d_fit);
+  if (ctx->d_wi) cudaFree(ctx->d_wi);
+  if (ctx->ev_built) cudaEventDestroy(ctx->ev_built);
+  if (ctx->ev_used) cudaEventDestroy(ctx->ev_used);
+  for (cudaEvent_t e : ctx->tev) cudaEventDestroy(e);
+  delete ctx;
+}
+
+lv_status lv_ctx_set_arith(lv_ctx *ctx, int32_t mode) {
+  if (!ctx || (mode != LV_ARITH_AUTO && mode != LV_ARITH_FP64)) return LV_EINVAL;
+  ctx->arith = mode;
+  return LV_OK;
+}
+
+lv_status lv_ctx_set_timing(lv_ctx *ctx, int32_t enable) {
+  if (!ctx) return LV_EINVAL;
+  ctx->timing = enable != 0;
+  return LV_OK;
+}
+
+lv_status lv_ctx_kernel_time(lv_ctx *ctx, double *ms, int64_t *launches) {
+  if (!ctx || !ms || !launches) return LV_EINVAL;
+  double tot = 0;
+  for (size_t k = 0; k + 1 < ctx->tev_used; k += 2) {
+    LV_CUDA(cudaEventSynchronize(ctx->tev[k + 1]));
+    float m = 0;
+    LV_CUDA(cudaEventElapsedTime(&m, ctx->tev[k], ctx->tev[k + 1]));
+    tot += m;
+  }
+  *ms = tot;
+  *launches = (int64_t)(ctx->tev_used / 2);
+  ctx->tev_used = 0;
+  return LV_OK;
+}
+
+lv_status lv_ctx_status(lv_ctx *ctx, void *stream) {
+  if (!ctx) return LV_EINVAL;
+  LV_CUDA(cudaStreamSynchronize((cudaStream_t)stream));
+  int h = 0;
+  LV_CUDA(cudaMemcpy(&h, ctx->d_status, sizeof(int), cudaMemcpyDeviceToHost));
+  LV_CUDA(cudaMemset(ctx->d_status, 0, sizeof(int)));
+  if (h & kStatusData) return LV_EDATA;
+  if (h & kStatusTimeout) return LV_ETIMEOUT;
+  return LV_OK;
+}
+
+lv_status lv_features(lv_ctx *ctx, const lv_arch *arch, const lv_model *model, const lv_batches *b,
+                      int64_t *req_feat, int64_t *batch_feat, uint8_t *batch_seg, void *stream_) {
+  if (!ctx) return LV_EINVAL;
+  lv_status st = check_batches(b, false);
+  if (st != LV_OK) return st;
+  if (req_feat && (!arch || !aligned(req_feat, 8))) return LV_EINVAL;
+  if (batch_seg && check_model(model) != LV_OK) return LV_EINVAL;
+  if (batch_feat && !aligned(batch_feat, 8)) return LV_EINVAL;
+  cudaStream_t stream = (cudaStream_t)stream_;
+  if (req_feat) {
+    int64_t phi[3], W;
+    st = lv_arch_constants(arch, phi, &W);
+    if (st != LV_OK) return st;
+    if (b->n_req > 0) {
+      const int64_t blocks = std::min<int64_t>((b->n_req + 255) / 256, (int64_t)ctx->sms * 8);
+      k_req_features<<<(unsigned)blocks, 256, 0, stream>>>(b->p, b->c, b->n_req, phi[0], phi[1], phi[2], req_feat,
+                                                           ctx->d_status);
+      LV_CUDA(cudaGetLastError());
+    }
+  }
+  if (batch_feat || batch_seg) {
+    TileArgs a{};
+    a.p = b->p;
+    a.c = b->c;
+    a.ph = b->phase;
+    a.off = b->offsets;
+    a.n_req = b->n_req;
+    a.n_batch = b->n_batch;
+    a.bfeat = batch_feat;
+    a.bseg = batch_seg;
+    a.status = ctx->d_status;
+    if (model) {
+      a.mp.split[0] = model->split[0];
+      a.mp.split[1] = model->split[1];
+    }
+    st = run_tiles(ctx, a, M_FEAT, stream);
+    if (st != LV_OK) return st;
+  }
+  return LV_OK;
+}
+
+lv_status lv_batch_latency(lv_ctx *ctx, const lv_model *model, const int64_t *batch_feat, const uint8_t *batch_seg,
+                           int64_t n_batch, double *T, void *stream_) {
+  if (!ctx || check_model(model) != LV_OK || n_batch < 0) return LV_EINVAL;
+  if (n_batch > 0 && (!batch_feat || !batch_seg || !T || !aligned(batch_feat, 8) || !aligned(T, 8)))
+    return LV_EINVAL;
+  if (n_batch == 0) return LV_OK;
+  cudaStream_t stream = (cudaStream_t)stream_;
+  ModelP mp;
+  lv_status st = prepare_model(ctx, model, stream, &mp);
+  if (st != LV_OK) return st;
+  const int64_t blocks = std::min<int64_t>((n_batch + 255) / 256, (int64_t)ctx->sms * 8);
+  if (mp.fixed)
+    k_batch_latency<true><<<(unsigned)blocks, 256, 0, stream>>>(mp, batch_feat, batch_seg, n_batch, T,
+                                                                ctx->d_status);
+  else
+    k_batch_latency<false><<<(unsigned)blocks, 256, 0, stream>>>(mp, batch_feat, batch_seg, n_batch, T,
+                                                                 ctx->d_status);
+  LV_CUDA(cudaGetLastError());
+  LV_CUDA(cudaEventRecord(ctx->ev_used, stream));
+  return LV_OK;
+}
+
+lv_status lv_attribute(lv_ctx *ctx, const lv_model *model, const lv_batches *b, double *T, double *share,
+                       lv_tenant_acc *acc, void *stream_) {
+  if (!ctx || check_model(model) != LV_OK) return LV_EINVAL;
+  lv_status st = check_batches(b, acc != nullptr);
+  if (st != LV_OK) return st;
+  if (T && !aligned(T, 8)) return LV_EINVAL;
+  if (share && !aligned(share, 8)) return LV_EINVAL;
+  if (b->n_batch > 0 && !T && !share && !acc) return LV_OK;
+  if (acc && (acc->ctx != ctx || acc->n_tenants != b->n_tenants)) return LV_EINVAL;
+  if (b->n_batch > 0 && b->n_req > 0 && !share && !acc && !T) return LV_OK;
+  cudaStream_t stream = (cudaStream_t)stream_;
+  ModelP mp;
+  st = prepare_model(ctx, model, stream, &mp);
+  if (st != LV_OK) return st;
+  TileArgs a{};
+  a.p = b->p;
+  a.c = b->c;
+  a.ph = b->phase;
+  a.ten = acc ? b->tenant : nullptr;
+  a.off = b->offsets;
+  a.n_req = b->n_req;
+  a.n_batch = b->n_batch;
+  a.T = T;
+  a.share = share;
+  a.status = ctx->d_status;
+  a.mp = mp;
+  int mode = M_ATTR | (mp.fixed ? M_FIX : 0);
+  if (acc) {
+    mode |= M_TEN;
+    a.ten_pend = acc->d_pend;
+    a.n_tenants = acc->n_tenants;
+    a.H = std::min<int32_t>(acc->n_tenants, kHotMax);
+  }
+  st = run_tiles(ctx, a, mode, stream);
+  if (st != LV_OK) return st;
+  LV_CUDA(cudaEventRecord(ctx->ev_used, stream));
+  if (acc) return fold_tenants(ctx, acc, stream);
+  return LV_OK;
+}
+
+lv_status lv_tenant_acc_create(lv_ctx *ctx, int32_t n_tenants, lv_tenant_acc **out) {
+  if (!ctx || !out || n_tenants <= 0) return LV_EINVAL;
+  *out = nullptr;
+  lv_tenant_acc *acc = new (std::nothrow) lv_tenant_acc();
+  if (!acc) return LV_ENOMEM;
+  acc->ctx = ctx;
+  acc->n_tenants = n_tenants;
+  if (cudaMalloc(&acc->d_pend, sizeof(unsigned long long) * 4 * (size_t)n_tenants) != cudaSuccess ||
+      cudaMalloc(&acc->d_state, sizeof(i128) * (size_t)n_tenants) != cudaSuccess) {
+    lv_tenant_acc_destroy(acc);
+    return LV_ENOMEM;
+  }
+  if (cudaMemset(acc->d_pend, 0, sizeof(unsigned long long) * 4 * (size_t)n_tenants) != cudaSuccess ||
+      cudaMemset(acc->d_state, 0, sizeof(i128) * (size_t)n_tenants) != cudaSuccess ||
+      cudaDeviceSynchronize() != cudaSuccess) {
+    lv_tenant_acc_destroy(acc);
+    return LV_ECUDA;
+  }
+  *out = acc;
+  return LV_OK;
+}
+
+void lv_tenant_acc_destroy(lv_tenant_acc *acc) {
+  if (!acc) return;
+  cudaDeviceSynchronize();
+  if (acc->d_pend) cudaFree(acc->d_pend);
+  if (acc->d_state) cudaFree(acc->d_state);
+  delete acc;
+}
+
+lv_status lv_tenant_acc_reset(lv_tenant_acc *acc, void *stream) {
+  if (!acc) return LV_EINVAL;
+  LV_CUDA(cudaMemsetAsync(acc->d_pend, 0, sizeof(unsigned long long) * 4 * (size_t)acc->n_tenants,
+                          (cudaStream_t)stream));
+  LV_CUDA(cudaMemsetAsync(acc->d_state, 0, sizeof(i128) * (size_t)acc->n_tenants, (cudaStream_t)stream));
+  return LV_OK;
+}
+
+lv_status lv_tenant_accumulate(lv_ctx *ctx, lv_tenant_acc *acc, const double *share, const int32_t *tenant,
+                               int64_t n_req, void *stream_) {
+  if (!ctx || !acc || acc->ctx != ctx || n_req < 0) return LV_EINVAL;
+  if (n_req > 0 && (!share || !tenant || !aligned(share, 8) || !aligned(tenant, 4))) return LV_EINVAL;
+  cudaStream_t stream = (cudaStream_t)stream_;
+  if (n_req > 0) {
+    const int H = std::min<int32_t>(acc->n_tenants, kHotMax);
+    const size_t smem = sizeof(uint32_t) * 4 * (size_t)H;
+    static bool configured = false;
+    if (!configured) {
+      LV_CUDA(cudaFuncSetAttribute(k_tenant_acc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   (int)(sizeof(uint32_t) * 4 * kHotMax)));
+      configured = true;
+    }
+    const int64_t blocks = std::min<int64_t>((n_req + kBlock - 1) / kBlock, (int64_t)ctx->sms * 4);
+    k_tenant_acc<<<(unsigned)blocks, kBlock, smem, stream>>>(share, tenant, n_req, acc->d_pend, acc->n_tenants, H,
+                                                              ctx->d_status);
+    LV_CUDA(cudaGetLastError());
+  }
+  return fold_tenants(ctx, acc, stream);
+}
+
+lv_status lv_tenant_totals(lv_ctx *ctx, lv_tenant_acc *acc, double *L, void *stream_) {
+  if (!ctx || !acc || acc->ctx != ctx || !L || !aligned(L, 8)) return LV_EINVAL;
+  const int n = acc->n_tenants;
+  k_tenant_totals<<<(n + 255) / 256, 256, 0, (cudaStream_t)stream_>>>(acc->d_state, L, n);
+  LV_CUDA(cudaGetLastError());
+  return LV_OK;
+}
+
+int64_t lv_tenant_acc_state_bytes(const lv_tenant_acc *acc) {
+  return acc ? (int64_t)sizeof(i128) * acc->n_tenants : 0;
+}
+
+lv_status lv_tenant_acc_export(lv_tenant_acc *acc, void *host_state, int64_t bytes, void *stream) {
+  if (!acc || !host_state || bytes != lv_tenant_acc_state_bytes(acc)) return LV_EINVAL;
+  LV_CUDA(cudaMemcpyAsync(host_state, acc->d_state, (size_t)bytes, cudaMemcpyDeviceToHost, (cudaStream_t)stream));
+  LV_CUDA(cudaStreamSynchronize((cudaStream_t)stream));
+  return LV_OK;
+}
+
+lv_status lv_tenant_acc_import(lv_tenant_acc *acc, const void *host_state, int64_t bytes, void *stream) {
+  if (!acc || !host_state || bytes != lv_tenant_acc_state_bytes(acc)) return LV_EINVAL;
+  LV_CUDA(cudaMemsetAsync(acc->d_pend, 0, sizeof(unsigned long long) * 4 * (size_t)acc->n_tenants,
+                          (cudaStream_t)stream));
+  LV_CUDA(cudaMemcpyAsync(acc->d_state, host_state, (size_t)bytes, cudaMemcpyHostToDevice, (cudaStream_t)stream));
+  LV_CUDA(cudaStreamSynchronize((cudaStream_t)stream));
+  return LV_OK;
+}
+
+}  // extern "C"
+
+extern "C" {
+
+lv_status lv_fit(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y, lv_model *inout,
+                 lv_fit_report *rep, void *stream) {
+  (void)ctx; (void)b; (void)y; (void)n_y; (void)inout; (void)rep; (void)stream;
+  return LV_EINVAL;
+}
+
+lv_status lv_whatif(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, const int32_t *p_new,
+                    const int32_t *c_new, const int32_t *phase_new, int64_t n_pending, double *T_new,
+                    double *share_new, void *stream) {
+  (void)ctx; (void)model; (void)cand; (void)p_new; (void)c_new; (void)phase_new; (void)n_pending;
+  (void)T_new; (void)share_new; (void)stream;
+  return LV_EINVAL;
+}
+
+}  // extern "C"
