@@ -119,6 +119,26 @@ __device__ __forceinline__ Rounded fix_to_double(i128 V, int E) {
   return r;
 }
 
+// Same as fix_to_double for the common case 2^64 <= V < 2^127 (V > 0, high
+// word non-zero): no sign handling and a branch-free normalisation.
+__device__ __forceinline__ Rounded fix_to_double_pos(i128 V, int E) {
+  if ((int64_t)V.hi <= 0) return fix_to_double(V, E);
+  const int lz = __clzll((long long)V.hi);  // 1..63
+  const uint64_t top = (V.hi << lz) | (V.lo >> (64 - lz));
+  const uint64_t rest = V.lo << lz;
+  uint64_t m = top >> 11;
+  const uint64_t rb = (top >> 10) & 1ull;
+  const uint64_t st = ((top & 0x3FFull) | rest) != 0 ? 1ull : 0ull;
+  m += rb & (st | (m & 1ull));
+  const int ex = 127 - lz + E;
+  Rounded r;
+  r.d = __longlong_as_double((long long)(((uint64_t)(ex + 1023) << 52) + (m - (1ull << 52))));
+  r.m = m;
+  r.ex = ex - 52;
+  r.neg = false;
+  return r;
+}
+
 // Exact double -> fixed point at 2^E, rounded to nearest (ties to even) when
 // the double has bits below 2^E.  Sets *ovf when the value needs >= 2^125.
 __host__ __device__ __forceinline__ i128 double_to_fix(double x, int E, bool *ovf) {

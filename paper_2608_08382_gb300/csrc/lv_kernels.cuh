@@ -36,7 +36,7 @@ constexpr int kCap = 1280;                         // requests staged per tile
 constexpr int kK = (kCap + kBlock - 1) / kBlock;   // max requests per thread per sub-tile
 constexpr int kBPT = kD / kBlock;                  // max batches per thread in the per-batch phase
 constexpr int kHotMax = 512;                       // tenants kept in shared memory per CTA
-constexpr int kNK = 128;                           // per-batch constants cached in shared memory for n <= kNK
+constexpr int kNK = 256;                           // per-batch constants cached in shared memory for n <= kNK
 constexpr int64_t kPMaxFix = 1ll << 24;            // p beyond this uses the fp64 share path
 constexpr int kTenLsb = -72;                       // tenant totals: shares rounded to 2^-72 s, summed exactly
 
@@ -263,7 +263,8 @@ __device__ __forceinline__ i128 a2_times(const SegFix &f, uint32_t c) {
 }
 
 // share = kf + (A1 + A3 p) p + A2 c, exact, then one rounding.  0 <= p <= 2^24.
-__device__ __forceinline__ Rounded share_fix(const SegFix &f, i128 kf, uint32_t p, uint32_t c) {
+template <class F>
+__device__ __forceinline__ Rounded share_fix(const F &f, i128 kf, uint32_t p, uint32_t c) {
   i128 V;
   if (p == 1) {
     V = add128(kf, f.A13);
@@ -271,8 +272,8 @@ __device__ __forceinline__ Rounded share_fix(const SegFix &f, i128 kf, uint32_t 
     const i128 r = add128(f.A1, mul128_u32(f.A3, p));
     V = add128(kf, mul128_u32(r, p));
   }
-  V = add128(V, a2_times(f, c));
-  return fix_to_double(V, f.E);
+  V = add128(V, f.a2_narrow ? mul_u64_u32(f.A2.lo, c) : mul128_u32(f.A2, c));
+  return fix_to_double_pos(V, f.E);
 }
 
 __device__ __forceinline__ Rounded decompose(double d) {
@@ -305,8 +306,9 @@ __device__ __forceinline__ Rounded decompose(double d) {
 // folded into the exact state by k_tenant_fold.
 
 __device__ __forceinline__ i128 share_to_tenant_fix(const Rounded &r, int *bad) {
-  if (r.m == 0) return mk128(0, 0);
   const int sh = r.ex - kTenLsb;
+  if (!r.neg && sh >= 0 && sh <= 10) return mk128(r.m << sh, 0);  // common case: fits 64 bits
+  if (r.m == 0) return mk128(0, 0);
   i128 q;
   if (sh >= 0) {
     if (sh > 127 - 54) {
@@ -402,6 +404,16 @@ struct TileHdr {
   int64_t b0, b1, r0, r1, staged, lo;
 };
 
+// Per-segment integers the share path needs, kept in shared memory so that a
+// runtime segment index is one shared-memory load (not a select over kernel
+// parameters).
+struct SegS {
+  i128 A1, A3, A13, A2;
+  int E;
+  int a2_narrow;
+  int pad[2];
+};
+
 struct Smem {
   Stage st[2];
   union U {
@@ -416,7 +428,8 @@ struct Smem {
       alignas(16) uint8_t seg[kD];
     } bp;
   } u;
-  alignas(16) i128 kc[4][kNK + 1];  // kf of the K table for n <= kNK
+  alignas(16) double kcd[4][kNK + 1];  // fl(fl(beta/n) + fl(a4*n)) for n <= kNK
+  alignas(16) SegS seg[4];
   TileHdr hdr[2];
   alignas(16) Sums scr[kBlock / 32];
   alignas(8) uint64_t full[2];
@@ -520,29 +533,41 @@ __device__ __forceinline__ void tenant_add(const TileArgs &a, uint32_t *tt, int3
     pend_add(a.ten_pend, u, q);
 }
 
-// Share of one request (kf: per-batch constant; in fp64 mode kf holds {q, a4n}).
-template <int MODE>
-__device__ __forceinline__ Rounded one_share(const TileArgs &a, int s, bool slow, i128 kf, int32_t p, int32_t c,
-                                             int64_t n) {
-  if ((MODE & M_FIX) && !slow && p <= kPMaxFix) return share_fix(a.mp.fx[s], kf, (uint32_t)p, (uint32_t)c);
+// Out-of-line fp64 share (fp64 mode, very large p, or a batch constant outside
+// the fixed-point range).
+__device__ __noinline__ Rounded share_slow(const ModelP &mp, int s, bool fixed, i128 kf, int32_t p, int32_t c,
+                                           int64_t n) {
   double q, a4n;
-  if (MODE & M_FIX) {
+  if (fixed) {
     bool dummy = false;
-    const KEntry e = batch_k(a.mp, s, n, &dummy);
+    const KEntry e = batch_k(mp, s, n, &dummy);
     q = e.q;
     a4n = e.a4n;
   } else {
     q = __longlong_as_double((long long)kf.lo);
     a4n = __longlong_as_double((long long)kf.hi);
   }
-  return decompose(share_fp64(a.mp.coef[s], q, a4n, p, c));
+  return decompose(share_fp64(mp.coef[s], q, a4n, p, c));
+}
+
+// Share of one request (kf: per-batch constant; in fp64 mode kf holds {q, a4n}).
+template <int MODE>
+__device__ __forceinline__ Rounded one_share(const TileArgs &a, const SegS *segs, int s, bool slow, i128 kf,
+                                             int32_t p, int32_t c, int64_t n) {
+  if ((MODE & M_FIX) && !slow && p <= kPMaxFix) return share_fix(segs[s], kf, (uint32_t)p, (uint32_t)c);
+  return share_slow(a.mp, s, (MODE & M_FIX) != 0, kf, p, c, n);
 }
 
 // Per-batch constant for the share phase, as stored in Smem::bp.
 template <int MODE>
 __device__ __forceinline__ i128 batch_const(const TileArgs &a, const Smem &sm, int s, int64_t n, bool *slow) {
   if (MODE & M_FIX) {
-    if (n >= 1 && n <= kNK) return sm.kc[s][n];
+    if (n >= 1 && n <= kNK) {
+      bool ovf = false;
+      const i128 kf = double_to_fix(sm.kcd[s][n], sm.seg[s].E, &ovf);
+      if (ovf) *slow = true;
+      return kf;
+    }
     return batch_k(a.mp, s, n, slow).kf;
   }
   bool dummy = false;
@@ -578,7 +603,7 @@ __device__ void jumbo_batch(const TileArgs &a, Smem &sm, uint32_t *tt, int64_t g
       int32_t p = a.p[i], c = a.c[i], ph = a.ph[i];
       int dummy = 0;
       check_req(p, c, ph, &dummy);
-      const Rounded r = one_share<MODE>(a, s, slow, kf, p, c, g.n);
+      const Rounded r = one_share<MODE>(a, sm.seg, s, slow, kf, p, c, g.n);
       if (a.share) __stcs(a.share + i, r.d);
       if (MODE & M_TEN) tenant_add(a, tt, a.ten[i], r, bad);
     }
@@ -701,7 +726,7 @@ __device__ __forceinline__ void sub_tile(const TileArgs &a, Smem &sm, Stage &st,
     if (k < K && i < i1) {
       while (win[jb + 1] - r0 <= i) ++jb;
       const uint8_t sg = sm.u.bp.seg[jb];
-      const Rounded r = one_share<MODE>(a, sg & 3, (sg & 0x80) != 0, sm.u.bp.kf[jb], rp[k], rc[k],
+      const Rounded r = one_share<MODE>(a, sm.seg, sg & 3, (sg & 0x80) != 0, sm.u.bp.kf[jb], rp[k], rc[k],
                                         win[jb + 1] - win[jb]);
       shs[i] = r.d;
       if (kTen) tenant_add(a, tt, rt[k], r, bad);
@@ -729,7 +754,24 @@ __global__ void __launch_bounds__(kBlock, 2) k_tiles(const TileArgs a) {
   if ((MODE & M_FIX) && (MODE & M_ATTR)) {
     for (int i = tid; i < 4 * (kNK + 1); i += kBlock) {
       const int s = i / (kNK + 1), n = i % (kNK + 1);
-      sm.kc[s][n] = (n >= 1 && n <= a.mp.nk) ? a.mp.ktab[s * (a.mp.nk + 1) + n].kf : mk128(0, 0);
+      double v = 0.0;
+      if (n >= 1 && n <= a.mp.nk) {
+        const KEntry e = a.mp.ktab[s * (a.mp.nk + 1) + n];
+        v = __dadd_rn(e.q, e.a4n);
+      }
+      sm.kcd[s][n] = v;
+    }
+    if (tid < 4) {
+      const SegFix &f = a.mp.fx[tid];
+      SegS g;
+      g.A1 = f.A1;
+      g.A3 = f.A3;
+      g.A13 = f.A13;
+      g.A2 = f.A2;
+      g.E = f.E;
+      g.a2_narrow = f.a2_narrow;
+      g.pad[0] = g.pad[1] = 0;
+      sm.seg[tid] = g;
     }
   }
   if (tid == 0) {
@@ -789,6 +831,7 @@ __global__ void __launch_bounds__(kBlock, 2) k_tiles(const TileArgs a) {
       while (bs < nb) {
         const int64_t r0s = win[bs];
         int lo = bs, hi = nb;  // largest be in (bs, nb] with win[be] - r0s <= kCap
+        if (win[nb] - r0s <= kCap) lo = nb;
         while (lo < hi) {
           const int mid = (lo + hi + 1) >> 1;
           if (win[mid] - r0s <= kCap) lo = mid; else hi = mid - 1;
