@@ -216,6 +216,35 @@ lv_status lv_whatif(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, 
                     const int32_t *c_new, const int32_t *phase_new, int64_t n_pending, double *T_new,
                     double *share_new, void *stream);
 
+/* Attribution without any allocation (the paper has no counterpart; this is a
+ * service to callers that cannot allocate device memory at call time).  A
+ * serving engine typically reserves nearly all GPU memory for its KV cache up
+ * front and must not grow its footprint inside the scheduling loop, and a
+ * cudaMalloc there would also synchronise the device on the latency-critical
+ * path; such a caller cannot create an lv_ctx (which allocates scratch).
+ *
+ * Computes exactly what lv_attribute computes for T and share (no tenant
+ * accumulation), with default arithmetic, using instead of an lv_ctx a fixed
+ * scratch area that lives in the library image as a static device array
+ * (about 1.6 MB on every GPU that loads the library, held until the process
+ * exits).  It calls no cudaMalloc, cudaFree or other allocating routine.
+ *  - Limit: n_batch + n_req must not exceed 67,108,864 (65,536 tiles of 1,024
+ *    batch boundaries and requests); larger inputs return LV_EINVAL before
+ *    anything is launched.
+ *  - status: optional DEVICE int32 (caller-owned).  It is set to 0 on the
+ *    stream, then kernels OR in 1 for invalid input data and 2 for a device
+ *    wait that timed out; read it after synchronising the stream.
+ *  - The first call on each device looks up the scratch array's device address
+ *    (cudaGetSymbolAddress) and caches it; make that first call before any
+ *    stream capture.
+ *  - Every call uses the same scratch array, which keeps the previous call's
+ *    contents (each call rewrites what it reads).  Calls whose work overlaps
+ *    on the GPU (different streams, or several host threads) race on it:
+ *    serialise them.
+ * Other arguments and errors as for lv_attribute. */
+lv_status lv_attribute_noalloc(const lv_model *model, const lv_batches *b, double *T, double *share,
+                               int32_t *status, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

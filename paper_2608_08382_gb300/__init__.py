@@ -28,7 +28,7 @@ EXPORTED = [
     "lv_ctx_set_timing", "lv_ctx_kernel_time",
     "lv_features", "lv_batch_latency", "lv_attribute", "lv_tenant_acc_create", "lv_tenant_acc_destroy",
     "lv_tenant_acc_reset", "lv_tenant_accumulate", "lv_tenant_totals", "lv_tenant_acc_state_bytes",
-    "lv_tenant_acc_export", "lv_tenant_acc_import", "lv_fit", "lv_whatif",
+    "lv_tenant_acc_export", "lv_tenant_acc_import", "lv_fit", "lv_whatif", "lv_attribute_noalloc",
 ]
 
 
@@ -90,6 +90,7 @@ def _load():
         "lv_tenant_acc_import": ([P, P, I64, P], I32),
         "lv_fit": ([P, P, P, I32, P, P, P], I32),
         "lv_whatif": ([P, P, P, P, P, P, I64, P, P, P], I32),
+        "lv_attribute_noalloc": ([P, P, P, P, P, P], I32),
     }
     for name, (args, res) in sig.items():
         f = getattr(L, name)

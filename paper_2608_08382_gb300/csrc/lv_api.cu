@@ -3,6 +3,7 @@
 #include <cuda_runtime.h>
 
 #include <cmath>
+#include <mutex>
 #include <cstdint>
 #include <cstdlib>
 #include <cstring>
@@ -631,3 +632,123 @@ lv_status lv_whatif(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, 
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------- allocation-free attribution
+//
+// lv_attribute_noalloc: the same kernels as lv_attribute (no tenant pass),
+// with the partition and the per-model constant table in a static device array
+// instead of a context's cudaMalloc'd scratch.
+
+namespace {
+
+constexpr int64_t kNoAllocMaxTiles = 1 << 16;  // => n_batch + n_req <= 65,536 * kD
+constexpr size_t kNoAllocPartBytes = sizeof(TilePart) * (size_t)(kNoAllocMaxTiles + 1);
+constexpr size_t kNoAllocTabOffset = (kNoAllocPartBytes + 255) & ~(size_t)255;
+constexpr size_t kNoAllocBytes = kNoAllocTabOffset + sizeof(KEntry) * 4 * (kKTableN + 1);
+
+}  // namespace
+
+// The scratch itself: one copy per device that loads the library.
+static __device__ __align__(256) unsigned char lv_noalloc_scratch[kNoAllocBytes];
+
+namespace {
+
+constexpr int kNoAllocMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void *g_noalloc_ptr[kNoAllocMaxDevices] = {};
+int g_noalloc_sms[kNoAllocMaxDevices] = {};
+
+// Device address of the scratch array on `dev` (looked up once per device, with
+// that device current).
+lv_status noalloc_scratch(int dev, void **ptr, int *sms) {
+  if (dev < 0 || dev >= kNoAllocMaxDevices) return LV_EINVAL;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, lv_noalloc_scratch) != cudaSuccess || !p) return LV_ECUDA;
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return LV_ECUDA;
+    g_noalloc_ptr[dev] = p;
+    g_noalloc_sms[dev] = n;
+  }
+  *ptr = g_noalloc_ptr[dev];
+  *sms = g_noalloc_sms[dev];
+  return LV_OK;
+}
+
+template <int MODE>
+lv_status noalloc_launch_tiles(int sms, const TileArgs &a, cudaStream_t stream) {
+  const size_t smem = sizeof(Smem);
+  LV_CUDA(cudaFuncSetAttribute(k_tiles<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)(sizeof(Smem) + sizeof(uint32_t) * 4 * kHotMax)));
+  int per_sm = 0;
+  LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_tiles<MODE>, kBlock, smem));
+  if (per_sm < 1) per_sm = 1;
+  const int64_t grid = std::min<int64_t>(a.n_tiles, (int64_t)sms * per_sm);
+  if (grid <= 0) return LV_OK;
+  k_tiles<MODE><<<(unsigned)grid, kBlock, smem, stream>>>(a);
+  LV_CUDA(cudaGetLastError());
+  return LV_OK;
+}
+
+}  // namespace
+
+extern "C" lv_status lv_attribute_noalloc(const lv_model *model, const lv_batches *b, double *T, double *share,
+                                          int32_t *status, void *stream_) {
+  if (check_model(model) != LV_OK) return LV_EINVAL;
+  lv_status st = check_batches(b, false);
+  if (st != LV_OK) return st;
+  if (T && !aligned(T, 8)) return LV_EINVAL;
+  if (share && !aligned(share, 8)) return LV_EINVAL;
+  if (status && !aligned(status, 4)) return LV_EINVAL;
+  const int64_t n_tiles = (b->n_batch + b->n_req + kD - 1) / kD;
+  if (n_tiles > kNoAllocMaxTiles) return LV_EINVAL;
+  int dev = 0;
+  LV_CUDA(cudaGetDevice(&dev));
+  void *scratch = nullptr;
+  int sms = 0;
+  st = noalloc_scratch(dev, &scratch, &sms);
+  if (st != LV_OK) return st;
+  cudaStream_t stream = (cudaStream_t)stream_;
+  if (status) LV_CUDA(cudaMemsetAsync(status, 0, sizeof(int32_t), stream));
+  if (b->n_batch == 0 || (!T && !share)) return LV_OK;
+
+  ModelP mp;
+  std::memset(&mp, 0, sizeof(mp));
+  for (int s = 0; s < 4; ++s) {
+    const lv_coef &k = model->seg[s >> 1][s & 1];
+    mp.coef[s][0] = k.beta;
+    mp.coef[s][1] = k.a1;
+    mp.coef[s][2] = k.a2;
+    mp.coef[s][3] = k.a3;
+    mp.coef[s][4] = k.a4;
+  }
+  mp.split[0] = model->split[0];
+  mp.split[1] = model->split[1];
+  mp.nk = kKTableN;
+  mp.fixed = derive_fixed(model, kKTableN, &mp) ? 1 : 0;
+  KEntry *ktab = reinterpret_cast<KEntry *>(static_cast<unsigned char *>(scratch) + kNoAllocTabOffset);
+  mp.ktab = ktab;
+  const int nk = 4 * (kKTableN + 1);
+  k_ktable<<<(nk + 255) / 256, 256, 0, stream>>>(mp, ktab);
+  LV_CUDA(cudaGetLastError());
+
+  TileArgs a{};
+  a.p = b->p;
+  a.c = b->c;
+  a.ph = b->phase;
+  a.off = b->offsets;
+  a.n_req = b->n_req;
+  a.n_batch = b->n_batch;
+  a.T = T;
+  a.share = share;
+  a.status = status;
+  a.mp = mp;
+  a.n_tiles = n_tiles;
+  TilePart *part = static_cast<TilePart *>(scratch);
+  a.part = part;
+  const int64_t pblocks = std::min<int64_t>((b->n_batch + 1 + 255) / 256, (int64_t)sms * 16);
+  k_partition<<<(unsigned)pblocks, 256, 0, stream>>>(a.off, a.n_batch, a.n_req, a.n_tiles, part, status);
+  LV_CUDA(cudaGetLastError());
+  return mp.fixed ? noalloc_launch_tiles<M_ATTR | M_FIX>(sms, a, stream) : noalloc_launch_tiles<M_ATTR>(sms, a, stream);
+}
