@@ -200,8 +200,14 @@ lv_status lv_tenant_acc_import(lv_tenant_acc *acc, const void *host_state, int64
  * lv_fit_report per y vector.  Decode batches have p_i = 1, so S1 == S3: when
  * that holds for every batch of a group the a3 column is dropped and a1
  * carries a1 + a3.  Empty batches are skipped.  The Gram matrix is accumulated
- * exactly in integers and X^T y exactly in fixed point; the solve runs in
- * double-double.  Synchronous: returns after the coefficients are on the host. */
+ * exactly in integers and X^T y exactly in fixed point (y on a 2^-100 s grid);
+ * the solve runs in double-double after power-of-two column scaling.
+ * Limits: 1 <= n_y <= 4; batch sums S1, S2, S3 and n^2 below 2^48 (else
+ * LV_EOVERFLOW); every y finite with |y| < 2^25 s (else LV_EDATA).  Returns LV_OK
+ * once the pass has completed, whatever the groups' outcomes (rep[k].status[g]);
+ * models are left untouched on any other return.  Synchronous: returns after
+ * the coefficients are on the host, and consumes the context's sticky status
+ * (a data error recorded by an earlier asynchronous call is reported here). */
 lv_status lv_fit(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y, lv_model *inout,
                  lv_fit_report *rep, void *stream);
 

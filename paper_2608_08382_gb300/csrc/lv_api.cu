@@ -34,6 +34,7 @@ struct lv_ctx {
   cudaStream_t ktab_stream = nullptr;
   void *d_fit = nullptr;      // fit partials + solve output
   size_t fit_cap = 0;
+  int64_t last_grid = 0;      // CTAs of the most recent tile-kernel launch
   void *d_wi = nullptr;       // what-if per-candidate / per-pending tables
   size_t wi_cap = 0;
   bool timing = false;
@@ -252,6 +253,7 @@ lv_status launch_tiles_mode(lv_ctx *ctx, TileArgs &a, int H, cudaStream_t stream
   LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_tiles<MODE>, kBlock, smem));
   if (per_sm < 1) per_sm = 1;
   const int64_t grid = std::min<int64_t>(a.n_tiles, (int64_t)ctx->sms * per_sm);
+  ctx->last_grid = grid > 0 ? grid : 0;
   if (grid <= 0) return LV_OK;
   cudaEvent_t stop;
   lv_status st = timing_begin(ctx, stream, &stop);
@@ -283,6 +285,7 @@ lv_status run_tiles(lv_ctx *ctx, TileArgs &a, int mode, cudaStream_t stream) {
     case M_ATTR | M_TEN: return launch_tiles_mode<M_ATTR | M_TEN>(ctx, a, H, stream);
     case M_ATTR | M_TEN | M_FIX: return launch_tiles_mode<M_ATTR | M_TEN | M_FIX>(ctx, a, H, stream);
     case M_FEAT: return launch_tiles_mode<M_FEAT>(ctx, a, 0, stream);
+    case M_FEAT | M_FIT: return launch_tiles_mode<M_FEAT | M_FIT>(ctx, a, 0, stream);
     default: return LV_EINVAL;
   }
 }
@@ -618,9 +621,84 @@ lv_status lv_tenant_acc_import(lv_tenant_acc *acc, const void *host_state, int64
 extern "C" {
 
 lv_status lv_fit(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y, lv_model *inout,
-                 lv_fit_report *rep, void *stream) {
-  (void)ctx; (void)b; (void)y; (void)n_y; (void)inout; (void)rep; (void)stream;
-  return LV_EINVAL;
+                 lv_fit_report *rep, void *stream_) {
+  if (!ctx || !inout || n_y < 1 || n_y > kFitMaxY) return LV_EINVAL;
+  lv_status st = check_batches(b, false);
+  if (st != LV_OK) return st;
+  if (b->n_batch > 0 && (!y || !aligned(y, 8))) return LV_EINVAL;
+  for (int k = 1; k < n_y; ++k)
+    if (inout[k].split[0] != inout[0].split[0] || inout[k].split[1] != inout[0].split[1]) return LV_EINVAL;
+  cudaStream_t stream = (cudaStream_t)stream_;
+  // scratch: per-CTA partials (at most 2048 / kBlock CTAs per SM), totals, solve output
+  const int NE = fit_entries(n_y), n_ent = 4 * NE;
+  const int64_t max_cta = (int64_t)ctx->sms * (2048 / kBlock);
+  const size_t o_tot = ((size_t)max_cta * n_ent * sizeof(FitAcc) + 255) & ~(size_t)255;
+  const size_t o_out = (o_tot + (size_t)n_ent * sizeof(FitAcc) + 255) & ~(size_t)255;
+  const size_t need = o_out + sizeof(FitOut) * 4 * kFitMaxY;
+  if (need > ctx->fit_cap) {
+    LV_CUDA(cudaDeviceSynchronize());
+    if (ctx->d_fit) cudaFree(ctx->d_fit);
+    ctx->d_fit = nullptr;
+    ctx->fit_cap = 0;
+    if (cudaMalloc(&ctx->d_fit, need) != cudaSuccess) return LV_ENOMEM;
+    ctx->fit_cap = need;
+  }
+  unsigned char *base = static_cast<unsigned char *>(ctx->d_fit);
+  FitAcc *partial = reinterpret_cast<FitAcc *>(base);
+  FitAcc *totals = reinterpret_cast<FitAcc *>(base + o_tot);
+  FitOut *out = reinterpret_cast<FitOut *>(base + o_out);
+
+  TileArgs a{};
+  a.p = b->p;
+  a.c = b->c;
+  a.ph = b->phase;
+  a.off = b->offsets;
+  a.n_req = b->n_req;
+  a.n_batch = b->n_batch;
+  a.status = ctx->d_status;
+  a.mp.split[0] = inout[0].split[0];
+  a.mp.split[1] = inout[0].split[1];
+  a.fit.y = y;
+  a.fit.n_y = n_y;
+  a.fit.partial = partial;
+  ctx->last_grid = 0;
+  st = run_tiles(ctx, a, M_FEAT | M_FIT, stream);
+  if (st != LV_OK) return st;
+  const int n_cta = (int)ctx->last_grid;
+  k_fit_reduce<<<(n_ent + 127) / 128, 128, 0, stream>>>(partial, n_cta, n_ent, totals);
+  LV_CUDA(cudaGetLastError());
+  k_fit_solve<<<1, 4 * kFitMaxY, 0, stream>>>(totals, n_y, out);
+  LV_CUDA(cudaGetLastError());
+  FitOut h[4 * kFitMaxY];
+  int hs = 0;
+  LV_CUDA(cudaMemcpyAsync(h, out, sizeof(FitOut) * 4 * (size_t)n_y, cudaMemcpyDeviceToHost, stream));
+  LV_CUDA(cudaMemcpyAsync(&hs, ctx->d_status, sizeof(int), cudaMemcpyDeviceToHost, stream));
+  LV_CUDA(cudaMemsetAsync(ctx->d_status, 0, sizeof(int), stream));
+  LV_CUDA(cudaStreamSynchronize(stream));
+  if (hs & kStatusData) return LV_EDATA;
+  if (hs & kStatusOverflow) return LV_EOVERFLOW;
+  if (hs & kStatusTimeout) return LV_ETIMEOUT;
+  for (int k = 0; k < n_y; ++k) {
+    for (int g = 0; g < 4; ++g) {
+      const FitOut &o = h[k * 4 + g];
+      if (rep) {
+        rep[k].n[g] = o.n;
+        rep[k].status[g] = o.status;
+        rep[k].dropped[g] = o.dropped;
+        rep[k].ssr[g] = o.ssr;
+        rep[k].r2[g] = o.r2;
+      }
+      if (o.status == LV_OK) {
+        lv_coef &c = inout[k].seg[g >> 1][g & 1];
+        c.beta = o.coef[0];
+        c.a1 = o.coef[1];
+        c.a2 = o.coef[2];
+        c.a3 = o.coef[3];
+        c.a4 = o.coef[4];
+      }
+    }
+  }
+  return LV_OK;
 }
 
 lv_status lv_whatif(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, const int32_t *p_new,

@@ -42,6 +42,7 @@ constexpr int kTenLsb = -72;                       // tenant totals: shares roun
 
 constexpr int kStatusData = 1;
 constexpr int kStatusTimeout = 2;
+constexpr int kStatusOverflow = 4;
 
 struct SegFix {
   i128 A1, A2, A3;   // exact a_k * 2^-E
@@ -67,6 +68,108 @@ struct ModelP {
   int fixed;           // 1: integer fixed-point path
 };
 
+constexpr int kFitMaxY = 4;             // latency vectors fitted per pass
+constexpr int kFitYLsb = -100;          // X^T y fixed point: y rounded to 2^-100 s
+constexpr int64_t kFitFeatMax = 1ll << 48;
+
+constexpr int kFitYYLsb = 2 * kFitYLsb + 64;  // y'y: floor(Y^2 / 2^64) summed, LSB 2^-136 s^2
+
+// Entries per group: 15 Gram pairs (a <= b), 5 X^T y per y, 1 y'y per y, 1 flag.
+__host__ __device__ constexpr int fit_entries(int n_y) { return 16 + 6 * n_y; }
+
+struct FitAcc {
+  uint64_t w[4];  // 256-bit two's complement (Gram: low 128 bits; flag: w[0])
+};
+
+struct FitArgs {
+  const double *y;  // [n_y][n_batch]
+  int n_y;
+  FitAcc *partial;  // [gridDim.x][4 * fit_entries(n_y)]
+};
+
+__device__ __forceinline__ void acc_add256(uint64_t *w, uint64_t a0, uint64_t a1, uint64_t a2, uint64_t a3) {
+  uint64_t s = w[0] + a0;
+  uint64_t c = s < a0 ? 1ull : 0ull;
+  w[0] = s;
+  s = w[1] + a1;
+  uint64_t c2 = s < a1 ? 1ull : 0ull;
+  s += c;
+  c2 |= (s < c) ? 1ull : 0ull;
+  w[1] = s;
+  s = w[2] + a2;
+  uint64_t c3 = s < a2 ? 1ull : 0ull;
+  s += c2;
+  c3 |= (s < c2) ? 1ull : 0ull;
+  w[2] = s;
+  w[3] = w[3] + a3 + c3;
+}
+
+// Exact y * 2^100 as a signed 128-bit integer (round to nearest even below 2^-100).
+__device__ __forceinline__ i128 y_fixed(double y, bool *ovf) {
+  return double_to_fix(y, kFitYLsb, ovf);
+}
+
+// One batch into the owner's accumulator.  x[0..4] = 1, S1, S2, S3, n^2.
+__device__ __forceinline__ void fit_owner_add(FitAcc &acc, int e, int n_y, const int64_t x[5], const double *yv,
+                                              int64_t nb, int64_t gb, bool s1_ne_s3, int *bad) {
+  if (e < 15) {
+    // Gram pair (a, b), a <= b, in row order
+    int a = 0, r = e;
+    while (r >= 5 - a) {
+      r -= 5 - a;
+      ++a;
+    }
+    const int b = a + r;
+    const uint64_t u = (uint64_t)x[a], v = (uint64_t)x[b];
+    acc_add256(acc.w, u * v, __umul64hi(u, v), 0, 0);
+  } else if (e < 15 + 5 * n_y) {
+    const int col = (e - 15) % 5, k = (e - 15) / 5;
+    bool ovf = false;
+    const i128 Y = y_fixed(yv[k * nb + gb], &ovf);
+    if (ovf) *bad = 1;
+    const bool neg = is_neg128(Y);
+    const i128 M = neg ? neg128(Y) : Y;
+    const uint64_t xv = (uint64_t)x[col];
+    // |Y| * x as 192 bits
+    const uint64_t p0 = M.lo * xv, p1 = __umul64hi(M.lo, xv);
+    const uint64_t q0 = M.hi * xv, q1 = __umul64hi(M.hi, xv);
+    uint64_t w0 = p0, w1 = p1 + q0, w2 = q1 + (w1 < p1 ? 1ull : 0ull), w3 = 0;
+    if (neg) {
+      w0 = ~w0;
+      w1 = ~w1;
+      w2 = ~w2;
+      w3 = ~w3;
+      w0 += 1;
+      if (w0 == 0) {
+        w1 += 1;
+        if (w1 == 0) {
+          w2 += 1;
+          if (w2 == 0) w3 += 1;
+        }
+      }
+    }
+    acc_add256(acc.w, w0, w1, w2, w3);
+  } else if (e < 15 + 6 * n_y) {
+    // y'y: Y^2 (below 2^250) shifted right by 64 bits; a sum of integers, so
+    // order independent, with an error below n * 2^-136 s^2
+    const int k = e - 15 - 5 * n_y;
+    bool ovf = false;
+    i128 Y = y_fixed(yv[k * nb + gb], &ovf);
+    if (ovf) *bad = 1;
+    if (is_neg128(Y)) Y = neg128(Y);
+    const uint64_t l = Y.lo, h = Y.hi;
+    const uint64_t ll1 = __umul64hi(l, l), hl0 = h * l, hl1 = __umul64hi(h, l);
+    const uint64_t hh0 = h * h, hh1 = __umul64hi(h, h);
+    // words 1..3 of l*l + 2^64 * 2*h*l + 2^128 * h*h (word 0 is dropped)
+    uint64_t w[4] = {ll1, hh0, hh1, 0};
+    acc_add256(w, hl0, hl1, 0, 0);
+    acc_add256(w, hl0, hl1, 0, 0);
+    acc_add256(acc.w, w[0], w[1], w[2], 0);
+  } else {
+    if (s1_ne_s3) acc.w[0] |= 1ull;
+  }
+}
+
 // First batch of a tile and its first request.
 struct TilePart {
   int64_t b;
@@ -86,6 +189,7 @@ struct TileArgs {
   int32_t n_tenants, H;
   int *status;
   ModelP mp;
+  FitArgs fit;
 };
 
 __device__ __forceinline__ void flag(int *status, int bit) {
@@ -389,6 +493,7 @@ enum : int {
   M_TEN = 4,     // accumulate tenant totals (with M_ATTR)
   M_FEAT = 8,    // write batch features / segment codes only
   M_FIX = 16,    // fixed-point arithmetic (else fp64)
+  M_FIT = 32,    // accumulate the least-squares statistics (with M_FEAT's reduction)
 };
 
 // One stage of the ring: offsets window and request arrays of one tile.
@@ -429,6 +534,7 @@ struct Smem {
     } bp;
   } u;
   alignas(16) double kcd[4][kNK + 1];  // fl(fl(beta/n) + fl(a4*n)) for n <= kNK
+  alignas(16) uint8_t fseg[kD + 16];   // fit mode: segment of each batch of the sub-tile
   alignas(16) SegS seg[4];
   TileHdr hdr[2];
   alignas(16) Sums scr[kBlock / 32];
@@ -578,7 +684,7 @@ __device__ __forceinline__ i128 batch_const(const TileArgs &a, const Smem &sm, i
 // Block-wide path for one batch with more than kCap requests (reads global memory).
 template <int MODE>
 __device__ void jumbo_batch(const TileArgs &a, Smem &sm, uint32_t *tt, int64_t gb, int64_t r0, int64_t r1,
-                            int *bad) {
+                            FitAcc &facc, int *bad) {
   Sums acc{0, 0, 0, 0};
   for (int64_t i = r0 + threadIdx.x; i < r1; i += kBlock) {
     int32_t p = a.p[i], c = a.c[i], ph = a.ph[i];
@@ -596,6 +702,14 @@ __device__ void jumbo_batch(const TileArgs &a, Smem &sm, uint32_t *tt, int64_t g
   const BatchAgg g{tot.s1, tot.s2, tot.s3, r1 - r0, tot.ph > 0};
   const int s = segment_of(a.mp, g);
   if (threadIdx.x == 0) emit_batch<MODE>(a, gb, g, s);
+  if (MODE & M_FIT) {
+    const int NE = fit_entries(a.fit.n_y);
+    const int64_t x[5] = {1, g.s1, g.s2, g.s3, g.n * g.n};
+    const bool in_range = g.s1 < kFitFeatMax && g.s2 < kFitFeatMax && g.s3 < kFitFeatMax && x[4] < kFitFeatMax;
+    if (!in_range && threadIdx.x == 0) flag(a.status, kStatusOverflow);
+    if ((int)threadIdx.x < 4 * NE && (int)threadIdx.x / NE == s && in_range)
+      fit_owner_add(facc, threadIdx.x % NE, a.fit.n_y, x, a.fit.y, a.n_batch, gb, g.s1 != g.s3, bad);
+  }
   if (MODE & M_ATTR) {
     bool slow = false;
     const i128 kf = batch_const<MODE>(a, sm, s, g.n, &slow);
@@ -614,7 +728,7 @@ __device__ void jumbo_batch(const TileArgs &a, Smem &sm, uint32_t *tt, int64_t g
 // index gb0 + j), staged in `st` from element `base`.
 template <int MODE>
 __device__ __forceinline__ void sub_tile(const TileArgs &a, Smem &sm, Stage &st, uint32_t *tt, const int64_t *win,
-                                         int64_t gb0, int nbt, int64_t r0, int64_t base, int *bad) {
+                                         int64_t gb0, int nbt, int64_t r0, int64_t base, FitAcc &facc, int *bad) {
   constexpr bool kTen = (MODE & M_TEN) != 0;
   constexpr bool kShares = (MODE & M_ATTR) != 0;
   const int tid = threadIdx.x;
@@ -696,6 +810,12 @@ __device__ __forceinline__ void sub_tile(const TileArgs &a, Smem &sm, Stage &st,
       const int s = segment_of(a.mp, g);
       segv[m] = s;
       emit_batch<MODE>(a, gb0 + jb, g, s);
+      if (MODE & M_FIT) {
+        const bool in_range = g.s1 < kFitFeatMax && g.s2 < kFitFeatMax && g.s3 < kFitFeatMax &&
+                              g.n * g.n < kFitFeatMax;
+        if (!in_range) flag(a.status, kStatusOverflow);
+        sm.fseg[jb] = (g.n > 0 && in_range) ? (uint8_t)s : (uint8_t)0xff;
+      }
       slowv[m] = false;
       kv[m] = mk128(0, 0);
       if (kShares && g.n > 0) kv[m] = batch_const<MODE>(a, sm, s, g.n, &slowv[m]);
@@ -703,6 +823,21 @@ __device__ __forceinline__ void sub_tile(const TileArgs &a, Smem &sm, Stage &st,
   }
   if (!kShares) {
     __syncthreads();
+    if (MODE & M_FIT) {
+      // owners: thread (g, e) adds the batches of group g of this sub-tile
+      const int NE = fit_entries(a.fit.n_y);
+      if (tid < 4 * NE) {
+        const int g = tid / NE, e = tid % NE;
+        for (int jb = 0; jb < nbt; ++jb) {
+          if (sm.fseg[jb] != g) continue;
+          const int64_t n = win[jb + 1] - win[jb];
+          const int64_t x[5] = {1, sm.u.pre.s1[jb + 1] - sm.u.pre.s1[jb], sm.u.pre.s2[jb + 1] - sm.u.pre.s2[jb],
+                                sm.u.pre.s3[jb + 1] - sm.u.pre.s3[jb], n * n};
+          fit_owner_add(facc, e, a.fit.n_y, x, a.fit.y, a.n_batch, gb0 + jb, x[1] != x[3], bad);
+        }
+      }
+      __syncthreads();
+    }
     return;
   }
   __syncthreads();  // pre[] is dead from here on; bp[] aliases it
@@ -747,6 +882,8 @@ __global__ void __launch_bounds__(kBlock, 2) k_tiles(const TileArgs a) {
   const int tid = threadIdx.x;
   constexpr bool kTen = (MODE & M_TEN) != 0;
   int bad = 0;
+  FitAcc facc;
+  facc.w[0] = facc.w[1] = facc.w[2] = facc.w[3] = 0;
 
   if (kTen) {
     for (int i = tid; i < 4 * a.H; i += kBlock) tt[i] = 0;
@@ -838,7 +975,7 @@ __global__ void __launch_bounds__(kBlock, 2) k_tiles(const TileArgs a) {
         }
         const int be = lo;
         if (be == bs) {
-          jumbo_batch<MODE>(a, sm, tt, h.b0 + bs, r0s, win[bs + 1], &bad);
+          jumbo_batch<MODE>(a, sm, tt, h.b0 + bs, r0s, win[bs + 1], facc, &bad);
           __syncthreads();
           bs = be + 1;
           continue;
@@ -857,13 +994,17 @@ __global__ void __launch_bounds__(kBlock, 2) k_tiles(const TileArgs a) {
           }
           __syncthreads();
         }
-        sub_tile<MODE>(a, sm, st, tt, win + bs, h.b0 + bs, be - bs, r0s, base, &bad);
+        sub_tile<MODE>(a, sm, st, tt, win + bs, h.b0 + bs, be - bs, r0s, base, facc, &bad);
         bs = be;
       }
     }
     __syncthreads();  // stage s is free for the next issue
   }
   if (bad) flag(a.status, kStatusData);
+  if (MODE & M_FIT) {
+    const int NE = fit_entries(a.fit.n_y);
+    if (tid < 4 * NE) a.fit.partial[(int64_t)blockIdx.x * 4 * NE + tid] = facc;
+  }
   if (kTen) {
     __syncthreads();
     for (int u = tid; u < a.H; u += kBlock) {
