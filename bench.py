@@ -8,7 +8,14 @@ tenant accumulator, then lv_tenant_totals).  Inputs are seeded synthetic
 arrays resident in HBM; they are ~2.2 GB, far larger than L2, so no flush is
 needed between steps.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload attr1|attr4|fit2|whatif3]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload attr1|attr4|fit2|whatif3] [--scale X] [--no-cpu-baseline]
+
+attr1 (the default) is the headline line.  attr4 is the skew stress, fit2 the
+coefficient fit over 2e6 profiled batches (one step = lv_fit of a noisy and a
+noiseless latency vector), whatif3 the what-if pairs (one step = lv_whatif over
+4096 pending x 1024 candidates); each prints a line of the same shape with its
+own metric and the roofline of its dominant kernel.
 
 Prints one JSON line.  Under torchrun each rank processes its own replica of
 the workload (weak scaling, no collective on the data path); timing takes the
@@ -153,33 +160,160 @@ def barrier(world):
 
 # ---------------------------------------------------------------------- workloads
 
+METRIC_FIT = "profiled requests/sec through the coefficient fit on 1 GB300"
+METRIC_WHATIF = "what-if (pending request, candidate batch) pairs/sec on 1 GB300"
+
 WORKLOADS = {
-    "attr1": (1, "qwen2.5-14b tp2 continuous batching: 1e6 batches U{16..256}, ~136M requests, 256 Zipf(1.1) tenants"),
-    "attr4": (4, "llama3.1-8b tp1 skew: 1e7 Pareto(1.5) batches <= 4096, ~25.8M requests, 65536 Zipf(1.2) tenants"),
+    "attr1": ("attr", 1, "qwen2.5-14b tp2 continuous batching: 1e6 batches U{16..256}, ~136M requests, "
+                         "256 Zipf(1.1) tenants"),
+    "attr4": ("attr", 4, "llama3.1-8b tp1 skew: 1e7 Pareto(1.5) batches <= 4096, ~25.8M requests, "
+                         "65536 Zipf(1.2) tenants"),
+    "fit2": ("fit", 2, "llama3.1-8b tp1 fit: 2e6 profiled batches U{1..256}, ~257M requests, noisy (sigma 0.03) "
+                       "and noiseless latency vectors fitted in one pass"),
+    "whatif3": ("whatif", 3, "qwen2.5-32b tp4 what-if: 1024 candidate batches U{32..256} x 4096 pending requests, "
+                             "4,194,304 pairs"),
 }
+
+
+def _workload(args):
+    import workloads
+    kind, k_cfg, desc = WORKLOADS[args.workload]
+    if kind == "whatif":
+        w = workloads.whatif_config(scale=args.scale)
+    else:
+        w = workloads.config(k_cfg, scale=args.scale)
+    if args.scale != 1.0:
+        desc = f"{desc} (scaled x{args.scale}: a profiling case, not the full workload)"
+    return kind, w, desc
+
+
+def _setup_attr(lv, ctx, w, stream):
+    """Step: lv_attribute (T, shares, fused tenant pass) + lv_tenant_totals over config 1 or 4."""
+    import torch
+    b = lv.batches_to_device(w.p, w.c, w.phase, w.offsets, w.tenant, w.n_tenants)
+    model = lv.make_model(w.coef, w.split)
+    T = torch.empty(w.n_batch, dtype=torch.float64, device="cuda")
+    share = torch.empty(w.n_req, dtype=torch.float64, device="cuda")
+    L = torch.empty(w.n_tenants, dtype=torch.float64, device="cuda")
+    acc = lv.TenantAcc(ctx, w.n_tenants)
+
+    def step():
+        lv.lv_attribute(ctx, model, b, T, share, acc, stream=stream)
+        lv.lv_tenant_totals(ctx, acc, L, stream=stream)
+
+    hp = {k: torch.from_numpy(np.ascontiguousarray(v)).pin_memory()
+          for k, v in dict(p=w.p, c=w.c, phase=w.phase, tenant=w.tenant, offsets=w.offsets).items()}
+    h_share = torch.empty(w.n_req, dtype=torch.float64).pin_memory()
+    h_T = torch.empty(w.n_batch, dtype=torch.float64).pin_memory()
+    h_L = torch.empty(w.n_tenants, dtype=torch.float64).pin_memory()
+
+    def e2e_step():
+        for name in ("p", "c", "phase", "tenant", "offsets"):
+            getattr(b, name).copy_(hp[name], non_blocking=True)
+        step()
+        h_share.copy_(share, non_blocking=True)
+        h_T.copy_(T, non_blocking=True)
+        h_L.copy_(L, non_blocking=True)
+
+    return dict(step=step, e2e_step=e2e_step, units=w.n_req, unit="requests/s", metric=METRIC,
+                h2d=sum(int(t.numel() * t.element_size()) for t in hp.values()),
+                d2h=8 * (w.n_req + w.n_batch + w.n_tenants), launches_per_step=4,
+                kernel="k_tiles", time_mask=lv.LV_TIME_TILES, bytes_per_launch=24.0 * w.n_req + 16.0 * w.n_batch,
+                bytes_rule="24 B/request (p, c, phase, tenant read; share written) + 16 B/batch (offset read; T written)",
+                config={"n_batch": w.n_batch, "n_req": w.n_req, "n_tenants": w.n_tenants, "seed": w.seed,
+                        "step": "lv_attribute(T, shares, tenant pass) + lv_tenant_totals"})
+
+
+def _setup_fit(lv, ctx, w, stream):
+    """Step: lv_fit of the noisy and the noiseless latency vectors of config 2 (one pass, synchronous)."""
+    import torch
+    b = lv.batches_to_device(w.p, w.c, w.phase, w.offsets)
+    # latencies of the ground-truth model, from the library's own Eq. 1, times the seeded noise
+    T = torch.empty(w.n_batch, dtype=torch.float64, device="cuda")
+    lv.lv_attribute(ctx, lv.make_model(w.coef, w.split), b, T, None, None, stream=stream)
+    noise = torch.as_tensor(w.noise, device="cuda")
+    Y = torch.stack([T * noise, T]).contiguous()
+    models = [lv.make_model(np.zeros((4, 5)), w.split) for _ in range(2)]
+    out = {}
+
+    def step():
+        out["rep"] = lv.lv_fit(ctx, b, Y, models, stream=stream)
+
+    hp = {k: torch.from_numpy(np.ascontiguousarray(v)).pin_memory()
+          for k, v in dict(p=w.p, c=w.c, phase=w.phase, offsets=w.offsets).items()}
+    hY = Y.cpu().pin_memory()
+
+    def e2e_step():
+        for name in ("p", "c", "phase", "offsets"):
+            getattr(b, name).copy_(hp[name], non_blocking=True)
+        Y.copy_(hY, non_blocking=True)
+        step()
+
+    return dict(step=step, e2e_step=e2e_step, units=w.n_req, unit="requests/s", metric=METRIC_FIT,
+                h2d=sum(int(t.numel() * t.element_size()) for t in hp.values()) + int(hY.numel() * 8),
+                d2h=72 * 4 * 2 + 4, launches_per_step=4, kernel="k_tiles<FEAT|FIT>", time_mask=lv.LV_TIME_TILES,
+                bytes_per_launch=12.0 * w.n_req + 8.0 * (w.n_batch + 1) + 16.0 * w.n_batch,
+                bytes_rule="12 B/request (p, c, phase read) + 8 B/batch offset + 2 x 8 B/batch latencies read",
+                config={"n_batch": w.n_batch, "n_req": w.n_req, "n_y": 2, "seed": w.seed,
+                        "step": "lv_fit(noisy y, noiseless y) incl. solve and coefficient read-back"},
+                check=lambda: out["rep"])
+
+
+def _setup_whatif(lv, ctx, q, stream):
+    """Step: lv_whatif over every (pending request, candidate batch) pair of config 3."""
+    import torch
+    c = q.cand
+    cand = lv.batches_to_device(c.p, c.c, c.phase, c.offsets)
+    t = lambda a: torch.as_tensor(np.ascontiguousarray(a, dtype=np.int32), device="cuda")  # noqa: E731
+    pn, cn, phn = t(q.p_new), t(q.c_new), t(q.phase_new)
+    model = lv.make_model(q.coef, q.split)
+    npairs = q.n_pending * c.n_batch
+    T = torch.empty((q.n_pending, c.n_batch), dtype=torch.float64, device="cuda")
+    S = torch.empty_like(T)
+
+    def step():
+        lv.lv_whatif(ctx, model, cand, pn, cn, phn, T, S, stream=stream)
+
+    hp = {k: torch.from_numpy(np.ascontiguousarray(v)).pin_memory()
+          for k, v in dict(p=c.p, c=c.c, phase=c.phase, offsets=c.offsets).items()}
+    hq = {k: torch.from_numpy(np.ascontiguousarray(v, dtype=np.int32)).pin_memory()
+          for k, v in dict(p=q.p_new, c=q.c_new, phase=q.phase_new).items()}
+    hT = torch.empty(T.shape, dtype=torch.float64).pin_memory()
+    hS = torch.empty(T.shape, dtype=torch.float64).pin_memory()
+
+    def e2e_step():
+        for name in ("p", "c", "phase", "offsets"):
+            getattr(cand, name).copy_(hp[name], non_blocking=True)
+        pn.copy_(hq["p"], non_blocking=True)
+        cn.copy_(hq["c"], non_blocking=True)
+        phn.copy_(hq["phase"], non_blocking=True)
+        step()
+        hT.copy_(T, non_blocking=True)
+        hS.copy_(S, non_blocking=True)
+
+    h2d = sum(int(x.numel() * x.element_size()) for x in list(hp.values()) + list(hq.values()))
+    return dict(step=step, e2e_step=e2e_step, units=npairs, unit="pairs/s", metric=METRIC_WHATIF,
+                h2d=h2d, d2h=16 * npairs, launches_per_step=5, kernel="k_wi_pairs", time_mask=lv.LV_TIME_PAIRS,
+                bytes_per_launch=16.0 * npairs,
+                bytes_rule="16 B/pair written (T_new, share_new); candidate and pending tables are cache-resident",
+                config={"n_cand": c.n_batch, "n_pending": q.n_pending, "pairs": npairs, "seed": q.seed,
+                        "l2": "working set below L2 size: a 512 MB buffer is overwritten before every timed step, "
+                              "outside the step's events",
+                        "step": "lv_whatif (candidate sums, tables, pair kernel)"},
+                flush=True)
 
 
 def run_ours(args, world, rank, local):
     import torch
 
     import paper_2608_08382_gb300 as lv
-    import workloads
 
     torch.cuda.set_device(local)
-    k_cfg, desc = WORKLOADS[args.workload]
-    w = workloads.config(k_cfg)
-    b = lv.batches_to_device(w.p, w.c, w.phase, w.offsets, w.tenant, w.n_tenants)
+    kind, w, desc = _workload(args)
     ctx = lv.Context()
-    model = lv.make_model(w.coef, w.split)
-    T = torch.empty(w.n_batch, dtype=torch.float64, device="cuda")
-    share = torch.empty(w.n_req, dtype=torch.float64, device="cuda")
-    L = torch.empty(w.n_tenants, dtype=torch.float64, device="cuda")
-    acc = lv.TenantAcc(ctx, w.n_tenants)
     stream = torch.cuda.current_stream()
-
-    def step():
-        lv.lv_attribute(ctx, model, b, T, share, acc, stream=stream)
-        lv.lv_tenant_totals(ctx, acc, L, stream=stream)
+    s = {"attr": _setup_attr, "fit": _setup_fit, "whatif": _setup_whatif}[kind](lv, ctx, w, stream)
+    step = s["step"]
 
     for _ in range(args.warmup):
         step()
@@ -190,53 +324,46 @@ def run_ours(args, world, rank, local):
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
-    ctx.set_timing(True)
+    ctx.set_timing(s["time_mask"])
     ctx.kernel_time()
     barrier(world)
     torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        step()
-    e1.record(stream)
-    torch.cuda.synchronize()
+    if s.get("flush"):
+        # the step's working set fits in L2: overwrite a 512 MB buffer before every step, outside its events
+        scrub = torch.empty(512 << 20, dtype=torch.uint8, device="cuda")
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        for a, z in ev:
+            scrub.fill_(1)
+            a.record(stream)
+            step()
+            z.record(stream)
+        torch.cuda.synchronize()
+        ms = sum(a.elapsed_time(z) for a, z in ev)
+        del scrub
+    else:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
     barrier(world)
-    ms = e0.elapsed_time(e1)
     kms, klaunch = ctx.kernel_time()
-    ctx.set_timing(False)
+    ctx.set_timing(0)
     clk = clocks.stop()
     ms_max = max_over_ranks(ms, world)
     status = ctx.status()
 
-    # ---- end to end through the public API with pinned host buffers
-    hp = {k: torch.from_numpy(np.ascontiguousarray(v)).pin_memory()
-          for k, v in dict(p=w.p, c=w.c, phase=w.phase, tenant=w.tenant, offsets=w.offsets).items()}
-    h_share = torch.empty(w.n_req, dtype=torch.float64).pin_memory()
-    h_T = torch.empty(w.n_batch, dtype=torch.float64).pin_memory()
-    h_L = torch.empty(w.n_tenants, dtype=torch.float64).pin_memory()
-    h2d = sum(int(t.numel() * t.element_size()) for t in hp.values())
-    d2h = int(h_share.numel() * 8 + h_T.numel() * 8 + h_L.numel() * 8)
-
-    def e2e_step():
-        b.p.copy_(hp["p"], non_blocking=True)
-        b.c.copy_(hp["c"], non_blocking=True)
-        b.phase.copy_(hp["phase"], non_blocking=True)
-        b.tenant.copy_(hp["tenant"], non_blocking=True)
-        b.offsets.copy_(hp["offsets"], non_blocking=True)
-        lv.lv_attribute(ctx, model, b, T, share, acc, stream=stream)
-        lv.lv_tenant_totals(ctx, acc, L, stream=stream)
-        h_share.copy_(share, non_blocking=True)
-        h_T.copy_(T, non_blocking=True)
-        h_L.copy_(L, non_blocking=True)
-
-    e2e_step()
+    # ---- end to end through the public API, inputs from pinned host memory, results back to the host
+    s["e2e_step"]()
     torch.cuda.synchronize()
     barrier(world)
     f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     n_e2e = max(1, min(args.steps, 5))
     f0.record(stream)
     for _ in range(n_e2e):
-        e2e_step()
+        s["e2e_step"]()
     f1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(f0.elapsed_time(f1), world) / n_e2e
@@ -245,16 +372,17 @@ def run_ours(args, world, rank, local):
         return None
 
     step_ms = ms_max / args.steps
-    value = world * w.n_req / (step_ms / 1e3)
-    bytes_per_launch = 24.0 * w.n_req + 16.0 * w.n_batch
+    value = world * s["units"] / (step_ms / 1e3)
     kavg_ms = kms / max(klaunch, 1)
-    achieved = bytes_per_launch / (kavg_ms / 1e3) / 1e9
+    achieved = s["bytes_per_launch"] / (kavg_ms / 1e3) / 1e9
     peak, peak_kind = measured_peaks()
-    traffic = ncu_traffic("k_tiles", args.workload)
+    traffic = ncu_traffic(s["kernel"].split("<")[0], args.workload)
+    config = {"workload": desc, **s["config"], "parallelism": f"replicas{world}"}
+    config.setdefault("l2", "inputs far larger than the 129 MB L2, no flush")
     line = {
-        "metric": METRIC,
+        "metric": s["metric"],
         "value": value,
-        "unit": "requests/s",
+        "unit": s["unit"],
         "n_gpus": world,
         "steps": args.steps,
         "warmup": args.warmup,
@@ -264,78 +392,94 @@ def run_ours(args, world, rank, local):
         "vs_baseline": None,
         "dtype": "f64",
         "data": "synthetic",
-        "config": {"workload": desc, "n_batch": w.n_batch, "n_req": w.n_req, "n_tenants": w.n_tenants,
-                   "seed": w.seed, "l2": "inputs 2.2 GB >> 129 MB L2, no flush", "parallelism": f"replicas{world}",
-                   "step": "lv_attribute(T, shares, tenant pass 1+2) + lv_tenant_totals"},
-        "hbm_gbs_step": bytes_per_launch / (step_ms / 1e3) / 1e9,
+        "config": config,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                     "traffic": traffic, "kernel": "k_tiles", "peak_source": peak_kind,
-                     "algorithmic_bytes_per_launch": bytes_per_launch, "kernel_ms_avg": kavg_ms,
-                     "kernel_launches": klaunch},
-        "e2e": {"value": world * w.n_req / (e2e_ms / 1e3), "unit": "requests/s", "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
-        "gpu_launches": 4 * args.steps,
+                     "traffic": traffic, "kernel": s["kernel"], "peak_source": peak_kind,
+                     "algorithmic_bytes_per_launch": s["bytes_per_launch"], "bytes_rule": s["bytes_rule"],
+                     "kernel_ms_avg": kavg_ms, "kernel_launches": klaunch},
+        "e2e": {"value": world * s["units"] / (e2e_ms / 1e3), "unit": s["unit"], "h2d_bytes_per_step": s["h2d"],
+                "d2h_bytes_per_step": s["d2h"], "ms_per_step": e2e_ms},
+        "gpu_launches": s["launches_per_step"] * args.steps,
         "clocks": clk,
         "status": lv.lv_status_string(status),
     }
     if not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(w, min_seconds=args.cpu_seconds)
+        line["cpu_baseline"] = cpu_baseline(kind, w, min_seconds=args.cpu_seconds)
     return line
 
 
-def cpu_baseline(w, min_seconds=10.0):
-    """The oracle as it stands, single-threaded, on a 10 % sample of the workload's batches."""
+def _oracle_sample(kind, w):
+    """A bounded piece of the workload for the oracle and the function that processes it once.
+
+    Returns (run, units per run, description)."""
     import oracle
-    nb = max(1, w.n_batch // 10)
+    oracle.build()
+    if kind == "whatif":
+        c = w.cand
+        rows = 64
+        pn, cn, phn = w.p_new[:rows], w.c_new[:rows], w.phase_new[:rows]
+
+        def run():
+            oracle.whatif(c.offsets, c.p, c.c, c.phase, pn, cn, phn, w.split, w.coef)
+        return run, rows * c.n_batch, f"first {rows} of {w.n_pending} pending requests x all {c.n_batch} candidates"
+    frac = 10 if kind == "attr" else 200
+    nb = max(1, w.n_batch // frac)
     hi = int(w.offsets[nb])
     off = w.offsets[:nb + 1]
-    p, c, ph, t = w.p[:hi], w.c[:hi], w.phase[:hi], w.tenant[:hi]
-    oracle.build()
+    p, c, ph = w.p[:hi], w.c[:hi], w.phase[:hi]
+    if kind == "attr":
+        t = w.tenant[:hi]
+
+        def run():
+            _, s = oracle.attribute(off, p, c, ph, w.split, w.coef)
+            oracle.tenant_totals(s, t, w.n_tenants)
+        return run, hi, f"first {nb} of {w.n_batch} batches ({hi} requests), attribution + tenant totals"
+    T, _ = oracle.attribute(off, p, c, ph, w.split, w.coef)
+    Y = np.stack([T * w.noise[:nb], T])
+
+    def run():
+        feat, seg = oracle.batch_features(off, p, c, ph, w.split)
+        for y in Y:
+            oracle.fit(feat, seg, y)
+    return run, hi, f"first {nb} of {w.n_batch} batches ({hi} requests), batch sums + exact fit of 2 latency vectors"
+
+
+def cpu_baseline(kind, w, min_seconds=10.0):
+    """The oracle as it stands, single-threaded, on a bounded sample of the workload."""
+    run, units, sample = _oracle_sample(kind, w)
     done, t0 = 0, time.perf_counter()
     while True:
-        _, s = oracle.attribute(off, p, c, ph, w.split, w.coef)
-        oracle.tenant_totals(s, t, w.n_tenants)
-        done += hi
+        run()
+        done += units
         el = time.perf_counter() - t0
         if el >= min_seconds:
             break
-    return {"value": done / el, "unit": "requests/s", "cores": 1, "kind": "oracle",
-            "sample": f"first {nb} of {w.n_batch} batches ({hi} requests) repeated for {el:.1f} s, "
-                      "attribution + tenant totals, single thread"}
+    unit = "pairs/s" if kind == "whatif" else "requests/s"
+    return {"value": done / el, "unit": unit, "cores": 1, "kind": "oracle",
+            "sample": f"{sample}; repeated for {el:.1f} s, single thread"}
 
 
 def run_reference(args, world, rank):
     if rank != 0:
         return None
-    import workloads
-    k_cfg, desc = WORKLOADS[args.workload]
-    w = workloads.config(k_cfg)
-    import oracle
-    oracle.build()
-    nb = max(1, w.n_batch // 10)
-    hi = int(w.offsets[nb])
-    off = w.offsets[:nb + 1]
-    p, c, ph, t = w.p[:hi], w.c[:hi], w.phase[:hi], w.tenant[:hi]
-
-    def step():
-        _, s = oracle.attribute(off, p, c, ph, w.split, w.coef)
-        oracle.tenant_totals(s, t, w.n_tenants)
-
+    kind, w, desc = _workload(args)
+    run, units, sample = _oracle_sample(kind, w)
     for _ in range(args.warmup):
-        step()
+        run()
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        step()
+        run()
     el = time.perf_counter() - t0
-    value = hi * args.steps / el
-    sample = f"first {nb} of {w.n_batch} batches ({hi} requests) per step, single thread"
-    return {"impl": "reference", "metric": METRIC, "value": value, "unit": "requests/s", "n_gpus": world,
+    value = units * args.steps / el
+    unit = "pairs/s" if kind == "whatif" else "requests/s"
+    metric = {"attr": METRIC, "fit": METRIC_FIT, "whatif": METRIC_WHATIF}[kind]
+    return {"impl": "reference", "metric": metric, "value": value, "unit": unit, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": desc, "n_batch": w.n_batch, "n_req": w.n_req, "n_tenants": w.n_tenants,
-                       "seed": w.seed, "parallelism": "host"},
-            "cpu_baseline": {"value": value, "unit": "requests/s", "cores": 1, "kind": "oracle", "sample": sample},
-            "e2e": {"value": value, "unit": "requests/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+            "config": {"workload": desc, "parallelism": "host", "sample": sample},
+            "cpu_baseline": {"value": value, "unit": unit, "cores": 1, "kind": "oracle",
+                             "sample": f"{sample} per step, single thread"},
+            "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
 def main():
@@ -347,6 +491,8 @@ def main():
     ap.add_argument("--workload", default="attr1", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--scale", type=float, default=1.0,
+                    help="batches x scale; values other than 1 make a smaller case for profiler captures")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

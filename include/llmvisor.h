@@ -122,13 +122,17 @@ lv_status lv_ctx_set_arith(lv_ctx *ctx, int32_t mode);
 lv_status lv_ctx_status(lv_ctx *ctx, void *stream);
 /* Static description of a status code. */
 const char *lv_status_string(lv_status s);
-/* Measurement support (no counterpart in the paper).  With timing enabled the
- * library brackets every launch of its request-streaming kernels (the tile
- * kernel of lv_attribute / lv_features / lv_fit, the pair kernel of lv_whatif)
- * with CUDA events on the launching stream.  lv_ctx_kernel_time synchronises
- * those events, returns the summed milliseconds and the number of launches
- * since the previous query, and resets the tally.  Off by default. */
-lv_status lv_ctx_set_timing(lv_ctx *ctx, int32_t enable);
+/* Measurement support (no counterpart in the paper).  `mask` selects which
+ * request-streaming kernels the library brackets with CUDA events on the
+ * launching stream: LV_TIME_TILES the tile kernel of lv_attribute /
+ * lv_features / lv_fit / lv_whatif's candidate pass, LV_TIME_PAIRS the pair
+ * kernel of lv_whatif; 0 (the default) none.  Other bits: LV_EINVAL.
+ * lv_ctx_kernel_time synchronises those events, returns the summed
+ * milliseconds and the number of launches since the previous query, and
+ * resets the tally. */
+#define LV_TIME_TILES 1
+#define LV_TIME_PAIRS 2
+lv_status lv_ctx_set_timing(lv_ctx *ctx, int32_t mask);
 lv_status lv_ctx_kernel_time(lv_ctx *ctx, double *ms, int64_t *launches);
 
 /* Architecture constants (Section 2.1: features proportional to FLOPs and to

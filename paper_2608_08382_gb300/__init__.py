@@ -22,6 +22,7 @@ LIB_PATH = os.path.join(_HERE, "_build", "libllmvisor.so")
 LV_OK, LV_EINVAL, LV_EOVERFLOW, LV_ENODATA, LV_ESINGULAR, LV_ECUDA, LV_EDATA, LV_ENOMEM, LV_ETIMEOUT = (
     0, -1, -2, -3, -4, -5, -6, -7, -8)
 LV_ARITH_AUTO, LV_ARITH_FP64 = 0, 1
+LV_TIME_TILES, LV_TIME_PAIRS = 1, 2
 
 EXPORTED = [
     "lv_status_string", "lv_arch_constants", "lv_ctx_create", "lv_ctx_destroy", "lv_ctx_set_arith", "lv_ctx_status",
@@ -203,8 +204,9 @@ class Context:
     def set_arith(self, mode: int):
         _check(_lib.lv_ctx_set_arith(self.h, int(mode)), "lv_ctx_set_arith")
 
-    def set_timing(self, enable: bool):
-        _check(_lib.lv_ctx_set_timing(self.h, int(bool(enable))), "lv_ctx_set_timing")
+    def set_timing(self, mask):
+        """mask: LV_TIME_TILES | LV_TIME_PAIRS, or 0 (True selects LV_TIME_TILES)."""
+        _check(_lib.lv_ctx_set_timing(self.h, int(mask)), "lv_ctx_set_timing")
 
     def kernel_time(self):
         """(milliseconds, launches) of the timed kernels since the previous query."""

@@ -37,7 +37,7 @@ struct lv_ctx {
   int64_t last_grid = 0;      // CTAs of the most recent tile-kernel launch
   void *d_wi = nullptr;       // what-if per-candidate / per-pending tables
   size_t wi_cap = 0;
-  bool timing = false;
+  int timing = 0;  // LV_TIME_* mask
   std::vector<cudaEvent_t> tev;  // start/stop pairs
   size_t tev_used = 0;
 };
@@ -218,9 +218,9 @@ lv_status prepare_model(lv_ctx *ctx, const lv_model *m, cudaStream_t stream, Mod
 }
 
 // Event pair around a measured launch (when timing is on).
-lv_status timing_begin(lv_ctx *ctx, cudaStream_t stream, cudaEvent_t *stop) {
+lv_status timing_begin(lv_ctx *ctx, int kind, cudaStream_t stream, cudaEvent_t *stop) {
   *stop = nullptr;
-  if (!ctx->timing) return LV_OK;
+  if (!(ctx->timing & kind)) return LV_OK;
   if (ctx->tev_used + 2 > ctx->tev.size()) {
     for (int k = 0; k < 2; ++k) {
       cudaEvent_t e;
@@ -256,7 +256,7 @@ lv_status launch_tiles_mode(lv_ctx *ctx, TileArgs &a, int H, cudaStream_t stream
   ctx->last_grid = grid > 0 ? grid : 0;
   if (grid <= 0) return LV_OK;
   cudaEvent_t stop;
-  lv_status st = timing_begin(ctx, stream, &stop);
+  lv_status st = timing_begin(ctx, LV_TIME_TILES, stream, &stop);
   if (st != LV_OK) return st;
   k_tiles<MODE><<<(unsigned)grid, kBlock, smem, stream>>>(a);
   LV_CUDA(cudaGetLastError());
@@ -395,7 +395,8 @@ lv_status lv_ctx_set_arith(lv_ctx *ctx, int32_t mode) {
 
 lv_status lv_ctx_set_timing(lv_ctx *ctx, int32_t enable) {
   if (!ctx) return LV_EINVAL;
-  ctx->timing = enable != 0;
+  if (enable & ~(LV_TIME_TILES | LV_TIME_PAIRS)) return LV_EINVAL;
+  ctx->timing = enable;
   return LV_OK;
 }
 
@@ -761,7 +762,7 @@ lv_status lv_whatif(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, 
     const int64_t rows = std::min<int64_t>(rows_per_launch, np - j);
     const dim3 grid((unsigned)gx, (unsigned)((rows + kWiRows - 1) / kWiRows));
     cudaEvent_t stop;
-    st = timing_begin(ctx, stream, &stop);
+    st = timing_begin(ctx, LV_TIME_PAIRS, stream, &stop);
     if (st != LV_OK) return st;
     k_wi_pairs<<<grid, kWiCols, 0, stream>>>(mp, candp, pendp, nc, np, j, T_new, share_new);
     LV_CUDA(cudaGetLastError());

@@ -87,3 +87,11 @@ def test_import_fails_loudly_without_library(tmp_path):
     r = subprocess.run([sys.executable, "-c", "import paper_2608_08382_gb300"], cwd=tmp_path, capture_output=True,
                        text=True)
     assert r.returncode != 0 and "not built" in r.stderr
+
+
+def test_binding_constants_match_header(lv):
+    src = open(os.path.join(ROOT, "include", "llmvisor.h")).read()
+    defs = dict(re.findall(r"#define\s+(LV_[A-Z_0-9]+)\s+\(?(-?\d+)\)?", src))
+    assert len(defs) >= 13
+    for name, value in defs.items():
+        assert getattr(lv, name) == int(value), name
