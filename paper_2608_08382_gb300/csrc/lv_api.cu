@@ -13,6 +13,7 @@
 #include "llmvisor.h"
 #include "lv_fit.cuh"
 #include "lv_kernels.cuh"
+#include "lv_warp.cuh"
 #include "lv_whatif.cuh"
 
 using namespace lv;
@@ -24,6 +25,9 @@ struct lv_ctx {
   int *d_status = nullptr;
   TilePart *d_tiles = nullptr;
   int64_t tiles_cap = 0;
+  unsigned long long *d_ctr = nullptr;  // [0] warp tiles handed out, [1] jumbo batches queued
+  int64_t *d_jumbo = nullptr;
+  int64_t jumbo_cap = 0;
   KEntry *d_ktab = nullptr;
   int ktab_nk = 0;
   bool ktab_valid = false;
@@ -240,52 +244,98 @@ lv_status timing_end(cudaEvent_t stop, cudaStream_t stream) {
   return LV_OK;
 }
 
+// Dynamic shared memory of k_warps for a tenant table of H entries and n_y fit vectors.
 template <int MODE>
-lv_status launch_tiles_mode(lv_ctx *ctx, TileArgs &a, int H, cudaStream_t stream) {
-  static bool configured = false;
-  const size_t smem = sizeof(Smem) + sizeof(uint32_t) * 4 * (size_t)H;
-  if (!configured) {
-    LV_CUDA(cudaFuncSetAttribute(k_tiles<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)(sizeof(Smem) + sizeof(uint32_t) * 4 * kHotMax)));
-    configured = true;
-  }
-  int per_sm = 0;
-  LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_tiles<MODE>, kBlock, smem));
-  if (per_sm < 1) per_sm = 1;
-  const int64_t grid = std::min<int64_t>(a.n_tiles, (int64_t)ctx->sms * per_sm);
-  ctx->last_grid = grid > 0 ? grid : 0;
-  if (grid <= 0) return LV_OK;
-  cudaEvent_t stop;
-  lv_status st = timing_begin(ctx, LV_TIME_TILES, stream, &stop);
-  if (st != LV_OK) return st;
-  k_tiles<MODE><<<(unsigned)grid, kBlock, smem, stream>>>(a);
-  LV_CUDA(cudaGetLastError());
-  return timing_end(stop, stream);
+size_t warps_smem(int H, int n_y) {
+  return sizeof(WSmem) + ((MODE & M_TEN) ? 16 * (size_t)H : 0) +
+         ((MODE & M_FIT) ? (size_t)kWarps * 4 * fit_entries(n_y) * sizeof(FitAcc) : 0);
 }
 
-// Partition + tile kernel for the given batches.
-lv_status run_tiles(lv_ctx *ctx, TileArgs &a, int mode, cudaStream_t stream) {
-  const int64_t units = a.n_batch + a.n_req;
-  a.n_tiles = (units + kD - 1) / kD;
-  if (a.n_batch == 0) {
-    return LV_OK;
+constexpr int kJumboCtasPerSm = 2;
+
+// Upper bound on the CTAs of one k_warps + k_jumbo pair (rows of fit partials).
+int64_t max_tile_ctas(int sms) { return (int64_t)sms * (2048 / kWThreads + kJumboCtasPerSm); }
+
+// k_warps then k_jumbo for the partitioned batches in `a` (a.part, a.ctr,
+// a.jumbo* set, counters zeroed on `stream`).  *ctas receives the number of
+// CTAs launched (fit partial rows).  ctx may be null (no timing).
+template <int MODE>
+lv_status launch_warps_mode(lv_ctx *ctx, int sms, TileArgs &a, cudaStream_t stream, int64_t *ctas) {
+  *ctas = 0;
+  const size_t smem = warps_smem<MODE>(a.H, a.fit.n_y);
+  LV_CUDA(cudaFuncSetAttribute(k_warps<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)warps_smem<MODE>(kHotMax, kFitMaxY)));
+  const size_t jsmem = sizeof(JSmem) + ((MODE & M_TEN) ? 16 * (size_t)a.H : 0);
+  LV_CUDA(cudaFuncSetAttribute(k_jumbo<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)(sizeof(JSmem) + 16 * (size_t)kHotMax)));
+  int per_sm = 0;
+  LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_warps<MODE>, kWThreads, smem));
+  if (per_sm < 1) per_sm = 1;
+  const int64_t grid = std::min<int64_t>(a.n_tiles, (int64_t)sms * per_sm);
+  if (grid <= 0) return LV_OK;
+  const int64_t jgrid = (int64_t)sms * kJumboCtasPerSm;
+  cudaEvent_t stop = nullptr;
+  if (ctx) {
+    lv_status st = timing_begin(ctx, LV_TIME_TILES, stream, &stop);
+    if (st != LV_OK) return st;
   }
+  k_warps<MODE><<<(unsigned)grid, kWThreads, smem, stream>>>(a);
+  LV_CUDA(cudaGetLastError());
+  k_jumbo<MODE><<<(unsigned)jgrid, kJBlock, jsmem, stream>>>(a, (int)grid);
+  LV_CUDA(cudaGetLastError());
+  *ctas = grid + jgrid;
+  return ctx ? timing_end(stop, stream) : LV_OK;
+}
+
+lv_status ensure_sched(lv_ctx *ctx, int64_t jumbo_cap) {
+  if (!ctx->d_ctr && cudaMalloc(&ctx->d_ctr, 2 * sizeof(unsigned long long)) != cudaSuccess) {
+    ctx->d_ctr = nullptr;
+    return LV_ENOMEM;
+  }
+  if (jumbo_cap <= ctx->jumbo_cap) return LV_OK;
+  LV_CUDA(cudaDeviceSynchronize());
+  if (ctx->d_jumbo) cudaFree(ctx->d_jumbo);
+  ctx->d_jumbo = nullptr;
+  ctx->jumbo_cap = 0;
+  const int64_t cap = std::max<int64_t>(jumbo_cap, 1 << 12);
+  if (cudaMalloc(&ctx->d_jumbo, sizeof(int64_t) * cap) != cudaSuccess) return LV_ENOMEM;
+  ctx->jumbo_cap = cap;
+  return LV_OK;
+}
+
+// Most batches of more than kJumbo requests that valid offsets allow.
+int64_t jumbo_bound(int64_t n_req) { return n_req / (kJumbo + 1) + 1; }
+
+// Partition + warp and jumbo kernels for the given batches.
+lv_status run_tiles(lv_ctx *ctx, TileArgs &a, int mode, cudaStream_t stream) {
+  ctx->last_grid = 0;
+  const int64_t units = a.n_batch + a.n_req;
+  a.n_tiles = (units + kDW - 1) / kDW;
+  if (a.n_batch == 0) return LV_OK;
   lv_status st = ensure_tiles(ctx, a.n_tiles + 1);
   if (st != LV_OK) return st;
+  st = ensure_sched(ctx, jumbo_bound(a.n_req));
+  if (st != LV_OK) return st;
   a.part = ctx->d_tiles;
+  a.ctr = ctx->d_ctr;
+  a.jumbo_n = ctx->d_ctr + 1;
+  a.jumbo = ctx->d_jumbo;
+  a.jumbo_cap = ctx->jumbo_cap;
+  LV_CUDA(cudaMemsetAsync(ctx->d_ctr, 0, 2 * sizeof(unsigned long long), stream));
   const int64_t nthreads = a.n_batch + 1;
   const int64_t pblocks = std::min<int64_t>((nthreads + 255) / 256, (int64_t)ctx->sms * 16);
-  k_partition<<<(unsigned)pblocks, 256, 0, stream>>>(a.off, a.n_batch, a.n_req, a.n_tiles, ctx->d_tiles,
+  k_partition<<<(unsigned)pblocks, 256, 0, stream>>>(a.off, a.n_batch, a.n_req, a.n_tiles, kDW, ctx->d_tiles,
                                                      ctx->d_status);
   LV_CUDA(cudaGetLastError());
-  const int H = a.H;
+  int64_t *g = &ctx->last_grid;
+  const int sms = ctx->sms;
   switch (mode) {
-    case M_ATTR: return launch_tiles_mode<M_ATTR>(ctx, a, H, stream);
-    case M_ATTR | M_FIX: return launch_tiles_mode<M_ATTR | M_FIX>(ctx, a, H, stream);
-    case M_ATTR | M_TEN: return launch_tiles_mode<M_ATTR | M_TEN>(ctx, a, H, stream);
-    case M_ATTR | M_TEN | M_FIX: return launch_tiles_mode<M_ATTR | M_TEN | M_FIX>(ctx, a, H, stream);
-    case M_FEAT: return launch_tiles_mode<M_FEAT>(ctx, a, 0, stream);
-    case M_FEAT | M_FIT: return launch_tiles_mode<M_FEAT | M_FIT>(ctx, a, 0, stream);
+    case M_ATTR: return launch_warps_mode<M_ATTR>(ctx, sms, a, stream, g);
+    case M_ATTR | M_FIX: return launch_warps_mode<M_ATTR | M_FIX>(ctx, sms, a, stream, g);
+    case M_ATTR | M_TEN: return launch_warps_mode<M_ATTR | M_TEN>(ctx, sms, a, stream, g);
+    case M_ATTR | M_TEN | M_FIX: return launch_warps_mode<M_ATTR | M_TEN | M_FIX>(ctx, sms, a, stream, g);
+    case M_FEAT: return launch_warps_mode<M_FEAT>(ctx, sms, a, stream, g);
+    case M_FEAT | M_FIT: return launch_warps_mode<M_FEAT | M_FIT>(ctx, sms, a, stream, g);
     default: return LV_EINVAL;
   }
 }
@@ -378,6 +428,8 @@ void lv_ctx_destroy(lv_ctx *ctx) {
   cudaDeviceSynchronize();
   if (ctx->d_status) cudaFree(ctx->d_status);
   if (ctx->d_tiles) cudaFree(ctx->d_tiles);
+  if (ctx->d_ctr) cudaFree(ctx->d_ctr);
+  if (ctx->d_jumbo) cudaFree(ctx->d_jumbo);
   if (ctx->d_ktab) cudaFree(ctx->d_ktab);
   if (ctx->d_fit) cudaFree(ctx->d_fit);
   if (ctx->d_wi) cudaFree(ctx->d_wi);
@@ -632,7 +684,7 @@ lv_status lv_fit(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y,
   cudaStream_t stream = (cudaStream_t)stream_;
   // scratch: per-CTA partials (at most 2048 / kBlock CTAs per SM), totals, solve output
   const int NE = fit_entries(n_y), n_ent = 4 * NE;
-  const int64_t max_cta = (int64_t)ctx->sms * (2048 / kBlock);
+  const int64_t max_cta = max_tile_ctas(ctx->sms);
   const size_t o_tot = ((size_t)max_cta * n_ent * sizeof(FitAcc) + 255) & ~(size_t)255;
   const size_t o_out = (o_tot + (size_t)n_ent * sizeof(FitAcc) + 255) & ~(size_t)255;
   const size_t need = o_out + sizeof(FitOut) * 4 * kFitMaxY;
@@ -783,10 +835,13 @@ lv_status lv_whatif(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, 
 
 namespace {
 
-constexpr int64_t kNoAllocMaxTiles = 1 << 16;  // => n_batch + n_req <= 65,536 * kD
+constexpr int64_t kNoAllocMaxTiles = 1 << 16;  // => n_batch + n_req <= 65,536 * kDW
 constexpr size_t kNoAllocPartBytes = sizeof(TilePart) * (size_t)(kNoAllocMaxTiles + 1);
 constexpr size_t kNoAllocTabOffset = (kNoAllocPartBytes + 255) & ~(size_t)255;
-constexpr size_t kNoAllocBytes = kNoAllocTabOffset + sizeof(KEntry) * 4 * (kKTableN + 1);
+constexpr size_t kNoAllocCtrOffset = (kNoAllocTabOffset + sizeof(KEntry) * 4 * (kKTableN + 1) + 255) & ~(size_t)255;
+constexpr size_t kNoAllocJumboOffset = kNoAllocCtrOffset + 256;
+constexpr int64_t kNoAllocJumboCap = kNoAllocMaxTiles * kDW / (kJumbo + 1) + 1;
+constexpr size_t kNoAllocBytes = kNoAllocJumboOffset + sizeof(int64_t) * (size_t)kNoAllocJumboCap;
 
 }  // namespace
 
@@ -818,21 +873,6 @@ lv_status noalloc_scratch(int dev, void **ptr, int *sms) {
   return LV_OK;
 }
 
-template <int MODE>
-lv_status noalloc_launch_tiles(int sms, const TileArgs &a, cudaStream_t stream) {
-  const size_t smem = sizeof(Smem);
-  LV_CUDA(cudaFuncSetAttribute(k_tiles<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)(sizeof(Smem) + sizeof(uint32_t) * 4 * kHotMax)));
-  int per_sm = 0;
-  LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_tiles<MODE>, kBlock, smem));
-  if (per_sm < 1) per_sm = 1;
-  const int64_t grid = std::min<int64_t>(a.n_tiles, (int64_t)sms * per_sm);
-  if (grid <= 0) return LV_OK;
-  k_tiles<MODE><<<(unsigned)grid, kBlock, smem, stream>>>(a);
-  LV_CUDA(cudaGetLastError());
-  return LV_OK;
-}
-
 }  // namespace
 
 extern "C" lv_status lv_attribute_noalloc(const lv_model *model, const lv_batches *b, double *T, double *share,
@@ -843,7 +883,7 @@ extern "C" lv_status lv_attribute_noalloc(const lv_model *model, const lv_batche
   if (T && !aligned(T, 8)) return LV_EINVAL;
   if (share && !aligned(share, 8)) return LV_EINVAL;
   if (status && !aligned(status, 4)) return LV_EINVAL;
-  const int64_t n_tiles = (b->n_batch + b->n_req + kD - 1) / kD;
+  const int64_t n_tiles = (b->n_batch + b->n_req + kDW - 1) / kDW;
   if (n_tiles > kNoAllocMaxTiles) return LV_EINVAL;
   int dev = 0;
   LV_CUDA(cudaGetDevice(&dev));
@@ -887,10 +927,18 @@ extern "C" lv_status lv_attribute_noalloc(const lv_model *model, const lv_batche
   a.status = status;
   a.mp = mp;
   a.n_tiles = n_tiles;
-  TilePart *part = static_cast<TilePart *>(scratch);
+  unsigned char *base = static_cast<unsigned char *>(scratch);
+  TilePart *part = reinterpret_cast<TilePart *>(base);
   a.part = part;
+  a.ctr = reinterpret_cast<unsigned long long *>(base + kNoAllocCtrOffset);
+  a.jumbo_n = a.ctr + 1;
+  a.jumbo = reinterpret_cast<int64_t *>(base + kNoAllocJumboOffset);
+  a.jumbo_cap = kNoAllocJumboCap;
+  LV_CUDA(cudaMemsetAsync(a.ctr, 0, 2 * sizeof(unsigned long long), stream));
   const int64_t pblocks = std::min<int64_t>((b->n_batch + 1 + 255) / 256, (int64_t)sms * 16);
-  k_partition<<<(unsigned)pblocks, 256, 0, stream>>>(a.off, a.n_batch, a.n_req, a.n_tiles, part, status);
+  k_partition<<<(unsigned)pblocks, 256, 0, stream>>>(a.off, a.n_batch, a.n_req, a.n_tiles, kDW, part, status);
   LV_CUDA(cudaGetLastError());
-  return mp.fixed ? noalloc_launch_tiles<M_ATTR | M_FIX>(sms, a, stream) : noalloc_launch_tiles<M_ATTR>(sms, a, stream);
+  int64_t ctas = 0;
+  return mp.fixed ? launch_warps_mode<M_ATTR | M_FIX>(nullptr, sms, a, stream, &ctas)
+                  : launch_warps_mode<M_ATTR>(nullptr, sms, a, stream, &ctas);
 }

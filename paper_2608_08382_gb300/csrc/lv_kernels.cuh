@@ -56,8 +56,12 @@ struct SegFix {
 struct KEntry {
   double q;    // fl(beta / n)
   double a4n;  // fl(a4 * n)
-  i128 kf;     // fl(q + a4n) at 2^E
+  i128 kf;     // fl(q + a4n) at 2^E, or kKSlowHi in the high word when it does not fit
 };
+
+// High word of KEntry::kf marking a constant outside the fixed-point range
+// (|K| < 2^125 otherwise, so this value never occurs).
+constexpr uint64_t kKSlowHi = 0x8000000000000000ull;
 
 struct ModelP {
   double coef[4][5];
@@ -190,6 +194,10 @@ struct TileArgs {
   int *status;
   ModelP mp;
   FitArgs fit;
+  unsigned long long *ctr;      // warp tiles handed out so far (zeroed before the launch)
+  unsigned long long *jumbo_n;  // batches queued for k_jumbo (zeroed before the launch)
+  int64_t *jumbo;               // [jumbo_cap] queued batch indices
+  int64_t jumbo_cap;
 };
 
 __device__ __forceinline__ void flag(int *status, int bit) {
@@ -202,11 +210,11 @@ __device__ __forceinline__ int64_t clampi(int64_t v, int64_t lo, int64_t hi) {
 
 // ---------------------------------------------------------------- merge-path partition
 
-// part[k] = {b, off[b]} for the first batch b with b + off[b] >= k*kD, for
+// part[k] = {b, off[b]} for the first batch b with b + off[b] >= k*D, for
 // k in [0, n_tiles); part[n_tiles] = {n_batch, n_req}.  Batch b writes the k in
-// (f(b-1)/kD, f(b)/kD], so every entry is written once by a coalesced pass.
+// (f(b-1)/D, f(b)/D], so every entry is written once by a coalesced pass.
 __global__ void k_partition(const int64_t *__restrict__ off, int64_t n_batch, int64_t n_req, int64_t n_tiles,
-                            TilePart *__restrict__ part, int *status) {
+                            int64_t D, TilePart *__restrict__ part, int *status) {
   int bad = 0;
   for (int64_t b = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; b <= n_batch;
        b += (int64_t)gridDim.x * blockDim.x) {
@@ -219,9 +227,9 @@ __global__ void k_partition(const int64_t *__restrict__ off, int64_t n_batch, in
     } else {
       const int64_t rp = __ldg(off + b - 1);
       if (rp > raw) bad = 1;
-      kmin = (b - 1 + clampi(rp, 0, n_req)) / kD + 1;
+      kmin = (b - 1 + clampi(rp, 0, n_req)) / D + 1;
     }
-    int64_t kmax = (b + ob) / kD;
+    int64_t kmax = (b + ob) / D;
     if (b == n_batch) {
       if (raw != n_req) bad = 1;
       kmax = n_tiles;
@@ -328,7 +336,11 @@ __device__ __forceinline__ double eq1_fix(const ModelP &mp, int s, const BatchAg
 
 // Per-batch share constant: q = fl(beta/n), a4n = fl(a4*n), kf = fix(fl(q+a4n)).
 __device__ __forceinline__ KEntry batch_k(const ModelP &mp, int s, int64_t n, bool *slow) {
-  if (n >= 1 && n <= mp.nk) return mp.ktab[s * (mp.nk + 1) + n];
+  if (n >= 1 && n <= mp.nk) {
+    const KEntry e = mp.ktab[s * (mp.nk + 1) + n];
+    if (mp.fixed && e.kf.hi == kKSlowHi) *slow = true;
+    return e;
+  }
   KEntry e;
   const double *k = mp.coef[s];
   const double dn = (double)n;
@@ -1089,6 +1101,7 @@ __global__ void k_ktable(ModelP mp, KEntry *tab) {
     e.a4n = __dmul_rn(k[4], (double)n);
     bool ovf = false;
     e.kf = mp.fixed ? double_to_fix(__dadd_rn(e.q, e.a4n), mp.fx[s].E, &ovf) : mk128(0, 0);
+    if (ovf) e.kf = mk128(0, kKSlowHi);
   }
   tab[idx] = e;
 }

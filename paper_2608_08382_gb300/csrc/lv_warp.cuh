@@ -1,0 +1,506 @@
+// Warp-centric attribution kernels (sm_103a).
+//
+// Every step of the path is a stream over request arrays, so the kernels are
+// built to keep many independent warps busy with coalesced loads and no
+// block-wide barrier while tiles are processed.
+//
+// Work decomposition.  The merge of batch boundaries and requests is cut every
+// kDW positions (k_partition); a warp tile owns the batches whose start falls
+// in its window (whole batches, no data shared with neighbours).  Persistent
+// warps take tiles from a global counter and walk each tile 32 batches at a
+// time, batch b0 + j on lane j:
+//   - a batch of kBig..kJumbo requests is reduced by the whole warp with
+//     coalesced strided loads and a butterfly sum; its segment and per-request
+//     constant follow (uniform across the warp) and its shares come from a
+//     second strided pass while its requests are still in L1;
+//   - batches of fewer than kBig requests are packed into rounds of up to 32
+//     requests (whole batches per round, one request per lane), reduced with a
+//     segmented scan across lanes and attributed in a second sweep of the same
+//     rounds;
+//   - a batch of more than kJumbo requests is queued for k_jumbo, where a whole
+//     CTA takes it, so that no warp holds a disproportionate share of the work;
+//   - T, the batch features and the fit statistics of the 32 batches are then
+//     produced with one lane per batch.
+// All sums are exact integers, so results do not depend on this schedule.
+#pragma once
+
+#include "lv_kernels.cuh"
+
+namespace lv {
+
+constexpr int kWarps = 16;                 // warps per CTA of k_warps
+constexpr int kWThreads = 32 * kWarps;
+constexpr int kDW = 1024;                  // merge positions per warp tile
+constexpr int kJumbo = 512;                // larger batches are attributed by k_jumbo
+constexpr int kBig = 32;                   // batches with at least this many requests are processed warp-strided
+constexpr int kJBlock = 512;               // threads per CTA of k_jumbo
+constexpr int kJWarps = kJBlock / 32;
+constexpr unsigned kFull = 0xffffffffu;
+
+static_assert(kJumbo <= kNK * 4, "jumbo threshold");
+
+// Shared memory of k_warps; the tenant table (4 x H words) and, in fit mode,
+// the per-warp fit accumulators ([kWarps][4 * NE]) follow it.
+struct WSmem {
+  alignas(16) i128 kfix[4][kNK + 1];     // K at 2^E for n <= kNK (fixed-point mode)
+  alignas(16) SegS seg[4];
+  alignas(16) uint8_t kslow[4][kNK + 4];  // 1: K outside the fixed-point range
+  alignas(16) uint8_t owner[kWarps][32];  // small-batch rounds: head slot -> lane
+};
+static_assert(sizeof(WSmem) % 16 == 0, "tenant table follows WSmem");
+
+// Shared memory of k_jumbo (tenant table follows).
+struct JSmem {
+  alignas(16) SegS seg[4];
+  alignas(16) Sums red[kJWarps];
+  alignas(16) Sums tot;
+};
+static_assert(sizeof(JSmem) % 16 == 0, "tenant table follows JSmem");
+
+__device__ __forceinline__ Sums add_sums(Sums a, const Sums &b) {
+  a.s1 += b.s1;
+  a.s2 += b.s2;
+  a.s3 += b.s3;
+  a.ph += b.ph;
+  return a;
+}
+
+__device__ __forceinline__ Sums shfl_sums(const Sums &v, int src) {
+  return Sums{__shfl_sync(kFull, v.s1, src), __shfl_sync(kFull, v.s2, src), __shfl_sync(kFull, v.s3, src),
+              __shfl_sync(kFull, v.ph, src)};
+}
+
+__device__ __forceinline__ Sums warp_sum(Sums v) {
+#pragma unroll
+  for (int d = 16; d; d >>= 1) {
+    v.s1 += __shfl_xor_sync(kFull, v.s1, d);
+    v.s2 += __shfl_xor_sync(kFull, v.s2, d);
+    v.s3 += __shfl_xor_sync(kFull, v.s3, d);
+    v.ph += __shfl_xor_sync(kFull, v.ph, d);
+  }
+  return v;
+}
+
+__device__ __forceinline__ int warp_excl_scan_int(int v, int lane) {
+  int x = v;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const int y = __shfl_up_sync(kFull, x, d);
+    if (lane >= d) x += y;
+  }
+  return x - v;
+}
+
+// One request's share, its store and its tenant contribution.
+template <int MODE>
+__device__ __forceinline__ void attribute_one(const TileArgs &a, uint32_t *tt, const SegS &sg, int s, bool slow,
+                                              i128 kf, int64_t n, int64_t i, int32_t p, int32_t c, int32_t u,
+                                              int *bad) {
+  Rounded r;
+  if ((MODE & M_FIX) && !slow && p <= kPMaxFix)
+    r = share_fix(sg, kf, (uint32_t)p, (uint32_t)c);
+  else
+    r = share_slow(a.mp, s, (MODE & M_FIX) != 0, kf, p, c, n);
+  if (a.share) __stcs(a.share + i, r.d);
+  if (MODE & M_TEN) tenant_add(a, tt, u, r, bad);
+}
+
+// Per-request constant of a batch: fixed-point K (from the shared table for
+// n <= kNK), or {fl(beta/n), fl(a4 n)} in fp64 mode.
+template <int MODE>
+__device__ __forceinline__ i128 batch_const_w(const TileArgs &a, const WSmem *ws, int s, int64_t n, bool *slow) {
+  if (MODE & M_FIX) {
+    if (ws && n >= 1 && n <= kNK) {
+      if (ws->kslow[s][n]) *slow = true;
+      return ws->kfix[s][n];
+    }
+    return batch_k(a.mp, s, n, slow).kf;
+  }
+  bool dummy = false;
+  const KEntry e = batch_k(a.mp, s, n, &dummy);
+  return mk128((uint64_t)__double_as_longlong(e.q), (uint64_t)__double_as_longlong(e.a4n));
+}
+
+// Warp-strided sums over requests [r0, r1); uniform result on every lane.
+__device__ __forceinline__ Sums big_reduce(const TileArgs &a, int64_t r0, int64_t r1, int lane, int *bad) {
+  Sums acc{0, 0, 0, 0};
+  for (int64_t i = r0 + lane; i < r1; i += 4 * 32) {
+    int32_t p[4], c[4], ph[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int64_t q = i + 32 * k;
+      const bool in = q < r1;
+      p[k] = in ? a.p[q] : 0;
+      c[k] = in ? a.c[q] : 0;
+      ph[k] = in ? a.ph[q] : 0;
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      check_req(p[k], c[k], ph[k], bad);
+      acc.s1 += p[k];
+      acc.s2 += c[k];
+      acc.s3 += (int64_t)p[k] * p[k];
+      acc.ph += ph[k];
+    }
+  }
+  return warp_sum(acc);
+}
+
+// Warp-strided shares of requests [r0, r1) of one batch (segment s, constant kf).
+template <int MODE>
+__device__ __forceinline__ void big_shares(const TileArgs &a, uint32_t *tt, const SegS &sg, int s, bool slow,
+                                           i128 kf, int64_t r0, int64_t r1, int lane, int *bad) {
+  const int64_t n = r1 - r0;
+  for (int64_t i = r0 + lane; i < r1; i += 4 * 32) {
+    int32_t p[4], c[4], u[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int64_t q = i + 32 * k;
+      const bool in = q < r1;
+      p[k] = in ? a.p[q] : 0;
+      c[k] = in ? a.c[q] : 0;
+      u[k] = (in && (MODE & M_TEN)) ? a.ten[q] : 0;
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int64_t q = i + 32 * k;
+      if (q < r1) {
+        const int32_t pk = p[k] < 0 ? 0 : p[k], ck = c[k] < 0 ? 0 : c[k];
+        attribute_one<MODE>(a, tt, sg, s, slow, kf, n, q, pk, ck, u[k], bad);
+      }
+    }
+  }
+}
+
+// Rounds over the small batches of a group (lanes with `small`): every round
+// takes the next batches whose requests fit in 32 slots, one request per lane.
+// Pass SHARE=false reduces (each small lane receives its batch's sums in
+// `mys`); SHARE=true attributes with the per-lane constants (myk, mymeta).
+// pn: the lane's request count (0 for other lanes); P: exclusive prefix of pn;
+// base = o0 - P so that slot q of the lane's batch is request base + q.
+template <int MODE, bool SHARE>
+__device__ __forceinline__ void small_rounds(const TileArgs &a, const WSmem &ws, uint32_t *tt, uint8_t *owner,
+                                             bool small, int pn, int P, int64_t base, Sums &mys, i128 myk,
+                                             int mymeta, int lane, int *bad) {
+  uint32_t rem = __ballot_sync(kFull, small);
+  while (rem) {
+    const int start = __shfl_sync(kFull, P, __ffs(rem) - 1);
+    const bool in = ((rem >> lane) & 1u) && (P + pn <= start + 32);
+    const uint32_t rm = __ballot_sync(kFull, in);
+    rem &= ~rm;
+    if (in) owner[P - start] = (uint8_t)lane;
+    const uint32_t H = __reduce_or_sync(kFull, in ? (1u << (P - start)) : 0u);
+    __syncwarp();
+    const int len = __shfl_sync(kFull, P + pn, 31 - __clz(rm)) - start;
+    const bool act = lane < len;
+    const int hp = act ? 31 - __clz(H & ((2u << lane) - 1u)) : 0;  // head slot of this lane's batch
+    const int j = owner[hp];
+    const int64_t r = __shfl_sync(kFull, base, j) + start + lane;
+    if (!SHARE) {
+      Sums v{0, 0, 0, 0};
+      if (act) {
+        int32_t p = a.p[r], c = a.c[r], ph = a.ph[r];
+        check_req(p, c, ph, bad);
+        v = Sums{p, c, (int64_t)p * p, ph};
+      }
+      const int maxn = __reduce_max_sync(kFull, in ? pn : 0);
+      for (int d = 1; d < maxn; d <<= 1) {
+        const Sums w{__shfl_up_sync(kFull, v.s1, d), __shfl_up_sync(kFull, v.s2, d),
+                     __shfl_up_sync(kFull, v.s3, d), __shfl_up_sync(kFull, v.ph, d)};
+        if (lane - d >= hp) v = add_sums(v, w);
+      }
+      const Sums tot = shfl_sums(v, in ? P - start + pn - 1 : 0);
+      if (in) mys = tot;
+    } else {
+      const uint64_t klo = __shfl_sync(kFull, myk.lo, j), khi = __shfl_sync(kFull, myk.hi, j);
+      const int meta = __shfl_sync(kFull, mymeta, j);
+      if (act) {
+        int32_t p = a.p[r], c = a.c[r];
+        const int32_t u = (MODE & M_TEN) ? a.ten[r] : 0;
+        p = p < 0 ? 0 : p;
+        c = c < 0 ? 0 : c;
+        const int s = meta & 3;
+        attribute_one<MODE>(a, tt, ws.seg[s], s, (meta & 4) != 0, mk128(klo, khi), meta >> 3, r, p, c, u, bad);
+      }
+    }
+    __syncwarp();  // owner[] is rewritten by the next round
+  }
+}
+
+// Fit statistics of the group's batches into this warp's accumulators: lane e
+// owns entries e, e+32, ... of [4 groups][NE].
+__device__ __forceinline__ void fit_group(const TileArgs &a, FitAcc *fw, int64_t g0, int ng, const Sums &mys,
+                                          int64_t n, int fseg, int lane, int *bad) {
+  const int NE = fit_entries(a.fit.n_y);
+  for (int j = 0; j < ng; ++j) {
+    const int sj = __shfl_sync(kFull, fseg, j);
+    if (sj < 0) continue;  // empty, jumbo or out of range
+    const int64_t nj = __shfl_sync(kFull, n, j);
+    const int64_t xx[5] = {1, __shfl_sync(kFull, mys.s1, j), __shfl_sync(kFull, mys.s2, j),
+                           __shfl_sync(kFull, mys.s3, j), nj * nj};
+    for (int t = lane; t < 4 * NE; t += 32) {
+      if (t / NE != sj) continue;
+      fit_owner_add(fw[t], t % NE, a.fit.n_y, xx, a.fit.y, a.n_batch, g0 + j, xx[1] != xx[3], bad);
+    }
+  }
+}
+
+// One group of up to 32 consecutive batches [g0, g0 + ng) of a tile.
+template <int MODE>
+__device__ __forceinline__ void process_group(const TileArgs &a, const WSmem &ws, uint32_t *tt, uint8_t *owner,
+                                              FitAcc *fw, int64_t g0, int ng, int lane, int *bad) {
+  constexpr bool kAttr = (MODE & M_ATTR) != 0;
+  const bool valid = lane < ng;
+  const int64_t b = g0 + lane;
+  int64_t o0 = valid ? a.off[b] : 0;
+  int64_t o1 = __shfl_down_sync(kFull, o0, 1);
+  if (valid && lane == ng - 1) o1 = a.off[b + 1];
+  if (valid) {
+    const int64_t c0 = clampi(o0, 0, a.n_req), c1 = clampi(o1, c0, a.n_req);
+    if (c0 != o0 || c1 != o1) *bad = 1;
+    o0 = c0;
+    o1 = c1;
+  }
+  const int64_t n = valid ? o1 - o0 : 0;
+  const bool jumbo = valid && n > kJumbo;
+  if (jumbo) {
+    const unsigned long long slot = atomicAdd(a.jumbo_n, 1ull);
+    if (slot < (unsigned long long)a.jumbo_cap)
+      a.jumbo[slot] = b;
+    else
+      *bad = 1;
+  }
+  Sums mys{0, 0, 0, 0};
+  i128 myk = mk128(0, 0);
+  int mymeta = 0;
+
+  // ---- big batches: reduce, constant and shares one batch at a time
+  uint32_t big = __ballot_sync(kFull, valid && !jumbo && n >= kBig);
+  while (big) {
+    const int j = __ffs(big) - 1;
+    big &= big - 1;
+    const int64_t r0 = __shfl_sync(kFull, o0, j), r1 = __shfl_sync(kFull, o1, j);
+    const Sums tot = big_reduce(a, r0, r1, lane, bad);
+    if (lane == j) mys = tot;
+    if (kAttr) {
+      const BatchAgg g{tot.s1, tot.s2, tot.s3, r1 - r0, tot.ph > 0};
+      const int s = segment_of(a.mp, g);
+      bool slow = false;
+      const i128 kf = batch_const_w<MODE>(a, &ws, s, r1 - r0, &slow);
+      const SegS sg = ws.seg[s];
+      big_shares<MODE>(a, tt, sg, s, slow, kf, r0, r1, lane, bad);
+    }
+  }
+
+  // ---- small batches: packed rounds
+  const bool small = valid && n > 0 && n < kBig;
+  if (__any_sync(kFull, small)) {
+    const int pn = small ? (int)n : 0;
+    const int P = warp_excl_scan_int(pn, lane);
+    const int64_t base = o0 - P;
+    small_rounds<MODE, false>(a, ws, tt, owner, small, pn, P, base, mys, myk, 0, lane, bad);
+    if (kAttr) {
+      if (small) {
+        const BatchAgg g{mys.s1, mys.s2, mys.s3, n, mys.ph > 0};
+        const int s = segment_of(a.mp, g);
+        bool slow = false;
+        myk = batch_const_w<MODE>(a, &ws, s, n, &slow);
+        mymeta = ((int)n << 3) | (slow ? 4 : 0) | s;
+      }
+      small_rounds<MODE, true>(a, ws, tt, owner, small, pn, P, base, mys, myk, mymeta, lane, bad);
+    }
+  }
+
+  // ---- per batch: T, features; fit statistics
+  int fseg = -1;
+  if (valid && !jumbo) {
+    const BatchAgg g{mys.s1, mys.s2, mys.s3, n, mys.ph > 0};
+    const int s = segment_of(a.mp, g);
+    emit_batch<MODE>(a, b, g, s);
+    if (MODE & M_FIT) {
+      const bool in_range = g.s1 < kFitFeatMax && g.s2 < kFitFeatMax && g.s3 < kFitFeatMax &&
+                            n * n < kFitFeatMax;
+      if (!in_range) flag(a.status, kStatusOverflow);
+      if (n > 0 && in_range) fseg = s;
+    }
+  }
+  if (MODE & M_FIT) fit_group(a, fw, g0, ng, mys, n, fseg, lane, bad);
+}
+
+// Shared-memory tables of a CTA: per-segment share parameters and, in
+// fixed-point attribution, the per-request constants for n <= kNK.
+template <int MODE>
+__device__ __forceinline__ void init_segs(const TileArgs &a, SegS *seg) {
+  if (threadIdx.x < 4) {
+    const SegFix &f = a.mp.fx[threadIdx.x];
+    SegS g;
+    g.A1 = f.A1;
+    g.A3 = f.A3;
+    g.A13 = f.A13;
+    g.A2 = f.A2;
+    g.E = f.E;
+    g.a2_narrow = f.a2_narrow;
+    g.pad[0] = g.pad[1] = 0;
+    seg[threadIdx.x] = g;
+  }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  WSmem &ws = *reinterpret_cast<WSmem *>(smem_raw);
+  uint32_t *tt = reinterpret_cast<uint32_t *>(smem_raw + sizeof(WSmem));
+  constexpr bool kTen = (MODE & M_TEN) != 0;
+  constexpr bool kFit = (MODE & M_FIT) != 0;
+  FitAcc *facc = reinterpret_cast<FitAcc *>(smem_raw + sizeof(WSmem) + (kTen ? 16 * (size_t)a.H : 0));
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const int NE4 = kFit ? 4 * fit_entries(a.fit.n_y) : 0;
+  int bad = 0;
+
+  if (kTen)
+    for (int i = tid; i < 4 * a.H; i += kWThreads) tt[i] = 0;
+  if (kFit)
+    for (int i = tid; i < kWarps * NE4; i += kWThreads) facc[i] = FitAcc{{0, 0, 0, 0}};
+  if (MODE & M_ATTR) {
+    init_segs<MODE>(a, ws.seg);
+    if (MODE & M_FIX) {
+      for (int i = tid; i < 4 * (kNK + 1); i += kWThreads) {
+        const int s = i / (kNK + 1), n = i % (kNK + 1);
+        i128 kf = mk128(0, 0);
+        bool ovf = false;
+        if (n >= 1 && n <= a.mp.nk) {
+          const KEntry e = a.mp.ktab[s * (a.mp.nk + 1) + n];
+          kf = double_to_fix(__dadd_rn(e.q, e.a4n), a.mp.fx[s].E, &ovf);
+        }
+        ws.kfix[s][n] = kf;
+        ws.kslow[s][n] = ovf ? 1 : 0;
+      }
+    }
+  }
+  __syncthreads();
+
+  uint8_t *owner = ws.owner[wid];
+  FitAcc *fw = facc + wid * NE4;
+  unsigned long long t = 0;
+  if (lane == 0) t = atomicAdd(a.ctr, 1ull);
+  t = __shfl_sync(kFull, t, 0);
+  while (t < (unsigned long long)a.n_tiles) {
+    unsigned long long tn = 0;
+    if (lane == 0) tn = atomicAdd(a.ctr, 1ull);  // next tile, fetched early
+    const int64_t b0 = clampi(a.part[t].b, 0, a.n_batch);
+    int64_t b1 = clampi(a.part[t + 1].b, b0, a.n_batch);
+    if (b1 - b0 > kDW) {
+      b1 = b0 + kDW;
+      bad = 1;
+    }
+    for (int64_t g0 = b0; g0 < b1; g0 += 32)
+      process_group<MODE>(a, ws, tt, owner, fw, g0, (int)(b1 - g0 < 32 ? b1 - g0 : 32), lane, &bad);
+    t = __shfl_sync(kFull, tn, 0);
+  }
+
+  if (bad) flag(a.status, kStatusData);
+  if (kTen || kFit) __syncthreads();
+  if (kTen) {
+    for (int u = tid; u < a.H; u += kWThreads) {
+      const i128 v = hot_value(tt + 4 * u);
+      if (v.lo | v.hi) pend_add(a.ten_pend, u, v);
+    }
+  }
+  if (kFit) {
+    // this CTA's partial: exact sum over its warps (flag entries ORed)
+    const int NE = fit_entries(a.fit.n_y);
+    for (int e = tid; e < NE4; e += kWThreads) {
+      FitAcc s{{0, 0, 0, 0}};
+      for (int w = 0; w < kWarps; ++w) {
+        const FitAcc &v = facc[w * NE4 + e];
+        if (e % NE == NE - 1)
+          s.w[0] |= v.w[0];
+        else
+          acc_add256(s.w, v.w[0], v.w[1], v.w[2], v.w[3]);
+      }
+      a.fit.partial[(int64_t)blockIdx.x * NE4 + e] = s;
+    }
+  }
+}
+
+// Batches of more than kJumbo requests, one CTA per batch (grid-stride over
+// the queue that k_warps filled).  Fit partials go to row fit_base + CTA.
+template <int MODE>
+__global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_base) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  JSmem &js = *reinterpret_cast<JSmem *>(smem_raw);
+  uint32_t *tt = reinterpret_cast<uint32_t *>(smem_raw + sizeof(JSmem));
+  constexpr bool kTen = (MODE & M_TEN) != 0;
+  constexpr bool kFit = (MODE & M_FIT) != 0;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  int bad = 0;
+  FitAcc facc{{0, 0, 0, 0}};
+  if (kTen)
+    for (int i = tid; i < 4 * a.H; i += kJBlock) tt[i] = 0;
+  if (MODE & M_ATTR) init_segs<MODE>(a, js.seg);
+  __syncthreads();
+
+  const unsigned long long q = *a.jumbo_n;
+  const int64_t nj = q < (unsigned long long)a.jumbo_cap ? (int64_t)q : a.jumbo_cap;
+  for (int64_t k = blockIdx.x; k < nj; k += gridDim.x) {
+    const int64_t b = clampi(a.jumbo[k], 0, a.n_batch - 1);
+    const int64_t r0 = clampi(a.off[b], 0, a.n_req), r1 = clampi(a.off[b + 1], r0, a.n_req);
+    Sums acc{0, 0, 0, 0};
+    for (int64_t i = r0 + tid; i < r1; i += kJBlock) {
+      int32_t p = a.p[i], c = a.c[i], ph = a.ph[i];
+      check_req(p, c, ph, &bad);
+      acc.s1 += p;
+      acc.s2 += c;
+      acc.s3 += (int64_t)p * p;
+      acc.ph += ph;
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) js.red[wid] = acc;
+    __syncthreads();
+    if (tid == 0) {
+      Sums t{0, 0, 0, 0};
+      for (int w = 0; w < kJWarps; ++w) t = add_sums(t, js.red[w]);
+      js.tot = t;
+    }
+    __syncthreads();
+    const Sums tot = js.tot;
+    const BatchAgg g{tot.s1, tot.s2, tot.s3, r1 - r0, tot.ph > 0};
+    const int s = segment_of(a.mp, g);
+    if (tid == 0) emit_batch<MODE>(a, b, g, s);
+    if (kFit) {
+      const int NE = fit_entries(a.fit.n_y);
+      const int64_t x[5] = {1, g.s1, g.s2, g.s3, g.n * g.n};
+      const bool in_range = g.s1 < kFitFeatMax && g.s2 < kFitFeatMax && g.s3 < kFitFeatMax && x[4] < kFitFeatMax;
+      if (!in_range && tid == 0) flag(a.status, kStatusOverflow);
+      if (tid < 4 * NE && tid / NE == s && in_range)
+        fit_owner_add(facc, tid % NE, a.fit.n_y, x, a.fit.y, a.n_batch, b, g.s1 != g.s3, &bad);
+    }
+    if (MODE & M_ATTR) {
+      bool slow = false;
+      const i128 kf = batch_const_w<MODE>(a, nullptr, s, g.n, &slow);
+      const SegS sg = js.seg[s];
+      for (int64_t i = r0 + tid; i < r1; i += kJBlock) {
+        int32_t p = a.p[i], c = a.c[i];
+        const int32_t u = kTen ? a.ten[i] : 0;
+        p = p < 0 ? 0 : p;
+        c = c < 0 ? 0 : c;
+        attribute_one<MODE>(a, tt, sg, s, slow, kf, g.n, i, p, c, u, &bad);
+      }
+    }
+    __syncthreads();  // js.red / js.tot are rewritten for the next batch
+  }
+  if (bad) flag(a.status, kStatusData);
+  if (kFit) {
+    const int NE4 = 4 * fit_entries(a.fit.n_y);
+    if (tid < NE4) a.fit.partial[((int64_t)fit_base + blockIdx.x) * NE4 + tid] = facc;
+  }
+  if (kTen) {
+    __syncthreads();
+    for (int u = tid; u < a.H; u += kJBlock) {
+      const i128 v = hot_value(tt + 4 * u);
+      if (v.lo | v.hi) pend_add(a.ten_pend, u, v);
+    }
+  }
+}
+
+}  // namespace lv
