@@ -1,40 +1,17 @@
-// Device code for the LLMVisor attribution path (sm_103a).
-//
-// Tiling.  The work is a merge of two sorted streams: batch boundaries
-// (offsets) and requests.  Batch b starts at merge position f(b) = b + off[b]
-// (b boundaries and off[b] requests precede it); f is strictly increasing, so
-// cutting the merge sequence every kD positions gives tiles that each own the
-// batches whose start falls inside them -- at most kD batches and about kD
-// requests, whatever the batch-size distribution (merge-based partitioning,
-// Merrill & Garland, SC'16).  A tile holds whole batches and needs no data from
-// its neighbours.  The partition is written by one coalesced pass over the
-// offsets (k_partition); no search is needed.
-//
-// Pipeline.  k_tiles runs persistent CTAs (two per SM).  Each CTA walks its
-// tiles with a two-stage ring in shared memory: while the threads compute tile
-// k, bulk asynchronous copies (TMA) bring the offsets window and the request
-// arrays of tile k+1.  Per tile, every thread takes K consecutive requests, the
-// per-batch sums S1 = sum p, S2 = sum c, S3 = sum p^2 and the prefill count
-// come from a block-wide prefix sum sampled at batch boundaries (exact integer
-// sums), then each batch's segment, T and per-request constant are computed
-// once and every request's share is produced from registers.  A batch with
-// more requests than the staging capacity takes a block-wide path that reads
-// global memory directly.
+// Device code shared by the LLMVisor kernels (sm_103a): model parameters, the
+// merge-path partition, exact fixed-point evaluation of Eq. 1 and of the
+// per-request shares, exact tenant accumulation, and the small kernels around
+// them.  The request-streaming kernels themselves are in lv_warp.cuh.
 #pragma once
 
 #include <cstddef>
 #include <cstdint>
 
 #include "lv_fixed.cuh"
-#include "lv_tma.cuh"
 
 namespace lv {
 
-constexpr int kBlock = 256;                        // threads per CTA
-constexpr int kD = 1024;                           // merge positions per tile (batches + requests)
-constexpr int kCap = 1280;                         // requests staged per tile
-constexpr int kK = (kCap + kBlock - 1) / kBlock;   // max requests per thread per sub-tile
-constexpr int kBPT = kD / kBlock;                  // max batches per thread in the per-batch phase
+constexpr int kBlock = 256;                        // threads per CTA of the small kernels
 constexpr int kHotMax = 512;                       // tenants kept in shared memory per CTA
 constexpr int kNK = 256;                           // per-batch constants cached in shared memory for n <= kNK
 constexpr int64_t kPMaxFix = 1ll << 24;            // p beyond this uses the fp64 share path
@@ -246,50 +223,12 @@ __global__ void k_partition(const int64_t *__restrict__ off, int64_t n_batch, in
   if (bad) flag(status, kStatusData);
 }
 
-// ---------------------------------------------------------------- block scan
+// ---------------------------------------------------------------- batch sums
 
 struct Sums {
   int64_t s1, s2, s3;
   int32_t ph;
 };
-
-__device__ __forceinline__ Sums warp_incl_scan(Sums v, int lane) {
-#pragma unroll
-  for (int d = 1; d < 32; d <<= 1) {
-    const int64_t a = __shfl_up_sync(0xffffffffu, v.s1, d);
-    const int64_t b = __shfl_up_sync(0xffffffffu, v.s2, d);
-    const int64_t c = __shfl_up_sync(0xffffffffu, v.s3, d);
-    const int32_t e = __shfl_up_sync(0xffffffffu, v.ph, d);
-    if (lane >= d) {
-      v.s1 += a;
-      v.s2 += b;
-      v.s3 += c;
-      v.ph += e;
-    }
-  }
-  return v;
-}
-
-// Exclusive block scan; `scr` holds kBlock/32 Sums.  Contains __syncthreads.
-__device__ __forceinline__ Sums block_excl_scan(Sums v, Sums *scr) {
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  Sums inc = warp_incl_scan(v, lane);
-  if (lane == 31) scr[wid] = inc;
-  __syncthreads();
-  if (wid == 0) {
-    Sums w = lane < kBlock / 32 ? scr[lane] : Sums{0, 0, 0, 0};
-    Sums wi = warp_incl_scan(w, lane);
-    if (lane < kBlock / 32) {
-      Sums ex{wi.s1 - w.s1, wi.s2 - w.s2, wi.s3 - w.s3, wi.ph - w.ph};
-      scr[lane] = ex;
-    }
-  }
-  __syncthreads();
-  Sums base = scr[wid];
-  Sums r{base.s1 + inc.s1 - v.s1, base.s2 + inc.s2 - v.s2, base.s3 + inc.s3 - v.s3, base.ph + inc.ph - v.ph};
-  __syncthreads();
-  return r;
-}
 
 // ---------------------------------------------------------------- model arithmetic
 
@@ -498,7 +437,7 @@ __device__ __forceinline__ i128 hot_value(const uint32_t *w) {
   return mk128((uint64_t)w[0] | ((uint64_t)w[1] << 32), (uint64_t)w[2] | ((uint64_t)w[3] << 32));
 }
 
-// ---------------------------------------------------------------- the tile kernel
+// ---------------------------------------------------------------- per-batch and per-request steps
 
 enum : int {
   M_ATTR = 1,    // T (if a.T) and shares (if a.share)
@@ -506,19 +445,6 @@ enum : int {
   M_FEAT = 8,    // write batch features / segment codes only
   M_FIX = 16,    // fixed-point arithmetic (else fp64)
   M_FIT = 32,    // accumulate the least-squares statistics (with M_FEAT's reduction)
-};
-
-// One stage of the ring: offsets window and request arrays of one tile.
-struct Stage {
-  alignas(16) int64_t win[kD + 4];
-  alignas(16) int32_t sp[kCap + 8];
-  alignas(16) int32_t sc[kCap + 8];
-  alignas(16) int32_t sph[kCap + 8];
-  alignas(16) int32_t sten[kCap + 8];
-};
-
-struct TileHdr {
-  int64_t b0, b1, r0, r1, staged, lo;
 };
 
 // Per-segment integers the share path needs, kept in shared memory so that a
@@ -530,90 +456,6 @@ struct SegS {
   int a2_narrow;
   int pad[2];
 };
-
-struct Smem {
-  Stage st[2];
-  union U {
-    struct {
-      alignas(16) int64_t s1[kD + 4];
-      alignas(16) int64_t s2[kD + 4];
-      alignas(16) int64_t s3[kD + 4];
-      alignas(16) int32_t ph[kD + 4];
-    } pre;
-    struct {
-      alignas(16) i128 kf[kD];  // per-batch constant (fixed) or {q, a4n} (fp64)
-      alignas(16) uint8_t seg[kD];
-    } bp;
-  } u;
-  alignas(16) double kcd[4][kNK + 1];  // fl(fl(beta/n) + fl(a4*n)) for n <= kNK
-  alignas(16) uint8_t fseg[kD + 16];   // fit mode: segment of each batch of the sub-tile
-  alignas(16) SegS seg[4];
-  TileHdr hdr[2];
-  alignas(16) Sums scr[kBlock / 32];
-  alignas(8) uint64_t full[2];
-  int flags;
-};
-static_assert(offsetof(Stage, win) % 16 == 0 && offsetof(Stage, sp) % 16 == 0 && offsetof(Stage, sc) % 16 == 0 &&
-                  offsetof(Stage, sph) % 16 == 0 && offsetof(Stage, sten) % 16 == 0 && sizeof(Stage) % 16 == 0,
-              "bulk-copy destinations must be 16-byte aligned");
-static_assert(offsetof(Stage, sc) - offsetof(Stage, sp) == sizeof(int32_t) * (kCap + 8) &&
-                  2 * sizeof(int32_t) * (kCap + 8) >= sizeof(double) * kCap,
-              "shares are staged over the consumed p and c arrays");
-static_assert(sizeof(Smem) % 16 == 0, "tenant table follows Smem");
-
-// Loads tile t's extent from the partition (clamped: never trusted blindly).
-__device__ __forceinline__ TileHdr tile_info(const TileArgs &a, int64_t t, int *bad) {
-  const TilePart p0 = a.part[t], p1 = a.part[t + 1];
-  TileHdr h;
-  h.b0 = clampi(p0.b, 0, a.n_batch);
-  h.b1 = clampi(p1.b, h.b0, a.n_batch);
-  if (h.b1 - h.b0 > kD) {
-    h.b1 = h.b0 + kD;
-    *bad = 1;
-  }
-  h.r0 = clampi(p0.r, 0, a.n_req);
-  h.r1 = clampi(p1.r, h.r0, a.n_req);
-  h.staged = h.r1 - h.r0 < kCap ? h.r1 - h.r0 : kCap;
-  h.lo = h.b0 & ~1ll;
-  return h;
-}
-
-// Thread 0: fill stage `s` with the tile described by h (window by bulk copy,
-// request arrays by bulk copy, ragged ends by plain loads), then arrive on the
-// stage's barrier with the byte count.
-template <bool TEN>
-__device__ __forceinline__ void issue_tile(const TileArgs &a, Smem &sm, int s, const TileHdr &h) {
-  Stage &st = sm.st[s];
-  uint64_t *bar = &sm.full[s];
-  sm.hdr[s] = h;
-  // window [lo, hi): 16-byte aligned start, even element count, never past off[n_batch]
-  const int64_t w_up = (h.b1 + 2) & ~1ll, w_cap = (a.n_batch + 1) & ~1ll;
-  const int64_t hi_w = w_up < w_cap ? w_up : w_cap;
-  if (hi_w <= h.b1) st.win[h.b1 - h.lo] = h.r1;  // last boundary not covered by the copy
-  // requests [base, vend) by bulk copy; [max(vend, base), r0 + staged) by plain loads
-  const int64_t base = h.r0 & ~3ll;
-  const int64_t rend = h.r0 + h.staged;
-  const int64_t vup = (rend + 3) & ~3ll, vcap = a.n_req & ~3ll;
-  const int64_t vend = vup < vcap ? vup : vcap;
-  for (int64_t g = (vend > base ? vend : base); g < rend; ++g) {
-    const int i = (int)(g - base);
-    st.sp[i] = a.p[g];
-    st.sc[i] = a.c[g];
-    st.sph[i] = a.ph[g];
-    if (TEN) st.sten[i] = a.ten[g];
-  }
-  const uint32_t wbytes = hi_w > h.lo ? (uint32_t)(hi_w - h.lo) * 8u : 0u;
-  const uint32_t rbytes = vend > base ? (uint32_t)(vend - base) * 4u : 0u;
-  const uint32_t bytes = wbytes + rbytes * (TEN ? 4u : 3u);
-  mbar_arrive_expect_tx(bar, bytes);
-  if (wbytes) bulk_g2s(st.win, a.off + h.lo, wbytes, bar);
-  if (rbytes) {
-    bulk_g2s(st.sp, a.p + base, rbytes, bar);
-    bulk_g2s(st.sc, a.c + base, rbytes, bar);
-    bulk_g2s(st.sph, a.ph + base, rbytes, bar);
-    if (TEN) bulk_g2s(st.sten, a.ten + base, rbytes, bar);
-  }
-}
 
 template <int MODE>
 __device__ __forceinline__ void emit_batch(const TileArgs &a, int64_t gb, const BatchAgg &g, int s) {
@@ -666,364 +508,6 @@ __device__ __noinline__ Rounded share_slow(const ModelP &mp, int s, bool fixed, 
     a4n = __longlong_as_double((long long)kf.hi);
   }
   return decompose(share_fp64(mp.coef[s], q, a4n, p, c));
-}
-
-// Share of one request (kf: per-batch constant; in fp64 mode kf holds {q, a4n}).
-template <int MODE>
-__device__ __forceinline__ Rounded one_share(const TileArgs &a, const SegS *segs, int s, bool slow, i128 kf,
-                                             int32_t p, int32_t c, int64_t n) {
-  if ((MODE & M_FIX) && !slow && p <= kPMaxFix) return share_fix(segs[s], kf, (uint32_t)p, (uint32_t)c);
-  return share_slow(a.mp, s, (MODE & M_FIX) != 0, kf, p, c, n);
-}
-
-// Per-batch constant for the share phase, as stored in Smem::bp.
-template <int MODE>
-__device__ __forceinline__ i128 batch_const(const TileArgs &a, const Smem &sm, int s, int64_t n, bool *slow) {
-  if (MODE & M_FIX) {
-    if (n >= 1 && n <= kNK) {
-      bool ovf = false;
-      const i128 kf = double_to_fix(sm.kcd[s][n], sm.seg[s].E, &ovf);
-      if (ovf) *slow = true;
-      return kf;
-    }
-    return batch_k(a.mp, s, n, slow).kf;
-  }
-  bool dummy = false;
-  const KEntry e = batch_k(a.mp, s, n, &dummy);
-  return mk128((uint64_t)__double_as_longlong(e.q), (uint64_t)__double_as_longlong(e.a4n));
-}
-
-// Block-wide path for one batch with more than kCap requests (reads global memory).
-template <int MODE>
-__device__ void jumbo_batch(const TileArgs &a, Smem &sm, uint32_t *tt, int64_t gb, int64_t r0, int64_t r1,
-                            FitAcc &facc, int *bad) {
-  Sums acc{0, 0, 0, 0};
-  for (int64_t i = r0 + threadIdx.x; i < r1; i += kBlock) {
-    int32_t p = a.p[i], c = a.c[i], ph = a.ph[i];
-    check_req(p, c, ph, bad);
-    acc.s1 += p;
-    acc.s2 += c;
-    acc.s3 += (int64_t)p * p;
-    acc.ph += ph;
-  }
-  const Sums ex = block_excl_scan(acc, sm.scr);
-  if (threadIdx.x == kBlock - 1) sm.scr[0] = Sums{ex.s1 + acc.s1, ex.s2 + acc.s2, ex.s3 + acc.s3, ex.ph + acc.ph};
-  __syncthreads();
-  const Sums tot = sm.scr[0];
-  __syncthreads();
-  const BatchAgg g{tot.s1, tot.s2, tot.s3, r1 - r0, tot.ph > 0};
-  const int s = segment_of(a.mp, g);
-  if (threadIdx.x == 0) emit_batch<MODE>(a, gb, g, s);
-  if (MODE & M_FIT) {
-    const int NE = fit_entries(a.fit.n_y);
-    const int64_t x[5] = {1, g.s1, g.s2, g.s3, g.n * g.n};
-    const bool in_range = g.s1 < kFitFeatMax && g.s2 < kFitFeatMax && g.s3 < kFitFeatMax && x[4] < kFitFeatMax;
-    if (!in_range && threadIdx.x == 0) flag(a.status, kStatusOverflow);
-    if ((int)threadIdx.x < 4 * NE && (int)threadIdx.x / NE == s && in_range)
-      fit_owner_add(facc, threadIdx.x % NE, a.fit.n_y, x, a.fit.y, a.n_batch, gb, g.s1 != g.s3, bad);
-  }
-  if (MODE & M_ATTR) {
-    bool slow = false;
-    const i128 kf = batch_const<MODE>(a, sm, s, g.n, &slow);
-    for (int64_t i = r0 + threadIdx.x; i < r1; i += kBlock) {
-      int32_t p = a.p[i], c = a.c[i], ph = a.ph[i];
-      int dummy = 0;
-      check_req(p, c, ph, &dummy);
-      const Rounded r = one_share<MODE>(a, sm.seg, s, slow, kf, p, c, g.n);
-      if (a.share) __stcs(a.share + i, r.d);
-      if (MODE & M_TEN) tenant_add(a, tt, a.ten[i], r, bad);
-    }
-  }
-}
-
-// Requests [r0, win[nbt]) of whole batches 0..nbt-1 of `win` (global batch
-// index gb0 + j), staged in `st` from element `base`.
-template <int MODE>
-__device__ __forceinline__ void sub_tile(const TileArgs &a, Smem &sm, Stage &st, uint32_t *tt, const int64_t *win,
-                                         int64_t gb0, int nbt, int64_t r0, int64_t base, FitAcc &facc, int *bad) {
-  constexpr bool kTen = (MODE & M_TEN) != 0;
-  constexpr bool kShares = (MODE & M_ATTR) != 0;
-  const int tid = threadIdx.x;
-  const int64_t r1 = win[nbt];
-  const int nr = (int)(r1 - r0);
-  const int o = (int)(r0 - base);
-
-  // ---- per-thread requests [i0, i1)
-  const int K = (nr + kBlock - 1) / kBlock;
-  const int i0 = min(tid * K, nr), i1 = min(i0 + K, nr);
-  const int t_last = nr > 0 ? (nr - 1) / K : 0;
-  int jf;  // first boundary j with q_j >= i0
-  {
-    int l = 0, h = nbt + 1;
-    while (l < h) {
-      const int m = (l + h) >> 1;
-      if (win[m] - r0 < i0) l = m + 1; else h = m;
-    }
-    jf = l;
-  }
-  Sums acc{0, 0, 0, 0};
-  int j = jf;
-  int32_t rp[kK], rc[kK], rt[kK];
-#pragma unroll
-  for (int k = 0; k < kK; ++k) {
-    const int i = i0 + k;
-    if (k < K && i < i1) {
-      while (j <= nbt && win[j] - r0 == i) {
-        sm.u.pre.s1[j] = acc.s1;
-        sm.u.pre.s2[j] = acc.s2;
-        sm.u.pre.s3[j] = acc.s3;
-        sm.u.pre.ph[j] = acc.ph;
-        ++j;
-      }
-      int32_t p = st.sp[o + i], c = st.sc[o + i], ph = st.sph[o + i];
-      check_req(p, c, ph, bad);
-      rp[k] = p;
-      rc[k] = c;
-      if (kTen) rt[k] = st.sten[o + i];
-      acc.s1 += p;
-      acc.s2 += c;
-      acc.s3 += (int64_t)p * p;
-      acc.ph += ph;
-    }
-  }
-  if (tid == t_last) {
-    while (j <= nbt && win[j] - r0 == nr) {
-      sm.u.pre.s1[j] = acc.s1;
-      sm.u.pre.s2[j] = acc.s2;
-      sm.u.pre.s3[j] = acc.s3;
-      sm.u.pre.ph[j] = acc.ph;
-      ++j;
-    }
-  }
-  const int jend = j;
-  const Sums base_s = block_excl_scan(acc, sm.scr);
-  for (int jj = jf; jj < jend; ++jj) {
-    sm.u.pre.s1[jj] += base_s.s1;
-    sm.u.pre.s2[jj] += base_s.s2;
-    sm.u.pre.s3[jj] += base_s.s3;
-    sm.u.pre.ph[jj] += base_s.ph;
-  }
-  __syncthreads();
-
-  // ---- per batch: aggregates, segment, outputs, share constant
-  int segv[kBPT];
-  i128 kv[kBPT];
-  bool slowv[kBPT];
-#pragma unroll
-  for (int m = 0; m < kBPT; ++m) {
-    const int jb = tid + m * kBlock;
-    if (jb < nbt) {
-      BatchAgg g;
-      g.s1 = sm.u.pre.s1[jb + 1] - sm.u.pre.s1[jb];
-      g.s2 = sm.u.pre.s2[jb + 1] - sm.u.pre.s2[jb];
-      g.s3 = sm.u.pre.s3[jb + 1] - sm.u.pre.s3[jb];
-      g.n = win[jb + 1] - win[jb];
-      g.prefill = (sm.u.pre.ph[jb + 1] - sm.u.pre.ph[jb]) > 0;
-      const int s = segment_of(a.mp, g);
-      segv[m] = s;
-      emit_batch<MODE>(a, gb0 + jb, g, s);
-      if (MODE & M_FIT) {
-        const bool in_range = g.s1 < kFitFeatMax && g.s2 < kFitFeatMax && g.s3 < kFitFeatMax &&
-                              g.n * g.n < kFitFeatMax;
-        if (!in_range) flag(a.status, kStatusOverflow);
-        sm.fseg[jb] = (g.n > 0 && in_range) ? (uint8_t)s : (uint8_t)0xff;
-      }
-      slowv[m] = false;
-      kv[m] = mk128(0, 0);
-      if (kShares && g.n > 0) kv[m] = batch_const<MODE>(a, sm, s, g.n, &slowv[m]);
-    }
-  }
-  if (!kShares) {
-    __syncthreads();
-    if (MODE & M_FIT) {
-      // owners: thread (g, e) adds the batches of group g of this sub-tile
-      const int NE = fit_entries(a.fit.n_y);
-      if (tid < 4 * NE) {
-        const int g = tid / NE, e = tid % NE;
-        for (int jb = 0; jb < nbt; ++jb) {
-          if (sm.fseg[jb] != g) continue;
-          const int64_t n = win[jb + 1] - win[jb];
-          const int64_t x[5] = {1, sm.u.pre.s1[jb + 1] - sm.u.pre.s1[jb], sm.u.pre.s2[jb + 1] - sm.u.pre.s2[jb],
-                                sm.u.pre.s3[jb + 1] - sm.u.pre.s3[jb], n * n};
-          fit_owner_add(facc, e, a.fit.n_y, x, a.fit.y, a.n_batch, gb0 + jb, x[1] != x[3], bad);
-        }
-      }
-      __syncthreads();
-    }
-    return;
-  }
-  __syncthreads();  // pre[] is dead from here on; bp[] aliases it
-#pragma unroll
-  for (int m = 0; m < kBPT; ++m) {
-    const int jb = tid + m * kBlock;
-    if (jb < nbt) {
-      sm.u.bp.kf[jb] = kv[m];
-      sm.u.bp.seg[jb] = (uint8_t)(segv[m] | (slowv[m] ? 0x80 : 0));
-    }
-  }
-  __syncthreads();
-
-  // ---- shares from registers; staged over the consumed p/c arrays
-  double *shs = reinterpret_cast<double *>(st.sp);
-  int jb = jf > 0 ? jf - 1 : 0;  // batch of request i0: last j with q_j <= i0
-  while (jb + 1 <= nbt && win[jb + 1] - r0 <= i0) ++jb;
-#pragma unroll
-  for (int k = 0; k < kK; ++k) {
-    const int i = i0 + k;
-    if (k < K && i < i1) {
-      while (win[jb + 1] - r0 <= i) ++jb;
-      const uint8_t sg = sm.u.bp.seg[jb];
-      const Rounded r = one_share<MODE>(a, sm.seg, sg & 3, (sg & 0x80) != 0, sm.u.bp.kf[jb], rp[k], rc[k],
-                                        win[jb + 1] - win[jb]);
-      shs[i] = r.d;
-      if (kTen) tenant_add(a, tt, rt[k], r, bad);
-    }
-  }
-  __syncthreads();
-  if (a.share) {
-    for (int i = tid; i < nr; i += kBlock) __stcs(a.share + r0 + i, shs[i]);
-  }
-  __syncthreads();
-}
-
-template <int MODE>
-__global__ void __launch_bounds__(kBlock, 2) k_tiles(const TileArgs a) {
-  extern __shared__ __align__(128) unsigned char smem_raw[];
-  Smem &sm = *reinterpret_cast<Smem *>(smem_raw);
-  uint32_t *tt = reinterpret_cast<uint32_t *>(smem_raw + sizeof(Smem));
-  const int tid = threadIdx.x;
-  constexpr bool kTen = (MODE & M_TEN) != 0;
-  int bad = 0;
-  FitAcc facc;
-  facc.w[0] = facc.w[1] = facc.w[2] = facc.w[3] = 0;
-
-  if (kTen) {
-    for (int i = tid; i < 4 * a.H; i += kBlock) tt[i] = 0;
-  }
-  if ((MODE & M_FIX) && (MODE & M_ATTR)) {
-    for (int i = tid; i < 4 * (kNK + 1); i += kBlock) {
-      const int s = i / (kNK + 1), n = i % (kNK + 1);
-      double v = 0.0;
-      if (n >= 1 && n <= a.mp.nk) {
-        const KEntry e = a.mp.ktab[s * (a.mp.nk + 1) + n];
-        v = __dadd_rn(e.q, e.a4n);
-      }
-      sm.kcd[s][n] = v;
-    }
-    if (tid < 4) {
-      const SegFix &f = a.mp.fx[tid];
-      SegS g;
-      g.A1 = f.A1;
-      g.A3 = f.A3;
-      g.A13 = f.A13;
-      g.A2 = f.A2;
-      g.E = f.E;
-      g.a2_narrow = f.a2_narrow;
-      g.pad[0] = g.pad[1] = 0;
-      sm.seg[tid] = g;
-    }
-  }
-  if (tid == 0) {
-    mbar_init(&sm.full[0], 1);
-    mbar_init(&sm.full[1], 1);
-    fence_mbar_init();
-  }
-  __syncthreads();
-
-  const int64_t G = gridDim.x;
-  TileHdr nxt{};
-  if (tid == 0 && (int64_t)blockIdx.x < a.n_tiles) {
-    const TileHdr h0 = tile_info(a, blockIdx.x, &bad);
-    issue_tile<kTen>(a, sm, 0, h0);
-    if ((int64_t)blockIdx.x + G < a.n_tiles) nxt = tile_info(a, blockIdx.x + G, &bad);
-  }
-
-  int64_t k = 0;
-  for (int64_t t = blockIdx.x; t < a.n_tiles; t += G, ++k) {
-    const int s = (int)(k & 1);
-    if (tid == 0 && t + G < a.n_tiles) {
-      fence_proxy_async_smem();  // the other stage was read and written by generic accesses
-      issue_tile<kTen>(a, sm, s ^ 1, nxt);
-      if (t + 2 * G < a.n_tiles) nxt = tile_info(a, t + 2 * G, &bad);
-    }
-    const bool ok = mbar_wait_bounded(&sm.full[s], (uint32_t)((k >> 1) & 1));
-    if (__syncthreads_or(!ok)) {
-      if (tid == 0) {
-        flag(a.status, kStatusTimeout);
-        // let the other stage's copies land before the CTA leaves
-        if (t + G < a.n_tiles) mbar_wait_bounded(&sm.full[s ^ 1], (uint32_t)(((k + 1) >> 1) & 1));
-      }
-      __syncthreads();
-      return;
-    }
-    Stage &st = sm.st[s];
-    const TileHdr h = sm.hdr[s];
-    const int nb = (int)(h.b1 - h.b0);
-    int64_t *win = st.win + (h.b0 - h.lo);
-    if (nb > 0) {
-      // clamp the window into the tile's request range and check it is monotone
-      for (int i = tid; i <= nb; i += kBlock) win[i] = clampi(win[i], h.r0, h.r1);
-      __syncthreads();
-      int nonmono = (tid == 0) && (win[0] != h.r0 || win[nb] != h.r1);
-      for (int i = tid; i < nb; i += kBlock) nonmono |= win[i + 1] < win[i];
-      if (__syncthreads_or(nonmono)) {
-        if (tid == 0) {
-          win[0] = h.r0;
-          for (int i = 1; i <= nb; ++i)
-            if (win[i] < win[i - 1]) win[i] = win[i - 1];
-          win[nb] = h.r1;
-        }
-        bad = 1;
-        __syncthreads();
-      }
-      int bs = 0;
-      while (bs < nb) {
-        const int64_t r0s = win[bs];
-        int lo = bs, hi = nb;  // largest be in (bs, nb] with win[be] - r0s <= kCap
-        if (win[nb] - r0s <= kCap) lo = nb;
-        while (lo < hi) {
-          const int mid = (lo + hi + 1) >> 1;
-          if (win[mid] - r0s <= kCap) lo = mid; else hi = mid - 1;
-        }
-        const int be = lo;
-        if (be == bs) {
-          jumbo_batch<MODE>(a, sm, tt, h.b0 + bs, r0s, win[bs + 1], facc, &bad);
-          __syncthreads();
-          bs = be + 1;
-          continue;
-        }
-        int64_t base = h.r0 & ~3ll;
-        if (bs > 0) {
-          // beyond the bulk-copied range: stage this sub-tile with plain loads
-          base = r0s & ~3ll;
-          const int64_t r1s = win[be];
-          for (int64_t g = base + tid; g < r1s; g += kBlock) {
-            const int i = (int)(g - base);
-            st.sp[i] = a.p[g];
-            st.sc[i] = a.c[g];
-            st.sph[i] = a.ph[g];
-            if (kTen) st.sten[i] = a.ten[g];
-          }
-          __syncthreads();
-        }
-        sub_tile<MODE>(a, sm, st, tt, win + bs, h.b0 + bs, be - bs, r0s, base, facc, &bad);
-        bs = be;
-      }
-    }
-    __syncthreads();  // stage s is free for the next issue
-  }
-  if (bad) flag(a.status, kStatusData);
-  if (MODE & M_FIT) {
-    const int NE = fit_entries(a.fit.n_y);
-    if (tid < 4 * NE) a.fit.partial[(int64_t)blockIdx.x * 4 * NE + tid] = facc;
-  }
-  if (kTen) {
-    __syncthreads();
-    for (int u = tid; u < a.H; u += kBlock) {
-      const i128 v = hot_value(tt + 4 * u);
-      if (v.lo | v.hi) pend_add(a.ten_pend, u, v);
-    }
-  }
 }
 
 // ---------------------------------------------------------------- tenant pass 2
