@@ -248,7 +248,8 @@ lv_status timing_end(cudaEvent_t stop, cudaStream_t stream) {
 template <int MODE>
 size_t warps_smem(int H, int n_y) {
   return sizeof(WSmem) + ((MODE & M_TEN) ? 16 * (size_t)H : 0) +
-         ((MODE & M_FIT) ? (size_t)kWarps * 4 * fit_entries(n_y) * sizeof(FitAcc) : 0);
+         ((MODE & M_FIT) ? (size_t)kWarps * 4 * fit_entries(n_y) * sizeof(FitAcc) : 0) +
+         ((MODE & M_ATTR) ? (size_t)kWarps * sizeof(DeferList) : 0);
 }
 
 constexpr int kJumboCtasPerSm = 2;

@@ -91,6 +91,87 @@ __device__ __forceinline__ int warp_excl_scan_int(int v, int lane) {
   return x - v;
 }
 
+// ---------------------------------------------------------------- decode fast path
+//
+// A decode request (p = 1) of a batch with constant K has the exact share
+// V = K13 + A2 c with K13 = K + A1 + A3.  When A2 < 2^64 (the segment's
+// a2_narrow) this is one 64x32-bit product and a 128-bit add; the result is
+// rounded to double with 32-bit funnel shifts.  Requests the fast path does not
+// cover (p != 1, V <= 0, a tenant contribution outside the three-word range)
+// are left to general_one.
+
+// v = k + (a1:a0) * c, four 32-bit words, exact (the sum stays below 2^128).
+__device__ __forceinline__ void mad_k13(uint32_t k0, uint32_t k1, uint32_t k2, uint32_t k3, uint32_t a0, uint32_t a1,
+                                        uint32_t c, uint32_t &v0, uint32_t &v1, uint32_t &v2, uint32_t &v3) {
+  asm("{\n\t"
+      ".reg .u32 l0, h0, l1, h1;\n\t"
+      "mul.lo.u32 l0, %4, %6;\n\t"
+      "mul.hi.u32 h0, %4, %6;\n\t"
+      "mul.lo.u32 l1, %5, %6;\n\t"
+      "mul.hi.u32 h1, %5, %6;\n\t"
+      "add.cc.u32 %0, %7, l0;\n\t"
+      "addc.cc.u32 %1, %8, h0;\n\t"
+      "addc.cc.u32 %2, %9, 0;\n\t"
+      "addc.u32 %3, %10, 0;\n\t"
+      "add.cc.u32 %1, %1, l1;\n\t"
+      "addc.cc.u32 %2, %2, h1;\n\t"
+      "addc.u32 %3, %3, 0;\n\t"
+      "}"
+      : "=r"(v0), "=r"(v1), "=r"(v2), "=r"(v3)
+      : "r"(a0), "r"(a1), "r"(c), "r"(k0), "r"(k1), "r"(k2), "r"(k3));
+}
+
+// V * 2^E rounded to the nearest double (ties to even) for 0 < V < 2^127
+// (v3 < 2^31, V nonzero).  m is the rounded significand (2^52 <= m <= 2^53)
+// and ex2 its exponent: the result equals m * 2^ex2.
+__device__ __forceinline__ double round_pos(uint32_t v0, uint32_t v1, uint32_t v2, uint32_t v3, int E, uint64_t &m,
+                                            int &ex2) {
+  const bool z = (v3 | v2) == 0u;  // high half zero: shift by two words
+  const uint32_t h1 = z ? v1 : v3, h0 = z ? v0 : v2, l1 = z ? 0u : v1, l0 = z ? 0u : v0;
+  const bool w = h1 == 0u;  // then by one more word if needed
+  const uint32_t b3 = w ? h0 : h1, b2 = w ? l1 : h0, b1 = w ? l0 : l1, b0 = w ? 0u : l0;
+  const int s = __clz(b3);
+  const uint32_t t3 = __funnelshift_l(b2, b3, s), t2 = __funnelshift_l(b1, b2, s);
+  const uint32_t t1 = __funnelshift_l(b0, b1, s), t0 = b0 << s;
+  const uint32_t mhi = t3 >> 11, mlo = __funnelshift_r(t2, t3, 11);
+  const uint32_t sticky = ((t2 & 0x3ffu) | t1 | t0) != 0u ? 1u : 0u;
+  const uint32_t inc = ((t2 >> 10) & 1u) & (sticky | (mlo & 1u));
+  m = (((uint64_t)mhi << 32) | mlo) + inc;
+  const int ex = 127 - (s + (w ? 32 : 0) + (z ? 64 : 0)) + E;  // exponent of the leading bit
+  ex2 = ex - 52;
+  return __longlong_as_double((long long)(((uint64_t)(ex + 1022) << 52) + m));
+}
+
+// Tenant contribution of a share m * 2^ex2 (m <= 2^53) when q = m 2^(ex2+72)
+// has at most three 32-bit words and the tenant id is valid; false otherwise
+// (nothing is added then).  Hot tenants: exact multi-word add in shared memory;
+// cold tenants: 32-bit limbs into the global 64-bit pending counters.
+__device__ __forceinline__ bool tenant_fast(const TileArgs &a, uint32_t *tt, int32_t u, uint64_t m, int ex2) {
+  const int sh = ex2 - kTenLsb;
+  if ((unsigned)sh > 42u || (unsigned)u >= (unsigned)a.n_tenants) return false;
+  const uint32_t ml = (uint32_t)m, mh = (uint32_t)(m >> 32);
+  const bool lowp = sh < 32;
+  const int t = lowp ? sh : sh - 32;
+  const uint32_t x0 = ml << t, x1 = __funnelshift_l(ml, mh, t), x2 = t ? mh >> (32 - t) : 0u;
+  const uint32_t q0 = lowp ? x0 : 0u, q1 = lowp ? x1 : x0, q2 = lowp ? x2 : x1;
+  if (u < a.H) {
+    uint32_t *w = tt + 4 * u;
+    const uint32_t o0 = atomicAdd(w, q0);
+    const uint32_t a1 = q1 + ((o0 + q0 < o0) ? 1u : 0u);
+    const uint32_t o1 = atomicAdd(w + 1, a1);
+    const uint32_t a2 = q2 + (((o1 + a1 < o1) || a1 < q1) ? 1u : 0u);  // q2 < 2^22: no wrap
+    if (a2) {
+      if (atomicAdd(w + 2, a2) + a2 < a2) atomicAdd(w + 3, 1u);
+    }
+  } else {
+    unsigned long long *pw = a.ten_pend + 4 * (int64_t)u;
+    atomicAdd(pw, (unsigned long long)q0);
+    atomicAdd(pw + 1, (unsigned long long)q1);
+    if (q2) atomicAdd(pw + 2, (unsigned long long)q2);
+  }
+  return true;
+}
+
 // One request's share, its store and its tenant contribution.
 template <int MODE>
 __device__ __forceinline__ void attribute_one(const TileArgs &a, uint32_t *tt, const SegS &sg, int s, bool slow,
@@ -103,6 +184,76 @@ __device__ __forceinline__ void attribute_one(const TileArgs &a, uint32_t *tt, c
     r = share_slow(a.mp, s, (MODE & M_FIX) != 0, kf, p, c, n);
   if (a.share) __stcs(a.share + i, r.d);
   if (MODE & M_TEN) tenant_add(a, tt, u, r, bad);
+}
+
+// The general path for one request q of a batch (segment s, constant kf):
+// reloads the request and takes the exact or fp64 share and the general tenant
+// add.  Out of line: the fast paths send it only the requests they do not cover.
+template <int MODE>
+__device__ __noinline__ void general_one(const TileArgs &a, uint32_t *tt, const SegS *segs, int s, bool slow, i128 kf,
+                                         int64_t n, int64_t q, int *bad) {
+  int32_t p = a.p[q], c = a.c[q];
+  const int32_t u = (MODE & M_TEN) ? a.ten[q] : 0;
+  p = p < 0 ? 0 : p;
+  c = c < 0 ? 0 : c;
+  attribute_one<MODE>(a, tt, segs[s], s, slow, kf, n, q, p, c, u, bad);
+}
+
+// Requests left to the general path, gathered per warp across batches so that
+// they are attributed 32 at a time with every lane busy (a batch of a
+// decode-dominated workload has only a few).  meta = n << 4 | slow << 2 | seg.
+constexpr int kDeferCap = 64;
+struct DeferList {
+  int64_t q[kDeferCap];
+  i128 kf[kDeferCap];
+  int meta[kDeferCap];
+};
+
+// Attribute the first min(cnt, 32) entries, one per lane, and move the rest
+// (at most 31 when cnt < kDeferCap) to the front.
+template <int MODE>
+__device__ __forceinline__ void defer_run(const TileArgs &a, uint32_t *tt, const SegS *segs, DeferList &L, int &cnt,
+                                          int lane, int *bad) {
+  const int take = cnt < 32 ? cnt : 32;
+  if (lane < take) {
+    const int m = L.meta[lane];
+    general_one<MODE>(a, tt, segs, m & 3, (m & 4) != 0, L.kf[lane], m >> 4, L.q[lane], bad);
+  }
+  const int rest = cnt - take;
+  int64_t q = 0;
+  i128 kf = mk128(0, 0);
+  int m = 0;
+  __syncwarp();
+  if (lane < rest) {
+    q = L.q[take + lane];
+    kf = L.kf[take + lane];
+    m = L.meta[take + lane];
+  }
+  __syncwarp();
+  if (lane < rest) {
+    L.q[lane] = q;
+    L.kf[lane] = kf;
+    L.meta[lane] = m;
+  }
+  __syncwarp();
+  cnt = rest;
+}
+
+// Append the request of every lane with `flag`; attribute a full 32 at once.
+template <int MODE>
+__device__ __forceinline__ void defer_push(const TileArgs &a, uint32_t *tt, const SegS *segs, DeferList &L, int &cnt,
+                                           bool flag, int64_t q, i128 kf, int meta, int lane, int *bad) {
+  const uint32_t bm = __ballot_sync(kFull, flag);
+  if (!bm) return;
+  if (flag) {
+    const int slot = cnt + __popc(bm & ((1u << lane) - 1u));
+    L.q[slot] = q;
+    L.kf[slot] = kf;
+    L.meta[slot] = meta;
+  }
+  cnt += __popc(bm);
+  __syncwarp();
+  if (cnt >= 32) defer_run<MODE>(a, tt, segs, L, cnt, lane, bad);
 }
 
 // Per-request constant of a batch: fixed-point K (from the shared table for
@@ -172,16 +323,71 @@ __device__ __forceinline__ void big_shares(const TileArgs &a, uint32_t *tt, cons
   }
 }
 
+// Warp-strided shares of a batch whose decode requests take the fast path
+// (fixed-point mode, in-range constant kf, A2 < 2^64).  Loads of four strided
+// requests are issued before any is used; one copy of the per-request body
+// walks them.  Requests the fast path does not cover are marked (a batch has at
+// most kJumbo requests, so 16 strided positions per lane) and returned: bit t
+// stands for request r0 + lane + 32 t.  ALLDEC: every p = 1, p is not loaded.
+template <int MODE, bool ALLDEC>
+__device__ __forceinline__ uint32_t big_shares_fast(const TileArgs &a, uint32_t *tt, const WSmem &ws, int s, i128 kf,
+                                                    int64_t r0, int64_t r1, int lane) {
+  static_assert(kJumbo <= 16 * 32, "strided positions fit in 16 bits per lane");
+  const SegS &sg = ws.seg[s];
+  const i128 K13 = add128(kf, sg.A13);
+  const uint32_t k0 = (uint32_t)K13.lo, k1 = (uint32_t)(K13.lo >> 32), k2 = (uint32_t)K13.hi,
+                 k3 = (uint32_t)(K13.hi >> 32);
+  const uint32_t a0 = (uint32_t)sg.A2.lo, a1 = (uint32_t)(sg.A2.lo >> 32);
+  const int E = sg.E;
+  uint32_t defer = 0;
+  int pos = 0;
+  for (int64_t i = r0 + lane; i < r1; i += 4 * 32, pos += 4) {
+    int32_t c[4], u[4], p[4];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      const int64_t q = i + 32 * t;
+      const bool in = q < r1;
+      c[t] = in ? a.c[q] : 0;
+      u[t] = (in && (MODE & M_TEN)) ? a.ten[q] : 0;
+      p[t] = (in && !ALLDEC) ? a.p[q] : 1;
+    }
+    int32_t c0 = c[0], c1 = c[1], c2 = c[2], c3 = c[3], u0 = u[0], u1 = u[1], u2 = u[2], u3 = u[3];
+    int32_t p0 = p[0], p1 = p[1], p2 = p[2], p3 = p[3];
+#pragma unroll 1
+    for (int t = 0; t < 4; ++t) {
+      const int64_t q = i + 32 * t;
+      if (q < r1) {
+        bool done = false;
+        if (ALLDEC || p0 == 1) {
+          uint32_t v0, v1, v2, v3;
+          mad_k13(k0, k1, k2, k3, a0, a1, (uint32_t)(c0 < 0 ? 0 : c0), v0, v1, v2, v3);
+          if ((v3 >> 31) == 0u && (v3 | v2 | v1 | v0) != 0u) {
+            uint64_t m;
+            int ex2;
+            const double d = round_pos(v0, v1, v2, v3, E, m, ex2);
+            done = !(MODE & M_TEN) || tenant_fast(a, tt, u0, m, ex2);
+            if (done && a.share) __stcs(a.share + q, d);
+          }
+        }
+        if (!done) defer |= 1u << (pos + t);
+      }
+      c0 = c1; c1 = c2; c2 = c3; u0 = u1; u1 = u2; u2 = u3; p0 = p1; p1 = p2; p2 = p3;
+    }
+  }
+  return defer;
+}
+
 // Rounds over the small batches of a group (lanes with `small`): every round
 // takes the next batches whose requests fit in 32 slots, one request per lane.
 // Pass SHARE=false reduces (each small lane receives its batch's sums in
 // `mys`); SHARE=true attributes with the per-lane constants (myk, mymeta).
 // pn: the lane's request count (0 for other lanes); P: exclusive prefix of pn;
 // base = o0 - P so that slot q of the lane's batch is request base + q.
+// mymeta = n << 4 | fast << 3 | slow << 2 | segment.
 template <int MODE, bool SHARE>
 __device__ __forceinline__ void small_rounds(const TileArgs &a, const WSmem &ws, uint32_t *tt, uint8_t *owner,
-                                             bool small, int pn, int P, int64_t base, Sums &mys, i128 myk,
-                                             int mymeta, int lane, int *bad) {
+                                             DeferList *dl, int &dcnt, bool small, int pn, int P, int64_t base,
+                                             Sums &mys, i128 myk, int mymeta, int lane, int *bad) {
   uint32_t rem = __ballot_sync(kFull, small);
   while (rem) {
     const int start = __shfl_sync(kFull, P, __ffs(rem) - 1);
@@ -214,14 +420,31 @@ __device__ __forceinline__ void small_rounds(const TileArgs &a, const WSmem &ws,
     } else {
       const uint64_t klo = __shfl_sync(kFull, myk.lo, j), khi = __shfl_sync(kFull, myk.hi, j);
       const int meta = __shfl_sync(kFull, mymeta, j);
+      const i128 kf = mk128(klo, khi);
+      bool done = true;
       if (act) {
-        int32_t p = a.p[r], c = a.c[r];
-        const int32_t u = (MODE & M_TEN) ? a.ten[r] : 0;
-        p = p < 0 ? 0 : p;
-        c = c < 0 ? 0 : c;
         const int s = meta & 3;
-        attribute_one<MODE>(a, tt, ws.seg[s], s, (meta & 4) != 0, mk128(klo, khi), meta >> 3, r, p, c, u, bad);
+        done = false;
+        if (meta & 8) {
+          const int32_t p = a.p[r], c = a.c[r];
+          const int32_t u = (MODE & M_TEN) ? a.ten[r] : 0;
+          if (p == 1) {
+            const SegS &sg = ws.seg[s];
+            const i128 K13 = add128(kf, sg.A13);
+            uint32_t v0, v1, v2, v3;
+            mad_k13((uint32_t)K13.lo, (uint32_t)(K13.lo >> 32), (uint32_t)K13.hi, (uint32_t)(K13.hi >> 32),
+                    (uint32_t)sg.A2.lo, (uint32_t)(sg.A2.lo >> 32), (uint32_t)(c < 0 ? 0 : c), v0, v1, v2, v3);
+            if ((v3 >> 31) == 0u && (v3 | v2 | v1 | v0) != 0u) {
+              uint64_t m;
+              int ex2;
+              const double d = round_pos(v0, v1, v2, v3, sg.E, m, ex2);
+              done = !(MODE & M_TEN) || tenant_fast(a, tt, u, m, ex2);
+              if (done && a.share) __stcs(a.share + r, d);
+            }
+          }
+        }
       }
+      defer_push<MODE>(a, tt, ws.seg, *dl, dcnt, !done, r, kf, meta & ~8, lane, bad);
     }
     __syncwarp();  // owner[] is rewritten by the next round
   }
@@ -248,7 +471,8 @@ __device__ __forceinline__ void fit_group(const TileArgs &a, FitAcc *fw, int64_t
 // One group of up to 32 consecutive batches [g0, g0 + ng) of a tile.
 template <int MODE>
 __device__ __forceinline__ void process_group(const TileArgs &a, const WSmem &ws, uint32_t *tt, uint8_t *owner,
-                                              FitAcc *fw, int64_t g0, int ng, int lane, int *bad) {
+                                              DeferList *dl, int &dcnt, FitAcc *fw, int64_t g0, int ng, int lane,
+                                              int *bad) {
   constexpr bool kAttr = (MODE & M_ATTR) != 0;
   const bool valid = lane < ng;
   const int64_t b = g0 + lane;
@@ -287,8 +511,21 @@ __device__ __forceinline__ void process_group(const TileArgs &a, const WSmem &ws
       const int s = segment_of(a.mp, g);
       bool slow = false;
       const i128 kf = batch_const_w<MODE>(a, &ws, s, r1 - r0, &slow);
-      const SegS sg = ws.seg[s];
-      big_shares<MODE>(a, tt, sg, s, slow, kf, r0, r1, lane, bad);
+      if ((MODE & M_FIX) && !slow && ws.seg[s].a2_narrow) {
+        uint32_t defer = (tot.s1 == r1 - r0 && tot.s3 == r1 - r0)
+                             ? big_shares_fast<MODE, true>(a, tt, ws, s, kf, r0, r1, lane)
+                             : big_shares_fast<MODE, false>(a, tt, ws, s, kf, r0, r1, lane);
+        const int meta = ((int)(r1 - r0) << 4) | s;
+        while (__any_sync(kFull, defer != 0u)) {
+          const bool has = defer != 0u;
+          const int t = has ? __ffs(defer) - 1 : 0;
+          if (has) defer &= defer - 1u;
+          defer_push<MODE>(a, tt, ws.seg, *dl, dcnt, has, r0 + lane + 32 * (int64_t)t, kf, meta, lane, bad);
+        }
+      } else {
+        const SegS sg = ws.seg[s];
+        big_shares<MODE>(a, tt, sg, s, slow, kf, r0, r1, lane, bad);
+      }
     }
   }
 
@@ -298,16 +535,17 @@ __device__ __forceinline__ void process_group(const TileArgs &a, const WSmem &ws
     const int pn = small ? (int)n : 0;
     const int P = warp_excl_scan_int(pn, lane);
     const int64_t base = o0 - P;
-    small_rounds<MODE, false>(a, ws, tt, owner, small, pn, P, base, mys, myk, 0, lane, bad);
+    small_rounds<MODE, false>(a, ws, tt, owner, dl, dcnt, small, pn, P, base, mys, myk, 0, lane, bad);
     if (kAttr) {
       if (small) {
         const BatchAgg g{mys.s1, mys.s2, mys.s3, n, mys.ph > 0};
         const int s = segment_of(a.mp, g);
         bool slow = false;
         myk = batch_const_w<MODE>(a, &ws, s, n, &slow);
-        mymeta = ((int)n << 3) | (slow ? 4 : 0) | s;
+        const bool fast = (MODE & M_FIX) && !slow && ws.seg[s].a2_narrow;
+        mymeta = ((int)n << 4) | (fast ? 8 : 0) | (slow ? 4 : 0) | s;
       }
-      small_rounds<MODE, true>(a, ws, tt, owner, small, pn, P, base, mys, myk, mymeta, lane, bad);
+      small_rounds<MODE, true>(a, ws, tt, owner, dl, dcnt, small, pn, P, base, mys, myk, mymeta, lane, bad);
     }
   }
 
@@ -353,6 +591,8 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
   constexpr bool kTen = (MODE & M_TEN) != 0;
   constexpr bool kFit = (MODE & M_FIT) != 0;
   FitAcc *facc = reinterpret_cast<FitAcc *>(smem_raw + sizeof(WSmem) + (kTen ? 16 * (size_t)a.H : 0));
+  DeferList *dlists = reinterpret_cast<DeferList *>(smem_raw + sizeof(WSmem) + (kTen ? 16 * (size_t)a.H : 0) +
+                                                    (kFit ? (size_t)kWarps * 4 * fit_entries(a.fit.n_y) * sizeof(FitAcc) : 0));
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
   const int NE4 = kFit ? 4 * fit_entries(a.fit.n_y) : 0;
   int bad = 0;
@@ -381,6 +621,8 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
 
   uint8_t *owner = ws.owner[wid];
   FitAcc *fw = facc + wid * NE4;
+  DeferList *dl = dlists + wid;
+  int dcnt = 0;
   unsigned long long t = 0;
   if (lane == 0) t = atomicAdd(a.ctr, 1ull);
   t = __shfl_sync(kFull, t, 0);
@@ -394,8 +636,11 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
       bad = 1;
     }
     for (int64_t g0 = b0; g0 < b1; g0 += 32)
-      process_group<MODE>(a, ws, tt, owner, fw, g0, (int)(b1 - g0 < 32 ? b1 - g0 : 32), lane, &bad);
+      process_group<MODE>(a, ws, tt, owner, dl, dcnt, fw, g0, (int)(b1 - g0 < 32 ? b1 - g0 : 32), lane, &bad);
     t = __shfl_sync(kFull, tn, 0);
+  }
+  if (MODE & M_ATTR) {
+    while (dcnt > 0) defer_run<MODE>(a, tt, ws.seg, *dl, dcnt, lane, &bad);
   }
 
   if (bad) flag(a.status, kStatusData);
