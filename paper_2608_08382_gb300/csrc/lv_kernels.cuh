@@ -257,8 +257,8 @@ __device__ __forceinline__ double eq1_fp64(const double *k, const BatchAgg &g) {
 }
 
 // Eq. 1 exactly in fixed point, one rounding; falls back to fp64 outside the
-// exact range.
-__device__ __forceinline__ double eq1_fix(const ModelP &mp, int s, const BatchAgg &g) {
+// exact range.  Once per batch, so kept out of line.
+__device__ __noinline__ double eq1_fix(const ModelP &mp, int s, const BatchAgg &g) {
   if (g.n == 0) return 0.0;
   const SegFix &f = mp.fx[s];
   const uint64_t F4 = (uint64_t)g.n * (uint64_t)g.n;

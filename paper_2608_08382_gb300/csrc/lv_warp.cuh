@@ -97,8 +97,8 @@ __device__ __forceinline__ int warp_excl_scan_int(int v, int lane) {
 // V = K13 + A2 c with K13 = K + A1 + A3.  When A2 < 2^64 (the segment's
 // a2_narrow) this is one 64x32-bit product and a 128-bit add; the result is
 // rounded to double with 32-bit funnel shifts.  Requests the fast path does not
-// cover (p != 1, V <= 0, a tenant contribution outside the three-word range)
-// are left to general_one.
+// cover (p != 1, V outside [2^64, 2^96), a tenant contribution outside the
+// three-word range) are left to general_one, which is exact for every case.
 
 // v = k + (a1:a0) * c, four 32-bit words, exact (the sum stays below 2^128).
 __device__ __forceinline__ void mad_k13(uint32_t k0, uint32_t k1, uint32_t k2, uint32_t k3, uint32_t a0, uint32_t a1,
@@ -121,23 +121,17 @@ __device__ __forceinline__ void mad_k13(uint32_t k0, uint32_t k1, uint32_t k2, u
       : "r"(a0), "r"(a1), "r"(c), "r"(k0), "r"(k1), "r"(k2), "r"(k3));
 }
 
-// V * 2^E rounded to the nearest double (ties to even) for 0 < V < 2^127
-// (v3 < 2^31, V nonzero).  m is the rounded significand (2^52 <= m <= 2^53)
-// and ex2 its exponent: the result equals m * 2^ex2.
-__device__ __forceinline__ double round_pos(uint32_t v0, uint32_t v1, uint32_t v2, uint32_t v3, int E, uint64_t &m,
-                                            int &ex2) {
-  const bool z = (v3 | v2) == 0u;  // high half zero: shift by two words
-  const uint32_t h1 = z ? v1 : v3, h0 = z ? v0 : v2, l1 = z ? 0u : v1, l0 = z ? 0u : v0;
-  const bool w = h1 == 0u;  // then by one more word if needed
-  const uint32_t b3 = w ? h0 : h1, b2 = w ? l1 : h0, b1 = w ? l0 : l1, b0 = w ? 0u : l0;
-  const int s = __clz(b3);
-  const uint32_t t3 = __funnelshift_l(b2, b3, s), t2 = __funnelshift_l(b1, b2, s);
-  const uint32_t t1 = __funnelshift_l(b0, b1, s), t0 = b0 << s;
-  const uint32_t mhi = t3 >> 11, mlo = __funnelshift_r(t2, t3, 11);
-  const uint32_t sticky = ((t2 & 0x3ffu) | t1 | t0) != 0u ? 1u : 0u;
-  const uint32_t inc = ((t2 >> 10) & 1u) & (sticky | (mlo & 1u));
+// V * 2^E rounded to the nearest double (ties to even) for the common
+// magnitude 2^64 <= V < 2^96 (v3 = 0, v2 != 0; the caller checks): the
+// leading word is v2.  m is the rounded significand (2^52 <= m <= 2^53) and
+// ex2 its exponent: the result equals m * 2^ex2.
+__device__ __forceinline__ double round96(uint32_t v0, uint32_t v1, uint32_t v2, int E, uint64_t &m, int &ex2) {
+  const int s = __clz(v2);
+  const uint32_t t2 = __funnelshift_l(v1, v2, s), t1 = __funnelshift_l(v0, v1, s), t0 = v0 << s;
+  const uint32_t mhi = t2 >> 11, mlo = __funnelshift_r(t1, t2, 11);
+  const uint32_t inc = ((t1 >> 10) & 1u) & ((((t1 & 0x3ffu) | t0) != 0u ? 1u : 0u) | (mlo & 1u));
   m = (((uint64_t)mhi << 32) | mlo) + inc;
-  const int ex = 127 - (s + (w ? 32 : 0) + (z ? 64 : 0)) + E;  // exponent of the leading bit
+  const int ex = 95 - s + E;  // exponent of the leading bit
   ex2 = ex - 52;
   return __longlong_as_double((long long)(((uint64_t)(ex + 1022) << 52) + m));
 }
@@ -272,34 +266,43 @@ __device__ __forceinline__ i128 batch_const_w(const TileArgs &a, const WSmem *ws
   return mk128((uint64_t)__double_as_longlong(e.q), (uint64_t)__double_as_longlong(e.a4n));
 }
 
-// Warp-strided sums over requests [r0, r1); uniform result on every lane.
+// Warp-strided sums over requests [r0, r1) (at most kJumbo); uniform result on
+// every lane.  Indices are 32-bit offsets from the batch's first request.
 __device__ __forceinline__ Sums big_reduce(const TileArgs &a, int64_t r0, int64_t r1, int lane, int *bad) {
+  const int32_t *P = a.p + r0, *C = a.c + r0, *PH = a.ph + r0;
+  const int n = (int)(r1 - r0);
   Sums acc{0, 0, 0, 0};
-  for (int64_t i = r0 + lane; i < r1; i += 4 * 32) {
+  int32_t sgn = 0, phx = 0;  // sign bits of p and c; bits of phase beyond 0/1
+  for (int i = lane; i < n; i += 4 * 32) {
     int32_t p[4], c[4], ph[4];
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int64_t q = i + 32 * k;
-      const bool in = q < r1;
-      p[k] = in ? a.p[q] : 0;
-      c[k] = in ? a.c[q] : 0;
-      ph[k] = in ? a.ph[q] : 0;
+    for (int t = 0; t < 4; ++t) {
+      const int q = i + 32 * t;
+      const bool in = q < n;
+      p[t] = in ? P[q] : 0;
+      c[t] = in ? C[q] : 0;
+      ph[t] = in ? PH[q] : 0;
     }
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      check_req(p[k], c[k], ph[k], bad);
-      acc.s1 += p[k];
-      acc.s2 += c[k];
-      acc.s3 += (int64_t)p[k] * p[k];
-      acc.ph += ph[k];
+    for (int t = 0; t < 4; ++t) {
+      sgn |= p[t] | c[t];
+      phx |= ph[t] & ~1;
+      const int32_t pt = p[t] < 0 ? 0 : p[t], ct = c[t] < 0 ? 0 : c[t];
+      acc.s1 += pt;
+      acc.s2 += ct;
+      acc.s3 += (int64_t)pt * pt;
+      acc.ph += ph[t] != 0;
     }
   }
+  if (sgn < 0 || phx != 0) *bad = 1;  // clamped as check_req does
   return warp_sum(acc);
 }
 
-// Warp-strided shares of requests [r0, r1) of one batch (segment s, constant kf).
+// Warp-strided shares of requests [r0, r1) of one batch (segment s, constant kf):
+// the general loop for fp64 mode, an out-of-range constant or a wide A2 (out
+// of line: the fast loop serves the common case).
 template <int MODE>
-__device__ __forceinline__ void big_shares(const TileArgs &a, uint32_t *tt, const SegS &sg, int s, bool slow,
+__device__ __noinline__ void big_shares(const TileArgs &a, uint32_t *tt, const SegS &sg, int s, bool slow,
                                            i128 kf, int64_t r0, int64_t r1, int lane, int *bad) {
   const int64_t n = r1 - r0;
   for (int64_t i = r0 + lane; i < r1; i += 4 * 32) {
@@ -339,36 +342,37 @@ __device__ __forceinline__ uint32_t big_shares_fast(const TileArgs &a, uint32_t 
                  k3 = (uint32_t)(K13.hi >> 32);
   const uint32_t a0 = (uint32_t)sg.A2.lo, a1 = (uint32_t)(sg.A2.lo >> 32);
   const int E = sg.E;
+  const int32_t *P = a.p + r0, *C = a.c + r0, *U = a.ten + r0;
+  double *S = a.share ? a.share + r0 : nullptr;
+  const int n = (int)(r1 - r0);
   uint32_t defer = 0;
-  int pos = 0;
-  for (int64_t i = r0 + lane; i < r1; i += 4 * 32, pos += 4) {
+  for (int i = lane, pos = 0; i < n; i += 4 * 32, pos += 4) {
     int32_t c[4], u[4], p[4];
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
-      const int64_t q = i + 32 * t;
-      const bool in = q < r1;
-      c[t] = in ? a.c[q] : 0;
-      u[t] = (in && (MODE & M_TEN)) ? a.ten[q] : 0;
-      p[t] = (in && !ALLDEC) ? a.p[q] : 1;
+      const int q = i + 32 * t;
+      const bool in = q < n;
+      c[t] = in ? C[q] : 0;
+      u[t] = (in && (MODE & M_TEN)) ? U[q] : 0;
+      p[t] = (in && !ALLDEC) ? P[q] : 1;
     }
+    // one copy of the body walks the four loaded requests (registers rotate)
     int32_t c0 = c[0], c1 = c[1], c2 = c[2], c3 = c[3], u0 = u[0], u1 = u[1], u2 = u[2], u3 = u[3];
     int32_t p0 = p[0], p1 = p[1], p2 = p[2], p3 = p[3];
 #pragma unroll 1
     for (int t = 0; t < 4; ++t) {
-      const int64_t q = i + 32 * t;
-      if (q < r1) {
-        bool done = false;
-        if (ALLDEC || p0 == 1) {
-          uint32_t v0, v1, v2, v3;
-          mad_k13(k0, k1, k2, k3, a0, a1, (uint32_t)(c0 < 0 ? 0 : c0), v0, v1, v2, v3);
-          if ((v3 >> 31) == 0u && (v3 | v2 | v1 | v0) != 0u) {
-            uint64_t m;
-            int ex2;
-            const double d = round_pos(v0, v1, v2, v3, E, m, ex2);
-            done = !(MODE & M_TEN) || tenant_fast(a, tt, u0, m, ex2);
-            if (done && a.share) __stcs(a.share + q, d);
-          }
+      const int q = i + 32 * t;
+      if (q < n) {
+        uint32_t v0, v1, v2, v3;
+        mad_k13(k0, k1, k2, k3, a0, a1, (uint32_t)(c0 < 0 ? 0 : c0), v0, v1, v2, v3);
+        uint64_t m;
+        int ex2;
+        const double d = round96(v0, v1, v2, E, m, ex2);
+        bool done = (ALLDEC || p0 == 1) && v3 == 0u && v2 != 0u;
+        if (MODE & M_TEN) {
+          if (done) done = tenant_fast(a, tt, u0, m, ex2);
         }
+        if (done && S) __stcs(S + q, d);
         if (!done) defer |= 1u << (pos + t);
       }
       c0 = c1; c1 = c2; c2 = c3; u0 = u1; u1 = u2; u2 = u3; p0 = p1; p1 = p2; p2 = p3;
@@ -428,20 +432,19 @@ __device__ __forceinline__ void small_rounds(const TileArgs &a, const WSmem &ws,
         if (meta & 8) {
           const int32_t p = a.p[r], c = a.c[r];
           const int32_t u = (MODE & M_TEN) ? a.ten[r] : 0;
-          if (p == 1) {
-            const SegS &sg = ws.seg[s];
-            const i128 K13 = add128(kf, sg.A13);
-            uint32_t v0, v1, v2, v3;
-            mad_k13((uint32_t)K13.lo, (uint32_t)(K13.lo >> 32), (uint32_t)K13.hi, (uint32_t)(K13.hi >> 32),
-                    (uint32_t)sg.A2.lo, (uint32_t)(sg.A2.lo >> 32), (uint32_t)(c < 0 ? 0 : c), v0, v1, v2, v3);
-            if ((v3 >> 31) == 0u && (v3 | v2 | v1 | v0) != 0u) {
-              uint64_t m;
-              int ex2;
-              const double d = round_pos(v0, v1, v2, v3, sg.E, m, ex2);
-              done = !(MODE & M_TEN) || tenant_fast(a, tt, u, m, ex2);
-              if (done && a.share) __stcs(a.share + r, d);
-            }
+          const SegS &sg = ws.seg[s];
+          const i128 K13 = add128(kf, sg.A13);
+          uint32_t v0, v1, v2, v3;
+          mad_k13((uint32_t)K13.lo, (uint32_t)(K13.lo >> 32), (uint32_t)K13.hi, (uint32_t)(K13.hi >> 32),
+                  (uint32_t)sg.A2.lo, (uint32_t)(sg.A2.lo >> 32), (uint32_t)(c < 0 ? 0 : c), v0, v1, v2, v3);
+          uint64_t m;
+          int ex2;
+          const double d = round96(v0, v1, v2, sg.E, m, ex2);
+          done = p == 1 && v3 == 0u && v2 != 0u;
+          if (MODE & M_TEN) {
+            if (done) done = tenant_fast(a, tt, u, m, ex2);
           }
+          if (done && a.share) __stcs(a.share + r, d);
         }
       }
       defer_push<MODE>(a, tt, ws.seg, *dl, dcnt, !done, r, kf, meta & ~8, lane, bad);
@@ -523,8 +526,7 @@ __device__ __forceinline__ void process_group(const TileArgs &a, const WSmem &ws
           defer_push<MODE>(a, tt, ws.seg, *dl, dcnt, has, r0 + lane + 32 * (int64_t)t, kf, meta, lane, bad);
         }
       } else {
-        const SegS sg = ws.seg[s];
-        big_shares<MODE>(a, tt, sg, s, slow, kf, r0, r1, lane, bad);
+        big_shares<MODE>(a, tt, ws.seg[s], s, slow, kf, r0, r1, lane, bad);
       }
     }
   }

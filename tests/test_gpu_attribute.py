@@ -196,6 +196,24 @@ def test_wide_coefficients_use_fp64_path(lv, ctx):
     _check_parity(w, T, share, L)
 
 
+@pytest.mark.parametrize("scale", ["low", "high"])
+def test_fixed_point_value_ranges(lv, ctx, scale):
+    """Shares whose exact fixed-point value lies below 2^64 or at or above 2^96 (outside the
+    decode fast path's window) are attributed exactly all the same, with and without tenants."""
+    rng = np.random.default_rng(11)
+    w = _from_sizes(rng, rng.integers(1, 300, 3000), pre=0.05)
+    if scale == "low":
+        # power-of-two coefficients: the scale is set by beta (2^-10 - 66), values near 2^59
+        w.coef[:] = [2.0 ** -10, 2.0 ** -20, 2.0 ** -27, 2.0 ** -33, 2.0 ** -27]
+    else:
+        # an odd multiple of 2^-130 in a4 puts the scale at 2^-130, values near 2^115
+        w.coef[:, 4] = 3.0 * 2.0 ** -130
+    for acc in (True, False):
+        T, share, L, st = _run(lv, ctx, w, acc=acc)
+        assert st == lv.LV_OK
+        _check_parity(w, T, share, L)
+
+
 def test_negative_coefficient_cancellation(lv, ctx):
     rng = np.random.default_rng(10)
     w = _from_sizes(rng, rng.integers(1, 200, 3000))
