@@ -267,18 +267,21 @@ __device__ __forceinline__ i128 batch_const_w(const TileArgs &a, const WSmem *ws
 }
 
 // Warp-strided sums over requests [r0, r1) (at most kJumbo); uniform result on
-// every lane.  Indices are 32-bit offsets from the batch's first request.
+// every lane.  Indices are 32-bit offsets from the batch's first request.  With
+// a tenant pass the tenant ids are loaded (and checked) here as well, so that
+// the share pass finds the whole batch in L1.
 __device__ __forceinline__ Sums big_reduce(const TileArgs &a, int64_t r0, int64_t r1, int lane, int *bad) {
   const int32_t *P = a.p + r0, *C = a.c + r0, *PH = a.ph + r0;
   const int n = (int)(r1 - r0);
   Sums acc{0, 0, 0, 0};
   int32_t sgn = 0, phx = 0;  // sign bits of p and c; bits of phase beyond 0/1
   for (int i = lane; i < n; i += 4 * 32) {
-    int32_t p[4], c[4], ph[4];
+    int32_t p[4], c[4], ph[4], u[4];
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
       const int q = i + 32 * t;
       const bool in = q < n;
+      u[t] = (in && a.ten) ? a.ten[r0 + q] : 0;
       p[t] = in ? P[q] : 0;
       c[t] = in ? C[q] : 0;
       ph[t] = in ? PH[q] : 0;
@@ -286,6 +289,7 @@ __device__ __forceinline__ Sums big_reduce(const TileArgs &a, int64_t r0, int64_
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
       sgn |= p[t] | c[t];
+      if (a.ten && (unsigned)u[t] >= (unsigned)a.n_tenants) sgn |= 0x80000000;
       phx |= ph[t] & ~1;
       const int32_t pt = p[t] < 0 ? 0 : p[t], ct = c[t] < 0 ? 0 : c[t];
       acc.s1 += pt;
@@ -327,11 +331,12 @@ __device__ __noinline__ void big_shares(const TileArgs &a, uint32_t *tt, const S
 }
 
 // Warp-strided shares of a batch whose decode requests take the fast path
-// (fixed-point mode, in-range constant kf, A2 < 2^64).  Loads of four strided
-// requests are issued before any is used; one copy of the per-request body
-// walks them.  Requests the fast path does not cover are marked (a batch has at
-// most kJumbo requests, so 16 strided positions per lane) and returned: bit t
-// stands for request r0 + lane + 32 t.  ALLDEC: every p = 1, p is not loaded.
+// (fixed-point mode, in-range constant kf, A2 < 2^64).  The batch was just
+// reduced, tenant ids included, so its requests are in L1 and the loop takes
+// one request per lane per step.  Requests the fast path does not cover are
+// marked (a batch has at most kJumbo requests, so 16 strided positions per
+// lane) and returned: bit t stands for request r0 + lane + 32 t.  ALLDEC:
+// every p = 1, p is not loaded.
 template <int MODE, bool ALLDEC>
 __device__ __forceinline__ uint32_t big_shares_fast(const TileArgs &a, uint32_t *tt, const WSmem &ws, int s, i128 kf,
                                                     int64_t r0, int64_t r1, int lane) {
@@ -346,37 +351,21 @@ __device__ __forceinline__ uint32_t big_shares_fast(const TileArgs &a, uint32_t 
   double *S = a.share ? a.share + r0 : nullptr;
   const int n = (int)(r1 - r0);
   uint32_t defer = 0;
-  for (int i = lane, pos = 0; i < n; i += 4 * 32, pos += 4) {
-    int32_t c[4], u[4], p[4];
-#pragma unroll
-    for (int t = 0; t < 4; ++t) {
-      const int q = i + 32 * t;
-      const bool in = q < n;
-      c[t] = in ? C[q] : 0;
-      u[t] = (in && (MODE & M_TEN)) ? U[q] : 0;
-      p[t] = (in && !ALLDEC) ? P[q] : 1;
+  for (int q = lane, pos = 0; q < n; q += 32, ++pos) {
+    const int32_t c0 = C[q];
+    const int32_t u0 = (MODE & M_TEN) ? U[q] : 0;
+    const int32_t p0 = ALLDEC ? 1 : P[q];
+    uint32_t v0, v1, v2, v3;
+    mad_k13(k0, k1, k2, k3, a0, a1, (uint32_t)(c0 < 0 ? 0 : c0), v0, v1, v2, v3);
+    uint64_t m;
+    int ex2;
+    const double d = round96(v0, v1, v2, E, m, ex2);
+    bool done = (ALLDEC || p0 == 1) && v3 == 0u && v2 != 0u;
+    if (MODE & M_TEN) {
+      if (done) done = tenant_fast(a, tt, u0, m, ex2);
     }
-    // one copy of the body walks the four loaded requests (registers rotate)
-    int32_t c0 = c[0], c1 = c[1], c2 = c[2], c3 = c[3], u0 = u[0], u1 = u[1], u2 = u[2], u3 = u[3];
-    int32_t p0 = p[0], p1 = p[1], p2 = p[2], p3 = p[3];
-#pragma unroll 1
-    for (int t = 0; t < 4; ++t) {
-      const int q = i + 32 * t;
-      if (q < n) {
-        uint32_t v0, v1, v2, v3;
-        mad_k13(k0, k1, k2, k3, a0, a1, (uint32_t)(c0 < 0 ? 0 : c0), v0, v1, v2, v3);
-        uint64_t m;
-        int ex2;
-        const double d = round96(v0, v1, v2, E, m, ex2);
-        bool done = (ALLDEC || p0 == 1) && v3 == 0u && v2 != 0u;
-        if (MODE & M_TEN) {
-          if (done) done = tenant_fast(a, tt, u0, m, ex2);
-        }
-        if (done && S) __stcs(S + q, d);
-        if (!done) defer |= 1u << (pos + t);
-      }
-      c0 = c1; c1 = c2; c2 = c3; u0 = u1; u1 = u2; u2 = u3; p0 = p1; p1 = p2; p2 = p3;
-    }
+    if (done && S) __stcs(S + q, d);
+    if (!done) defer |= 1u << pos;
   }
   return defer;
 }
