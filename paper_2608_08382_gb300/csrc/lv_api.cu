@@ -39,6 +39,7 @@ struct lv_ctx {
   void *d_fit = nullptr;      // fit partials + solve output
   size_t fit_cap = 0;
   int64_t last_grid = 0;      // CTAs of the most recent tile-kernel launch
+  std::vector<std::pair<uint64_t, int>> occ;  // (mode << 32 | dynamic smem) -> k_warps CTAs per SM
   void *d_wi = nullptr;       // what-if per-candidate / per-pending tables
   size_t wi_cap = 0;
   int timing = 0;  // LV_TIME_* mask
@@ -264,14 +265,23 @@ template <int MODE>
 lv_status launch_warps_mode(lv_ctx *ctx, int sms, TileArgs &a, cudaStream_t stream, int64_t *ctas) {
   *ctas = 0;
   const size_t smem = warps_smem<MODE>(a.H, a.fit.n_y);
-  LV_CUDA(cudaFuncSetAttribute(k_warps<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)warps_smem<MODE>(kHotMax, kFitMaxY)));
   const size_t jsmem = sizeof(JSmem) + ((MODE & M_TEN) ? 16 * (size_t)a.H : 0);
-  LV_CUDA(cudaFuncSetAttribute(k_jumbo<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)(sizeof(JSmem) + 16 * (size_t)kHotMax)));
+  const uint64_t key = ((uint64_t)MODE << 32) | smem;
   int per_sm = 0;
-  LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_warps<MODE>, kWThreads, smem));
-  if (per_sm < 1) per_sm = 1;
+  if (ctx) {
+    for (const auto &e : ctx->occ)
+      if (e.first == key) per_sm = e.second;
+  }
+  if (per_sm == 0) {
+    // kernel attributes and occupancy: once per (context, mode, shared-memory size)
+    LV_CUDA(cudaFuncSetAttribute(k_warps<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)warps_smem<MODE>(kHotMax, kFitMaxY)));
+    LV_CUDA(cudaFuncSetAttribute(k_jumbo<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)(sizeof(JSmem) + 16 * (size_t)kHotMax)));
+    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_warps<MODE>, kWThreads, smem));
+    if (per_sm < 1) per_sm = 1;
+    if (ctx) ctx->occ.emplace_back(key, per_sm);
+  }
   const int64_t grid = std::min<int64_t>(a.n_tiles, (int64_t)sms * per_sm);
   if (grid <= 0) return LV_OK;
   const int64_t jgrid = (int64_t)sms * kJumboCtasPerSm;
@@ -719,7 +729,7 @@ lv_status lv_fit(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y,
   st = run_tiles(ctx, a, M_FEAT | M_FIT, stream);
   if (st != LV_OK) return st;
   const int n_cta = (int)ctx->last_grid;
-  k_fit_reduce<<<(n_ent + 127) / 128, 128, 0, stream>>>(partial, n_cta, n_ent, totals);
+  k_fit_reduce<<<n_ent, kFitRedThreads, 0, stream>>>(partial, n_cta, n_ent, totals);
   LV_CUDA(cudaGetLastError());
   k_fit_solve<<<1, 4 * kFitMaxY, 0, stream>>>(totals, n_y, out);
   LV_CUDA(cudaGetLastError());

@@ -23,22 +23,38 @@ namespace lv {
 
 // ---------------------------------------------------------------- reduction across CTAs
 
-// totals[ge] = sum over CTAs of partial[cta][ge] (exact integer adds; the flag entry is ORed).
-__global__ void k_fit_reduce(const FitAcc *__restrict__ partial, int n_cta, int n_ent, FitAcc *__restrict__ totals) {
-  const int ge = blockIdx.x * blockDim.x + threadIdx.x;
-  if (ge >= n_ent) return;
+// totals[ge] = sum over CTAs of partial[cta][ge]: one block per entry, threads
+// striding over the CTAs, then a tree in shared memory.  Integer addition is
+// associative, so the exact result does not depend on the order; the flag
+// entries are ORed.
+constexpr int kFitRedThreads = 256;
+__global__ void __launch_bounds__(kFitRedThreads) k_fit_reduce(const FitAcc *__restrict__ partial, int n_cta,
+                                                               int n_ent, FitAcc *__restrict__ totals) {
+  __shared__ FitAcc red[kFitRedThreads];
+  const int ge = blockIdx.x;
+  const bool is_flag = ge % (n_ent / 4) == n_ent / 4 - 1;
   FitAcc t;
   t.w[0] = t.w[1] = t.w[2] = t.w[3] = 0;
-  const int e = ge % (n_ent / 4);
-  const bool is_flag = e == n_ent / 4 - 1;
-  for (int c = 0; c < n_cta; ++c) {
-    const FitAcc &p = partial[(int64_t)c * n_ent + ge];
+  for (int c = threadIdx.x; c < n_cta; c += kFitRedThreads) {
+    const FitAcc p = partial[(int64_t)c * n_ent + ge];
     if (is_flag)
       t.w[0] |= p.w[0];
     else
       acc_add256(t.w, p.w[0], p.w[1], p.w[2], p.w[3]);
   }
-  totals[ge] = t;
+  red[threadIdx.x] = t;
+  __syncthreads();
+  for (int h = kFitRedThreads / 2; h > 0; h >>= 1) {
+    if ((int)threadIdx.x < h) {
+      const FitAcc o = red[threadIdx.x + h];
+      if (is_flag)
+        red[threadIdx.x].w[0] |= o.w[0];
+      else
+        acc_add256(red[threadIdx.x].w, o.w[0], o.w[1], o.w[2], o.w[3]);
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) totals[ge] = red[0];
 }
 
 // ---------------------------------------------------------------- double-double arithmetic
@@ -137,61 +153,69 @@ struct FitOut {
   int32_t status, dropped;
 };
 
+// Index of Gram pair (a, b) in the accumulator order (row-major upper triangle).
+__host__ __device__ constexpr int gram_idx(int a, int b) {
+  return a <= b ? a * 5 - a * (a - 1) / 2 + (b - a) : b * 5 - b * (b - 1) / 2 + (a - b);
+}
+
 // One thread per (y vector, group): builds, scales and solves the normal
-// equations from the exact totals.
-__global__ void k_fit_solve(const FitAcc *__restrict__ totals, int n_y, FitOut *__restrict__ out) {
+// equations from the exact totals.  Every loop has constant bounds, so the
+// 5x5 system lives in registers; a dropped a3 column becomes a unit row and
+// column with a zero right-hand side (its coefficient solves to 0).  Each
+// pivot is inverted once in double-double and the eliminations multiply.
+__global__ void __launch_bounds__(32) k_fit_solve(const FitAcc *__restrict__ totals, int n_y, FitOut *__restrict__ out) {
   const int t = threadIdx.x;
   if (t >= 4 * n_y) return;
   const int k = t / 4, g = t % 4;
   const int NE = fit_entries(n_y);
   const FitAcc *T = totals + g * NE;
   FitOut o;
+#pragma unroll
   for (int i = 0; i < 5; ++i) o.coef[i] = 0.0;
   o.ssr = 0.0;
   o.r2 = 0.0;
   o.dropped = 0;
   const int64_t n = (int64_t)T[0].w[0];  // Gram (0,0) = number of batches
   o.n = n;
-  const bool any_ne = (T[NE - 1].w[0] & 1ull) != 0;
-  int cols[5], kc = 0;
-  for (int a = 0; a < 5; ++a) {
-    if (a == 3 && n > 0 && !any_ne) {
-      o.dropped |= 1 << 3;
-      continue;
-    }
-    cols[kc++] = a;
-  }
-  if (n < kc) {
+  const bool drop3 = n > 0 && (T[NE - 1].w[0] & 1ull) == 0ull;
+  if (drop3) o.dropped = 1 << 3;
+  if (n < (drop3 ? 4 : 5)) {
     o.status = LV_ENODATA;
     out[k * 4 + g] = o;
     return;
   }
-  // Gram in double-double; index of pair (a, b), a <= b
-  auto gidx = [](int a, int b) {
-    if (a > b) {
-      const int tt = a;
-      a = b;
-      b = tt;
-    }
-    return a * 5 - a * (a - 1) / 2 + (b - a);
-  };
-  dd G[5][5], r[5];
+  // exact totals as double-double, each converted once
+  dd Gu[15], ru[5];
+#pragma unroll
+  for (int i = 0; i < 15; ++i) Gu[i] = int256_to_dd(T[i].w, 0);
+#pragma unroll
+  for (int a = 0; a < 5; ++a) ru[a] = int256_to_dd(T[15 + k * 5 + a].w, kFitYLsb);
+  if (drop3) {
+#pragma unroll
+    for (int a = 0; a < 5; ++a) Gu[gram_idx(a, 3)] = dd{a == 3 ? 1.0 : 0.0, 0.0};
+    ru[3] = dd{0.0, 0.0};
+  }
+  // power-of-two column scaling: scaled diagonal near 1
   int sc[5];
-  for (int i = 0; i < kc; ++i) {
-    const FitAcc &d = T[gidx(cols[i], cols[i])];
-    const dd gii = int256_to_dd(d.w, 0);
+#pragma unroll
+  for (int i = 0; i < 5; ++i) {
     int ex;
-    frexp(gii.hi, &ex);
-    sc[i] = -(ex / 2);  // column scale 2^sc, makes the scaled diagonal ~1
+    frexp(Gu[gram_idx(i, i)].hi, &ex);
+    sc[i] = -(ex / 2);
   }
-  for (int i = 0; i < kc; ++i) {
-    for (int j = 0; j < kc; ++j) G[i][j] = dd_scale(int256_to_dd(T[gidx(cols[i], cols[j])].w, 0), sc[i] + sc[j]);
-    r[i] = dd_scale(int256_to_dd(T[15 + k * 5 + cols[i]].w, kFitYLsb), sc[i]);
+  dd L[15], r[5], inv[5];
+#pragma unroll
+  for (int i = 0; i < 5; ++i) {
+#pragma unroll
+    for (int j = 0; j <= i; ++j) L[gram_idx(i, j)] = dd_scale(Gu[gram_idx(i, j)], sc[i] + sc[j]);
+    r[i] = dd_scale(ru[i], sc[i]);
   }
-  // Cholesky G = L L^T (in place, lower triangle)
-  for (int j = 0; j < kc; ++j) {
-    dd d = G[j][j];
-    for (int m = 0; m < j; ++m) d = dd_add(d, dd_neg(dd_mul(G[j][m], G[j][m])));
+  // Cholesky G = L L^T (lower triangle in L, indexed symmetrically)
+#pragma unroll
+  for (int j = 0; j < 5; ++j) {
+    dd d = L[gram_idx(j, j)];
+#pragma unroll
+    for (int m = 0; m < j; ++m) d = dd_add(d, dd_neg(dd_mul(L[gram_idx(j, m)], L[gram_idx(j, m)])));
     if (!(d.hi > 1e-24)) {
       o.status = LV_ESINGULAR;
       out[k * 4 + g] = o;
@@ -200,35 +224,44 @@ __global__ void k_fit_solve(const FitAcc *__restrict__ totals, int n_y, FitOut *
     // square root in double-double: s0 = sqrt(d.hi), one Newton step
     const double s0 = sqrt(d.hi);
     const dd s0sq = dd_mul(dd{s0, 0.0}, dd{s0, 0.0});
-    const dd corr = dd_div(dd_add(d, dd_neg(s0sq)), dd{2.0 * s0, 0.0});
-    const dd s = dd_add(dd{s0, 0.0}, corr);
-    G[j][j] = s;
-    for (int i = j + 1; i < kc; ++i) {
-      dd v = G[i][j];
-      for (int m = 0; m < j; ++m) v = dd_add(v, dd_neg(dd_mul(G[i][m], G[j][m])));
-      G[i][j] = dd_div(v, s);
+    const dd s = dd_add(dd{s0, 0.0}, dd_div(dd_add(d, dd_neg(s0sq)), dd{2.0 * s0, 0.0}));
+    L[gram_idx(j, j)] = s;
+    inv[j] = dd_div(dd{1.0, 0.0}, s);
+#pragma unroll
+    for (int i = j + 1; i < 5; ++i) {
+      dd v = L[gram_idx(i, j)];
+#pragma unroll
+      for (int m = 0; m < j; ++m) v = dd_add(v, dd_neg(dd_mul(L[gram_idx(i, m)], L[gram_idx(j, m)])));
+      L[gram_idx(i, j)] = dd_mul(v, inv[j]);
     }
   }
   dd z[5], a[5];
-  for (int i = 0; i < kc; ++i) {
+#pragma unroll
+  for (int i = 0; i < 5; ++i) {
     dd v = r[i];
-    for (int m = 0; m < i; ++m) v = dd_add(v, dd_neg(dd_mul(G[i][m], z[m])));
-    z[i] = dd_div(v, G[i][i]);
+#pragma unroll
+    for (int m = 0; m < i; ++m) v = dd_add(v, dd_neg(dd_mul(L[gram_idx(i, m)], z[m])));
+    z[i] = dd_mul(v, inv[i]);
   }
-  for (int i = kc - 1; i >= 0; --i) {
+#pragma unroll
+  for (int i = 4; i >= 0; --i) {
     dd v = z[i];
-    for (int m = i + 1; m < kc; ++m) v = dd_add(v, dd_neg(dd_mul(G[m][i], a[m])));
-    a[i] = dd_div(v, G[i][i]);
+#pragma unroll
+    for (int m = i + 1; m < 5; ++m) v = dd_add(v, dd_neg(dd_mul(L[gram_idx(m, i)], a[m])));
+    a[i] = dd_mul(v, inv[i]);
   }
-  for (int i = 0; i < kc; ++i) o.coef[cols[i]] = ldexp(a[i].hi + a[i].lo, sc[i]);
+#pragma unroll
+  for (int i = 0; i < 5; ++i) o.coef[i] = (drop3 && i == 3) ? 0.0 : ldexp(a[i].hi + a[i].lo, sc[i]);
   // residuals of the rounded coefficients: SSR = y'y - 2 c'X'y + c'Gc (unscaled)
-  dd cxy{0.0, 0.0}, cgc{0.0, 0.0}, sy = int256_to_dd(T[15 + k * 5 + 0].w, kFitYLsb);
-  for (int i = 0; i < kc; ++i) {
-    const dd ci{o.coef[cols[i]], 0.0};
-    cxy = dd_add(cxy, dd_mul(ci, int256_to_dd(T[15 + k * 5 + cols[i]].w, kFitYLsb)));
-    for (int j = 0; j < kc; ++j)
-      cgc = dd_add(cgc, dd_mul(dd_mul(ci, dd{o.coef[cols[j]], 0.0}), int256_to_dd(T[gidx(cols[i], cols[j])].w, 0)));
+  dd cxy{0.0, 0.0}, cgc{0.0, 0.0};
+#pragma unroll
+  for (int i = 0; i < 5; ++i) {
+    const dd ci{o.coef[i], 0.0};
+    cxy = dd_add(cxy, dd_mul(ci, ru[i]));
+#pragma unroll
+    for (int j = 0; j < 5; ++j) cgc = dd_add(cgc, dd_mul(dd_mul(ci, dd{o.coef[j], 0.0}), Gu[gram_idx(i, j)]));
   }
+  const dd sy = ru[0];
   const dd yy = int256_to_dd(T[15 + 5 * n_y + k].w, kFitYYLsb);
   const dd ssr = dd_add(dd_add(yy, dd_neg(dd_scale(cxy, 1))), cgc);
   const dd sst = dd_add(yy, dd_neg(dd_div(dd_mul(sy, sy), dd{(double)n, 0.0})));
