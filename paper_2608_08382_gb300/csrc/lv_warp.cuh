@@ -442,20 +442,111 @@ __device__ __forceinline__ void small_rounds(const TileArgs &a, const WSmem &ws,
   }
 }
 
-// Fit statistics of the group's batches into this warp's accumulators: lane e
-// owns entries e, e+32, ... of [4 groups][NE].
-__device__ __forceinline__ void fit_group(const TileArgs &a, FitAcc *fw, int64_t g0, int ng, const Sums &mys,
-                                          int64_t n, int fseg, int lane, int *bad) {
-  const int NE = fit_entries(a.fit.n_y);
-  for (int j = 0; j < ng; ++j) {
-    const int sj = __shfl_sync(kFull, fseg, j);
-    if (sj < 0) continue;  // empty, jumbo or out of range
-    const int64_t nj = __shfl_sync(kFull, n, j);
-    const int64_t xx[5] = {1, __shfl_sync(kFull, mys.s1, j), __shfl_sync(kFull, mys.s2, j),
-                           __shfl_sync(kFull, mys.s3, j), nj * nj};
-    for (int t = lane; t < 4 * NE; t += 32) {
-      if (t / NE != sj) continue;
-      fit_owner_add(fw[t], t % NE, a.fit.n_y, xx, a.fit.y, a.n_batch, g0 + j, xx[1] != xx[3], bad);
+// Fit statistics of the group's batches into this warp's accumulators
+// fw[group][entry].  Every lane converts its own batch's latencies to fixed
+// point once (Y = y * 2^100 and floor(Y^2 / 2^64)); then, for each batch of
+// segment g in turn, lane e adds that batch's contribution to entry e of
+// group g (and e + 32 when a group has more than 32 entries), the batch's sums
+// and Y values arriving by shuffle.  Entry order: 15 Gram pairs (a <= b, row
+// order), 5 X^T y columns per y vector, one y'y per y vector, one flag.
+__device__ __forceinline__ int64_t fit_x(int i, int64_t s1, int64_t s2, int64_t s3, int64_t n2) {
+  return i == 0 ? 1 : i == 1 ? s1 : i == 2 ? s2 : i == 3 ? s3 : n2;
+}
+
+__device__ __forceinline__ void fit_entry_add(FitAcc &acc, int e, int n_y, int64_t s1, int64_t s2, int64_t s3,
+                                              int64_t n2, const i128 *Y, const uint64_t (*YY)[3]) {
+  if (e < 15) {
+    int a = 0, r = e;
+    while (r >= 5 - a) {
+      r -= 5 - a;
+      ++a;
+    }
+    const uint64_t u = (uint64_t)fit_x(a, s1, s2, s3, n2), v = (uint64_t)fit_x(a + r, s1, s2, s3, n2);
+    acc_add256(acc.w, u * v, __umul64hi(u, v), 0, 0);
+  } else if (e < 15 + 5 * n_y) {
+    const int col = (e - 15) % 5, kk = (e - 15) / 5;
+    i128 y = Y[0];
+#pragma unroll
+    for (int q = 1; q < kFitMaxY; ++q)
+      if (kk == q) y = Y[q];
+    const bool neg = is_neg128(y);
+    const i128 M = neg ? neg128(y) : y;
+    const uint64_t xv = (uint64_t)fit_x(col, s1, s2, s3, n2);
+    const uint64_t p0 = M.lo * xv, p1 = __umul64hi(M.lo, xv);
+    const uint64_t q0 = M.hi * xv, q1 = __umul64hi(M.hi, xv);
+    uint64_t w0 = p0, w1 = p1 + q0, w2 = q1 + (w1 < p1 ? 1ull : 0ull), w3 = 0;
+    if (neg) {
+      w0 = ~w0 + 1;
+      w1 = ~w1 + (w0 == 0 ? 1ull : 0ull);
+      w2 = ~w2 + ((w0 | w1) == 0 ? 1ull : 0ull);
+      w3 = ~w3 + ((w0 | w1 | w2) == 0 ? 1ull : 0ull);
+    }
+    acc_add256(acc.w, w0, w1, w2, w3);
+  } else if (e < 15 + 6 * n_y) {
+    const int kk = e - 15 - 5 * n_y;
+    uint64_t a0 = YY[0][0], a1 = YY[0][1], a2 = YY[0][2];
+#pragma unroll
+    for (int q = 1; q < kFitMaxY; ++q)
+      if (kk == q) {
+        a0 = YY[q][0];
+        a1 = YY[q][1];
+        a2 = YY[q][2];
+      }
+    acc_add256(acc.w, a0, a1, a2, 0);
+  } else {
+    if (s1 != s3) acc.w[0] |= 1ull;
+  }
+}
+
+__device__ __forceinline__ void fit_group(const TileArgs &a, FitAcc *fw, int64_t g0, const Sums &mys, int64_t n,
+                                          int fseg, int lane, int *bad) {
+  const int NE = fit_entries(a.fit.n_y), n_y = a.fit.n_y;
+  // this lane's batch: latencies in fixed point
+  i128 Ym[kFitMaxY];
+  uint64_t YYm[kFitMaxY][3];
+#pragma unroll
+  for (int q = 0; q < kFitMaxY; ++q) {
+    Ym[q] = mk128(0, 0);
+    YYm[q][0] = YYm[q][1] = YYm[q][2] = 0;
+    if (q < n_y && fseg >= 0) {
+      bool ovf = false;
+      i128 Y = y_fixed(a.fit.y[q * a.n_batch + g0 + lane], &ovf);
+      if (ovf) *bad = 1;
+      Ym[q] = Y;
+      if (is_neg128(Y)) Y = neg128(Y);
+      const uint64_t l = Y.lo, h = Y.hi;
+      uint64_t w[4] = {__umul64hi(l, l), h * h, __umul64hi(h, h), 0};
+      acc_add256(w, h * l, __umul64hi(h, l), 0, 0);
+      acc_add256(w, h * l, __umul64hi(h, l), 0, 0);
+      YYm[q][0] = w[0];
+      YYm[q][1] = w[1];
+      YYm[q][2] = w[2];
+    }
+  }
+  const int64_t n2 = n * n;
+#pragma unroll 1
+  for (int g = 0; g < 4; ++g) {
+    uint32_t m = __ballot_sync(kFull, fseg == g);
+    while (m) {
+      const int j = __ffs(m) - 1;
+      m &= m - 1;
+      const int64_t s1 = __shfl_sync(kFull, mys.s1, j), s2 = __shfl_sync(kFull, mys.s2, j),
+                    s3 = __shfl_sync(kFull, mys.s3, j), nn = __shfl_sync(kFull, n2, j);
+      i128 Y[kFitMaxY];
+      uint64_t YY[kFitMaxY][3];
+#pragma unroll
+      for (int q = 0; q < kFitMaxY; ++q) {
+        if (q < n_y) {
+          Y[q] = mk128(__shfl_sync(kFull, Ym[q].lo, j), __shfl_sync(kFull, Ym[q].hi, j));
+          YY[q][0] = __shfl_sync(kFull, YYm[q][0], j);
+          YY[q][1] = __shfl_sync(kFull, YYm[q][1], j);
+          YY[q][2] = __shfl_sync(kFull, YYm[q][2], j);
+        } else {
+          Y[q] = mk128(0, 0);
+          YY[q][0] = YY[q][1] = YY[q][2] = 0;
+        }
+      }
+      for (int e = lane; e < NE; e += 32) fit_entry_add(fw[g * NE + e], e, n_y, s1, s2, s3, nn, Y, YY);
     }
   }
 }
@@ -553,7 +644,7 @@ __device__ __forceinline__ void process_group(const TileArgs &a, const WSmem &ws
       if (n > 0 && in_range) fseg = s;
     }
   }
-  if (MODE & M_FIT) fit_group(a, fw, g0, ng, mys, n, fseg, lane, bad);
+  if (MODE & M_FIT) fit_group(a, fw, g0, mys, n, fseg, lane, bad);
 }
 
 // Shared-memory tables of a CTA: per-segment share parameters and, in

@@ -16,6 +16,7 @@
 #pragma once
 
 #include "lv_kernels.cuh"
+#include "lv_warp.cuh"
 
 namespace lv {
 
@@ -97,6 +98,18 @@ __global__ void k_wi_pend(ModelP mp, const int32_t *__restrict__ p_new, const in
   out[j] = q;
 }
 
+// V * 2^E rounded to double: the leading-word rounding for the common
+// magnitude 2^64 <= V < 2^96, the general rounding otherwise.
+__device__ __forceinline__ double round_fix(i128 V, int E) {
+  const uint32_t v3 = (uint32_t)(V.hi >> 32), v2 = (uint32_t)V.hi;
+  if (v3 == 0u && v2 != 0u) {
+    uint64_t m;
+    int ex2;
+    return round96((uint32_t)V.lo, (uint32_t)(V.lo >> 32), v2, E, m, ex2);
+  }
+  return fix_to_double(V, E).d;
+}
+
 // Left-to-right fp64 evaluation of one pair (fp64 mode, or outside the exact range).
 __device__ __noinline__ void wi_pair_slow(const ModelP &mp, int s, int64_t s1, int64_t s2, int64_t s3, int64_t n1,
                                           int32_t p, int32_t c, double *T, double *share) {
@@ -140,8 +153,8 @@ __global__ void __launch_bounds__(kWiCols) k_wi_pairs(ModelP mp, const CandP *__
       wi_pair_slow(mp, s, s1 + p, s2 + c, s3 + (int64_t)p * p, n1, p, c, &T, &sh);
     } else {
       const i128 V = sp[r].V[s];
-      T = fix_to_double(add128(cb->U[s], V), sE[s]).d;
-      sh = fix_to_double(add128(cb->W[s], V), sE[s]).d;
+      T = round_fix(add128(cb->U[s], V), sE[s]);
+      sh = round_fix(add128(cb->W[s], V), sE[s]);
     }
     const int64_t o = (j0 + r) * nc + b;
     if (T_new) __stcs(T_new + o, T);
