@@ -248,7 +248,7 @@ lv_status timing_end(cudaEvent_t stop, cudaStream_t stream) {
 // Dynamic shared memory of k_warps for a tenant table of H entries and n_y fit vectors.
 template <int MODE>
 size_t warps_smem(int H, int n_y) {
-  return sizeof(WSmem) + ((MODE & M_TEN) ? 16 * (size_t)H : 0) +
+  return sizeof(WSmem) + ((MODE & M_TEN) ? ten_bytes(H) : 0) +
          ((MODE & M_FIT) ? (size_t)kWarps * 4 * fit_entries(n_y) * sizeof(FitAcc) : 0) +
          ((MODE & M_ATTR) ? (size_t)kWarps * sizeof(DeferList) : 0);
 }
@@ -265,7 +265,7 @@ template <int MODE>
 lv_status launch_warps_mode(lv_ctx *ctx, int sms, TileArgs &a, cudaStream_t stream, int64_t *ctas) {
   *ctas = 0;
   const size_t smem = warps_smem<MODE>(a.H, a.fit.n_y);
-  const size_t jsmem = sizeof(JSmem) + ((MODE & M_TEN) ? 16 * (size_t)a.H : 0);
+  const size_t jsmem = sizeof(JSmem) + ((MODE & M_TEN) ? ten_bytes(a.H) : 0);
   const uint64_t key = ((uint64_t)MODE << 32) | smem;
   int per_sm = 0;
   if (ctx) {
@@ -277,7 +277,7 @@ lv_status launch_warps_mode(lv_ctx *ctx, int sms, TileArgs &a, cudaStream_t stre
     LV_CUDA(cudaFuncSetAttribute(k_warps<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)warps_smem<MODE>(kHotMax, kFitMaxY)));
     LV_CUDA(cudaFuncSetAttribute(k_jumbo<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)(sizeof(JSmem) + 16 * (size_t)kHotMax)));
+                                 (int)(sizeof(JSmem) + ten_bytes(kHotMax))));
     LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_warps<MODE>, kWThreads, smem));
     if (per_sm < 1) per_sm = 1;
     if (ctx) ctx->occ.emplace_back(key, per_sm);
@@ -637,11 +637,11 @@ lv_status lv_tenant_accumulate(lv_ctx *ctx, lv_tenant_acc *acc, const double *sh
   cudaStream_t stream = (cudaStream_t)stream_;
   if (n_req > 0) {
     const int H = std::min<int32_t>(acc->n_tenants, kHotMax);
-    const size_t smem = sizeof(uint32_t) * 4 * (size_t)H;
+    const size_t smem = ten_bytes(H);
     static bool configured = false;
     if (!configured) {
       LV_CUDA(cudaFuncSetAttribute(k_tenant_acc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                   (int)(sizeof(uint32_t) * 4 * kHotMax)));
+                                   (int)ten_bytes(kHotMax)));
       configured = true;
     }
     const int64_t blocks = std::min<int64_t>((n_req + kBlock - 1) / kBlock, (int64_t)ctx->sms * 4);

@@ -395,30 +395,27 @@ __device__ __forceinline__ void pend_add(unsigned long long *pend, int64_t u, i1
   if (l3) atomicAdd(w + 3, (unsigned long long)l3);
 }
 
-// Exact q into the 128-bit integer held as four 32-bit shared-memory words.
-// Each word's atomic returns its old value, so the thread whose addition
-// wraps a word is the one that carries into the next: the multi-word sum stays
-// exact (mod 2^128) under any interleaving.
-__device__ __forceinline__ void hot_add(uint32_t *w, i128 q) {
-  if (q.hi == 0) {
-    const uint32_t lo = (uint32_t)q.lo, hi = (uint32_t)(q.lo >> 32);
-    uint32_t c = 0;
-    if (lo) {
-      const uint32_t o = atomicAdd(w, lo);
-      c = (o + lo < o) ? 1u : 0u;
-    }
-    const uint32_t add1 = hi + c;
-    uint32_t c1 = (add1 < hi) ? 1u : 0u;
-    if (add1) {
-      const uint32_t o = atomicAdd(w + 1, add1);
-      c1 |= (o + add1 < o) ? 1u : 0u;
-    }
-    if (c1) {
-      const uint32_t o = atomicAdd(w + 2, 1u);
-      if (o == 0xffffffffu) atomicAdd(w + 3, 1u);
-    }
-    return;
-  }
+// Shared-memory tenant table.  Each hot tenant has kTenRep replicas of a
+// 128-bit integer held as four 32-bit words; a thread adds into replica
+// (threadIdx.x & (kTenRep - 1)), which divides same-tenant conflicts within a
+// warp.  Word k of replica r of tenant u is tt[k * plane + r * stride + u]:
+// consecutive tenants fall in consecutive banks and, the stride being 8 mod
+// 32 words, one tenant's replicas fall in different banks.
+constexpr int kTenRep = 4;
+__host__ __device__ constexpr int ten_stride(int H) { return ((H + 31) & ~31) + 8; }
+__host__ __device__ constexpr int ten_plane(int H) { return kTenRep * ten_stride(H); }
+__host__ __device__ constexpr size_t ten_bytes(int H) { return 4 * sizeof(uint32_t) * (size_t)ten_plane(H); }
+
+// Word 0 of this thread's replica of tenant u (word k is k * ten_plane(H) further).
+__device__ __forceinline__ uint32_t *ten_word0(uint32_t *tt, int H, int u) {
+  return tt + (threadIdx.x & (kTenRep - 1)) * ten_stride(H) + u;
+}
+
+// Exact q into the 128-bit integer whose word k is w[k * plane].  Each word's
+// atomic returns its old value, so the thread whose addition wraps a word is
+// the one that carries into the next: the multi-word sum stays exact (mod
+// 2^128) under any interleaving.
+__device__ __forceinline__ void hot_add(uint32_t *w, int plane, i128 q) {
   const uint32_t v[4] = {(uint32_t)q.lo, (uint32_t)(q.lo >> 32), (uint32_t)q.hi, (uint32_t)(q.hi >> 32)};
   uint32_t c = 0;
 #pragma unroll
@@ -426,15 +423,23 @@ __device__ __forceinline__ void hot_add(uint32_t *w, i128 q) {
     const uint32_t add = v[k] + c;
     uint32_t cc = (add < v[k]) ? 1u : 0u;
     if (add) {
-      const uint32_t o = atomicAdd(w + k, add);
+      const uint32_t o = atomicAdd(w + k * plane, add);
       cc |= (o + add < o) ? 1u : 0u;
     }
     c = cc;
   }
 }
 
-__device__ __forceinline__ i128 hot_value(const uint32_t *w) {
-  return mk128((uint64_t)w[0] | ((uint64_t)w[1] << 32), (uint64_t)w[2] | ((uint64_t)w[3] << 32));
+// Tenant u's total over the replicas (mod 2^128).
+__device__ __forceinline__ i128 hot_value(const uint32_t *tt, int H, int u) {
+  const int S = ten_stride(H), P = ten_plane(H);
+  i128 v = mk128(0, 0);
+#pragma unroll
+  for (int r = 0; r < kTenRep; ++r) {
+    const uint32_t *w = tt + r * S + u;
+    v = add128(v, mk128((uint64_t)w[0] | ((uint64_t)w[P] << 32), (uint64_t)w[2 * P] | ((uint64_t)w[3 * P] << 32)));
+  }
+  return v;
 }
 
 // ---------------------------------------------------------------- per-batch and per-request steps
@@ -488,7 +493,7 @@ __device__ __forceinline__ void tenant_add(const TileArgs &a, uint32_t *tt, int3
   const i128 q = share_to_tenant_fix(r, bad);
   if ((q.lo | q.hi) == 0) return;
   if (u < a.H)
-    hot_add(tt + 4 * u, q);
+    hot_add(ten_word0(tt, a.H, u), ten_plane(a.H), q);
   else
     pend_add(a.ten_pend, u, q);
 }
@@ -546,7 +551,7 @@ __global__ void __launch_bounds__(kBlock) k_tenant_acc(const double *__restrict_
                                                         int *status) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   uint32_t *tt = reinterpret_cast<uint32_t *>(smem_raw);
-  for (int i = threadIdx.x; i < 4 * H; i += kBlock) tt[i] = 0;
+  for (int i = threadIdx.x; i < 4 * ten_plane(H); i += kBlock) tt[i] = 0;
   __syncthreads();
   int bad = 0;
   TileArgs a{};
@@ -560,7 +565,7 @@ __global__ void __launch_bounds__(kBlock) k_tenant_acc(const double *__restrict_
   if (bad) flag(status, kStatusData);
   __syncthreads();
   for (int u = threadIdx.x; u < H; u += kBlock) {
-    const i128 v = hot_value(tt + 4 * u);
+    const i128 v = hot_value(tt, H, u);
     if (v.lo | v.hi) pend_add(pend, u, v);
   }
 }

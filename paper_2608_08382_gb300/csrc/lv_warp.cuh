@@ -142,6 +142,20 @@ __device__ __forceinline__ double round96(uint32_t v0, uint32_t v1, uint32_t v2,
 // cold tenants: 32-bit limbs into the global 64-bit pending counters.
 __device__ __forceinline__ bool tenant_fast(const TileArgs &a, uint32_t *tt, int32_t u, uint64_t m, int ex2) {
   const int sh = ex2 - kTenLsb;
+  if ((unsigned)sh <= 10u && (unsigned)u < (unsigned)a.H) {
+    // the common case: q = m 2^sh <= 2^63, two words
+    const uint64_t q = m << sh;
+    uint32_t *w = ten_word0(tt, a.H, u);
+    const int P = ten_plane(a.H);
+    const uint32_t lo = (uint32_t)q, hi = (uint32_t)(q >> 32);
+    const uint32_t o0 = atomicAdd(w, lo);
+    const uint32_t a1 = hi + ((o0 + lo < o0) ? 1u : 0u);  // hi <= 2^31: no wrap
+    const uint32_t o1 = atomicAdd(w + P, a1);
+    if (o1 + a1 < o1) {
+      if (atomicAdd(w + 2 * P, 1u) == 0xffffffffu) atomicAdd(w + 3 * P, 1u);
+    }
+    return true;
+  }
   if ((unsigned)sh > 42u || (unsigned)u >= (unsigned)a.n_tenants) return false;
   const uint32_t ml = (uint32_t)m, mh = (uint32_t)(m >> 32);
   const bool lowp = sh < 32;
@@ -149,13 +163,14 @@ __device__ __forceinline__ bool tenant_fast(const TileArgs &a, uint32_t *tt, int
   const uint32_t x0 = ml << t, x1 = __funnelshift_l(ml, mh, t), x2 = t ? mh >> (32 - t) : 0u;
   const uint32_t q0 = lowp ? x0 : 0u, q1 = lowp ? x1 : x0, q2 = lowp ? x2 : x1;
   if (u < a.H) {
-    uint32_t *w = tt + 4 * u;
+    uint32_t *w = ten_word0(tt, a.H, u);
+    const int P = ten_plane(a.H);
     const uint32_t o0 = atomicAdd(w, q0);
     const uint32_t a1 = q1 + ((o0 + q0 < o0) ? 1u : 0u);
-    const uint32_t o1 = atomicAdd(w + 1, a1);
+    const uint32_t o1 = atomicAdd(w + P, a1);
     const uint32_t a2 = q2 + (((o1 + a1 < o1) || a1 < q1) ? 1u : 0u);  // q2 < 2^22: no wrap
     if (a2) {
-      if (atomicAdd(w + 2, a2) + a2 < a2) atomicAdd(w + 3, 1u);
+      if (atomicAdd(w + 2 * P, a2) + a2 < a2) atomicAdd(w + 3 * P, 1u);
     }
   } else {
     unsigned long long *pw = a.ten_pend + 4 * (int64_t)u;
@@ -672,15 +687,15 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
   uint32_t *tt = reinterpret_cast<uint32_t *>(smem_raw + sizeof(WSmem));
   constexpr bool kTen = (MODE & M_TEN) != 0;
   constexpr bool kFit = (MODE & M_FIT) != 0;
-  FitAcc *facc = reinterpret_cast<FitAcc *>(smem_raw + sizeof(WSmem) + (kTen ? 16 * (size_t)a.H : 0));
-  DeferList *dlists = reinterpret_cast<DeferList *>(smem_raw + sizeof(WSmem) + (kTen ? 16 * (size_t)a.H : 0) +
+  FitAcc *facc = reinterpret_cast<FitAcc *>(smem_raw + sizeof(WSmem) + (kTen ? ten_bytes(a.H) : 0));
+  DeferList *dlists = reinterpret_cast<DeferList *>(smem_raw + sizeof(WSmem) + (kTen ? ten_bytes(a.H) : 0) +
                                                     (kFit ? (size_t)kWarps * 4 * fit_entries(a.fit.n_y) * sizeof(FitAcc) : 0));
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
   const int NE4 = kFit ? 4 * fit_entries(a.fit.n_y) : 0;
   int bad = 0;
 
   if (kTen)
-    for (int i = tid; i < 4 * a.H; i += kWThreads) tt[i] = 0;
+    for (int i = tid; i < 4 * ten_plane(a.H); i += kWThreads) tt[i] = 0;
   if (kFit)
     for (int i = tid; i < kWarps * NE4; i += kWThreads) facc[i] = FitAcc{{0, 0, 0, 0}};
   if (MODE & M_ATTR) {
@@ -729,7 +744,7 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
   if (kTen || kFit) __syncthreads();
   if (kTen) {
     for (int u = tid; u < a.H; u += kWThreads) {
-      const i128 v = hot_value(tt + 4 * u);
+      const i128 v = hot_value(tt, a.H, u);
       if (v.lo | v.hi) pend_add(a.ten_pend, u, v);
     }
   }
@@ -763,7 +778,7 @@ __global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_bas
   int bad = 0;
   FitAcc facc{{0, 0, 0, 0}};
   if (kTen)
-    for (int i = tid; i < 4 * a.H; i += kJBlock) tt[i] = 0;
+    for (int i = tid; i < 4 * ten_plane(a.H); i += kJBlock) tt[i] = 0;
   if (MODE & M_ATTR) init_segs<MODE>(a, js.seg);
   __syncthreads();
 
@@ -824,7 +839,7 @@ __global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_bas
   if (kTen) {
     __syncthreads();
     for (int u = tid; u < a.H; u += kJBlock) {
-      const i128 v = hot_value(tt + 4 * u);
+      const i128 v = hot_value(tt, a.H, u);
       if (v.lo | v.hi) pend_add(a.ten_pend, u, v);
     }
   }
