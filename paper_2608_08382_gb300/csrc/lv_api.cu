@@ -321,7 +321,11 @@ int64_t jumbo_bound(int64_t n_req) { return n_req / (kJumbo + 1) + 1; }
 lv_status run_tiles(lv_ctx *ctx, TileArgs &a, int mode, cudaStream_t stream) {
   ctx->last_grid = 0;
   const int64_t units = a.n_batch + a.n_req;
-  a.n_tiles = (units + kDW - 1) / kDW;
+  // larger tiles fill the per-lane batch groups better; keep at least six tiles
+  // per resident warp for the dynamic schedule's tail
+  const int64_t warps = (int64_t)ctx->sms * (2048 / kWThreads) * kWarps;
+  a.D = units / (2 * kDW) >= 6 * warps ? 2 * kDW : kDW;
+  a.n_tiles = (units + a.D - 1) / a.D;
   if (a.n_batch == 0) return LV_OK;
   lv_status st = ensure_tiles(ctx, a.n_tiles + 1);
   if (st != LV_OK) return st;
@@ -335,7 +339,7 @@ lv_status run_tiles(lv_ctx *ctx, TileArgs &a, int mode, cudaStream_t stream) {
   LV_CUDA(cudaMemsetAsync(ctx->d_ctr, 0, 2 * sizeof(unsigned long long), stream));
   const int64_t nthreads = a.n_batch + 1;
   const int64_t pblocks = std::min<int64_t>((nthreads + 255) / 256, (int64_t)ctx->sms * 16);
-  k_partition<<<(unsigned)pblocks, 256, 0, stream>>>(a.off, a.n_batch, a.n_req, a.n_tiles, kDW, ctx->d_tiles,
+  k_partition<<<(unsigned)pblocks, 256, 0, stream>>>(a.off, a.n_batch, a.n_req, a.n_tiles, a.D, ctx->d_tiles,
                                                      ctx->d_status);
   LV_CUDA(cudaGetLastError());
   int64_t *g = &ctx->last_grid;
@@ -938,6 +942,7 @@ extern "C" lv_status lv_attribute_noalloc(const lv_model *model, const lv_batche
   a.status = status;
   a.mp = mp;
   a.n_tiles = n_tiles;
+  a.D = kDW;
   unsigned char *base = static_cast<unsigned char *>(scratch);
   TilePart *part = reinterpret_cast<TilePart *>(base);
   a.part = part;

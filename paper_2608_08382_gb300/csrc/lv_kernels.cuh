@@ -163,6 +163,7 @@ struct TileArgs {
   int64_t n_req, n_batch;
   const TilePart *part;  // [n_tiles + 1]
   int64_t n_tiles;
+  int64_t D;             // merge positions per tile
   double *T, *share;
   int64_t *bfeat;   // [5][n_batch] or null
   uint8_t *bseg;    // [n_batch] or null

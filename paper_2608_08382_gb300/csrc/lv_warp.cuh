@@ -30,7 +30,7 @@ namespace lv {
 
 constexpr int kWarps = 16;                 // warps per CTA of k_warps
 constexpr int kWThreads = 32 * kWarps;
-constexpr int kDW = 1024;                  // merge positions per warp tile
+constexpr int kDW = 1024;                  // merge positions per warp tile (large inputs: 2 kDW)
 constexpr int kJumbo = 512;                // larger batches are attributed by k_jumbo
 constexpr int kBig = 32;                   // batches with at least this many requests are processed warp-strided
 constexpr int kJBlock = 512;               // threads per CTA of k_jumbo
@@ -728,8 +728,8 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
     if (lane == 0) tn = atomicAdd(a.ctr, 1ull);  // next tile, fetched early
     const int64_t b0 = clampi(a.part[t].b, 0, a.n_batch);
     int64_t b1 = clampi(a.part[t + 1].b, b0, a.n_batch);
-    if (b1 - b0 > kDW) {
-      b1 = b0 + kDW;
+    if (b1 - b0 > a.D) {
+      b1 = b0 + a.D;
       bad = 1;
     }
     for (int64_t g0 = b0; g0 < b1; g0 += 32)
