@@ -28,6 +28,8 @@ struct SegFix {
   uint64_t lim[4];   // exact T path valid when S1, S2, S3, n^2 <= lim[0..3]
   int E;
   int a2_narrow;     // 1: 0 <= A2 < 2^64 (64-bit multiply suffices)
+  int t_narrow;      // 1: B, A1..A4 all in [0, 2^64) (eq1_fast applies)
+  int pad;
 };
 
 struct KEntry {
@@ -274,6 +276,30 @@ __device__ __noinline__ double eq1_fix(const ModelP &mp, int s, const BatchAgg &
   return fix_to_double(V, f.E).d;
 }
 
+// Eq. 1 in fixed point for the common case: every coefficient in [0, 2^64)
+// (t_narrow), each product below 2^96 and the sum in [2^64, 2^96); four
+// 64x64-bit products and the leading-word rounding.  False when any of these
+// does not hold (the caller then takes eq1_fix).
+__device__ __forceinline__ bool eq1_fast(const SegFix &f, const BatchAgg &g, double *T) {
+  if (!f.t_narrow || g.n == 0 || g.n > 0x7fffffffll) return false;
+  uint64_t lo = f.B.lo, hi = 0;
+  bool ok = true;
+  const uint64_t A[4] = {f.A1.lo, f.A2.lo, f.A3.lo, f.A4.lo};
+  const uint64_t S[4] = {(uint64_t)g.s1, (uint64_t)g.s2, (uint64_t)g.s3, (uint64_t)g.n * (uint64_t)g.n};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint64_t pl = A[i] * S[i], ph = __umul64hi(A[i], S[i]);
+    ok &= ph < (1ull << 32);  // product below 2^96: the sum of five stays below 2^99
+    lo += pl;
+    hi += ph + (lo < pl ? 1ull : 0ull);
+  }
+  if (!ok || hi == 0 || hi >= (1ull << 32)) return false;
+  uint64_t m;
+  int ex2;
+  *T = round96((uint32_t)lo, (uint32_t)(lo >> 32), (uint32_t)hi, f.E, m, ex2);
+  return true;
+}
+
 // Per-batch share constant: q = fl(beta/n), a4n = fl(a4*n), kf = fix(fl(q+a4n)).
 __device__ __forceinline__ KEntry batch_k(const ModelP &mp, int s, int64_t n, bool *slow) {
   if (n >= 1 && n <= mp.nk) {
@@ -398,11 +424,12 @@ __device__ __forceinline__ void pend_add(unsigned long long *pend, int64_t u, i1
 
 // Shared-memory tenant table.  Each hot tenant has kTenRep replicas of a
 // 128-bit integer held as four 32-bit words; a thread adds into replica
-// (threadIdx.x & (kTenRep - 1)), which divides same-tenant conflicts within a
-// warp.  Word k of replica r of tenant u is tt[k * plane + r * stride + u]:
-// consecutive tenants fall in consecutive banks and, the stride being 8 mod
-// 32 words, one tenant's replicas fall in different banks.
-constexpr int kTenRep = 4;
+// (threadIdx.x & (kTenRep - 1)).  Word k of replica r of tenant u is
+// tt[k * plane + r * stride + u]: consecutive tenants fall in consecutive
+// banks and, the stride being 8 mod 32 words, one tenant's replicas would fall
+// in different banks.  One replica measured fastest on the Zipf workloads (more
+// divide same-tenant conflicts but cost shared memory and flush work).
+constexpr int kTenRep = 1;
 __host__ __device__ constexpr int ten_stride(int H) { return ((H + 31) & ~31) + 8; }
 __host__ __device__ constexpr int ten_plane(int H) { return kTenRep * ten_stride(H); }
 __host__ __device__ constexpr size_t ten_bytes(int H) { return 4 * sizeof(uint32_t) * (size_t)ten_plane(H); }
@@ -476,7 +503,12 @@ __device__ __forceinline__ void emit_batch(const TileArgs &a, int64_t gb, const 
     if (a.bseg) a.bseg[gb] = (uint8_t)s;
   }
   if ((MODE & M_ATTR) && a.T) {
-    a.T[gb] = (MODE & M_FIX) ? eq1_fix(a.mp, s, g) : eq1_fp64(a.mp.coef[s], g);
+    double T;
+    if (!(MODE & M_FIX))
+      T = eq1_fp64(a.mp.coef[s], g);
+    else if (!eq1_fast(a.mp.fx[s], g, &T))
+      T = eq1_fix(a.mp, s, g);
+    a.T[gb] = T;
   }
 }
 

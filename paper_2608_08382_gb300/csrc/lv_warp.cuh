@@ -121,21 +121,6 @@ __device__ __forceinline__ void mad_k13(uint32_t k0, uint32_t k1, uint32_t k2, u
       : "r"(a0), "r"(a1), "r"(c), "r"(k0), "r"(k1), "r"(k2), "r"(k3));
 }
 
-// V * 2^E rounded to the nearest double (ties to even) for the common
-// magnitude 2^64 <= V < 2^96 (v3 = 0, v2 != 0; the caller checks): the
-// leading word is v2.  m is the rounded significand (2^52 <= m <= 2^53) and
-// ex2 its exponent: the result equals m * 2^ex2.
-__device__ __forceinline__ double round96(uint32_t v0, uint32_t v1, uint32_t v2, int E, uint64_t &m, int &ex2) {
-  const int s = __clz(v2);
-  const uint32_t t2 = __funnelshift_l(v1, v2, s), t1 = __funnelshift_l(v0, v1, s), t0 = v0 << s;
-  const uint32_t mhi = t2 >> 11, mlo = __funnelshift_r(t1, t2, 11);
-  const uint32_t inc = ((t1 >> 10) & 1u) & ((((t1 & 0x3ffu) | t0) != 0u ? 1u : 0u) | (mlo & 1u));
-  m = (((uint64_t)mhi << 32) | mlo) + inc;
-  const int ex = 95 - s + E;  // exponent of the leading bit
-  ex2 = ex - 52;
-  return __longlong_as_double((long long)(((uint64_t)(ex + 1022) << 52) + m));
-}
-
 // Tenant contribution of a share m * 2^ex2 (m <= 2^53) when q = m 2^(ex2+72)
 // has at most three 32-bit words and the tenant id is valid; false otherwise
 // (nothing is added then).  Hot tenants: exact multi-word add in shared memory;
