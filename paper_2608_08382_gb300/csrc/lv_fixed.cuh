@@ -146,12 +146,15 @@ __device__ __forceinline__ Rounded fix_to_double_pos(i128 V, int E) {
 __device__ __forceinline__ double round96(uint32_t v0, uint32_t v1, uint32_t v2, int E, uint64_t &m, int &ex2) {
   const int s = __clz(v2);
   const uint32_t t2 = __funnelshift_l(v1, v2, s), t1 = __funnelshift_l(v0, v1, s), t0 = v0 << s;
-  const uint32_t mhi = t2 >> 11, mlo = __funnelshift_r(t1, t2, 11);
+  uint32_t mhi = t2 >> 11, mlo = __funnelshift_r(t1, t2, 11);
   const uint32_t inc = ((t1 >> 10) & 1u) & ((((t1 & 0x3ffu) | t0) != 0u ? 1u : 0u) | (mlo & 1u));
-  m = (((uint64_t)mhi << 32) | mlo) + inc;
+  mlo += inc;
+  mhi += mlo < inc ? 1u : 0u;
   const int ex = 95 - s + E;  // exponent of the leading bit
+  m = ((uint64_t)mhi << 32) | mlo;
   ex2 = ex - 52;
-  return __longlong_as_double((long long)(((uint64_t)(ex + 1022) << 52) + m));
+  // bits = (ex + 1022) 2^52 + m: m's implicit bit (2^52, or 2^53 after a carry) completes the exponent
+  return __hiloint2double((int)(((uint32_t)(ex + 1022) << 20) + mhi), (int)mlo);
 }
 
 // Exact double -> fixed point at 2^E, rounded to nearest (ties to even) when

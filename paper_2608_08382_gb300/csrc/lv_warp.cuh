@@ -129,10 +129,10 @@ __device__ __forceinline__ bool tenant_fast(const TileArgs &a, uint32_t *tt, int
   const int sh = ex2 - kTenLsb;
   if ((unsigned)sh <= 10u && (unsigned)u < (unsigned)a.H) {
     // the common case: q = m 2^sh <= 2^63, two words
-    const uint64_t q = m << sh;
+    const uint32_t ml = (uint32_t)m, mh = (uint32_t)(m >> 32);
     uint32_t *w = ten_word0(tt, a.H, u);
     const int P = ten_plane(a.H);
-    const uint32_t lo = (uint32_t)q, hi = (uint32_t)(q >> 32);
+    const uint32_t lo = ml << sh, hi = __funnelshift_l(ml, mh, sh);
     const uint32_t o0 = atomicAdd(w, lo);
     const uint32_t a1 = hi + ((o0 + lo < o0) ? 1u : 0u);  // hi <= 2^31: no wrap
     const uint32_t o1 = atomicAdd(w + P, a1);
