@@ -487,7 +487,8 @@ struct SegS {
   i128 A1, A3, A13, A2;
   int E;
   int a2_narrow;
-  int pad[2];
+  int p_narrow;  // 1: 0 <= A1 < 2^95 and 0 <= A3 < 2^64 (prefill constant in 128 bits)
+  int pad;
 };
 
 template <int MODE>

@@ -46,6 +46,7 @@ struct WSmem {
   alignas(16) SegS seg[4];
   alignas(16) uint8_t kslow[4][kNK + 4];  // 1: K outside the fixed-point range
   alignas(16) uint8_t owner[kWarps][32];  // small-batch rounds: head slot -> lane
+  alignas(16) Sums gsum[kWarps][32];      // sums of the group's big batches (kept out of registers)
 };
 static_assert(sizeof(WSmem) % 16 == 0, "tenant table follows WSmem");
 
@@ -81,6 +82,25 @@ __device__ __forceinline__ Sums warp_sum(Sums v) {
   return v;
 }
 
+// Warp sum of per-lane sums over at most 16 requests each (s1, s2 below 2^35,
+// ph at most 16; s3 modulo 2^64, as 64-bit adds take it), from 32-bit warp
+// reductions of 27-bit pieces: 32 of them sum below 2^32.
+__device__ __forceinline__ Sums warp_sum16(const Sums &v) {
+  constexpr uint32_t kM27 = (1u << 27) - 1u;
+  const uint64_t a = (uint64_t)v.s1, b = (uint64_t)v.s2, c = (uint64_t)v.s3;
+  const uint32_t a0 = __reduce_add_sync(kFull, (uint32_t)a & kM27), a1 = __reduce_add_sync(kFull, (uint32_t)(a >> 27));
+  const uint32_t b0 = __reduce_add_sync(kFull, (uint32_t)b & kM27), b1 = __reduce_add_sync(kFull, (uint32_t)(b >> 27));
+  const uint32_t c0 = __reduce_add_sync(kFull, (uint32_t)c & kM27);
+  const uint32_t c1 = __reduce_add_sync(kFull, (uint32_t)(c >> 27) & kM27);
+  const uint32_t c2 = __reduce_add_sync(kFull, (uint32_t)(c >> 54));
+  Sums r;
+  r.s1 = (int64_t)(((uint64_t)a1 << 27) + a0);
+  r.s2 = (int64_t)(((uint64_t)b1 << 27) + b0);
+  r.s3 = (int64_t)(((uint64_t)c2 << 54) + ((uint64_t)c1 << 27) + c0);
+  r.ph = (int32_t)__reduce_add_sync(kFull, (uint32_t)v.ph);
+  return r;
+}
+
 __device__ __forceinline__ int warp_excl_scan_int(int v, int lane) {
   int x = v;
 #pragma unroll
@@ -96,9 +116,11 @@ __device__ __forceinline__ int warp_excl_scan_int(int v, int lane) {
 // A decode request (p = 1) of a batch with constant K has the exact share
 // V = K13 + A2 c with K13 = K + A1 + A3.  When A2 < 2^64 (the segment's
 // a2_narrow) this is one 64x32-bit product and a 128-bit add; the result is
-// rounded to double with 32-bit funnel shifts.  Requests the fast path does not
+// rounded to double with 32-bit funnel shifts.  Requests the fast loops do not
 // cover (p != 1, V outside [2^64, 2^96), a tenant contribution outside the
-// three-word range) are left to general_one, which is exact for every case.
+// three-word range) are left to defer_one, 32 at a time: it takes the same
+// steps with K + p (A1 + A3 p) in place of K13 (prefill_const) where that is
+// exact, and the general path, exact for every case, otherwise.
 
 // v = k + (a1:a0) * c, four 32-bit words, exact (the sum stays below 2^128).
 __device__ __forceinline__ void mad_k13(uint32_t k0, uint32_t k1, uint32_t k2, uint32_t k3, uint32_t a0, uint32_t a1,
@@ -119,6 +141,20 @@ __device__ __forceinline__ void mad_k13(uint32_t k0, uint32_t k1, uint32_t k2, u
       "}"
       : "=r"(v0), "=r"(v1), "=r"(v2), "=r"(v3)
       : "r"(a0), "r"(a1), "r"(c), "r"(k0), "r"(k1), "r"(k2), "r"(k3));
+}
+
+// Constant part of a prefill request's share, kf + p (A1 + A3 p), for a
+// segment with p_narrow and p <= 2^24: A1 + A3 p < 2^96 and its product with p
+// stays below 2^120, so the 128-bit sum is exact whenever the share itself is
+// below 2^128 (which the caller's V < 2^96 test then confirms).
+__device__ __forceinline__ void prefill_const(const SegS &sg, i128 kf, uint32_t p, uint32_t &b0, uint32_t &b1,
+                                              uint32_t &b2, uint32_t &b3) {
+  const i128 r = add128(sg.A1, mul_u64_u32(sg.A3.lo, p));
+  const i128 b = add128(kf, mul128_u32(r, p));
+  b0 = (uint32_t)b.lo;
+  b1 = (uint32_t)(b.lo >> 32);
+  b2 = (uint32_t)b.hi;
+  b3 = (uint32_t)(b.hi >> 32);
 }
 
 // Tenant contribution of a share m * 2^ex2 (m <= 2^53) when q = m 2^(ex2+72)
@@ -180,76 +216,6 @@ __device__ __forceinline__ void attribute_one(const TileArgs &a, uint32_t *tt, c
   if (MODE & M_TEN) tenant_add(a, tt, u, r, bad);
 }
 
-// The general path for one request q of a batch (segment s, constant kf):
-// reloads the request and takes the exact or fp64 share and the general tenant
-// add.  Out of line: the fast paths send it only the requests they do not cover.
-template <int MODE>
-__device__ __noinline__ void general_one(const TileArgs &a, uint32_t *tt, const SegS *segs, int s, bool slow, i128 kf,
-                                         int64_t n, int64_t q, int *bad) {
-  int32_t p = a.p[q], c = a.c[q];
-  const int32_t u = (MODE & M_TEN) ? a.ten[q] : 0;
-  p = p < 0 ? 0 : p;
-  c = c < 0 ? 0 : c;
-  attribute_one<MODE>(a, tt, segs[s], s, slow, kf, n, q, p, c, u, bad);
-}
-
-// Requests left to the general path, gathered per warp across batches so that
-// they are attributed 32 at a time with every lane busy (a batch of a
-// decode-dominated workload has only a few).  meta = n << 4 | slow << 2 | seg.
-constexpr int kDeferCap = 64;
-struct DeferList {
-  int64_t q[kDeferCap];
-  i128 kf[kDeferCap];
-  int meta[kDeferCap];
-};
-
-// Attribute the first min(cnt, 32) entries, one per lane, and move the rest
-// (at most 31 when cnt < kDeferCap) to the front.
-template <int MODE>
-__device__ __forceinline__ void defer_run(const TileArgs &a, uint32_t *tt, const SegS *segs, DeferList &L, int &cnt,
-                                          int lane, int *bad) {
-  const int take = cnt < 32 ? cnt : 32;
-  if (lane < take) {
-    const int m = L.meta[lane];
-    general_one<MODE>(a, tt, segs, m & 3, (m & 4) != 0, L.kf[lane], m >> 4, L.q[lane], bad);
-  }
-  const int rest = cnt - take;
-  int64_t q = 0;
-  i128 kf = mk128(0, 0);
-  int m = 0;
-  __syncwarp();
-  if (lane < rest) {
-    q = L.q[take + lane];
-    kf = L.kf[take + lane];
-    m = L.meta[take + lane];
-  }
-  __syncwarp();
-  if (lane < rest) {
-    L.q[lane] = q;
-    L.kf[lane] = kf;
-    L.meta[lane] = m;
-  }
-  __syncwarp();
-  cnt = rest;
-}
-
-// Append the request of every lane with `flag`; attribute a full 32 at once.
-template <int MODE>
-__device__ __forceinline__ void defer_push(const TileArgs &a, uint32_t *tt, const SegS *segs, DeferList &L, int &cnt,
-                                           bool flag, int64_t q, i128 kf, int meta, int lane, int *bad) {
-  const uint32_t bm = __ballot_sync(kFull, flag);
-  if (!bm) return;
-  if (flag) {
-    const int slot = cnt + __popc(bm & ((1u << lane) - 1u));
-    L.q[slot] = q;
-    L.kf[slot] = kf;
-    L.meta[slot] = meta;
-  }
-  cnt += __popc(bm);
-  __syncwarp();
-  if (cnt >= 32) defer_run<MODE>(a, tt, segs, L, cnt, lane, bad);
-}
-
 // Per-request constant of a batch: fixed-point K (from the shared table for
 // n <= kNK), or {fl(beta/n), fl(a4 n)} in fp64 mode.
 template <int MODE>
@@ -264,6 +230,105 @@ __device__ __forceinline__ i128 batch_const_w(const TileArgs &a, const WSmem *ws
   bool dummy = false;
   const KEntry e = batch_k(a.mp, s, n, &dummy);
   return mk128((uint64_t)__double_as_longlong(e.q), (uint64_t)__double_as_longlong(e.a4n));
+}
+
+// The general path for one request (segment s, constant kf, fields p, c, u as
+// loaded): the exact fixed-point share with prefill_const where the segment
+// allows it, else the exact or fp64 share and the general tenant add.  Out of
+// line: the fast loops send it only the requests they do not cover.
+template <int MODE>
+__device__ __forceinline__ void defer_one(const TileArgs &a, uint32_t *tt, const SegS *segs, int s, bool slow, i128 kf,
+                                          int64_t n, int64_t q, int32_t p, int32_t c, int32_t u, int *bad) {
+  p = p < 0 ? 0 : p;
+  c = c < 0 ? 0 : c;
+  const SegS &sg = segs[s];
+  if ((MODE & M_FIX) && !slow && sg.a2_narrow && sg.p_narrow && p <= kPMaxFix) {
+    uint32_t b0, b1, b2, b3, v0, v1, v2, v3;
+    prefill_const(sg, kf, (uint32_t)p, b0, b1, b2, b3);
+    mad_k13(b0, b1, b2, b3, (uint32_t)sg.A2.lo, (uint32_t)(sg.A2.lo >> 32), (uint32_t)c, v0, v1, v2, v3);
+    if (v3 == 0u && v2 != 0u) {
+      uint64_t m;
+      int ex2;
+      const double d = round96(v0, v1, v2, sg.E, m, ex2);
+      if (!(MODE & M_TEN) || tenant_fast(a, tt, u, m, ex2)) {
+        if (a.share) __stcs(a.share + q, d);
+        return;
+      }
+    }
+  }
+  attribute_one<MODE>(a, tt, sg, s, slow, kf, n, q, p, c, u, bad);
+}
+
+// Requests left to the general path, gathered per warp across batches so that
+// they are attributed 32 at a time with every lane busy (a batch of a
+// decode-dominated workload has only a few).  meta = n << 4 | segment (other
+// bits ignored); p, c, u: the request's fields as loaded (unclamped).
+constexpr int kDeferCap = 64;
+struct DeferList {
+  int64_t q[kDeferCap];
+  int meta[kDeferCap];
+  int32_t p[kDeferCap], c[kDeferCap], u[kDeferCap];
+};
+
+// Attribute the first min(cnt, 32) entries, one per lane (the batch constant
+// looked up again), move the rest (at most 31 when cnt < kDeferCap) to the
+// front and return their number.  Out of line: once per 32 deferred requests;
+// bad data is flagged in the status word directly.
+template <int MODE>
+__device__ __noinline__ int defer_flush(const TileArgs &a, uint32_t *tt, const WSmem &ws, DeferList &L, int cnt,
+                                        int lane) {
+  const int take = cnt < 32 ? cnt : 32;
+  if (lane < take) {
+    const int m = L.meta[lane];
+    const int s = m & 3;
+    const int64_t n = m >> 4;
+    bool slow = false;
+    int bad = 0;
+    const i128 kf = batch_const_w<MODE>(a, &ws, s, n, &slow);
+    defer_one<MODE>(a, tt, ws.seg, s, slow, kf, n, L.q[lane], L.p[lane], L.c[lane], L.u[lane], &bad);
+    if (bad) flag(a.status, kStatusData);
+  }
+  const int rest = cnt - take;
+  int64_t q = 0;
+  int m = 0, p = 0, c = 0, u = 0;
+  __syncwarp();
+  if (lane < rest) {
+    q = L.q[take + lane];
+    m = L.meta[take + lane];
+    p = L.p[take + lane];
+    c = L.c[take + lane];
+    u = L.u[take + lane];
+  }
+  __syncwarp();
+  if (lane < rest) {
+    L.q[lane] = q;
+    L.meta[lane] = m;
+    L.p[lane] = p;
+    L.c[lane] = c;
+    L.u[lane] = u;
+  }
+  __syncwarp();
+  return rest;
+}
+
+// Append the request of every lane with `flag` (all lanes call); attribute 32
+// at once when the list holds that many.
+template <int MODE>
+__device__ __forceinline__ void defer_push(const TileArgs &a, uint32_t *tt, const WSmem &ws, DeferList &L, int &cnt,
+                                           bool flag, int64_t q, int meta, int32_t p, int32_t c, int32_t u, int lane) {
+  const uint32_t bm = __ballot_sync(kFull, flag);
+  if (!bm) return;
+  if (flag) {
+    const int slot = cnt + __popc(bm & ((1u << lane) - 1u));
+    L.q[slot] = q;
+    L.meta[slot] = meta;
+    L.p[slot] = p;
+    L.c[slot] = c;
+    L.u[slot] = u;
+  }
+  cnt += __popc(bm);
+  __syncwarp();
+  if (cnt >= 32) cnt = defer_flush<MODE>(a, tt, ws, L, cnt, lane);
 }
 
 // Warp-strided sums over requests [r0, r1) (at most kJumbo); uniform result on
@@ -299,7 +364,8 @@ __device__ __forceinline__ Sums big_reduce(const TileArgs &a, int64_t r0, int64_
     }
   }
   if (sgn < 0 || phx != 0) *bad = 1;  // clamped as check_req does
-  return warp_sum(acc);
+  static_assert(kJumbo <= 4 * 4 * 32, "at most 16 requests per lane");
+  return warp_sum16(acc);
 }
 
 // Warp-strided shares of requests [r0, r1) of one batch (segment s, constant kf):
@@ -307,8 +373,9 @@ __device__ __forceinline__ Sums big_reduce(const TileArgs &a, int64_t r0, int64_
 // of line: the fast loop serves the common case).
 template <int MODE>
 __device__ __noinline__ void big_shares(const TileArgs &a, uint32_t *tt, const SegS &sg, int s, bool slow,
-                                           i128 kf, int64_t r0, int64_t r1, int lane, int *bad) {
+                                           i128 kf, int64_t r0, int64_t r1, int lane) {
   const int64_t n = r1 - r0;
+  int bad = 0;
   for (int64_t i = r0 + lane; i < r1; i += 4 * 32) {
     int32_t p[4], c[4], u[4];
 #pragma unroll
@@ -324,23 +391,22 @@ __device__ __noinline__ void big_shares(const TileArgs &a, uint32_t *tt, const S
       const int64_t q = i + 32 * k;
       if (q < r1) {
         const int32_t pk = p[k] < 0 ? 0 : p[k], ck = c[k] < 0 ? 0 : c[k];
-        attribute_one<MODE>(a, tt, sg, s, slow, kf, n, q, pk, ck, u[k], bad);
+        attribute_one<MODE>(a, tt, sg, s, slow, kf, n, q, pk, ck, u[k], &bad);
       }
     }
   }
+  if (bad) flag(a.status, kStatusData);
 }
 
-// Warp-strided shares of a batch whose decode requests take the fast path
+// Warp-strided shares of a batch whose requests take the fast path
 // (fixed-point mode, in-range constant kf, A2 < 2^64).  The batch was just
 // reduced, tenant ids included, so its requests are in L1 and the loop takes
-// one request per lane per step.  Requests the fast path does not cover are
-// marked (a batch has at most kJumbo requests, so 16 strided positions per
-// lane) and returned: bit t stands for request r0 + lane + 32 t.  ALLDEC:
+// one request per lane per step; every lane runs every step, so the requests
+// the fast path does not cover go to the defer list as they appear.  ALLDEC:
 // every p = 1, p is not loaded.
 template <int MODE, bool ALLDEC>
-__device__ __forceinline__ uint32_t big_shares_fast(const TileArgs &a, uint32_t *tt, const WSmem &ws, int s, i128 kf,
-                                                    int64_t r0, int64_t r1, int lane) {
-  static_assert(kJumbo <= 16 * 32, "strided positions fit in 16 bits per lane");
+__device__ __forceinline__ void big_shares_fast(const TileArgs &a, uint32_t *tt, const WSmem &ws, DeferList &L,
+                                                int &cnt, int s, i128 kf, int64_t r0, int64_t r1, int lane) {
   const SegS &sg = ws.seg[s];
   const i128 K13 = add128(kf, sg.A13);
   const uint32_t k0 = (uint32_t)K13.lo, k1 = (uint32_t)(K13.lo >> 32), k2 = (uint32_t)K13.hi,
@@ -350,24 +416,28 @@ __device__ __forceinline__ uint32_t big_shares_fast(const TileArgs &a, uint32_t 
   const int32_t *P = a.p + r0, *C = a.c + r0, *U = a.ten + r0;
   double *S = a.share ? a.share + r0 : nullptr;
   const int n = (int)(r1 - r0);
-  uint32_t defer = 0;
-  for (int q = lane, pos = 0; q < n; q += 32, ++pos) {
-    const int32_t c0 = C[q];
-    const int32_t u0 = (MODE & M_TEN) ? U[q] : 0;
-    const int32_t p0 = ALLDEC ? 1 : P[q];
-    uint32_t v0, v1, v2, v3;
-    mad_k13(k0, k1, k2, k3, a0, a1, (uint32_t)(c0 < 0 ? 0 : c0), v0, v1, v2, v3);
-    uint64_t m;
-    int ex2;
-    const double d = round96(v0, v1, v2, E, m, ex2);
-    bool done = (ALLDEC || p0 == 1) && v3 == 0u && v2 != 0u;
-    if (MODE & M_TEN) {
-      if (done) done = tenant_fast(a, tt, u0, m, ex2);
+  const int meta = (n << 4) | s;
+  for (int q0 = 0; q0 < n; q0 += 32) {
+    const int q = q0 + lane;
+    bool done = true;
+    int32_t c0 = 0, u0 = 0, p0 = 1;
+    if (q < n) {
+      c0 = C[q];
+      u0 = (MODE & M_TEN) ? U[q] : 0;
+      p0 = ALLDEC ? 1 : P[q];
+      uint32_t v0, v1, v2, v3;
+      mad_k13(k0, k1, k2, k3, a0, a1, (uint32_t)(c0 < 0 ? 0 : c0), v0, v1, v2, v3);
+      uint64_t m;
+      int ex2;
+      const double d = round96(v0, v1, v2, E, m, ex2);
+      done = (ALLDEC || p0 == 1) && v3 == 0u && v2 != 0u;
+      if (MODE & M_TEN) {
+        if (done) done = tenant_fast(a, tt, u0, m, ex2);
+      }
+      if (done && S) __stcs(S + q, d);
     }
-    if (done && S) __stcs(S + q, d);
-    if (!done) defer |= 1u << pos;
+    defer_push<MODE>(a, tt, ws, L, cnt, !done, r0 + q, meta, p0, c0, u0, lane);
   }
-  return defer;
 }
 
 // Rounds over the small batches of a group (lanes with `small`): every round
@@ -415,12 +485,14 @@ __device__ __forceinline__ void small_rounds(const TileArgs &a, const WSmem &ws,
       const int meta = __shfl_sync(kFull, mymeta, j);
       const i128 kf = mk128(klo, khi);
       bool done = true;
+      int32_t p = 0, c = 0, u = 0;
       if (act) {
         const int s = meta & 3;
         done = false;
+        p = a.p[r];
+        c = a.c[r];
+        u = (MODE & M_TEN) ? a.ten[r] : 0;
         if (meta & 8) {
-          const int32_t p = a.p[r], c = a.c[r];
-          const int32_t u = (MODE & M_TEN) ? a.ten[r] : 0;
           const SegS &sg = ws.seg[s];
           const i128 K13 = add128(kf, sg.A13);
           uint32_t v0, v1, v2, v3;
@@ -436,7 +508,7 @@ __device__ __forceinline__ void small_rounds(const TileArgs &a, const WSmem &ws,
           if (done && a.share) __stcs(a.share + r, d);
         }
       }
-      defer_push<MODE>(a, tt, ws.seg, *dl, dcnt, !done, r, kf, meta & ~8, lane, bad);
+      defer_push<MODE>(a, tt, ws, *dl, dcnt, !done, r, meta, p, c, u, lane);
     }
     __syncwarp();  // owner[] is rewritten by the next round
   }
@@ -553,68 +625,68 @@ __device__ __forceinline__ void fit_group(const TileArgs &a, FitAcc *fw, int64_t
 
 // One group of up to 32 consecutive batches [g0, g0 + ng) of a tile.
 template <int MODE>
-__device__ __forceinline__ void process_group(const TileArgs &a, const WSmem &ws, uint32_t *tt, uint8_t *owner,
+__device__ __forceinline__ void process_group(const TileArgs &a, WSmem &ws, uint32_t *tt, uint8_t *owner,
                                               DeferList *dl, int &dcnt, FitAcc *fw, int64_t g0, int ng, int lane,
                                               int *bad) {
   constexpr bool kAttr = (MODE & M_ATTR) != 0;
   const bool valid = lane < ng;
-  const int64_t b = g0 + lane;
-  int64_t o0 = valid ? a.off[b] : 0;
-  int64_t o1 = __shfl_down_sync(kFull, o0, 1);
-  if (valid && lane == ng - 1) o1 = a.off[b + 1];
-  if (valid) {
-    const int64_t c0 = clampi(o0, 0, a.n_req), c1 = clampi(o1, c0, a.n_req);
-    if (c0 != o0 || c1 != o1) *bad = 1;
-    o0 = c0;
-    o1 = c1;
+  int64_t o0 = valid ? a.off[g0 + lane] : 0;
+  int n = 0;  // requests of this lane's batch; 0 for jumbo batches (k_jumbo's)
+  bool jumbo = false;
+  {
+    int64_t o1 = __shfl_down_sync(kFull, o0, 1);
+    if (valid && lane == ng - 1) o1 = a.off[g0 + lane + 1];
+    if (valid) {
+      const int64_t c0 = clampi(o0, 0, a.n_req), c1 = clampi(o1, c0, a.n_req);
+      if (c0 != o0 || c1 != o1) *bad = 1;
+      o0 = c0;
+      jumbo = c1 - c0 > kJumbo;
+      n = jumbo ? 0 : (int)(c1 - c0);
+    }
   }
-  const int64_t n = valid ? o1 - o0 : 0;
-  const bool jumbo = valid && n > kJumbo;
   if (jumbo) {
     const unsigned long long slot = atomicAdd(a.jumbo_n, 1ull);
     if (slot < (unsigned long long)a.jumbo_cap)
-      a.jumbo[slot] = b;
+      a.jumbo[slot] = g0 + lane;
     else
       *bad = 1;
   }
   Sums mys{0, 0, 0, 0};
   i128 myk = mk128(0, 0);
   int mymeta = 0;
+  Sums *gsum = ws.gsum[threadIdx.x >> 5];
 
   // ---- big batches: reduce, constant and shares one batch at a time
-  uint32_t big = __ballot_sync(kFull, valid && !jumbo && n >= kBig);
+  const uint32_t big0 = __ballot_sync(kFull, n >= kBig);
+  uint32_t big = big0;
   while (big) {
     const int j = __ffs(big) - 1;
     big &= big - 1;
-    const int64_t r0 = __shfl_sync(kFull, o0, j), r1 = __shfl_sync(kFull, o1, j);
+    const int64_t r0 = __shfl_sync(kFull, o0, j), r1 = r0 + __shfl_sync(kFull, n, j);
     const Sums tot = big_reduce(a, r0, r1, lane, bad);
-    if (lane == j) mys = tot;
+    if (lane == j) gsum[j] = tot;
     if (kAttr) {
       const BatchAgg g{tot.s1, tot.s2, tot.s3, r1 - r0, tot.ph > 0};
       const int s = segment_of(a.mp, g);
       bool slow = false;
       const i128 kf = batch_const_w<MODE>(a, &ws, s, r1 - r0, &slow);
       if ((MODE & M_FIX) && !slow && ws.seg[s].a2_narrow) {
-        uint32_t defer = (tot.s1 == r1 - r0 && tot.s3 == r1 - r0)
-                             ? big_shares_fast<MODE, true>(a, tt, ws, s, kf, r0, r1, lane)
-                             : big_shares_fast<MODE, false>(a, tt, ws, s, kf, r0, r1, lane);
-        const int meta = ((int)(r1 - r0) << 4) | s;
-        while (__any_sync(kFull, defer != 0u)) {
-          const bool has = defer != 0u;
-          const int t = has ? __ffs(defer) - 1 : 0;
-          if (has) defer &= defer - 1u;
-          defer_push<MODE>(a, tt, ws.seg, *dl, dcnt, has, r0 + lane + 32 * (int64_t)t, kf, meta, lane, bad);
-        }
+        if (tot.s1 == r1 - r0 && tot.s3 == r1 - r0)
+          big_shares_fast<MODE, true>(a, tt, ws, *dl, dcnt, s, kf, r0, r1, lane);
+        else
+          big_shares_fast<MODE, false>(a, tt, ws, *dl, dcnt, s, kf, r0, r1, lane);
       } else {
-        big_shares<MODE>(a, tt, ws.seg[s], s, slow, kf, r0, r1, lane, bad);
+        big_shares<MODE>(a, tt, ws.seg[s], s, slow, kf, r0, r1, lane);
       }
     }
   }
 
+  if ((big0 >> lane) & 1u) mys = gsum[lane];  // slot j is written and read by lane j only
+
   // ---- small batches: packed rounds
-  const bool small = valid && n > 0 && n < kBig;
+  const bool small = n > 0 && n < kBig;
   if (__any_sync(kFull, small)) {
-    const int pn = small ? (int)n : 0;
+    const int pn = small ? n : 0;
     const int P = warp_excl_scan_int(pn, lane);
     const int64_t base = o0 - P;
     small_rounds<MODE, false>(a, ws, tt, owner, dl, dcnt, small, pn, P, base, mys, myk, 0, lane, bad);
@@ -625,7 +697,7 @@ __device__ __forceinline__ void process_group(const TileArgs &a, const WSmem &ws
         bool slow = false;
         myk = batch_const_w<MODE>(a, &ws, s, n, &slow);
         const bool fast = (MODE & M_FIX) && !slow && ws.seg[s].a2_narrow;
-        mymeta = ((int)n << 4) | (fast ? 8 : 0) | (slow ? 4 : 0) | s;
+        mymeta = (n << 4) | (fast ? 8 : 0) | (slow ? 4 : 0) | s;
       }
       small_rounds<MODE, true>(a, ws, tt, owner, dl, dcnt, small, pn, P, base, mys, myk, mymeta, lane, bad);
     }
@@ -636,10 +708,10 @@ __device__ __forceinline__ void process_group(const TileArgs &a, const WSmem &ws
   if (valid && !jumbo) {
     const BatchAgg g{mys.s1, mys.s2, mys.s3, n, mys.ph > 0};
     const int s = segment_of(a.mp, g);
-    emit_batch<MODE>(a, b, g, s);
+    emit_batch<MODE>(a, g0 + lane, g, s);
     if (MODE & M_FIT) {
       const bool in_range = g.s1 < kFitFeatMax && g.s2 < kFitFeatMax && g.s3 < kFitFeatMax &&
-                            n * n < kFitFeatMax;
+                            (int64_t)n * n < kFitFeatMax;
       if (!in_range) flag(a.status, kStatusOverflow);
       if (n > 0 && in_range) fseg = s;
     }
@@ -660,7 +732,8 @@ __device__ __forceinline__ void init_segs(const TileArgs &a, SegS *seg) {
     g.A2 = f.A2;
     g.E = f.E;
     g.a2_narrow = f.a2_narrow;
-    g.pad[0] = g.pad[1] = 0;
+    g.p_narrow = ((uint64_t)f.A1.hi < (1ull << 31) && f.A3.hi == 0) ? 1 : 0;
+    g.pad = 0;
     seg[threadIdx.x] = g;
   }
 }
@@ -722,7 +795,7 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
     t = __shfl_sync(kFull, tn, 0);
   }
   if (MODE & M_ATTR) {
-    while (dcnt > 0) defer_run<MODE>(a, tt, ws.seg, *dl, dcnt, lane, &bad);
+    while (dcnt > 0) dcnt = defer_flush<MODE>(a, tt, ws, *dl, dcnt, lane);
   }
 
   if (bad) flag(a.status, kStatusData);
