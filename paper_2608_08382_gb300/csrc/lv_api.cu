@@ -141,7 +141,7 @@ bool derive_fixed(const lv_model *m, int nk, ModelP *mp) {
     if (std::ldexp(kmax, -E) >= std::ldexp(1.0, 123) || mag(f.B) >= std::ldexp(1.0, 124)) return false;
     f.A13 = add128(f.A1, f.A3);
     f.a2_narrow = (f.A2.hi == 0) ? 1 : 0;
-    f.t_narrow = (f.B.hi | f.A1.hi | f.A2.hi | f.A3.hi | f.A4.hi) == 0 ? 1 : 0;
+    f.t_narrow = (f.B.hi | f.A1.hi | f.A2.hi | f.A3.hi | f.A4.hi) < (1ull << 32) ? 1 : 0;
     f.pad = 0;
     f.lim[0] = limit_for(f.A1);
     f.lim[1] = limit_for(f.A2);

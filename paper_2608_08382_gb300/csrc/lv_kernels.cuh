@@ -28,7 +28,7 @@ struct SegFix {
   uint64_t lim[4];   // exact T path valid when S1, S2, S3, n^2 <= lim[0..3]
   int E;
   int a2_narrow;     // 1: 0 <= A2 < 2^64 (64-bit multiply suffices)
-  int t_narrow;      // 1: B, A1..A4 all in [0, 2^64) (eq1_fast applies)
+  int t_narrow;      // 1: B, A1..A4 all in [0, 2^96) (eq1_fast applies)
   int pad;
 };
 
@@ -276,19 +276,24 @@ __device__ __noinline__ double eq1_fix(const ModelP &mp, int s, const BatchAgg &
   return fix_to_double(V, f.E).d;
 }
 
-// Eq. 1 in fixed point for the common case: every coefficient in [0, 2^64)
-// (t_narrow), each product below 2^96 and the sum in [2^64, 2^96); four
-// 64x64-bit products and the leading-word rounding.  False when any of these
-// does not hold (the caller then takes eq1_fix).
+// Eq. 1 in fixed point for the common case: every coefficient in [0, 2^96)
+// (t_narrow), each product A_k S_k below 2^96 and the sum in [2^64, 2^96);
+// 64x64-bit products with the coefficients' high words folded in, and the
+// leading-word rounding.  False when any of these does not hold (the caller
+// then takes eq1_fix, which gives the same value wherever this one applies).
 __device__ __forceinline__ bool eq1_fast(const SegFix &f, const BatchAgg &g, double *T) {
   if (!f.t_narrow || g.n == 0 || g.n > 0x7fffffffll) return false;
-  uint64_t lo = f.B.lo, hi = 0;
+  uint64_t lo = f.B.lo, hi = f.B.hi;
   bool ok = true;
-  const uint64_t A[4] = {f.A1.lo, f.A2.lo, f.A3.lo, f.A4.lo};
+  const i128 A[4] = {f.A1, f.A2, f.A3, f.A4};
   const uint64_t S[4] = {(uint64_t)g.s1, (uint64_t)g.s2, (uint64_t)g.s3, (uint64_t)g.n * (uint64_t)g.n};
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const uint64_t pl = A[i] * S[i], ph = __umul64hi(A[i], S[i]);
+    const uint64_t pl = A[i].lo * S[i];
+    uint64_t ph = __umul64hi(A[i].lo, S[i]);
+    // A_hi < 2^32; A_hi S 2^64 stays below 2^96 only for S < 2^32 (then no wrap)
+    ok &= A[i].hi == 0 || (S[i] >> 32) == 0;
+    ph += (uint64_t)(uint32_t)A[i].hi * (uint32_t)S[i];
     ok &= ph < (1ull << 32);  // product below 2^96: the sum of five stays below 2^99
     lo += pl;
     hi += ph + (lo < pl ? 1ull : 0ull);
