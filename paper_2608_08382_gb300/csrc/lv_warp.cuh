@@ -111,6 +111,8 @@ __device__ __forceinline__ int warp_excl_scan_int(int v, int lane) {
   return x - v;
 }
 
+__device__ __forceinline__ void prefetch_l2(const void *p) { asm volatile("prefetch.global.L2 [%0];" ::"l"(p)); }
+
 // ---------------------------------------------------------------- decode fast path
 //
 // A decode request (p = 1) of a batch with constant K has the exact share
@@ -663,6 +665,14 @@ __device__ __forceinline__ void process_group(const TileArgs &a, WSmem &ws, uint
     const int j = __ffs(big) - 1;
     big &= big - 1;
     const int64_t r0 = __shfl_sync(kFull, o0, j), r1 = r0 + __shfl_sync(kFull, n, j);
+    {
+      // the next 256 requests (the batches after this one) into L2 while this
+      // batch is reduced and attributed: one line per lane, 8 per array.  Not
+      // bounded by the tile: measured faster than stopping at its end.
+      const int32_t *arr = lane < 8 ? a.p : lane < 16 ? a.c : lane < 24 ? a.ph : a.ten;
+      const int64_t pq = (r1 & ~(int64_t)31) + 32 * (lane & 7);
+      if (arr && pq < a.n_req) prefetch_l2(arr + pq);
+    }
     const Sums tot = big_reduce(a, r0, r1, lane, bad);
     if (lane == j) gsum[j] = tot;
     if (kAttr) {
