@@ -131,19 +131,41 @@ __global__ void __launch_bounds__(kWiCols) k_wi_pairs(ModelP mp, const CandP *__
                                                        const PendP *__restrict__ pend, int64_t nc, int64_t np,
                                                        int64_t j_base, double *__restrict__ T_new,
                                                        double *__restrict__ share_new) {
+  static_assert(kWiRows <= kWiCols, "one pending row per thread at most");
   __shared__ PendP sp[kWiRows];
   __shared__ int sE[4];
   const int64_t b = blockIdx.x * (int64_t)kWiCols + threadIdx.x;
   const int64_t j0 = j_base + blockIdx.y * (int64_t)kWiRows;
   const int rows = (int)(np - j0 < kWiRows ? np - j0 : kWiRows);
-  for (int r = threadIdx.x; r < rows; r += kWiCols) sp[r] = pend[j0 + r];
+  int rslow = 0;
+  if (threadIdx.x < rows) {
+    sp[threadIdx.x] = pend[j0 + threadIdx.x];
+    rslow = sp[threadIdx.x].slow;
+  }
   if (threadIdx.x < 4) sE[threadIdx.x] = mp.fx[threadIdx.x].E;
-  __syncthreads();
+  rslow = __syncthreads_or(rslow);
   if (b >= nc) return;
   const CandP *cb = cand + b;
   const int64_t s1 = cb->s1, s2 = cb->s2, s3 = cb->s3, n1 = cb->n + 1;
   const int prefill = cb->prefill, cslow = cb->slow;
   const int64_t sp0 = mp.split[0], sp1 = mp.split[1];
+  if (!cslow && !rslow && rows == kWiRows) {
+    // every pair of the block exact: no out-of-line call, rows unrolled for
+    // independent loads and roundings in flight
+#pragma unroll 4
+    for (int r = 0; r < kWiRows; ++r) {
+      const int32_t p = sp[r].p;
+      const int phase = (prefill | sp[r].phase) ? 1 : 0;
+      const int s = phase * 2 + ((s1 + p >= (phase ? sp1 : sp0)) ? 1 : 0);
+      const i128 V = sp[r].V[s];
+      const double T = round_fix(add128(cb->U[s], V), sE[s]);
+      const double sh = round_fix(add128(cb->W[s], V), sE[s]);
+      const int64_t o = (j0 + r) * nc + b;
+      if (T_new) __stcs(T_new + o, T);
+      if (share_new) __stcs(share_new + o, sh);
+    }
+    return;
+  }
   for (int r = 0; r < rows; ++r) {
     const int32_t p = sp[r].p, c = sp[r].c;
     const int phase = (prefill | sp[r].phase) ? 1 : 0;
