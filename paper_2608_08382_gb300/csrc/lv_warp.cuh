@@ -517,65 +517,64 @@ __device__ __forceinline__ void small_rounds(const TileArgs &a, const WSmem &ws,
 }
 
 // Fit statistics of the group's batches into this warp's accumulators
-// fw[group][entry].  Every lane converts its own batch's latencies to fixed
-// point once (Y = y * 2^100 and floor(Y^2 / 2^64)); then, for each batch of
-// segment g in turn, lane e adds that batch's contribution to entry e of
-// group g (and e + 32 when a group has more than 32 entries), the batch's sums
-// and Y values arriving by shuffle.  Entry order: 15 Gram pairs (a <= b, row
-// order), 5 X^T y columns per y vector, one y'y per y vector, one flag.
-__device__ __forceinline__ int64_t fit_x(int i, int64_t s1, int64_t s2, int64_t s3, int64_t n2) {
-  return i == 0 ? 1 : i == 1 ? s1 : i == 2 ? s2 : i == 3 ? s3 : n2;
-}
+// fw[group][entry].  Entry order: 15 Gram pairs (a <= b, row order), 5 X^T y
+// columns per y vector, one y'y per y vector, one flag.  Every entry adds
+// x[a] * B for each batch of its group, B a 192-bit two's complement operand:
+// a feature (Gram), the batch's Y = y * 2^100 (X^T y), or floor(Y^2 / 2^64)
+// with x[a] = 1 (y'y).  The batches of segment g are taken in turn: the owner
+// lane writes the batch's record (kFitRecWords words: x0..x4 = 1, S1, S2, S3,
+// n^2, a zero word, then Y and floor(Y^2 / 2^64), three words each, per y
+// vector) to the warp's slot in shared memory, and lane e reads entry e's two
+// operands from it and multiply-adds in registers, the same instructions for
+// every kind of entry.  The accumulators are loaded and stored once per
+// segment and group.
+constexpr int kFitRecWords = 6 + 6 * kFitMaxY;
 
-__device__ __forceinline__ void fit_entry_add(FitAcc &acc, int e, int n_y, int64_t s1, int64_t s2, int64_t s3,
-                                              int64_t n2, const i128 *Y, const uint64_t (*YY)[3]) {
+struct FitRole {
+  int xa, b0, b1, b2;  // record words of x and of B's three words
+};
+
+__device__ __forceinline__ FitRole fit_role(int e, int n_y) {
   if (e < 15) {
     int a = 0, r = e;
     while (r >= 5 - a) {
       r -= 5 - a;
       ++a;
     }
-    const uint64_t u = (uint64_t)fit_x(a, s1, s2, s3, n2), v = (uint64_t)fit_x(a + r, s1, s2, s3, n2);
-    acc_add256(acc.w, u * v, __umul64hi(u, v), 0, 0);
-  } else if (e < 15 + 5 * n_y) {
-    const int col = (e - 15) % 5, kk = (e - 15) / 5;
-    i128 y = Y[0];
-#pragma unroll
-    for (int q = 1; q < kFitMaxY; ++q)
-      if (kk == q) y = Y[q];
-    const bool neg = is_neg128(y);
-    const i128 M = neg ? neg128(y) : y;
-    const uint64_t xv = (uint64_t)fit_x(col, s1, s2, s3, n2);
-    const uint64_t p0 = M.lo * xv, p1 = __umul64hi(M.lo, xv);
-    const uint64_t q0 = M.hi * xv, q1 = __umul64hi(M.hi, xv);
-    uint64_t w0 = p0, w1 = p1 + q0, w2 = q1 + (w1 < p1 ? 1ull : 0ull), w3 = 0;
-    if (neg) {
-      w0 = ~w0 + 1;
-      w1 = ~w1 + (w0 == 0 ? 1ull : 0ull);
-      w2 = ~w2 + ((w0 | w1) == 0 ? 1ull : 0ull);
-      w3 = ~w3 + ((w0 | w1 | w2) == 0 ? 1ull : 0ull);
-    }
-    acc_add256(acc.w, w0, w1, w2, w3);
-  } else if (e < 15 + 6 * n_y) {
-    const int kk = e - 15 - 5 * n_y;
-    uint64_t a0 = YY[0][0], a1 = YY[0][1], a2 = YY[0][2];
-#pragma unroll
-    for (int q = 1; q < kFitMaxY; ++q)
-      if (kk == q) {
-        a0 = YY[q][0];
-        a1 = YY[q][1];
-        a2 = YY[q][2];
-      }
-    acc_add256(acc.w, a0, a1, a2, 0);
-  } else {
-    if (s1 != s3) acc.w[0] |= 1ull;
+    return FitRole{a, a + r, 5, 5};
   }
+  if (e < 15 + 5 * n_y) {
+    const int col = (e - 15) % 5, kk = (e - 15) / 5;
+    return FitRole{col, 6 + 6 * kk, 7 + 6 * kk, 8 + 6 * kk};
+  }
+  if (e < 15 + 6 * n_y) {
+    const int kk = e - 15 - 5 * n_y;
+    return FitRole{0, 9 + 6 * kk, 10 + 6 * kk, 11 + 6 * kk};
+  }
+  return FitRole{1, 3, 5, 5};  // the flag (S1 != S3) and lanes past the last entry
 }
 
-__device__ __forceinline__ void fit_group(const TileArgs &a, FitAcc *fw, int64_t g0, const Sums &mys, int64_t n,
-                                          int fseg, int lane, int *bad) {
+// acc += x * B (mod 2^256) for B = b0 + b1 2^64 + b2 2^128, b2 sign-extended.
+__device__ __forceinline__ void fit_mac(uint64_t *acc, uint64_t x, uint64_t b0, uint64_t b1, uint64_t b2) {
+  const uint64_t b3 = (uint64_t)((int64_t)b2 >> 63);
+  acc_add256(acc, x * b0, __umul64hi(x, b0), __umul64hi(x, b1), __umul64hi(x, b2));
+  acc_add256(acc, 0, x * b1, x * b2, x * b3);
+}
+
+// One entry's update for the record in `rec`; the flag entry ORs S1 != S3.
+__device__ __forceinline__ void fit_entry(uint64_t *acc, const uint64_t *rec, const FitRole &r, bool flag) {
+  const uint64_t x = rec[r.xa], b0 = rec[r.b0];
+  if (flag)
+    acc[0] |= x != b0 ? 1ull : 0ull;
+  else
+    fit_mac(acc, x, b0, rec[r.b1], rec[r.b2]);
+}
+
+__device__ __forceinline__ void fit_group(const TileArgs &a, FitAcc *fw, uint64_t *rec, int64_t g0, const Sums &mys,
+                                          int64_t n, int fseg, int lane, int *bad) {
+  if (!__any_sync(kFull, fseg >= 0)) return;
   const int NE = fit_entries(a.fit.n_y), n_y = a.fit.n_y;
-  // this lane's batch: latencies in fixed point
+  // this lane's batch: latencies in fixed point and floor(Y^2 / 2^64)
   i128 Ym[kFitMaxY];
   uint64_t YYm[kFitMaxY][3];
 #pragma unroll
@@ -597,39 +596,68 @@ __device__ __forceinline__ void fit_group(const TileArgs &a, FitAcc *fw, int64_t
       YYm[q][2] = w[2];
     }
   }
-  const int64_t n2 = n * n;
+  const FitRole r0 = fit_role(lane, n_y), r1 = fit_role(lane + 32, n_y);
+  const bool two = NE > 32;  // lanes 0..NE-33 also own entry lane + 32
+  if (lane == 0) {
+    rec[0] = 1;
+    rec[5] = 0;
+  }
 #pragma unroll 1
   for (int g = 0; g < 4; ++g) {
     uint32_t m = __ballot_sync(kFull, fseg == g);
+    if (!m) continue;
+    uint64_t acc0[4] = {0, 0, 0, 0}, acc1[4] = {0, 0, 0, 0};
+    FitAcc *f0 = fw + g * NE + lane, *f1 = f0 + 32;
+    if (lane < NE) {
+#pragma unroll
+      for (int w = 0; w < 4; ++w) acc0[w] = f0->w[w];
+    }
+    if (two && lane + 32 < NE) {
+#pragma unroll
+      for (int w = 0; w < 4; ++w) acc1[w] = f1->w[w];
+    }
     while (m) {
       const int j = __ffs(m) - 1;
       m &= m - 1;
-      const int64_t s1 = __shfl_sync(kFull, mys.s1, j), s2 = __shfl_sync(kFull, mys.s2, j),
-                    s3 = __shfl_sync(kFull, mys.s3, j), nn = __shfl_sync(kFull, n2, j);
-      i128 Y[kFitMaxY];
-      uint64_t YY[kFitMaxY][3];
+      __syncwarp();  // the previous record has been read
+      if (lane == j) {
+        rec[1] = (uint64_t)mys.s1;
+        rec[2] = (uint64_t)mys.s2;
+        rec[3] = (uint64_t)mys.s3;
+        rec[4] = (uint64_t)(n * n);
 #pragma unroll
-      for (int q = 0; q < kFitMaxY; ++q) {
-        if (q < n_y) {
-          Y[q] = mk128(__shfl_sync(kFull, Ym[q].lo, j), __shfl_sync(kFull, Ym[q].hi, j));
-          YY[q][0] = __shfl_sync(kFull, YYm[q][0], j);
-          YY[q][1] = __shfl_sync(kFull, YYm[q][1], j);
-          YY[q][2] = __shfl_sync(kFull, YYm[q][2], j);
-        } else {
-          Y[q] = mk128(0, 0);
-          YY[q][0] = YY[q][1] = YY[q][2] = 0;
+        for (int q = 0; q < kFitMaxY; ++q) {
+          if (q < n_y) {
+            rec[6 + 6 * q] = Ym[q].lo;
+            rec[7 + 6 * q] = Ym[q].hi;
+            rec[8 + 6 * q] = (uint64_t)((int64_t)Ym[q].hi >> 63);
+            rec[9 + 6 * q] = YYm[q][0];
+            rec[10 + 6 * q] = YYm[q][1];
+            rec[11 + 6 * q] = YYm[q][2];
+          }
         }
       }
-      for (int e = lane; e < NE; e += 32) fit_entry_add(fw[g * NE + e], e, n_y, s1, s2, s3, nn, Y, YY);
+      __syncwarp();
+      fit_entry(acc0, rec, r0, lane == NE - 1);
+      if (two) fit_entry(acc1, rec, r1, lane + 32 == NE - 1);
+    }
+    if (lane < NE) {
+#pragma unroll
+      for (int w = 0; w < 4; ++w) f0->w[w] = acc0[w];
+    }
+    if (two && lane + 32 < NE) {
+#pragma unroll
+      for (int w = 0; w < 4; ++w) f1->w[w] = acc1[w];
     }
   }
+  __syncwarp();  // the record slot is rewritten by the next group
 }
 
 // One group of up to 32 consecutive batches [g0, g0 + ng) of a tile.
 template <int MODE>
 __device__ __forceinline__ void process_group(const TileArgs &a, WSmem &ws, uint32_t *tt, uint8_t *owner,
-                                              DeferList *dl, int &dcnt, FitAcc *fw, int64_t g0, int ng, int lane,
-                                              int *bad) {
+                                              DeferList *dl, int &dcnt, FitAcc *fw, uint64_t *frec, int64_t g0, int ng,
+                                              int lane, int *bad) {
   constexpr bool kAttr = (MODE & M_ATTR) != 0;
   const bool valid = lane < ng;
   int64_t o0 = valid ? a.off[g0 + lane] : 0;
@@ -726,7 +754,7 @@ __device__ __forceinline__ void process_group(const TileArgs &a, WSmem &ws, uint
       if (n > 0 && in_range) fseg = s;
     }
   }
-  if (MODE & M_FIT) fit_group(a, fw, g0, mys, n, fseg, lane, bad);
+  if (MODE & M_FIT) fit_group(a, fw, frec, g0, mys, n, fseg, lane, bad);
 }
 
 // Shared-memory tables of a CTA: per-segment share parameters and, in
@@ -758,6 +786,8 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
   FitAcc *facc = reinterpret_cast<FitAcc *>(smem_raw + sizeof(WSmem) + (kTen ? ten_bytes(a.H) : 0));
   DeferList *dlists = reinterpret_cast<DeferList *>(smem_raw + sizeof(WSmem) + (kTen ? ten_bytes(a.H) : 0) +
                                                     (kFit ? (size_t)kWarps * 4 * fit_entries(a.fit.n_y) * sizeof(FitAcc) : 0));
+  uint64_t *frecs = reinterpret_cast<uint64_t *>(reinterpret_cast<unsigned char *>(dlists) +
+                                                 ((MODE & M_ATTR) ? kWarps * sizeof(DeferList) : 0));
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
   const int NE4 = kFit ? 4 * fit_entries(a.fit.n_y) : 0;
   int bad = 0;
@@ -787,6 +817,7 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
   uint8_t *owner = ws.owner[wid];
   FitAcc *fw = facc + wid * NE4;
   DeferList *dl = dlists + wid;
+  uint64_t *frec = frecs + wid * kFitRecWords;
   int dcnt = 0;
   unsigned long long t = 0;
   if (lane == 0) t = atomicAdd(a.ctr, 1ull);
@@ -801,7 +832,7 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
       bad = 1;
     }
     for (int64_t g0 = b0; g0 < b1; g0 += 32)
-      process_group<MODE>(a, ws, tt, owner, dl, dcnt, fw, g0, (int)(b1 - g0 < 32 ? b1 - g0 : 32), lane, &bad);
+      process_group<MODE>(a, ws, tt, owner, dl, dcnt, fw, frec, g0, (int)(b1 - g0 < 32 ? b1 - g0 : 32), lane, &bad);
     t = __shfl_sync(kFull, tn, 0);
   }
   if (MODE & M_ATTR) {
