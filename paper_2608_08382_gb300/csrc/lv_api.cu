@@ -252,8 +252,7 @@ template <int MODE>
 size_t warps_smem(int H, int n_y) {
   return sizeof(WSmem) + ((MODE & M_TEN) ? ten_bytes(H) : 0) +
          ((MODE & M_FIT) ? (size_t)kWarps * 4 * fit_entries(n_y) * sizeof(FitAcc) : 0) +
-         ((MODE & M_ATTR) ? (size_t)kWarps * sizeof(DeferList) : 0) +
-         ((MODE & M_FIT) ? (size_t)kWarps * kFitRecWords * sizeof(uint64_t) : 0);
+         ((MODE & M_ATTR) ? (size_t)kWarps * sizeof(DeferList) : 0);
 }
 
 constexpr int kJumboCtasPerSm = 2;

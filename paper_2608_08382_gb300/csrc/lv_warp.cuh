@@ -521,14 +521,18 @@ __device__ __forceinline__ void small_rounds(const TileArgs &a, const WSmem &ws,
 // columns per y vector, one y'y per y vector, one flag.  Every entry adds
 // x[a] * B for each batch of its group, B a 192-bit two's complement operand:
 // a feature (Gram), the batch's Y = y * 2^100 (X^T y), or floor(Y^2 / 2^64)
-// with x[a] = 1 (y'y).  The batches of segment g are taken in turn: the owner
-// lane writes the batch's record (kFitRecWords words: x0..x4 = 1, S1, S2, S3,
-// n^2, a zero word, then Y and floor(Y^2 / 2^64), three words each, per y
-// vector) to the warp's slot in shared memory, and lane e reads entry e's two
-// operands from it and multiply-adds in registers, the same instructions for
-// every kind of entry.  The accumulators are loaded and stored once per
-// segment and group.
+// with x[a] = 1 (y'y).  The batches of segment g are taken kFitRecs at a time:
+// their owner lanes write the batches' records (kFitRecWords words: x0..x4 =
+// 1, S1, S2, S3, n^2, a zero word, then Y and floor(Y^2 / 2^64), three words
+// each, per y vector) to the warp's slots in shared memory, and lane e reads
+// entry e's two operands from each and multiply-adds in registers, the same
+// instructions for every kind of entry.  The accumulators are loaded and
+// stored once per segment and group.  The record slots use the shared table
+// of per-request constants, which the fit does not use.
 constexpr int kFitRecWords = 6 + 6 * kFitMaxY;
+constexpr int kFitRecs = 4;
+static_assert(sizeof(uint64_t) * kWarps * kFitRecs * kFitRecWords <= sizeof(i128) * 4 * (kNK + 1),
+              "fit record slots fit in the per-request constant table");
 
 struct FitRole {
   int xa, b0, b1, b2;  // record words of x and of B's three words
@@ -598,9 +602,9 @@ __device__ __forceinline__ void fit_group(const TileArgs &a, FitAcc *fw, uint64_
   }
   const FitRole r0 = fit_role(lane, n_y), r1 = fit_role(lane + 32, n_y);
   const bool two = NE > 32;  // lanes 0..NE-33 also own entry lane + 32
-  if (lane == 0) {
-    rec[0] = 1;
-    rec[5] = 0;
+  if (lane < kFitRecs) {
+    rec[lane * kFitRecWords] = 1;
+    rec[lane * kFitRecWords + 5] = 0;
   }
 #pragma unroll 1
   for (int g = 0; g < 4; ++g) {
@@ -617,29 +621,38 @@ __device__ __forceinline__ void fit_group(const TileArgs &a, FitAcc *fw, uint64_
       for (int w = 0; w < 4; ++w) acc1[w] = f1->w[w];
     }
     while (m) {
-      const int j = __ffs(m) - 1;
-      m &= m - 1;
-      __syncwarp();  // the previous record has been read
-      if (lane == j) {
-        rec[1] = (uint64_t)mys.s1;
-        rec[2] = (uint64_t)mys.s2;
-        rec[3] = (uint64_t)mys.s3;
-        rec[4] = (uint64_t)(n * n);
+      uint32_t sel = 0;  // the next (at most) kFitRecs batches of the segment
+#pragma unroll
+      for (int i = 0; i < kFitRecs; ++i) {
+        sel |= m & (0u - m);
+        m &= m - 1;
+      }
+      const int cnt = __popc(sel);
+      __syncwarp();  // the previous records have been read
+      if ((sel >> lane) & 1u) {
+        uint64_t *rw = rec + __popc(sel & ((1u << lane) - 1u)) * kFitRecWords;
+        rw[1] = (uint64_t)mys.s1;
+        rw[2] = (uint64_t)mys.s2;
+        rw[3] = (uint64_t)mys.s3;
+        rw[4] = (uint64_t)(n * n);
 #pragma unroll
         for (int q = 0; q < kFitMaxY; ++q) {
           if (q < n_y) {
-            rec[6 + 6 * q] = Ym[q].lo;
-            rec[7 + 6 * q] = Ym[q].hi;
-            rec[8 + 6 * q] = (uint64_t)((int64_t)Ym[q].hi >> 63);
-            rec[9 + 6 * q] = YYm[q][0];
-            rec[10 + 6 * q] = YYm[q][1];
-            rec[11 + 6 * q] = YYm[q][2];
+            rw[6 + 6 * q] = Ym[q].lo;
+            rw[7 + 6 * q] = Ym[q].hi;
+            rw[8 + 6 * q] = (uint64_t)((int64_t)Ym[q].hi >> 63);
+            rw[9 + 6 * q] = YYm[q][0];
+            rw[10 + 6 * q] = YYm[q][1];
+            rw[11 + 6 * q] = YYm[q][2];
           }
         }
       }
       __syncwarp();
-      fit_entry(acc0, rec, r0, lane == NE - 1);
-      if (two) fit_entry(acc1, rec, r1, lane + 32 == NE - 1);
+      for (int i = 0; i < cnt; ++i) {
+        const uint64_t *rr = rec + i * kFitRecWords;
+        fit_entry(acc0, rr, r0, lane == NE - 1);
+        if (two) fit_entry(acc1, rr, r1, lane + 32 == NE - 1);
+      }
     }
     if (lane < NE) {
 #pragma unroll
@@ -783,11 +796,10 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
   uint32_t *tt = reinterpret_cast<uint32_t *>(smem_raw + sizeof(WSmem));
   constexpr bool kTen = (MODE & M_TEN) != 0;
   constexpr bool kFit = (MODE & M_FIT) != 0;
+  static_assert(!(kFit && (MODE & M_ATTR)), "fit records share the attribution constant table");
   FitAcc *facc = reinterpret_cast<FitAcc *>(smem_raw + sizeof(WSmem) + (kTen ? ten_bytes(a.H) : 0));
   DeferList *dlists = reinterpret_cast<DeferList *>(smem_raw + sizeof(WSmem) + (kTen ? ten_bytes(a.H) : 0) +
                                                     (kFit ? (size_t)kWarps * 4 * fit_entries(a.fit.n_y) * sizeof(FitAcc) : 0));
-  uint64_t *frecs = reinterpret_cast<uint64_t *>(reinterpret_cast<unsigned char *>(dlists) +
-                                                 ((MODE & M_ATTR) ? kWarps * sizeof(DeferList) : 0));
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
   const int NE4 = kFit ? 4 * fit_entries(a.fit.n_y) : 0;
   int bad = 0;
@@ -817,7 +829,7 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
   uint8_t *owner = ws.owner[wid];
   FitAcc *fw = facc + wid * NE4;
   DeferList *dl = dlists + wid;
-  uint64_t *frec = frecs + wid * kFitRecWords;
+  uint64_t *frec = reinterpret_cast<uint64_t *>(&ws.kfix[0][0]) + wid * kFitRecs * kFitRecWords;  // fit mode only
   int dcnt = 0;
   unsigned long long t = 0;
   if (lane == 0) t = atomicAdd(a.ctr, 1ull);
