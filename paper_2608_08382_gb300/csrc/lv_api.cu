@@ -737,7 +737,7 @@ lv_status lv_fit(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y,
   const int n_cta = (int)ctx->last_grid;
   k_fit_reduce<<<n_ent, kFitRedThreads, 0, stream>>>(partial, n_cta, n_ent, totals);
   LV_CUDA(cudaGetLastError());
-  k_fit_solve<<<1, 4 * kFitMaxY, 0, stream>>>(totals, n_y, out);
+  k_fit_solve<<<4 * kFitMaxY, 32, 0, stream>>>(totals, n_y, out);
   LV_CUDA(cudaGetLastError());
   FitOut h[4 * kFitMaxY];
   int hs = 0;

@@ -158,19 +158,38 @@ __host__ __device__ constexpr int gram_idx(int a, int b) {
   return a <= b ? a * 5 - a * (a - 1) / 2 + (b - a) : b * 5 - b * (b - 1) / 2 + (a - b);
 }
 
-// One thread per (y vector, group): builds, scales and solves the normal
-// equations from the exact totals.  Every loop has constant bounds, so the
-// 5x5 system lives in registers; a dropped a3 column becomes a unit row and
-// column with a zero right-hand side (its coefficient solves to 0).  Each
-// pivot is inverted once in double-double and the eliminations multiply.
+// Row and column of Gram entry e (inverse of gram_idx: a <= b, row order).
+__device__ __forceinline__ void gram_ab(int e, int &a, int &b) {
+  a = 0;
+  while (e >= 5 - a) {
+    e -= 5 - a;
+    ++a;
+  }
+  b = a + e;
+}
+
+__device__ __forceinline__ dd dd_sub(dd x, dd y) { return dd_add(x, dd_neg(y)); }
+
+// One warp per (y vector k, group g), block k * 4 + g: builds, scales and
+// solves the normal equations from the exact totals.  Lanes convert the 21
+// totals at once; the Cholesky factorisation goes column by column, the pivot
+// on one lane and the rest of the column on the lanes of its rows; the
+// substitutions run on lane 0; the residual sum of squares adds its 30 terms
+// on 30 lanes.  A dropped a3 column becomes a unit row and column with a zero
+// right-hand side (its coefficient solves to 0).  Each pivot is inverted once
+// in double-double and the eliminations multiply.  Loops stay rolled: the
+// kernel runs once per fit, so its code is fetched cold.
 __global__ void __launch_bounds__(32) k_fit_solve(const FitAcc *__restrict__ totals, int n_y, FitOut *__restrict__ out) {
-  const int t = threadIdx.x;
-  if (t >= 4 * n_y) return;
-  const int k = t / 4, g = t % 4;
+  __shared__ dd G[15], R[5], L[15], rs[5], inv[5], zz[5];
+  __shared__ dd YY;
+  __shared__ double cf[5];
+  __shared__ int sc[5], sing;
+  const int lane = threadIdx.x;
+  const int k = blockIdx.x / 4, g = blockIdx.x % 4;
+  if (k >= n_y) return;
   const int NE = fit_entries(n_y);
   const FitAcc *T = totals + g * NE;
   FitOut o;
-#pragma unroll
   for (int i = 0; i < 5; ++i) o.coef[i] = 0.0;
   o.ssr = 0.0;
   o.r2 = 0.0;
@@ -181,95 +200,102 @@ __global__ void __launch_bounds__(32) k_fit_solve(const FitAcc *__restrict__ tot
   if (drop3) o.dropped = 1 << 3;
   if (n < (drop3 ? 4 : 5)) {
     o.status = LV_ENODATA;
-    out[k * 4 + g] = o;
+    if (lane == 0) out[k * 4 + g] = o;
     return;
   }
-  // exact totals as double-double, each converted once
-  dd Gu[15], ru[5];
-#pragma unroll
-  for (int i = 0; i < 15; ++i) Gu[i] = int256_to_dd(T[i].w, 0);
-#pragma unroll
-  for (int a = 0; a < 5; ++a) ru[a] = int256_to_dd(T[15 + k * 5 + a].w, kFitYLsb);
-  if (drop3) {
-#pragma unroll
-    for (int a = 0; a < 5; ++a) Gu[gram_idx(a, 3)] = dd{a == 3 ? 1.0 : 0.0, 0.0};
-    ru[3] = dd{0.0, 0.0};
-  }
+  // exact totals as double-double, one per lane
+  if (lane < 15)
+    G[lane] = int256_to_dd(T[lane].w, 0);
+  else if (lane < 20)
+    R[lane - 15] = int256_to_dd(T[15 + k * 5 + (lane - 15)].w, kFitYLsb);
+  else if (lane == 20)
+    YY = int256_to_dd(T[15 + 5 * n_y + k].w, kFitYYLsb);
+  if (lane == 0) sing = 0;
+  __syncwarp();
+  if (drop3 && lane < 5) G[gram_idx(lane, 3)] = dd{lane == 3 ? 1.0 : 0.0, 0.0};
+  if (drop3 && lane == 5) R[3] = dd{0.0, 0.0};
+  __syncwarp();
   // power-of-two column scaling: scaled diagonal near 1
-  int sc[5];
-#pragma unroll
-  for (int i = 0; i < 5; ++i) {
+  if (lane < 5) {
     int ex;
-    frexp(Gu[gram_idx(i, i)].hi, &ex);
-    sc[i] = -(ex / 2);
+    frexp(G[gram_idx(lane, lane)].hi, &ex);
+    sc[lane] = -(ex / 2);
   }
-  dd L[15], r[5], inv[5];
-#pragma unroll
-  for (int i = 0; i < 5; ++i) {
-#pragma unroll
-    for (int j = 0; j <= i; ++j) L[gram_idx(i, j)] = dd_scale(Gu[gram_idx(i, j)], sc[i] + sc[j]);
-    r[i] = dd_scale(ru[i], sc[i]);
+  __syncwarp();
+  if (lane < 15) {
+    int a, b;
+    gram_ab(lane, a, b);
+    L[lane] = dd_scale(G[lane], sc[a] + sc[b]);
+  } else if (lane < 20) {
+    rs[lane - 15] = dd_scale(R[lane - 15], sc[lane - 15]);
   }
+  __syncwarp();
   // Cholesky G = L L^T (lower triangle in L, indexed symmetrically)
-#pragma unroll
   for (int j = 0; j < 5; ++j) {
-    dd d = L[gram_idx(j, j)];
-#pragma unroll
-    for (int m = 0; m < j; ++m) d = dd_add(d, dd_neg(dd_mul(L[gram_idx(j, m)], L[gram_idx(j, m)])));
-    if (!(d.hi > 1e-24)) {
+    if (lane == j) {
+      dd d = L[gram_idx(j, j)];
+      for (int m = 0; m < j; ++m) d = dd_sub(d, dd_mul(L[gram_idx(j, m)], L[gram_idx(j, m)]));
+      if (!(d.hi > 1e-24)) {
+        sing = 1;
+      } else {
+        // square root in double-double: s0 = sqrt(d.hi), one Newton step
+        const double s0 = sqrt(d.hi);
+        const dd s0sq = dd_mul(dd{s0, 0.0}, dd{s0, 0.0});
+        const dd s = dd_add(dd{s0, 0.0}, dd_div(dd_sub(d, s0sq), dd{2.0 * s0, 0.0}));
+        L[gram_idx(j, j)] = s;
+        inv[j] = dd_div(dd{1.0, 0.0}, s);
+      }
+    }
+    __syncwarp();
+    if (sing) {
       o.status = LV_ESINGULAR;
-      out[k * 4 + g] = o;
+      if (lane == 0) out[k * 4 + g] = o;
       return;
     }
-    // square root in double-double: s0 = sqrt(d.hi), one Newton step
-    const double s0 = sqrt(d.hi);
-    const dd s0sq = dd_mul(dd{s0, 0.0}, dd{s0, 0.0});
-    const dd s = dd_add(dd{s0, 0.0}, dd_div(dd_add(d, dd_neg(s0sq)), dd{2.0 * s0, 0.0}));
-    L[gram_idx(j, j)] = s;
-    inv[j] = dd_div(dd{1.0, 0.0}, s);
-#pragma unroll
-    for (int i = j + 1; i < 5; ++i) {
-      dd v = L[gram_idx(i, j)];
-#pragma unroll
-      for (int m = 0; m < j; ++m) v = dd_add(v, dd_neg(dd_mul(L[gram_idx(i, m)], L[gram_idx(j, m)])));
-      L[gram_idx(i, j)] = dd_mul(v, inv[j]);
+    if (lane > j && lane < 5) {
+      dd v = L[gram_idx(lane, j)];
+      for (int m = 0; m < j; ++m) v = dd_sub(v, dd_mul(L[gram_idx(lane, m)], L[gram_idx(j, m)]));
+      L[gram_idx(lane, j)] = dd_mul(v, inv[j]);
+    }
+    __syncwarp();
+  }
+  if (lane == 0) {
+    for (int i = 0; i < 5; ++i) {
+      dd v = rs[i];
+      for (int m = 0; m < i; ++m) v = dd_sub(v, dd_mul(L[gram_idx(i, m)], zz[m]));
+      zz[i] = dd_mul(v, inv[i]);
+    }
+    for (int i = 4; i >= 0; --i) {
+      dd v = zz[i];
+      for (int m = i + 1; m < 5; ++m) v = dd_sub(v, dd_mul(L[gram_idx(m, i)], zz[m]));
+      zz[i] = dd_mul(v, inv[i]);  // the solution overwrites z, highest index first
+      cf[i] = (drop3 && i == 3) ? 0.0 : ldexp(zz[i].hi + zz[i].lo, sc[i]);
     }
   }
-  dd z[5], a[5];
-#pragma unroll
-  for (int i = 0; i < 5; ++i) {
-    dd v = r[i];
-#pragma unroll
-    for (int m = 0; m < i; ++m) v = dd_add(v, dd_neg(dd_mul(L[gram_idx(i, m)], z[m])));
-    z[i] = dd_mul(v, inv[i]);
+  __syncwarp();
+  for (int i = 0; i < 5; ++i) o.coef[i] = cf[i];
+  // residuals of the rounded coefficients: SSR = y'y - 2 c'X'y + c'Gc (unscaled),
+  // one term per lane, summed across the warp
+  dd term{0.0, 0.0};
+  if (lane < 25) {
+    const int i = lane / 5, j = lane % 5;
+    term = dd_mul(dd_mul(dd{cf[i], 0.0}, dd{cf[j], 0.0}), G[gram_idx(i, j)]);
+  } else if (lane < 30) {
+    term = dd_neg(dd_scale(dd_mul(dd{cf[lane - 25], 0.0}, R[lane - 25]), 1));
   }
 #pragma unroll
-  for (int i = 4; i >= 0; --i) {
-    dd v = z[i];
-#pragma unroll
-    for (int m = i + 1; m < 5; ++m) v = dd_add(v, dd_neg(dd_mul(L[gram_idx(m, i)], a[m])));
-    a[i] = dd_mul(v, inv[i]);
+  for (int d = 16; d; d >>= 1)
+    term = dd_add(term, dd{__shfl_xor_sync(0xffffffffu, term.hi, d), __shfl_xor_sync(0xffffffffu, term.lo, d)});
+  if (lane == 0) {
+    const dd sy = R[0];
+    const dd ssr = dd_add(YY, term);
+    const dd sst = dd_sub(YY, dd_div(dd_mul(sy, sy), dd{(double)n, 0.0}));
+    o.ssr = ssr.hi + ssr.lo;
+    const double sstv = sst.hi + sst.lo;
+    o.r2 = sstv != 0.0 ? 1.0 - o.ssr / sstv : __longlong_as_double(0x7ff8000000000000ll);
+    o.status = LV_OK;
+    out[k * 4 + g] = o;
   }
-#pragma unroll
-  for (int i = 0; i < 5; ++i) o.coef[i] = (drop3 && i == 3) ? 0.0 : ldexp(a[i].hi + a[i].lo, sc[i]);
-  // residuals of the rounded coefficients: SSR = y'y - 2 c'X'y + c'Gc (unscaled)
-  dd cxy{0.0, 0.0}, cgc{0.0, 0.0};
-#pragma unroll
-  for (int i = 0; i < 5; ++i) {
-    const dd ci{o.coef[i], 0.0};
-    cxy = dd_add(cxy, dd_mul(ci, ru[i]));
-#pragma unroll
-    for (int j = 0; j < 5; ++j) cgc = dd_add(cgc, dd_mul(dd_mul(ci, dd{o.coef[j], 0.0}), Gu[gram_idx(i, j)]));
-  }
-  const dd sy = ru[0];
-  const dd yy = int256_to_dd(T[15 + 5 * n_y + k].w, kFitYYLsb);
-  const dd ssr = dd_add(dd_add(yy, dd_neg(dd_scale(cxy, 1))), cgc);
-  const dd sst = dd_add(yy, dd_neg(dd_div(dd_mul(sy, sy), dd{(double)n, 0.0})));
-  o.ssr = ssr.hi + ssr.lo;
-  const double sstv = sst.hi + sst.lo;
-  o.r2 = sstv != 0.0 ? 1.0 - o.ssr / sstv : __longlong_as_double(0x7ff8000000000000ll);
-  o.status = LV_OK;
-  out[k * 4 + g] = o;
 }
 
 }  // namespace lv
