@@ -238,12 +238,15 @@ __global__ void __launch_bounds__(32) k_fit_solve(const FitAcc *__restrict__ tot
       if (!(d.hi > 1e-24)) {
         sing = 1;
       } else {
-        // square root in double-double: s0 = sqrt(d.hi), one Newton step
-        const double s0 = sqrt(d.hi);
+        // square root in double-double: s0 = sqrt(d.hi) and one Newton step, whose
+        // correction needs only a double factor 1/(2 s0); the inverse by one
+        // Newton step from the double reciprocal r0 = 1/s0
+        const double s0 = sqrt(d.hi), r0 = 1.0 / s0;
         const dd s0sq = dd_mul(dd{s0, 0.0}, dd{s0, 0.0});
-        const dd s = dd_add(dd{s0, 0.0}, dd_div(dd_sub(d, s0sq), dd{2.0 * s0, 0.0}));
+        const dd s = dd_add(dd{s0, 0.0}, dd_mul(dd_sub(d, s0sq), dd{0.5 * r0, 0.0}));
         L[gram_idx(j, j)] = s;
-        inv[j] = dd_div(dd{1.0, 0.0}, s);
+        const dd e = dd_sub(dd{1.0, 0.0}, dd_mul(s, dd{r0, 0.0}));
+        inv[j] = dd_add(dd{r0, 0.0}, dd_mul(dd{r0, 0.0}, e));
       }
     }
     __syncwarp();
