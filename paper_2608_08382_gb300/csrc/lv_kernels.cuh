@@ -496,8 +496,10 @@ struct SegS {
   int pad;
 };
 
+// fx: the segments' fixed-point parameters (a shared-memory copy in k_warps,
+// where the lanes of a warp take different segments).
 template <int MODE>
-__device__ __forceinline__ void emit_batch(const TileArgs &a, int64_t gb, const BatchAgg &g, int s) {
+__device__ __forceinline__ void emit_batch(const TileArgs &a, int64_t gb, const BatchAgg &g, int s, const SegFix *fx) {
   if (MODE & M_FEAT) {
     if (a.bfeat) {
       a.bfeat[gb] = g.s1;
@@ -512,7 +514,7 @@ __device__ __forceinline__ void emit_batch(const TileArgs &a, int64_t gb, const 
     double T;
     if (!(MODE & M_FIX))
       T = eq1_fp64(a.mp.coef[s], g);
-    else if (!eq1_fast(a.mp.fx[s], g, &T))
+    else if (!eq1_fast(fx[s], g, &T))
       T = eq1_fix(a.mp, s, g);
     a.T[gb] = T;
   }

@@ -47,6 +47,7 @@ struct WSmem {
   alignas(16) uint8_t kslow[4][kNK + 4];  // 1: K outside the fixed-point range
   alignas(16) uint8_t owner[kWarps][32];  // small-batch rounds: head slot -> lane
   alignas(16) Sums gsum[kWarps][32];      // sums of the group's big batches (kept out of registers)
+  alignas(16) SegFix fx[4];               // Eq. 1 parameters (lanes of a warp read different segments)
 };
 static_assert(sizeof(WSmem) % 16 == 0, "tenant table follows WSmem");
 
@@ -759,7 +760,7 @@ __device__ __forceinline__ void process_group(const TileArgs &a, WSmem &ws, uint
   if (valid && !jumbo) {
     const BatchAgg g{mys.s1, mys.s2, mys.s3, n, mys.ph > 0};
     const int s = segment_of(a.mp, g);
-    emit_batch<MODE>(a, g0 + lane, g, s);
+    emit_batch<MODE>(a, g0 + lane, g, s, ws.fx);
     if (MODE & M_FIT) {
       const bool in_range = g.s1 < kFitFeatMax && g.s2 < kFitFeatMax && g.s3 < kFitFeatMax &&
                             (int64_t)n * n < kFitFeatMax;
@@ -808,6 +809,7 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
     for (int i = tid; i < 4 * ten_plane(a.H); i += kWThreads) tt[i] = 0;
   if (kFit)
     for (int i = tid; i < kWarps * NE4; i += kWThreads) facc[i] = FitAcc{{0, 0, 0, 0}};
+  if ((MODE & M_ATTR) && tid < 4) ws.fx[tid] = a.mp.fx[tid];
   if (MODE & M_ATTR) {
     init_segs<MODE>(a, ws.seg);
     if (MODE & M_FIX) {
@@ -919,7 +921,7 @@ __global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_bas
     const Sums tot = js.tot;
     const BatchAgg g{tot.s1, tot.s2, tot.s3, r1 - r0, tot.ph > 0};
     const int s = segment_of(a.mp, g);
-    if (tid == 0) emit_batch<MODE>(a, b, g, s);
+    if (tid == 0) emit_batch<MODE>(a, b, g, s, a.mp.fx);
     if (kFit) {
       const int NE = fit_entries(a.fit.n_y);
       const int64_t x[5] = {1, g.s1, g.s2, g.s3, g.n * g.n};
