@@ -445,15 +445,17 @@ __device__ __forceinline__ void big_shares_fast(const TileArgs &a, uint32_t *tt,
 
 // Rounds over the small batches of a group (lanes with `small`): every round
 // takes the next batches whose requests fit in 32 slots, one request per lane.
-// Pass SHARE=false reduces (each small lane receives its batch's sums in
-// `mys`); SHARE=true attributes with the per-lane constants (myk, mymeta).
-// pn: the lane's request count (0 for other lanes); P: exclusive prefix of pn;
-// base = o0 - P so that slot q of the lane's batch is request base + q.
-// mymeta = n << 4 | fast << 3 | slow << 2 | segment.
-template <int MODE, bool SHARE>
+// A segmented scan gives each batch's sums to its lane (`mys`).  With
+// attribution the same round then forms those batches' constants on their
+// lanes and attributes the round's requests, whose fields are still in
+// registers: a batch lies within one round.  pn: the lane's request count (0
+// for other lanes); P: exclusive prefix of pn; base = o0 - P so that slot q of
+// the lane's batch is request base + q.  meta = n << 4 | fast << 3 | slow << 2
+// | segment.
+template <int MODE>
 __device__ __forceinline__ void small_rounds(const TileArgs &a, const WSmem &ws, uint32_t *tt, uint8_t *owner,
                                              DeferList *dl, int &dcnt, bool small, int pn, int P, int64_t base,
-                                             Sums &mys, i128 myk, int mymeta, int lane, int *bad) {
+                                             Sums &mys, int lane, int *bad) {
   uint32_t rem = __ballot_sync(kFull, small);
   while (rem) {
     const int start = __shfl_sync(kFull, P, __ffs(rem) - 1);
@@ -468,39 +470,47 @@ __device__ __forceinline__ void small_rounds(const TileArgs &a, const WSmem &ws,
     const int hp = act ? 31 - __clz(H & ((2u << lane) - 1u)) : 0;  // head slot of this lane's batch
     const int j = owner[hp];
     const int64_t r = __shfl_sync(kFull, base, j) + start + lane;
-    if (!SHARE) {
-      Sums v{0, 0, 0, 0};
-      if (act) {
-        int32_t p = a.p[r], c = a.c[r], ph = a.ph[r];
-        check_req(p, c, ph, bad);
-        v = Sums{p, c, (int64_t)p * p, ph};
+    Sums v{0, 0, 0, 0};
+    int32_t p = 0, c = 0, ph = 0;
+    if (act) {
+      p = a.p[r];
+      c = a.c[r];
+      ph = a.ph[r];
+      check_req(p, c, ph, bad);  // clamped: the share paths clamp the same way
+      v = Sums{p, c, (int64_t)p * p, ph};
+    }
+    const int maxn = __reduce_max_sync(kFull, in ? pn : 0);
+    for (int d = 1; d < maxn; d <<= 1) {
+      const Sums w{__shfl_up_sync(kFull, v.s1, d), __shfl_up_sync(kFull, v.s2, d),
+                   __shfl_up_sync(kFull, v.s3, d), __shfl_up_sync(kFull, v.ph, d)};
+      if (lane - d >= hp) v = add_sums(v, w);
+    }
+    const Sums tot = shfl_sums(v, in ? P - start + pn - 1 : 0);
+    if (in) mys = tot;
+    if (MODE & M_ATTR) {
+      i128 myk = mk128(0, 0);
+      int mymeta = 0;
+      if (in) {
+        const BatchAgg g{mys.s1, mys.s2, mys.s3, pn, mys.ph > 0};
+        const int s = segment_of(a.mp, g);
+        bool slow = false;
+        myk = batch_const_w<MODE>(a, &ws, s, pn, &slow);
+        const bool fast = (MODE & M_FIX) && !slow && ws.seg[s].a2_narrow;
+        mymeta = (pn << 4) | (fast ? 8 : 0) | (slow ? 4 : 0) | s;
       }
-      const int maxn = __reduce_max_sync(kFull, in ? pn : 0);
-      for (int d = 1; d < maxn; d <<= 1) {
-        const Sums w{__shfl_up_sync(kFull, v.s1, d), __shfl_up_sync(kFull, v.s2, d),
-                     __shfl_up_sync(kFull, v.s3, d), __shfl_up_sync(kFull, v.ph, d)};
-        if (lane - d >= hp) v = add_sums(v, w);
-      }
-      const Sums tot = shfl_sums(v, in ? P - start + pn - 1 : 0);
-      if (in) mys = tot;
-    } else {
       const uint64_t klo = __shfl_sync(kFull, myk.lo, j), khi = __shfl_sync(kFull, myk.hi, j);
       const int meta = __shfl_sync(kFull, mymeta, j);
-      const i128 kf = mk128(klo, khi);
       bool done = true;
-      int32_t p = 0, c = 0, u = 0;
+      int32_t u = 0;
       if (act) {
-        const int s = meta & 3;
         done = false;
-        p = a.p[r];
-        c = a.c[r];
         u = (MODE & M_TEN) ? a.ten[r] : 0;
         if (meta & 8) {
-          const SegS &sg = ws.seg[s];
-          const i128 K13 = add128(kf, sg.A13);
+          const SegS &sg = ws.seg[meta & 3];
+          const i128 K13 = add128(mk128(klo, khi), sg.A13);
           uint32_t v0, v1, v2, v3;
           mad_k13((uint32_t)K13.lo, (uint32_t)(K13.lo >> 32), (uint32_t)K13.hi, (uint32_t)(K13.hi >> 32),
-                  (uint32_t)sg.A2.lo, (uint32_t)(sg.A2.lo >> 32), (uint32_t)(c < 0 ? 0 : c), v0, v1, v2, v3);
+                  (uint32_t)sg.A2.lo, (uint32_t)(sg.A2.lo >> 32), (uint32_t)c, v0, v1, v2, v3);
           uint64_t m;
           int ex2;
           const double d = round96(v0, v1, v2, sg.E, m, ex2);
@@ -696,8 +706,6 @@ __device__ __forceinline__ void process_group(const TileArgs &a, WSmem &ws, uint
       *bad = 1;
   }
   Sums mys{0, 0, 0, 0};
-  i128 myk = mk128(0, 0);
-  int mymeta = 0;
   Sums *gsum = ws.gsum[threadIdx.x >> 5];
 
   // ---- big batches: reduce, constant and shares one batch at a time
@@ -741,18 +749,7 @@ __device__ __forceinline__ void process_group(const TileArgs &a, WSmem &ws, uint
     const int pn = small ? n : 0;
     const int P = warp_excl_scan_int(pn, lane);
     const int64_t base = o0 - P;
-    small_rounds<MODE, false>(a, ws, tt, owner, dl, dcnt, small, pn, P, base, mys, myk, 0, lane, bad);
-    if (kAttr) {
-      if (small) {
-        const BatchAgg g{mys.s1, mys.s2, mys.s3, n, mys.ph > 0};
-        const int s = segment_of(a.mp, g);
-        bool slow = false;
-        myk = batch_const_w<MODE>(a, &ws, s, n, &slow);
-        const bool fast = (MODE & M_FIX) && !slow && ws.seg[s].a2_narrow;
-        mymeta = (n << 4) | (fast ? 8 : 0) | (slow ? 4 : 0) | s;
-      }
-      small_rounds<MODE, true>(a, ws, tt, owner, dl, dcnt, small, pn, P, base, mys, myk, mymeta, lane, bad);
-    }
+    small_rounds<MODE>(a, ws, tt, owner, dl, dcnt, small, pn, P, base, mys, lane, bad);
   }
 
   // ---- per batch: T, features; fit statistics
