@@ -9,13 +9,15 @@ arrays resident in HBM; they are ~2.2 GB, far larger than L2, so no flush is
 needed between steps.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--workload attr1|attr4|fit2|whatif3] [--scale X] [--no-cpu-baseline]
+                    [--workload attr1|attr4|fit2|whatif3|step] [--scale X] [--no-cpu-baseline]
 
 attr1 (the default) is the headline line.  attr4 is the skew stress, fit2 the
 coefficient fit over 2e6 profiled batches (one step = lv_fit of a noisy and a
 noiseless latency vector), whatif3 the what-if pairs (one step = lv_whatif over
-4096 pending x 1024 candidates); each prints a line of the same shape with its
-own metric and the roofline of its dominant kernel.
+4096 pending x 1024 candidates), step the single-step scheduler mode (one
+batch of 2048 requests per step, replayed from a CUDA graph; the line adds
+us_per_step); each prints a line of the same shape with its own metric and the
+roofline of its dominant kernel.
 
 Prints one JSON line.  Under torchrun each rank processes its own replica of
 the workload (weak scaling, no collective on the data path); timing takes the
@@ -165,6 +167,7 @@ def barrier(world):
 
 METRIC_FIT = "profiled requests/sec through the coefficient fit on 1 GB300"
 METRIC_WHATIF = "what-if (pending request, candidate batch) pairs/sec on 1 GB300"
+METRIC_STEP = "attributed requests/sec, one 2048-request serving step per CUDA-graph replay on 1 GB300"
 
 WORKLOADS = {
     "attr1": ("attr", 1, "qwen2.5-14b tp2 continuous batching: 1e6 batches U{16..256}, ~136M requests, "
@@ -175,6 +178,8 @@ WORKLOADS = {
                        "and noiseless latency vectors fitted in one pass"),
     "whatif3": ("whatif", 3, "qwen2.5-32b tp4 what-if: 1024 candidate batches U{32..256} x 4096 pending requests, "
                              "4,194,304 pairs"),
+    "step": ("step", 5, "qwen2.5-14b tp2 serving step: one batch of 2048 requests (4 chunked prefills), "
+                        "256 Zipf(1.1) tenants, replayed from a CUDA graph"),
 }
 
 
@@ -183,6 +188,8 @@ def _workload(args):
     kind, k_cfg, desc = WORKLOADS[args.workload]
     if kind == "whatif":
         w = workloads.whatif_config(scale=args.scale)
+    elif kind == "step":
+        w = workloads.step_config(n_req=max(1, int(round(2048 * args.scale))))
     else:
         w = workloads.config(k_cfg, scale=args.scale)
     if args.scale != 1.0:
@@ -225,6 +232,64 @@ def _setup_attr(lv, ctx, w, stream):
                 bytes_rule="24 B/request (p, c, phase, tenant read; share written) + 16 B/batch (offset read; T written)",
                 config={"n_batch": w.n_batch, "n_req": w.n_req, "n_tenants": w.n_tenants, "seed": w.seed,
                         "step": "lv_attribute(T, shares, tenant pass) + lv_tenant_totals"})
+
+
+def _setup_step(lv, ctx, w, stream):
+    """Step: one serving batch through a CUDA graph of lv_tenant_acc_reset + lv_attribute (T, shares, tenant
+    pass) + lv_tenant_totals, captured once on a side stream (after eager warm-up there) and replayed."""
+    import torch
+    b = lv.batches_to_device(w.p, w.c, w.phase, w.offsets, w.tenant, w.n_tenants)
+    model = lv.make_model(w.coef, w.split)
+    T = torch.empty(w.n_batch, dtype=torch.float64, device="cuda")
+    share = torch.empty(w.n_req, dtype=torch.float64, device="cuda")
+    L = torch.empty(w.n_tenants, dtype=torch.float64, device="cuda")
+    acc = lv.TenantAcc(ctx, w.n_tenants)
+
+    def eager(st):
+        acc.reset(stream=st)
+        lv.lv_attribute(ctx, model, b, T, share, acc, stream=st)
+        lv.lv_tenant_totals(ctx, acc, L, stream=st)
+
+    cs = torch.cuda.Stream()
+    cs.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(cs):
+        for _ in range(3):
+            eager(cs)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=cs):
+        eager(cs)
+    torch.cuda.synchronize()
+
+    def step():
+        graph.replay()
+
+    hp = {k: torch.from_numpy(np.ascontiguousarray(v)).pin_memory()
+          for k, v in dict(p=w.p, c=w.c, phase=w.phase, tenant=w.tenant, offsets=w.offsets).items()}
+    h_share = torch.empty(w.n_req, dtype=torch.float64).pin_memory()
+    h_T = torch.empty(w.n_batch, dtype=torch.float64).pin_memory()
+    h_L = torch.empty(w.n_tenants, dtype=torch.float64).pin_memory()
+
+    def e2e_step():
+        for name in ("p", "c", "phase", "tenant", "offsets"):
+            getattr(b, name).copy_(hp[name], non_blocking=True)
+        eager(stream)
+        h_share.copy_(share, non_blocking=True)
+        h_T.copy_(T, non_blocking=True)
+        h_L.copy_(L, non_blocking=True)
+
+    return dict(step=step, e2e_step=e2e_step, units=w.n_req, unit="requests/s", metric=METRIC_STEP,
+                h2d=sum(int(t.numel() * t.element_size()) for t in hp.values()),
+                d2h=8 * (w.n_req + w.n_batch + w.n_tenants), launches_per_step=5,
+                kernel="graph", time_mask=0, graph=True, flush=True,
+                bytes_per_launch=24.0 * w.n_req + 16.0 * w.n_batch,
+                bytes_rule="24 B/request + 16 B/batch over the whole replay (memsets, k_partition, k_warps, k_jumbo, "
+                           "k_tenant_fold, k_tenant_totals): a single batch is bound by launch latency, not HBM",
+                config={"n_batch": w.n_batch, "n_req": w.n_req, "n_tenants": w.n_tenants, "seed": w.seed,
+                        "l2": "working set below L2 size: a 512 MB buffer is overwritten before every timed step, "
+                              "outside the step's events",
+                        "step": "CUDA-graph replay of lv_tenant_acc_reset + lv_attribute(T, shares, tenant pass) + "
+                                "lv_tenant_totals"})
 
 
 def _setup_fit(lv, ctx, w, stream):
@@ -315,7 +380,8 @@ def run_ours(args, world, rank, local):
     kind, w, desc = _workload(args)
     ctx = lv.Context()
     stream = torch.cuda.current_stream()
-    s = {"attr": _setup_attr, "fit": _setup_fit, "whatif": _setup_whatif}[kind](lv, ctx, w, stream)
+    s = {"attr": _setup_attr, "fit": _setup_fit, "whatif": _setup_whatif, "step": _setup_step}[kind](
+        lv, ctx, w, stream)
     step = s["step"]
 
     for _ in range(args.warmup):
@@ -377,10 +443,13 @@ def run_ours(args, world, rank, local):
     step_ms = ms_max / args.steps
     value = world * s["units"] / (step_ms / 1e3)
     kavg_ms = kms / max(klaunch, 1)
+    if s.get("graph"):
+        kavg_ms, klaunch = step_ms, args.steps  # the replay is the timed unit
     achieved = s["bytes_per_launch"] / (kavg_ms / 1e3) / 1e9
     peak, peak_kind = measured_peaks()
     traffic = ncu_traffic(s["kernel"], args.workload)
-    timed = ("k_warps + k_jumbo, one event pair per launch pair" if s["kernel"] == "k_warps" else s["kernel"])
+    timed = ("k_warps + k_jumbo, one event pair per launch pair" if s["kernel"] == "k_warps" else
+             "the whole CUDA-graph replay, CUDA events on the launching stream" if s.get("graph") else s["kernel"])
     config = {"workload": desc, **s["config"], "parallelism": f"replicas{world}"}
     config.setdefault("l2", "inputs far larger than the 129 MB L2, no flush")
     line = {
@@ -407,6 +476,8 @@ def run_ours(args, world, rank, local):
         "clocks": clk,
         "status": lv.lv_status_string(status),
     }
+    if s.get("graph"):
+        line["us_per_step"] = step_ms * 1e3
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(kind, w, min_seconds=args.cpu_seconds)
     return line
@@ -426,6 +497,13 @@ def _oracle_sample(kind, w):
         def run():
             oracle.whatif(c.offsets, c.p, c.c, c.phase, pn, cn, phn, w.split, w.coef)
         return run, rows * c.n_batch, f"first {rows} of {w.n_pending} pending requests x all {c.n_batch} candidates"
+    if kind == "step":
+        t = w.tenant
+
+        def run():
+            _, s = oracle.attribute(w.offsets, w.p, w.c, w.phase, w.split, w.coef)
+            oracle.tenant_totals(s, t, w.n_tenants)
+        return run, w.n_req, f"the whole batch ({w.n_req} requests), attribution + tenant totals"
     frac = 10 if kind == "attr" else 200
     nb = max(1, w.n_batch // frac)
     hi = int(w.offsets[nb])
@@ -476,7 +554,7 @@ def run_reference(args, world, rank):
     el = time.perf_counter() - t0
     value = units * args.steps / el
     unit = "pairs/s" if kind == "whatif" else "requests/s"
-    metric = {"attr": METRIC, "fit": METRIC_FIT, "whatif": METRIC_WHATIF}[kind]
+    metric = {"attr": METRIC, "fit": METRIC_FIT, "whatif": METRIC_WHATIF, "step": METRIC_STEP}[kind]
     return {"impl": "reference", "metric": metric, "value": value, "unit": unit, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",

@@ -37,6 +37,15 @@
  *    16-byte aligned (they are read with bulk asynchronous copies), fp64 outputs
  *    8-byte aligned; otherwise LV_EINVAL.
  *  - One lv_ctx must not be used from two host threads at once.
+ *  - CUDA graphs: lv_features, lv_batch_latency, lv_attribute,
+ *    lv_tenant_acc_reset, lv_tenant_accumulate, lv_tenant_totals and
+ *    lv_whatif may be captured into a CUDA graph once an uncaptured call with
+ *    the same context, model and sizes has run (it creates the context's
+ *    buffers and caches the kernel configuration; a capture never allocates).
+ *    The context's ordering events are then recorded and waited for by the
+ *    graph itself at each replay; library timing (lv_ctx_set_timing) skips
+ *    captured launches.  lv_fit, lv_ctx_status and lv_tenant_acc_export /
+ *    import synchronise and cannot be captured.
  */
 #ifndef LLMVISOR_H
 #define LLMVISOR_H

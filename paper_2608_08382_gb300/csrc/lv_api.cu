@@ -186,6 +186,25 @@ lv_status ensure_tiles(lv_ctx *ctx, int64_t n) {
 }
 
 // Builds (or reuses) the per-model parameters and K table on `stream`.
+// Event record and wait that stay valid while `stream` is being captured into a
+// CUDA graph: the graph then records (waits for) the event itself at every
+// replay, so a captured call still orders itself after the context's earlier
+// work on other streams, and later calls after the replay.
+bool capturing(cudaStream_t stream) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  return cudaStreamIsCapturing(stream, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusActive;
+}
+
+lv_status record_event(cudaEvent_t ev, cudaStream_t stream) {
+  LV_CUDA(cudaEventRecordWithFlags(ev, stream, capturing(stream) ? cudaEventRecordExternal : cudaEventRecordDefault));
+  return LV_OK;
+}
+
+lv_status wait_event(cudaStream_t stream, cudaEvent_t ev) {
+  LV_CUDA(cudaStreamWaitEvent(stream, ev, capturing(stream) ? cudaEventWaitExternal : cudaEventWaitDefault));
+  return LV_OK;
+}
+
 lv_status prepare_model(lv_ctx *ctx, const lv_model *m, cudaStream_t stream, ModelP *mp) {
   std::memset(mp, 0, sizeof(*mp));
   for (int s = 0; s < 4; ++s) {
@@ -209,25 +228,29 @@ lv_status prepare_model(lv_ctx *ctx, const lv_model *m, cudaStream_t stream, Mod
                     std::memcmp(&ctx->ktab_model, m, sizeof(lv_model)) == 0;
   if (!same) {
     // wait for earlier users of the table on any stream
-    LV_CUDA(cudaStreamWaitEvent(stream, ctx->ev_used, 0));
+    lv_status st = wait_event(stream, ctx->ev_used);
+    if (st != LV_OK) return st;
     const int n = 4 * (kKTableN + 1);
     k_ktable<<<(n + 255) / 256, 256, 0, stream>>>(*mp, ctx->d_ktab);
     LV_CUDA(cudaGetLastError());
-    LV_CUDA(cudaEventRecord(ctx->ev_built, stream));
+    st = record_event(ctx->ev_built, stream);
+    if (st != LV_OK) return st;
     ctx->ktab_model = *m;
     ctx->ktab_fixed = mp->fixed;
     ctx->ktab_valid = true;
     ctx->ktab_stream = stream;
   } else if (stream != ctx->ktab_stream) {
-    LV_CUDA(cudaStreamWaitEvent(stream, ctx->ev_built, 0));
+    lv_status st = wait_event(stream, ctx->ev_built);
+    if (st != LV_OK) return st;
   }
   return LV_OK;
 }
 
-// Event pair around a measured launch (when timing is on).
+// Event pair around a measured launch (when timing is on; not while the stream
+// is being captured into a graph).
 lv_status timing_begin(lv_ctx *ctx, int kind, cudaStream_t stream, cudaEvent_t *stop) {
   *stop = nullptr;
-  if (!(ctx->timing & kind)) return LV_OK;
+  if (!(ctx->timing & kind) || capturing(stream)) return LV_OK;
   if (ctx->tev_used + 2 > ctx->tev.size()) {
     for (int k = 0; k < 2; ++k) {
       cudaEvent_t e;
@@ -286,7 +309,9 @@ lv_status launch_warps_mode(lv_ctx *ctx, int sms, TileArgs &a, cudaStream_t stre
   }
   const int64_t grid = std::min<int64_t>(a.n_tiles, (int64_t)sms * per_sm);
   if (grid <= 0) return LV_OK;
-  const int64_t jgrid = (int64_t)sms * kJumboCtasPerSm;
+  // k_jumbo: at most one CTA per batch that can exceed kJumbo requests (none
+  // for small inputs, e.g. a single serving step of a few hundred requests)
+  const int64_t jgrid = std::min<int64_t>((int64_t)sms * kJumboCtasPerSm, a.n_req / (kJumbo + 1));
   cudaEvent_t stop = nullptr;
   if (ctx) {
     lv_status st = timing_begin(ctx, LV_TIME_TILES, stream, &stop);
@@ -294,8 +319,10 @@ lv_status launch_warps_mode(lv_ctx *ctx, int sms, TileArgs &a, cudaStream_t stre
   }
   k_warps<MODE><<<(unsigned)grid, kWThreads, smem, stream>>>(a);
   LV_CUDA(cudaGetLastError());
-  k_jumbo<MODE><<<(unsigned)jgrid, kJBlock, jsmem, stream>>>(a, (int)grid);
-  LV_CUDA(cudaGetLastError());
+  if (jgrid > 0) {
+    k_jumbo<MODE><<<(unsigned)jgrid, kJBlock, jsmem, stream>>>(a, (int)grid);
+    LV_CUDA(cudaGetLastError());
+  }
   *ctas = grid + jgrid;
   return ctx ? timing_end(stop, stream) : LV_OK;
 }
@@ -554,7 +581,8 @@ lv_status lv_batch_latency(lv_ctx *ctx, const lv_model *model, const int64_t *ba
     k_batch_latency<false><<<(unsigned)blocks, 256, 0, stream>>>(mp, batch_feat, batch_seg, n_batch, T,
                                                                  ctx->d_status);
   LV_CUDA(cudaGetLastError());
-  LV_CUDA(cudaEventRecord(ctx->ev_used, stream));
+  st = record_event(ctx->ev_used, stream);
+  if (st != LV_OK) return st;
   return LV_OK;
 }
 
@@ -593,7 +621,8 @@ lv_status lv_attribute(lv_ctx *ctx, const lv_model *model, const lv_batches *b, 
   }
   st = run_tiles(ctx, a, mode, stream);
   if (st != LV_OK) return st;
-  LV_CUDA(cudaEventRecord(ctx->ev_used, stream));
+  st = record_event(ctx->ev_used, stream);
+  if (st != LV_OK) return st;
   if (acc) return fold_tenants(ctx, acc, stream);
   return LV_OK;
 }
@@ -838,7 +867,8 @@ lv_status lv_whatif(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, 
     st = timing_end(stop, stream);
     if (st != LV_OK) return st;
   }
-  LV_CUDA(cudaEventRecord(ctx->ev_used, stream));
+  st = record_event(ctx->ev_used, stream);
+  if (st != LV_OK) return st;
   return LV_OK;
 }
 

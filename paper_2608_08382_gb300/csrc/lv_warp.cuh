@@ -815,8 +815,8 @@ __global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
         i128 kf = mk128(0, 0);
         bool ovf = false;
         if (n >= 1 && n <= a.mp.nk) {
-          const KEntry e = a.mp.ktab[s * (a.mp.nk + 1) + n];
-          kf = double_to_fix(__dadd_rn(e.q, e.a4n), a.mp.fx[s].E, &ovf);
+          kf = a.mp.ktab[s * (a.mp.nk + 1) + n].kf;  // fix(fl(q + a4n)), built once per model
+          ovf = kf.hi == kKSlowHi;
         }
         ws.kfix[s][n] = kf;
         ws.kslow[s][n] = ovf ? 1 : 0;
@@ -931,12 +931,30 @@ __global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_bas
       bool slow = false;
       const i128 kf = batch_const_w<MODE>(a, nullptr, s, g.n, &slow);
       const SegS sg = js.seg[s];
+      // decode requests through the same fast path as k_warps; the rest general
+      const bool fast = (MODE & M_FIX) && !slow && sg.a2_narrow;
+      const i128 K13 = add128(kf, sg.A13);
       for (int64_t i = r0 + tid; i < r1; i += kJBlock) {
         int32_t p = a.p[i], c = a.c[i];
         const int32_t u = kTen ? a.ten[i] : 0;
         p = p < 0 ? 0 : p;
         c = c < 0 ? 0 : c;
-        attribute_one<MODE>(a, tt, sg, s, slow, kf, g.n, i, p, c, u, &bad);
+        bool done = false;
+        if (fast && p == 1) {
+          uint32_t v0, v1, v2, v3;
+          mad_k13((uint32_t)K13.lo, (uint32_t)(K13.lo >> 32), (uint32_t)K13.hi, (uint32_t)(K13.hi >> 32),
+                  (uint32_t)sg.A2.lo, (uint32_t)(sg.A2.lo >> 32), (uint32_t)c, v0, v1, v2, v3);
+          if (v3 == 0u && v2 != 0u) {
+            uint64_t m;
+            int ex2;
+            const double d = round96(v0, v1, v2, sg.E, m, ex2);
+            if (!kTen || tenant_fast(a, tt, u, m, ex2)) {
+              if (a.share) __stcs(a.share + i, d);
+              done = true;
+            }
+          }
+        }
+        if (!done) attribute_one<MODE>(a, tt, sg, s, slow, kf, g.n, i, p, c, u, &bad);
       }
     }
     __syncthreads();  // js.red / js.tot are rewritten for the next batch

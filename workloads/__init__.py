@@ -29,7 +29,7 @@ import math
 import numpy as np
 
 __all__ = [
-    "ARCHS", "Workload", "WhatIf", "config", "whatif_config", "random_batches",
+    "ARCHS", "Workload", "WhatIf", "config", "whatif_config", "step_config", "random_batches",
     "draw_coefficients", "zipf_tenants", "SEED_BASE",
 ]
 
@@ -262,6 +262,32 @@ def config(k: int, scale: float = 1.0) -> Workload:
     return Workload(name=f"config{k}", arch=np.asarray(ARCHS[model], dtype=np.int32), p=p, c=c,
                     phase=ph, tenant=t, offsets=off, n_tenants=nt, coef=coef, split=split,
                     noise=noise, seed=seed)
+
+
+def step_config(n_req: int = 2048, n_prefill: int = 4) -> Workload:
+    """One serving step: a single Qwen2.5-14B tp2 continuous batch of ``n_req``
+    requests (the paper's 128-2048 concurrent requests), drawn as in workload 1:
+    ``n_prefill`` chunked prefills of 512 new tokens with prior context
+    U{0..32256} at random positions, decodes with lognormal(7.5, 1.2) contexts in
+    [1, 32768], Zipf(1.1) tenants over 256.
+    """
+    seed = SEED_BASE + 5
+    rng = np.random.default_rng(seed)
+    n = int(n_req)
+    k = min(int(n_prefill), n)
+    phase = np.zeros(n, dtype=np.int32)
+    phase[rng.choice(n, size=k, replace=False)] = 1
+    pre = phase == 1
+    p = np.ones(n, dtype=np.int32)
+    c = np.empty(n, dtype=np.int32)
+    p[pre] = 512
+    c[pre] = rng.integers(0, 32257, size=k, dtype=np.int32)
+    c[~pre] = _lognormal_int(rng, n - k, 7.5, 1.2, 1, 32768)
+    tenant = zipf_tenants(rng, n, 256, 1.1)
+    off = np.array([0, n], dtype=np.int64)
+    coef, split = draw_coefficients(rng, "qwen2.5-14b")
+    return Workload(name="step", arch=np.asarray(ARCHS["qwen2.5-14b"], dtype=np.int32), p=p, c=c, phase=phase,
+                    tenant=tenant, offsets=off, n_tenants=256, coef=coef, split=split, seed=seed)
 
 
 def whatif_config(scale: float = 1.0, n_pending: int | None = None) -> WhatIf:
