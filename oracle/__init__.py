@@ -160,6 +160,22 @@ def tenant_totals(share, tenant, n_tenants):
     return TenantSums(n_tenants).add(share, tenant).totals()
 
 
+def admit(T_new, share_new, tenant_new, L, budget, slo):
+    """Admission over what-if pairs (Section 1: what-if planning for admission
+    control).  Pending request j may join candidate batch b when its tenant's
+    running total plus its share in the merged batch stays within the tenant's
+    budget, L[u_j] + share_new[j, b] <= budget[u_j] (one fp64 addition), and
+    the merged batch meets the latency objective, T_new[j, b] <= slo.
+    Returns uint8[n_pending, n_cand] (1 = admissible)."""
+    T_new = np.asarray(T_new, dtype=np.float64)
+    share_new = np.asarray(share_new, dtype=np.float64)
+    u = np.asarray(tenant_new, dtype=np.int64)
+    Lu = np.asarray(L, dtype=np.float64)[u][:, None]
+    Bu = np.asarray(budget, dtype=np.float64)[u][:, None]
+    ok = ((Lu + share_new) <= Bu) & (T_new <= float(slo))
+    return ok.astype(np.uint8)
+
+
 def whatif(offsets, p, c, phase, p_new, c_new, phase_new, split, coef):
     """Returns (T_new, share_new), each float64[n_pending, n_cand]."""
     off = _c(offsets, np.int64)

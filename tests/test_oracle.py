@@ -248,6 +248,32 @@ def test_whatif_brute_force():
             assert abs(Fraction(float(Sn[j, b])) - exS) <= 10 * 2.0**-53 * exS
 
 
+def test_admit_hand_case(golden_dir):
+    """The admission predicate on a hand-worked case: equality admits, the
+    tenant is the pending request's, and both conditions are required."""
+    g = _load(golden_dir, "admit_hand_case.json")
+    m = oracle.admit(np.array(g["T_new"]), np.array(g["share_new"]), g["tenant_new"], g["L"], g["budget"], g["slo"])
+    assert m.dtype == np.uint8 and m.shape == (2, 3)
+    assert np.array_equal(m, np.array(g["expected"], dtype=np.uint8))
+
+
+def test_admit_brute_force():
+    """Against a per-pair restatement in exact rationals on random what-if outputs
+    (dyadic values, so the single fp64 addition is exact)."""
+    rng = np.random.default_rng(7)
+    npd, nc, nt = 13, 17, 5
+    T = rng.integers(0, 64, (npd, nc)) / 32.0
+    S = rng.integers(0, 64, (npd, nc)) / 64.0
+    u = rng.integers(0, nt, npd)
+    L = rng.integers(0, 64, nt) / 64.0
+    B = rng.integers(0, 128, nt) / 64.0
+    m = oracle.admit(T, S, u, L, B, 1.0)
+    for j in range(npd):
+        for b in range(nc):
+            want = Fraction(float(L[u[j]])) + Fraction(float(S[j, b])) <= Fraction(float(B[u[j]])) and T[j, b] <= 1.0
+            assert m[j, b] == int(want)
+
+
 # ---------------------------------------------------------------- fit
 
 def _fit_data(scale=0.004, seed_noise=True):
