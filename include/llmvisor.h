@@ -38,8 +38,8 @@
  *    8-byte aligned; otherwise LV_EINVAL.
  *  - One lv_ctx must not be used from two host threads at once.
  *  - CUDA graphs: lv_features, lv_batch_latency, lv_attribute,
- *    lv_tenant_acc_reset, lv_tenant_accumulate, lv_tenant_totals and
- *    lv_whatif may be captured into a CUDA graph once an uncaptured call with
+ *    lv_tenant_acc_reset, lv_tenant_accumulate, lv_tenant_totals, lv_whatif
+ *    and lv_whatif_admit may be captured into a CUDA graph once an uncaptured call with
  *    the same context, model and sizes has run (it creates the context's
  *    buffers and caches the kernel configuration; a capture never allocates).
  *    The context's ordering events are then recorded and waited for by the
@@ -234,6 +234,22 @@ lv_status lv_fit(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y,
 lv_status lv_whatif(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, const int32_t *p_new,
                     const int32_t *c_new, const int32_t *phase_new, int64_t n_pending, double *T_new,
                     double *share_new, void *stream);
+
+/* What-if with admission (Section 1: what-if planning for admission control).
+ * lv_whatif's outputs, plus
+ *   admit[j][k] = 1 if L[u_j] + share_new[j][k] <= budget[u_j] (one fp64
+ *                 addition) and T_new[j][k] <= slo, else 0,
+ * with u_j = tenant_new[j] (device int32[n_pending]); L and budget are device
+ * double[n_tenants] (L, e.g., from lv_tenant_totals: each tenant's attributed
+ * latency so far; budget its allowance), slo in seconds.  admit: device
+ * uint8[n_pending][n_cand], required; T_new and share_new may be NULL.  A
+ * tenant id outside [0, n_tenants) records LV_EDATA and that request's pairs
+ * get 0.  Pointers misaligned for their type, n_tenants <= 0 or a NULL admit,
+ * L or budget: LV_EINVAL. */
+lv_status lv_whatif_admit(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, const int32_t *p_new,
+                          const int32_t *c_new, const int32_t *phase_new, const int32_t *tenant_new,
+                          int64_t n_pending, const double *L, const double *budget, int32_t n_tenants, double slo,
+                          double *T_new, double *share_new, uint8_t *admit, void *stream);
 
 /* Attribution without any allocation (the paper has no counterpart; this is a
  * service to callers that cannot allocate device memory at call time).  A

@@ -29,7 +29,7 @@ EXPORTED = [
     "lv_ctx_set_timing", "lv_ctx_kernel_time",
     "lv_features", "lv_batch_latency", "lv_attribute", "lv_tenant_acc_create", "lv_tenant_acc_destroy",
     "lv_tenant_acc_reset", "lv_tenant_accumulate", "lv_tenant_totals", "lv_tenant_acc_state_bytes",
-    "lv_tenant_acc_export", "lv_tenant_acc_import", "lv_fit", "lv_whatif", "lv_attribute_noalloc",
+    "lv_tenant_acc_export", "lv_tenant_acc_import", "lv_fit", "lv_whatif", "lv_whatif_admit", "lv_attribute_noalloc",
 ]
 
 
@@ -91,6 +91,7 @@ def _load():
         "lv_tenant_acc_import": ([P, P, I64, P], I32),
         "lv_fit": ([P, P, P, I32, P, P, P], I32),
         "lv_whatif": ([P, P, P, P, P, P, I64, P, P, P], I32),
+        "lv_whatif_admit": ([P, P, P, P, P, P, P, I64, P, P, I32, ctypes.c_double, P, P, P, P], I32),
         "lv_attribute_noalloc": ([P, P, P, P, P, P], I32),
     }
     for name, (args, res) in sig.items():
@@ -324,3 +325,12 @@ def lv_whatif(ctx: Context, model: lv_model, cand: Batches, p_new, c_new, phase_
     bs = cand.struct()
     _check(_lib.lv_whatif(ctx.h, ctypes.byref(model), ctypes.byref(bs), _ptr(p_new), _ptr(c_new), _ptr(phase_new),
                           int(p_new.numel()), _ptr(T_new), _ptr(share_new), _stream(stream)), "lv_whatif")
+
+
+def lv_whatif_admit(ctx: Context, model: lv_model, cand: Batches, p_new, c_new, phase_new, tenant_new, L, budget,
+                    slo: float, admit, T_new=None, share_new=None, stream=None):
+    bs = cand.struct()
+    _check(_lib.lv_whatif_admit(ctx.h, ctypes.byref(model), ctypes.byref(bs), _ptr(p_new), _ptr(c_new),
+                                _ptr(phase_new), _ptr(tenant_new), int(p_new.numel()), _ptr(L), _ptr(budget),
+                                int(L.numel()), float(slo), _ptr(T_new), _ptr(share_new), _ptr(admit),
+                                _stream(stream)), "lv_whatif_admit")

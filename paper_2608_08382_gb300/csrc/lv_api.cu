@@ -391,6 +391,79 @@ lv_status fold_tenants(lv_ctx *ctx, lv_tenant_acc *acc, cudaStream_t stream) {
   return LV_OK;
 }
 
+// lv_whatif and lv_whatif_admit (adm.admit null for the former).
+lv_status whatif_run(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, const int32_t *p_new,
+                     const int32_t *c_new, const int32_t *phase_new, int64_t n_pending, double *T_new,
+                     double *share_new, const AdmitArgs &adm, void *stream_) {
+  if (!ctx || check_model(model) != LV_OK || n_pending < 0) return LV_EINVAL;
+  lv_status st = check_batches(cand, false);
+  if (st != LV_OK) return st;
+  if (n_pending > 0 && (!p_new || !c_new || !phase_new || !aligned(p_new, 4) || !aligned(c_new, 4) ||
+                        !aligned(phase_new, 4)))
+    return LV_EINVAL;
+  if ((T_new && !aligned(T_new, 8)) || (share_new && !aligned(share_new, 8))) return LV_EINVAL;
+  const int64_t nc = cand->n_batch, np = n_pending;
+  if (nc == 0 || np == 0 || (!T_new && !share_new && !adm.admit)) return LV_OK;
+  cudaStream_t stream = (cudaStream_t)stream_;
+  ModelP mp;
+  st = prepare_model(ctx, model, stream, &mp);
+  if (st != LV_OK) return st;
+  // scratch: candidate sums, segment codes, candidate and pending tables
+  const size_t o_feat = 0;
+  const size_t o_seg = o_feat + sizeof(int64_t) * 5 * (size_t)nc;
+  const size_t o_cand = (o_seg + (size_t)nc + 255) & ~(size_t)255;
+  const size_t o_pend = (o_cand + sizeof(CandP) * (size_t)nc + 255) & ~(size_t)255;
+  const size_t need = o_pend + sizeof(PendP) * (size_t)np;
+  if (need > ctx->wi_cap) {
+    LV_CUDA(cudaDeviceSynchronize());
+    if (ctx->d_wi) cudaFree(ctx->d_wi);
+    ctx->d_wi = nullptr;
+    ctx->wi_cap = 0;
+    if (cudaMalloc(&ctx->d_wi, need) != cudaSuccess) return LV_ENOMEM;
+    ctx->wi_cap = need;
+  }
+  unsigned char *base = static_cast<unsigned char *>(ctx->d_wi);
+  int64_t *bfeat = reinterpret_cast<int64_t *>(base + o_feat);
+  uint8_t *bseg = base + o_seg;
+  CandP *candp = reinterpret_cast<CandP *>(base + o_cand);
+  PendP *pendp = reinterpret_cast<PendP *>(base + o_pend);
+
+  TileArgs a{};
+  a.p = cand->p;
+  a.c = cand->c;
+  a.ph = cand->phase;
+  a.off = cand->offsets;
+  a.n_req = cand->n_req;
+  a.n_batch = nc;
+  a.bfeat = bfeat;
+  a.bseg = bseg;
+  a.status = ctx->d_status;
+  a.mp = mp;
+  st = run_tiles(ctx, a, M_FEAT, stream);
+  if (st != LV_OK) return st;
+  k_wi_cand<<<(unsigned)((nc + 127) / 128), 128, 0, stream>>>(mp, bfeat, bseg, nc, candp);
+  LV_CUDA(cudaGetLastError());
+  k_wi_pend<<<(unsigned)((np + 127) / 128), 128, 0, stream>>>(mp, p_new, c_new, phase_new, np, pendp, adm,
+                                                              ctx->d_status);
+  LV_CUDA(cudaGetLastError());
+  const int64_t gx = (nc + kWiCols - 1) / kWiCols;
+  const int64_t rows_per_launch = (int64_t)65535 * kWiRows;
+  for (int64_t j = 0; j < np; j += rows_per_launch) {
+    const int64_t rows = std::min<int64_t>(rows_per_launch, np - j);
+    const dim3 grid((unsigned)gx, (unsigned)((rows + kWiRows - 1) / kWiRows));
+    cudaEvent_t stop;
+    st = timing_begin(ctx, LV_TIME_PAIRS, stream, &stop);
+    if (st != LV_OK) return st;
+    k_wi_pairs<<<grid, kWiCols, 0, stream>>>(mp, candp, pendp, nc, np, j, T_new, share_new, adm.slo, adm.admit);
+    LV_CUDA(cudaGetLastError());
+    st = timing_end(stop, stream);
+    if (st != LV_OK) return st;
+  }
+  st = record_event(ctx->ev_used, stream);
+  if (st != LV_OK) return st;
+  return LV_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -803,73 +876,18 @@ lv_status lv_fit(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y,
 lv_status lv_whatif(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, const int32_t *p_new,
                     const int32_t *c_new, const int32_t *phase_new, int64_t n_pending, double *T_new,
                     double *share_new, void *stream_) {
-  if (!ctx || check_model(model) != LV_OK || n_pending < 0) return LV_EINVAL;
-  lv_status st = check_batches(cand, false);
-  if (st != LV_OK) return st;
-  if (n_pending > 0 && (!p_new || !c_new || !phase_new || !aligned(p_new, 4) || !aligned(c_new, 4) ||
-                        !aligned(phase_new, 4)))
-    return LV_EINVAL;
-  if ((T_new && !aligned(T_new, 8)) || (share_new && !aligned(share_new, 8))) return LV_EINVAL;
-  const int64_t nc = cand->n_batch, np = n_pending;
-  if (nc == 0 || np == 0 || (!T_new && !share_new)) return LV_OK;
-  cudaStream_t stream = (cudaStream_t)stream_;
-  ModelP mp;
-  st = prepare_model(ctx, model, stream, &mp);
-  if (st != LV_OK) return st;
-  // scratch: candidate sums, segment codes, candidate and pending tables
-  const size_t o_feat = 0;
-  const size_t o_seg = o_feat + sizeof(int64_t) * 5 * (size_t)nc;
-  const size_t o_cand = (o_seg + (size_t)nc + 255) & ~(size_t)255;
-  const size_t o_pend = (o_cand + sizeof(CandP) * (size_t)nc + 255) & ~(size_t)255;
-  const size_t need = o_pend + sizeof(PendP) * (size_t)np;
-  if (need > ctx->wi_cap) {
-    LV_CUDA(cudaDeviceSynchronize());
-    if (ctx->d_wi) cudaFree(ctx->d_wi);
-    ctx->d_wi = nullptr;
-    ctx->wi_cap = 0;
-    if (cudaMalloc(&ctx->d_wi, need) != cudaSuccess) return LV_ENOMEM;
-    ctx->wi_cap = need;
-  }
-  unsigned char *base = static_cast<unsigned char *>(ctx->d_wi);
-  int64_t *bfeat = reinterpret_cast<int64_t *>(base + o_feat);
-  uint8_t *bseg = base + o_seg;
-  CandP *candp = reinterpret_cast<CandP *>(base + o_cand);
-  PendP *pendp = reinterpret_cast<PendP *>(base + o_pend);
+  return whatif_run(ctx, model, cand, p_new, c_new, phase_new, n_pending, T_new, share_new, AdmitArgs{}, stream_);
+}
 
-  TileArgs a{};
-  a.p = cand->p;
-  a.c = cand->c;
-  a.ph = cand->phase;
-  a.off = cand->offsets;
-  a.n_req = cand->n_req;
-  a.n_batch = nc;
-  a.bfeat = bfeat;
-  a.bseg = bseg;
-  a.status = ctx->d_status;
-  a.mp = mp;
-  st = run_tiles(ctx, a, M_FEAT, stream);
-  if (st != LV_OK) return st;
-  k_wi_cand<<<(unsigned)((nc + 127) / 128), 128, 0, stream>>>(mp, bfeat, bseg, nc, candp);
-  LV_CUDA(cudaGetLastError());
-  k_wi_pend<<<(unsigned)((np + 127) / 128), 128, 0, stream>>>(mp, p_new, c_new, phase_new, np, pendp,
-                                                              ctx->d_status);
-  LV_CUDA(cudaGetLastError());
-  const int64_t gx = (nc + kWiCols - 1) / kWiCols;
-  const int64_t rows_per_launch = (int64_t)65535 * kWiRows;
-  for (int64_t j = 0; j < np; j += rows_per_launch) {
-    const int64_t rows = std::min<int64_t>(rows_per_launch, np - j);
-    const dim3 grid((unsigned)gx, (unsigned)((rows + kWiRows - 1) / kWiRows));
-    cudaEvent_t stop;
-    st = timing_begin(ctx, LV_TIME_PAIRS, stream, &stop);
-    if (st != LV_OK) return st;
-    k_wi_pairs<<<grid, kWiCols, 0, stream>>>(mp, candp, pendp, nc, np, j, T_new, share_new);
-    LV_CUDA(cudaGetLastError());
-    st = timing_end(stop, stream);
-    if (st != LV_OK) return st;
-  }
-  st = record_event(ctx->ev_used, stream);
-  if (st != LV_OK) return st;
-  return LV_OK;
+lv_status lv_whatif_admit(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, const int32_t *p_new,
+                          const int32_t *c_new, const int32_t *phase_new, const int32_t *tenant_new,
+                          int64_t n_pending, const double *L, const double *budget, int32_t n_tenants, double slo,
+                          double *T_new, double *share_new, uint8_t *admit, void *stream_) {
+  if (!admit || n_tenants <= 0 || (n_pending > 0 && (!tenant_new || !aligned(tenant_new, 4))) || !L || !budget ||
+      !aligned(L, 8) || !aligned(budget, 8))
+    return LV_EINVAL;
+  AdmitArgs adm{tenant_new, L, budget, n_tenants, slo, admit};
+  return whatif_run(ctx, model, cand, p_new, c_new, phase_new, n_pending, T_new, share_new, adm, stream_);
 }
 
 }  // extern "C"

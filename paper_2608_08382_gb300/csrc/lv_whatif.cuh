@@ -31,6 +31,18 @@ struct CandP {
 struct PendP {
   i128 V[4];
   int32_t p, c, phase, slow;
+  double Lu, Bu;  // admission: the request's tenant's running total and budget
+};
+
+// Admission inputs (null: plain what-if).  A pair (j, b) is admissible when
+// L[u_j] + share_new[j][b] <= budget[u_j] (one fp64 addition) and
+// T_new[j][b] <= slo (Section 1: what-if planning for admission control).
+struct AdmitArgs {
+  const int32_t *tenant;  // [n_pending]
+  const double *L, *budget;  // [n_tenants]
+  int32_t n_tenants;
+  double slo;
+  uint8_t *admit;  // [n_pending][n_cand]
 };
 
 // Per candidate: U_b[s], W_b[s] for every segment, from the batch sums.
@@ -72,19 +84,34 @@ __global__ void k_wi_cand(ModelP mp, const int64_t *__restrict__ bfeat, const ui
 }
 
 // Per pending request: V_j[s] = a1 p + a2 c + a3 p^2 for every segment.
+// With admission, also the request's tenant's total and budget (a tenant id
+// out of range records a data error and makes every pair of the request
+// inadmissible: NaN compares false).
 __global__ void k_wi_pend(ModelP mp, const int32_t *__restrict__ p_new, const int32_t *__restrict__ c_new,
-                          const int32_t *__restrict__ ph_new, int64_t np, PendP *__restrict__ out, int *status) {
+                          const int32_t *__restrict__ ph_new, int64_t np, PendP *__restrict__ out, AdmitArgs adm,
+                          int *status) {
   const int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (j >= np) return;
   int32_t p = p_new[j], c = c_new[j], ph = ph_new[j];
   int bad = 0;
   check_req(p, c, ph, &bad);
-  if (bad) flag(status, kStatusData);
   PendP q;
   q.p = p;
   q.c = c;
   q.phase = ph;
   q.slow = (!mp.fixed || p > kPMaxFix) ? 1 : 0;
+  q.Lu = q.Bu = 0.0;
+  if (adm.admit) {
+    const int32_t u = adm.tenant[j];
+    if (u < 0 || u >= adm.n_tenants) {
+      bad = 1;
+      q.Lu = __longlong_as_double(0x7ff8000000000000ll);
+    } else {
+      q.Lu = adm.L[u];
+      q.Bu = adm.budget[u];
+    }
+  }
+  if (bad) flag(status, kStatusData);
 #pragma unroll
   for (int s = 0; s < 4; ++s) {
     q.V[s] = mk128(0, 0);
@@ -130,7 +157,8 @@ constexpr int kWiRows = 32;   // pending requests per block
 __global__ void __launch_bounds__(kWiCols) k_wi_pairs(ModelP mp, const CandP *__restrict__ cand,
                                                        const PendP *__restrict__ pend, int64_t nc, int64_t np,
                                                        int64_t j_base, double *__restrict__ T_new,
-                                                       double *__restrict__ share_new) {
+                                                       double *__restrict__ share_new, double slo,
+                                                       uint8_t *__restrict__ admit) {
   static_assert(kWiRows <= kWiCols, "one pending row per thread at most");
   __shared__ PendP sp[kWiRows];
   __shared__ int sE[4];
@@ -163,6 +191,7 @@ __global__ void __launch_bounds__(kWiCols) k_wi_pairs(ModelP mp, const CandP *__
       const int64_t o = (j0 + r) * nc + b;
       if (T_new) __stcs(T_new + o, T);
       if (share_new) __stcs(share_new + o, sh);
+      if (admit) admit[o] = (__dadd_rn(sp[r].Lu, sh) <= sp[r].Bu && T <= slo) ? 1 : 0;
     }
     return;
   }
@@ -181,6 +210,7 @@ __global__ void __launch_bounds__(kWiCols) k_wi_pairs(ModelP mp, const CandP *__
     const int64_t o = (j0 + r) * nc + b;
     if (T_new) __stcs(T_new + o, T);
     if (share_new) __stcs(share_new + o, sh);
+    if (admit) admit[o] = (__dadd_rn(sp[r].Lu, sh) <= sp[r].Bu && T <= slo) ? 1 : 0;
   }
 }
 

@@ -108,3 +108,67 @@ def test_whatif_deterministic_and_outputs_optional(lv, ctx):
     S = torch.empty((q.n_pending, c.n_batch), dtype=torch.float64, device="cuda")
     lv.lv_whatif(ctx, lv.make_model(q.coef, q.split), cand, t(q.p_new), t(q.c_new), t(q.phase_new), None, S)
     assert np.array_equal(S.cpu().numpy(), a[1])
+
+
+def _admit_inputs(q, n_tenants=8, seed=3):
+    """Tenants of the pending requests, running totals, budgets and an SLO around
+    the workload's own magnitudes, so that both outcomes occur often."""
+    rng = np.random.default_rng(seed)
+    To, So = oracle.whatif(q.cand.offsets, q.cand.p, q.cand.c, q.cand.phase, q.p_new, q.c_new, q.phase_new,
+                           q.split, q.coef)
+    u = rng.integers(0, n_tenants, q.n_pending).astype(np.int32)
+    L = rng.uniform(0.0, 1.0, n_tenants) * float(np.median(So)) * 100
+    B = L + rng.uniform(0.0, 2.0, n_tenants) * float(np.median(So))
+    slo = float(np.median(To))
+    return u, L, B, slo, To, So
+
+
+@pytest.mark.parametrize("scale", [0.25, 1.0])
+def test_whatif_admit_config3(lv, ctx, scale):
+    """admit equals the oracle's predicate on the device's own T_new and shares
+    bit for bit, and on the oracle's everywhere but at exact-margin ties; the
+    admit-only call (no T_new, share_new) gives the same mask."""
+    import torch
+    q = workloads.whatif_config(scale=scale)
+    c = q.cand
+    u, L, B, slo, To, So = _admit_inputs(q)
+    cand = lv.batches_to_device(c.p, c.c, c.phase, c.offsets)
+    t = lambda a: torch.as_tensor(np.ascontiguousarray(a, dtype=np.int32), device="cuda")  # noqa: E731
+    d = lambda a: torch.as_tensor(np.ascontiguousarray(a, dtype=np.float64), device="cuda")  # noqa: E731
+    npd, nc = q.n_pending, c.n_batch
+    T = torch.full((npd, nc), float("nan"), dtype=torch.float64, device="cuda")
+    S = torch.full((npd, nc), float("nan"), dtype=torch.float64, device="cuda")
+    A = torch.full((npd, nc), 7, dtype=torch.uint8, device="cuda")
+    model = lv.make_model(q.coef, q.split)
+    lv.lv_whatif_admit(ctx, model, cand, t(q.p_new), t(q.c_new), t(q.phase_new), t(u), d(L), d(B), slo, A, T, S)
+    assert ctx.status() == lv.LV_OK
+    T, S, A = T.cpu().numpy(), S.cpu().numpy(), A.cpu().numpy()
+    _check(c.offsets, c.p, c.c, c.phase, q.p_new, q.c_new, q.phase_new, q.coef, q.split, T, S)
+    assert np.array_equal(A, oracle.admit(T, S, u, L, B, slo))
+    Ao = oracle.admit(To, So, u, L, B, slo)
+    margin = np.minimum(np.abs(L[u][:, None] + So - B[u][:, None]) / B[u][:, None], np.abs(To - slo) / slo)
+    assert np.all((A == Ao) | (margin <= 4 * TOL))
+    assert 0.05 < A.mean() < 0.95
+    A2 = torch.full((npd, nc), 7, dtype=torch.uint8, device="cuda")
+    lv.lv_whatif_admit(ctx, model, cand, t(q.p_new), t(q.c_new), t(q.phase_new), t(u), d(L), d(B), slo, A2)
+    assert np.array_equal(A2.cpu().numpy(), A)
+
+
+def test_whatif_admit_invalid_tenant_and_arguments(lv, ctx):
+    import torch
+    q = workloads.whatif_config(scale=0.05)
+    c = q.cand
+    u, L, B, slo, _, _ = _admit_inputs(q)
+    u[3] = 8  # out of range: data error, that request's pairs inadmissible
+    cand = lv.batches_to_device(c.p, c.c, c.phase, c.offsets)
+    t = lambda a: torch.as_tensor(np.ascontiguousarray(a, dtype=np.int32), device="cuda")  # noqa: E731
+    d = lambda a: torch.as_tensor(np.ascontiguousarray(a, dtype=np.float64), device="cuda")  # noqa: E731
+    A = torch.full((q.n_pending, c.n_batch), 7, dtype=torch.uint8, device="cuda")
+    model = lv.make_model(q.coef, q.split)
+    lv.lv_whatif_admit(ctx, model, cand, t(q.p_new), t(q.c_new), t(q.phase_new), t(u), d(L), d(B), slo, A)
+    assert ctx.status() == lv.LV_EDATA
+    A = A.cpu().numpy()
+    assert np.all(A[3] == 0) and np.all(A <= 1)
+    with pytest.raises(lv.LVError) as ei:
+        lv.lv_whatif_admit(ctx, model, cand, t(q.p_new), t(q.c_new), t(q.phase_new), t(u), d(L), d(B), slo, None)
+    assert ei.value.status == lv.LV_EINVAL
