@@ -9,12 +9,13 @@ arrays resident in HBM; they are ~2.2 GB, far larger than L2, so no flush is
 needed between steps.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--workload attr1|attr4|fit2|whatif3|step] [--scale X] [--no-cpu-baseline]
+                    [--workload attr1|attr4|fit2|whatif3|admit3|step] [--scale X] [--no-cpu-baseline]
 
 attr1 (the default) is the headline line.  attr4 is the skew stress, fit2 the
 coefficient fit over 2e6 profiled batches (one step = lv_fit of a noisy and a
 noiseless latency vector), whatif3 the what-if pairs (one step = lv_whatif over
-4096 pending x 1024 candidates), step the single-step scheduler mode (one
+4096 pending x 1024 candidates), admit3 the same pairs with the admission
+epilogue (lv_whatif_admit), step the single-step scheduler mode (one
 batch of 2048 requests per step, replayed from a CUDA graph; the line adds
 us_per_step); each prints a line of the same shape with its own metric and the
 roofline of its dominant kernel.
@@ -167,6 +168,7 @@ def barrier(world):
 
 METRIC_FIT = "profiled requests/sec through the coefficient fit on 1 GB300"
 METRIC_WHATIF = "what-if (pending request, candidate batch) pairs/sec on 1 GB300"
+METRIC_ADMIT = "what-if pairs/sec with SLO-aware admission (per-tenant budget, latency objective) on 1 GB300"
 METRIC_STEP = "attributed requests/sec, one 2048-request serving step per CUDA-graph replay on 1 GB300"
 
 WORKLOADS = {
@@ -178,6 +180,8 @@ WORKLOADS = {
                        "and noiseless latency vectors fitted in one pass"),
     "whatif3": ("whatif", 3, "qwen2.5-32b tp4 what-if: 1024 candidate batches U{32..256} x 4096 pending requests, "
                              "4,194,304 pairs"),
+    "admit3": ("admit", 3, "qwen2.5-32b tp4 what-if with admission: 1024 candidate batches x 4096 pending requests "
+                           "of 64 tenants, per-tenant budgets and a latency objective, 4,194,304 pairs"),
     "step": ("step", 5, "qwen2.5-14b tp2 serving step: one batch of 2048 requests (4 chunked prefills), "
                         "256 Zipf(1.1) tenants, replayed from a CUDA graph"),
 }
@@ -186,7 +190,7 @@ WORKLOADS = {
 def _workload(args):
     import workloads
     kind, k_cfg, desc = WORKLOADS[args.workload]
-    if kind == "whatif":
+    if kind in ("whatif", "admit"):
         w = workloads.whatif_config(scale=args.scale)
     elif kind == "step":
         w = workloads.step_config(n_req=max(1, int(round(2048 * args.scale))))
@@ -327,8 +331,10 @@ def _setup_fit(lv, ctx, w, stream):
                 check=lambda: out["rep"])
 
 
-def _setup_whatif(lv, ctx, q, stream):
-    """Step: lv_whatif over every (pending request, candidate batch) pair of config 3."""
+def _setup_whatif(lv, ctx, q, stream, admit=False):
+    """Step: lv_whatif over every (pending request, candidate batch) pair of config 3 (admit: lv_whatif_admit,
+    with the pending requests spread over 64 tenants whose running totals, budgets and the latency objective sit
+    at the workload's own magnitudes)."""
     import torch
     c = q.cand
     cand = lv.batches_to_device(c.p, c.c, c.phase, c.offsets)
@@ -339,8 +345,22 @@ def _setup_whatif(lv, ctx, q, stream):
     T = torch.empty((q.n_pending, c.n_batch), dtype=torch.float64, device="cuda")
     S = torch.empty_like(T)
 
-    def step():
+    if admit:
         lv.lv_whatif(ctx, model, cand, pn, cn, phn, T, S, stream=stream)
+        med_T, med_S = float(T.median()), float(S.median())
+        rng = np.random.default_rng(q.seed)
+        nt = 64
+        tn = t(rng.integers(0, nt, q.n_pending))
+        Lh = rng.uniform(0.0, 1.0, nt) * med_S * 100
+        L = torch.as_tensor(Lh, device="cuda")
+        B = torch.as_tensor(Lh + rng.uniform(0.0, 2.0, nt) * med_S, device="cuda")
+        A = torch.empty((q.n_pending, c.n_batch), dtype=torch.uint8, device="cuda")
+
+        def step():
+            lv.lv_whatif_admit(ctx, model, cand, pn, cn, phn, tn, L, B, med_T, A, T, S, stream=stream)
+    else:
+        def step():
+            lv.lv_whatif(ctx, model, cand, pn, cn, phn, T, S, stream=stream)
 
     hp = {k: torch.from_numpy(np.ascontiguousarray(v)).pin_memory()
           for k, v in dict(p=c.p, c=c.c, phase=c.phase, offsets=c.offsets).items()}
@@ -358,16 +378,23 @@ def _setup_whatif(lv, ctx, q, stream):
         step()
         hT.copy_(T, non_blocking=True)
         hS.copy_(S, non_blocking=True)
+        if admit:
+            hA.copy_(A, non_blocking=True)
 
+    hA = torch.empty(T.shape, dtype=torch.uint8).pin_memory() if admit else None
     h2d = sum(int(x.numel() * x.element_size()) for x in list(hp.values()) + list(hq.values()))
-    return dict(step=step, e2e_step=e2e_step, units=npairs, unit="pairs/s", metric=METRIC_WHATIF,
-                h2d=h2d, d2h=16 * npairs, launches_per_step=6, kernel="k_wi_pairs", time_mask=lv.LV_TIME_PAIRS,
-                bytes_per_launch=16.0 * npairs,
-                bytes_rule="16 B/pair written (T_new, share_new); candidate and pending tables are cache-resident",
+    per_pair = 17 if admit else 16
+    return dict(step=step, e2e_step=e2e_step, units=npairs, unit="pairs/s",
+                metric=METRIC_ADMIT if admit else METRIC_WHATIF,
+                h2d=h2d, d2h=per_pair * npairs, launches_per_step=6, kernel="k_wi_pairs",
+                time_mask=lv.LV_TIME_PAIRS, bytes_per_launch=float(per_pair) * npairs,
+                bytes_rule=(f"{per_pair} B/pair written (T_new, share_new" + (", admit" if admit else "") +
+                            "); candidate and pending tables are cache-resident"),
                 config={"n_cand": c.n_batch, "n_pending": q.n_pending, "pairs": npairs, "seed": q.seed,
                         "l2": "working set below L2 size: a 512 MB buffer is overwritten before every timed step, "
                               "outside the step's events",
-                        "step": "lv_whatif (candidate sums, tables, pair kernel)"},
+                        "step": ("lv_whatif_admit" if admit else "lv_whatif") +
+                                " (candidate sums, tables, pair kernel)"},
                 flush=True)
 
 
@@ -380,8 +407,8 @@ def run_ours(args, world, rank, local):
     kind, w, desc = _workload(args)
     ctx = lv.Context()
     stream = torch.cuda.current_stream()
-    s = {"attr": _setup_attr, "fit": _setup_fit, "whatif": _setup_whatif, "step": _setup_step}[kind](
-        lv, ctx, w, stream)
+    s = {"attr": _setup_attr, "fit": _setup_fit, "whatif": _setup_whatif, "step": _setup_step,
+         "admit": lambda *x: _setup_whatif(*x, admit=True)}[kind](lv, ctx, w, stream)
     step = s["step"]
 
     for _ in range(args.warmup):
@@ -489,13 +516,17 @@ def _oracle_sample(kind, w):
     Returns (run, units per run, description)."""
     import oracle
     oracle.build()
-    if kind == "whatif":
+    if kind in ("whatif", "admit"):
         c = w.cand
         rows = 64
         pn, cn, phn = w.p_new[:rows], w.c_new[:rows], w.phase_new[:rows]
+        rng = np.random.default_rng(w.seed)
+        un, Lh, Bh = rng.integers(0, 64, rows), rng.uniform(0, 1e-3, 64), rng.uniform(0, 2e-3, 64)
 
         def run():
-            oracle.whatif(c.offsets, c.p, c.c, c.phase, pn, cn, phn, w.split, w.coef)
+            T, S = oracle.whatif(c.offsets, c.p, c.c, c.phase, pn, cn, phn, w.split, w.coef)
+            if kind == "admit":
+                oracle.admit(T, S, un, Lh, Bh, 0.05)
         return run, rows * c.n_batch, f"first {rows} of {w.n_pending} pending requests x all {c.n_batch} candidates"
     if kind == "step":
         t = w.tenant
@@ -536,7 +567,7 @@ def cpu_baseline(kind, w, min_seconds=10.0):
         el = time.perf_counter() - t0
         if el >= min_seconds:
             break
-    unit = "pairs/s" if kind == "whatif" else "requests/s"
+    unit = "pairs/s" if kind in ("whatif", "admit") else "requests/s"
     return {"value": done / el, "unit": unit, "cores": 1, "kind": "oracle",
             "sample": f"{sample}; repeated for {el:.1f} s, single thread"}
 
@@ -553,8 +584,9 @@ def run_reference(args, world, rank):
         run()
     el = time.perf_counter() - t0
     value = units * args.steps / el
-    unit = "pairs/s" if kind == "whatif" else "requests/s"
-    metric = {"attr": METRIC, "fit": METRIC_FIT, "whatif": METRIC_WHATIF, "step": METRIC_STEP}[kind]
+    unit = "pairs/s" if kind in ("whatif", "admit") else "requests/s"
+    metric = {"attr": METRIC, "fit": METRIC_FIT, "whatif": METRIC_WHATIF, "admit": METRIC_ADMIT,
+              "step": METRIC_STEP}[kind]
     return {"impl": "reference", "metric": metric, "value": value, "unit": unit, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
