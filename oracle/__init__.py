@@ -16,7 +16,7 @@ import subprocess
 import numpy as np
 
 from . import fit as _fit  # noqa: F401  (re-exported)
-from .fit import fit, fit_group, OK, ENODATA, ESINGULAR  # noqa: F401
+from .fit import fit, fit_group, vtc_fit, accuracy, OK, ENODATA, ESINGULAR  # noqa: F401
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "lvo.c")

@@ -127,3 +127,62 @@ def fit(feat: np.ndarray, seg: np.ndarray, y: np.ndarray):
                       feat[4, sel]], axis=1)
         out.append(fit_group(X, y[sel]))
     return out
+
+
+def vtc_fit(S1: np.ndarray, n: np.ndarray, y: np.ndarray):
+    """The token-count baseline the paper compares against (VTC, Tables 1-2): one
+    least-squares line T = beta + a * S1 over every profiled batch, whatever its
+    phase and regime, S1 being the batch's total new tokens.  Exact normal
+    equations in rationals, rounded once; empty batches (n = 0) are skipped.
+    Returns (beta, a, status, count); beta and a are NaN unless status is OK."""
+    S1 = np.asarray(S1, dtype=np.int64)
+    sel = np.asarray(n) > 0
+    S = [int(v) for v in S1[sel].tolist()]
+    Y, E = _exact_targets(np.asarray(y, dtype=np.float64)[sel])
+    m = len(S)
+    if m < 2:
+        return float("nan"), float("nan"), ENODATA, m
+    G = [[m, sum(S)], [sum(S), sum(v * v for v in S)]]
+    scale = Fraction(2) ** E
+    r = [Fraction(sum(Y.tolist())) * scale, Fraction(sum(s * yv for s, yv in zip(S, Y.tolist()))) * scale]
+    sol = _solve_exact(G, r)
+    if sol is None:
+        return float("nan"), float("nan"), ESINGULAR, m
+    return float(sol[0]), float(sol[1]), OK, m
+
+
+def accuracy(y: np.ndarray, T: np.ndarray):
+    """Accuracy of predicted batch latencies T against measured y, as the paper
+    reports it (Section 3.2, Tables 1-2): R^2 in both of its usual forms and
+    percentiles of the relative error, over the batches with y > 0 (m of them).
+      r2_ssr   = 1 - sum (y - T)^2 / sum (y - mean y)^2
+      r2_corr  = (sum (y - mean y)(T - mean T))^2 / (sum (y - mean y)^2 sum (T - mean T)^2)
+      rel_b    = |T_b - y_b| / y_b; mean_rel is its mean, and p50, p90, p99 are
+                 nearest-rank percentiles: the ceil(q m)-th smallest of the m.
+    Sums are correctly rounded (math.fsum); an R^2 whose denominator is 0 is
+    NaN; with m = 0 every value is NaN."""
+    import math
+    y = np.asarray(y, dtype=np.float64)
+    T = np.asarray(T, dtype=np.float64)
+    sel = y > 0
+    y, T = y[sel], T[sel]
+    m = int(y.size)
+    nan = float("nan")
+    out = {"n": m, "r2_ssr": nan, "r2_corr": nan, "mean_rel": nan, "p50": nan, "p90": nan, "p99": nan}
+    if m == 0:
+        return out
+    my, mT = math.fsum(y.tolist()) / m, math.fsum(T.tolist()) / m
+    dy, dT = y - my, T - mT
+    sxx = math.fsum((dy * dy).tolist())
+    syy = math.fsum((dT * dT).tolist())
+    sxy = math.fsum((dy * dT).tolist())
+    ssr = math.fsum(((y - T) ** 2).tolist())
+    out["r2_ssr"] = 1.0 - ssr / sxx if sxx != 0 else nan
+    out["r2_corr"] = sxy * sxy / (sxx * syy) if sxx != 0 and syy != 0 else nan
+    rel = np.abs(T - y) / y
+    out["mean_rel"] = math.fsum(rel.tolist()) / m
+    srt = np.sort(rel)
+    for name, q in (("p50", 50), ("p90", 90), ("p99", 99)):
+        k = -(-q * m // 100)  # ceil(q m / 100), exact in integers
+        out[name] = float(srt[k - 1])
+    return out

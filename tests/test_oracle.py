@@ -276,6 +276,62 @@ def test_admit_brute_force():
 
 # ---------------------------------------------------------------- fit
 
+def test_accuracy_hand_case():
+    """Worked by hand: y = [1, 2, 4, 8], T = [1, 2.2, 3, 8] plus a non-positive
+    measurement that must be ignored; R^2 restated in exact rationals."""
+    y = np.array([1.0, 2.0, 4.0, 0.0, 8.0])
+    T = np.array([1.0, 2.2, 3.0, 5.0, 8.0])
+    a = oracle.accuracy(y, T)
+    assert a["n"] == 4
+    rel = sorted([0.0, abs(2.2 - 2.0) / 2.0, 0.25, 0.0])
+    assert a["p50"] == rel[1] and a["p90"] == rel[3] and a["p99"] == rel[3]
+    assert abs(a["mean_rel"] - sum(rel) / 4) <= 1e-16
+    ys = [Fraction(v) for v in (1.0, 2.0, 4.0, 8.0)]
+    ts = [Fraction(v) for v in (1.0, 2.2, 3.0, 8.0)]
+    my, mt = sum(ys) / 4, sum(ts) / 4
+    sxx = sum((v - my) ** 2 for v in ys)
+    syy = sum((v - mt) ** 2 for v in ts)
+    sxy = sum((u - my) * (v - mt) for u, v in zip(ys, ts))
+    ssr = sum((u - v) ** 2 for u, v in zip(ys, ts))
+    assert abs(a["r2_ssr"] - float(1 - ssr / sxx)) <= 1e-15
+    assert abs(a["r2_corr"] - float(sxy * sxy / (sxx * syy))) <= 1e-15
+
+
+def test_accuracy_invariants_and_ranks():
+    rng = np.random.default_rng(2)
+    y = rng.uniform(0.5, 2.0, 1000)
+    a = oracle.accuracy(y, y)
+    assert a["r2_ssr"] == 1.0 and a["r2_corr"] == 1.0 and a["p99"] == 0.0 and a["mean_rel"] == 0.0
+    assert oracle.accuracy(y, 2 * y)["r2_corr"] == 1.0  # an affine prediction is perfectly correlated
+    assert oracle.accuracy(y, 2 * y)["p50"] == 1.0
+    # nearest rank: with relative errors 1..100 (x 1/128) the q-th percentile is the q-th value
+    e = np.arange(1, 101) / 128.0
+    a = oracle.accuracy(np.ones(100), 1.0 + rng.permutation(e))
+    assert (a["p50"], a["p90"], a["p99"]) == (e[49], e[89], e[98])
+    a = oracle.accuracy(np.ones(1), np.array([1.5]))
+    assert a["p50"] == a["p99"] == 0.5
+    assert math.isnan(oracle.accuracy(np.zeros(3), np.ones(3))["r2_ssr"])
+
+
+def test_vtc_fit_pins():
+    """Exact recovery of a noiseless line, the line through two points, empty
+    batches skipped, degenerate cases, and agreement with numpy's least squares."""
+    S1 = np.array([3, 7, 1, 12, 5], dtype=np.int64)
+    n = np.array([1, 2, 1, 3, 0])
+    y = 0.25 + 0.0625 * S1.astype(np.float64)
+    assert oracle.vtc_fit(S1, n, y) == (0.25, 0.0625, oracle.OK, 4)
+    b, a, st, m = oracle.vtc_fit(np.array([2, 6]), np.array([1, 1]), np.array([1.0, 3.0]))
+    assert (b, a, st, m) == (0.0, 0.5, oracle.OK, 2)
+    assert oracle.vtc_fit(np.array([4, 4, 4]), np.ones(3), np.array([1.0, 2.0, 3.0]))[2] == oracle.ESINGULAR
+    assert oracle.vtc_fit(np.array([4]), np.ones(1), np.array([1.0]))[2] == oracle.ENODATA
+    rng = np.random.default_rng(4)
+    S1 = rng.integers(1, 4000, 300)
+    y = 1e-3 + 2e-6 * S1 * np.exp(0.05 * rng.standard_normal(300))
+    b, a, st, m = oracle.vtc_fit(S1, np.ones(300), y)
+    ref = np.linalg.lstsq(np.stack([np.ones(300), S1.astype(np.float64)], 1), y, rcond=None)[0]
+    assert st == oracle.OK and abs(b - ref[0]) <= 1e-9 * abs(ref[0]) and abs(a - ref[1]) <= 1e-9 * abs(ref[1])
+
+
 def _fit_data(scale=0.004, seed_noise=True):
     x = workloads.config(2, scale=scale)
     feat, seg = oracle.batch_features(x.offsets, x.p, x.c, x.phase, x.split)
