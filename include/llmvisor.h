@@ -111,6 +111,15 @@ typedef struct {
     double r2[4];        /* 1 - ssr/sst */
 } lv_fit_report;
 
+/* Accuracy of predicted batch latencies (lv_accuracy). */
+typedef struct {
+    int64_t n;           /* batches with y > 0 (the samples) */
+    double r2_ssr;       /* 1 - sum (y - T)^2 / sum (y - mean y)^2 */
+    double r2_corr;      /* squared Pearson correlation of y and T */
+    double mean_rel;     /* mean of |T - y| / y */
+    double p50, p90, p99;  /* nearest-rank percentiles of |T - y| / y */
+} lv_accuracy_report;
+
 typedef struct lv_ctx lv_ctx;
 typedef struct lv_tenant_acc lv_tenant_acc;
 
@@ -223,6 +232,29 @@ lv_status lv_tenant_acc_import(lv_tenant_acc *acc, const void *host_state, int64
  * (a data error recorded by an earlier asynchronous call is reported here). */
 lv_status lv_fit(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y, lv_model *inout,
                  lv_fit_report *rep, void *stream);
+
+/* The token-count baseline the paper compares against (VTC, Tables 1-2): for
+ * each of n_y latency vectors y (device double[n_y][n_batch], as lv_fit), one
+ * least-squares line T = beta + a * S1 over every non-empty batch, whatever its
+ * phase and regime (S1: the batch's total new tokens).  The sums come from the
+ * same exact pass as lv_fit; the 2x2 normal equations are solved with an exact
+ * integer determinant and double-double numerators.  coef: host
+ * double[n_y][2] (beta, a), written where status[k] is LV_OK; status: host
+ * int32[n_y] (LV_OK, LV_ENODATA for fewer than 2 batches, LV_ESINGULAR when
+ * every batch has the same S1); count: host int64[n_y] (batches used) or NULL.
+ * Synchronous.  Errors as lv_fit. */
+lv_status lv_fit_vtc(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y, double *coef, int32_t *status,
+                     int64_t *count, void *stream);
+
+/* Accuracy of predicted batch latencies T against measured y (both device
+ * double[n]; Section 3.2, Tables 1-2), over the batches with y > 0: both forms
+ * of R^2, the mean relative error and its nearest-rank p50/p90/p99 (the
+ * ceil(q m / 100)-th smallest of the m relative errors, exact).  Sums are fp64
+ * in a fixed order, so results repeat bit for bit.  rep: host.  With no sample
+ * every value is NaN and n = 0; an R^2 whose denominator is 0 is NaN.
+ * Synchronous. */
+lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, lv_accuracy_report *rep,
+                      void *stream);
 
 /* What-if (Section 1: admission control and what-if planning over alternative
  * batch mixes).  For every pending request j (p_new, c_new, phase_new: device

@@ -29,7 +29,8 @@ EXPORTED = [
     "lv_ctx_set_timing", "lv_ctx_kernel_time",
     "lv_features", "lv_batch_latency", "lv_attribute", "lv_tenant_acc_create", "lv_tenant_acc_destroy",
     "lv_tenant_acc_reset", "lv_tenant_accumulate", "lv_tenant_totals", "lv_tenant_acc_state_bytes",
-    "lv_tenant_acc_export", "lv_tenant_acc_import", "lv_fit", "lv_whatif", "lv_whatif_admit", "lv_attribute_noalloc",
+    "lv_tenant_acc_export", "lv_tenant_acc_import", "lv_fit", "lv_fit_vtc", "lv_accuracy", "lv_whatif",
+    "lv_whatif_admit", "lv_attribute_noalloc",
 ]
 
 
@@ -63,6 +64,12 @@ class lv_fit_report(ctypes.Structure):
                 ("ssr", ctypes.c_double * 4), ("r2", ctypes.c_double * 4)]
 
 
+class lv_accuracy_report(ctypes.Structure):
+    _fields_ = [("n", ctypes.c_int64), ("r2_ssr", ctypes.c_double), ("r2_corr", ctypes.c_double),
+                ("mean_rel", ctypes.c_double), ("p50", ctypes.c_double), ("p90", ctypes.c_double),
+                ("p99", ctypes.c_double)]
+
+
 def _load():
     if not os.path.exists(LIB_PATH):
         raise ImportError(f"LLMVisor CUDA library not built: {LIB_PATH} is missing "
@@ -90,6 +97,8 @@ def _load():
         "lv_tenant_acc_export": ([P, P, I64, P], I32),
         "lv_tenant_acc_import": ([P, P, I64, P], I32),
         "lv_fit": ([P, P, P, I32, P, P, P], I32),
+        "lv_fit_vtc": ([P, P, P, I32, P, P, P, P], I32),
+        "lv_accuracy": ([P, P, P, I64, P, P], I32),
         "lv_whatif": ([P, P, P, P, P, P, I64, P, P, P], I32),
         "lv_whatif_admit": ([P, P, P, P, P, P, P, I64, P, P, I32, ctypes.c_double, P, P, P, P], I32),
         "lv_attribute_noalloc": ([P, P, P, P, P, P], I32),
@@ -318,6 +327,27 @@ def lv_fit(ctx: Context, b: Batches, y, models: list, stream=None):
         out.append(dict(n=list(r.n), status=list(r.status), dropped=list(r.dropped), ssr=list(r.ssr),
                         r2=list(r.r2)))
     return out
+
+
+def lv_fit_vtc(ctx: Context, b: Batches, y, stream=None):
+    """y: device float64 tensor [n_y, n_batch].  Returns a list of (beta, a, status, count), one per y vector."""
+    n_y = int(y.shape[0])
+    coef = (ctypes.c_double * (2 * n_y))()
+    st = (ctypes.c_int32 * n_y)()
+    cnt = (ctypes.c_int64 * n_y)()
+    bs = b.struct()
+    _check(_lib.lv_fit_vtc(ctx.h, ctypes.byref(bs), _ptr(y), n_y, coef, st, cnt, _stream(stream)), "lv_fit_vtc")
+    nan = float("nan")
+    return [(coef[2 * k] if st[k] == 0 else nan, coef[2 * k + 1] if st[k] == 0 else nan, st[k], cnt[k])
+            for k in range(n_y)]
+
+
+def lv_accuracy(ctx: Context, y, T, stream=None) -> dict:
+    """Accuracy of predictions T against measurements y (device float64 tensors of one length)."""
+    r = lv_accuracy_report()
+    _check(_lib.lv_accuracy(ctx.h, _ptr(y), _ptr(T), int(y.numel()), ctypes.byref(r), _stream(stream)),
+           "lv_accuracy")
+    return dict(n=r.n, r2_ssr=r.r2_ssr, r2_corr=r.r2_corr, mean_rel=r.mean_rel, p50=r.p50, p90=r.p90, p99=r.p99)
 
 
 def lv_whatif(ctx: Context, model: lv_model, cand: Batches, p_new, c_new, phase_new, T_new=None, share_new=None,

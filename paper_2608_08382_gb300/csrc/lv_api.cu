@@ -13,6 +13,7 @@
 #include "llmvisor.h"
 #include "lv_fit.cuh"
 #include "lv_kernels.cuh"
+#include "lv_metrics.cuh"
 #include "lv_warp.cuh"
 #include "lv_whatif.cuh"
 
@@ -42,6 +43,8 @@ struct lv_ctx {
   std::vector<std::pair<uint64_t, int>> occ;  // (mode << 32 | dynamic smem) -> k_warps CTAs per SM
   void *d_wi = nullptr;       // what-if per-candidate / per-pending tables
   size_t wi_cap = 0;
+  void *d_acc = nullptr;      // accuracy metrics: relative-error bits, partials, histograms
+  size_t acc_cap = 0;
   int timing = 0;  // LV_TIME_* mask
   std::vector<cudaEvent_t> tev;  // start/stop pairs
   size_t tev_used = 0;
@@ -391,6 +394,69 @@ lv_status fold_tenants(lv_ctx *ctx, lv_tenant_acc *acc, cudaStream_t stream) {
   return LV_OK;
 }
 
+// The exact pass of lv_fit and lv_fit_vtc: per-CTA partials of the fit
+// statistics, reduced into totals[4 * NE]; *out points at room for the solves'
+// outputs (4 * kFitMaxY FitOut).
+lv_status fit_pass(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y, const int64_t split[2],
+                   cudaStream_t stream, FitAcc **totals_out, FitOut **out_out) {
+  lv_status st = check_batches(b, false);
+  if (st != LV_OK) return st;
+  if (b->n_batch > 0 && (!y || !aligned(y, 8))) return LV_EINVAL;
+  // scratch: per-CTA partials (at most 2048 / kBlock CTAs per SM), totals, solve output
+  const int NE = fit_entries(n_y), n_ent = 4 * NE;
+  const int64_t max_cta = max_tile_ctas(ctx->sms);
+  const size_t o_tot = ((size_t)max_cta * n_ent * sizeof(FitAcc) + 255) & ~(size_t)255;
+  const size_t o_out = (o_tot + (size_t)n_ent * sizeof(FitAcc) + 255) & ~(size_t)255;
+  const size_t need = o_out + sizeof(FitOut) * 4 * kFitMaxY;
+  if (need > ctx->fit_cap) {
+    LV_CUDA(cudaDeviceSynchronize());
+    if (ctx->d_fit) cudaFree(ctx->d_fit);
+    ctx->d_fit = nullptr;
+    ctx->fit_cap = 0;
+    if (cudaMalloc(&ctx->d_fit, need) != cudaSuccess) return LV_ENOMEM;
+    ctx->fit_cap = need;
+  }
+  unsigned char *base = static_cast<unsigned char *>(ctx->d_fit);
+  FitAcc *partial = reinterpret_cast<FitAcc *>(base);
+  FitAcc *totals = reinterpret_cast<FitAcc *>(base + o_tot);
+  FitOut *out = reinterpret_cast<FitOut *>(base + o_out);
+
+  TileArgs a{};
+  a.p = b->p;
+  a.c = b->c;
+  a.ph = b->phase;
+  a.off = b->offsets;
+  a.n_req = b->n_req;
+  a.n_batch = b->n_batch;
+  a.status = ctx->d_status;
+  a.mp.split[0] = split[0];
+  a.mp.split[1] = split[1];
+  a.fit.y = y;
+  a.fit.n_y = n_y;
+  a.fit.partial = partial;
+  ctx->last_grid = 0;
+  st = run_tiles(ctx, a, M_FEAT | M_FIT, stream);
+  if (st != LV_OK) return st;
+  const int n_cta = (int)ctx->last_grid;
+  k_fit_reduce<<<n_ent, kFitRedThreads, 0, stream>>>(partial, n_cta, n_ent, totals);
+  LV_CUDA(cudaGetLastError());
+  *totals_out = totals;
+  *out_out = out;
+  return LV_OK;
+}
+
+// Reads and clears the sticky status after a synchronous fit (syncs `stream`).
+lv_status fit_status(lv_ctx *ctx, cudaStream_t stream) {
+  int hs = 0;
+  LV_CUDA(cudaMemcpyAsync(&hs, ctx->d_status, sizeof(int), cudaMemcpyDeviceToHost, stream));
+  LV_CUDA(cudaMemsetAsync(ctx->d_status, 0, sizeof(int), stream));
+  LV_CUDA(cudaStreamSynchronize(stream));
+  if (hs & kStatusData) return LV_EDATA;
+  if (hs & kStatusOverflow) return LV_EOVERFLOW;
+  if (hs & kStatusTimeout) return LV_ETIMEOUT;
+  return LV_OK;
+}
+
 // lv_whatif and lv_whatif_admit (adm.admit null for the former).
 lv_status whatif_run(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, const int32_t *p_new,
                      const int32_t *c_new, const int32_t *phase_new, int64_t n_pending, double *T_new,
@@ -550,6 +616,7 @@ void lv_ctx_destroy(lv_ctx *ctx) {
   if (ctx->d_ktab) cudaFree(ctx->d_ktab);
   if (ctx->d_fit) cudaFree(ctx->d_fit);
   if (ctx->d_wi) cudaFree(ctx->d_wi);
+  if (ctx->d_acc) cudaFree(ctx->d_acc);
   if (ctx->ev_built) cudaEventDestroy(ctx->ev_built);
   if (ctx->ev_used) cudaEventDestroy(ctx->ev_used);
   for (cudaEvent_t e : ctx->tev) cudaEventDestroy(e);
@@ -795,61 +862,19 @@ extern "C" {
 lv_status lv_fit(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y, lv_model *inout,
                  lv_fit_report *rep, void *stream_) {
   if (!ctx || !inout || n_y < 1 || n_y > kFitMaxY) return LV_EINVAL;
-  lv_status st = check_batches(b, false);
-  if (st != LV_OK) return st;
-  if (b->n_batch > 0 && (!y || !aligned(y, 8))) return LV_EINVAL;
   for (int k = 1; k < n_y; ++k)
     if (inout[k].split[0] != inout[0].split[0] || inout[k].split[1] != inout[0].split[1]) return LV_EINVAL;
   cudaStream_t stream = (cudaStream_t)stream_;
-  // scratch: per-CTA partials (at most 2048 / kBlock CTAs per SM), totals, solve output
-  const int NE = fit_entries(n_y), n_ent = 4 * NE;
-  const int64_t max_cta = max_tile_ctas(ctx->sms);
-  const size_t o_tot = ((size_t)max_cta * n_ent * sizeof(FitAcc) + 255) & ~(size_t)255;
-  const size_t o_out = (o_tot + (size_t)n_ent * sizeof(FitAcc) + 255) & ~(size_t)255;
-  const size_t need = o_out + sizeof(FitOut) * 4 * kFitMaxY;
-  if (need > ctx->fit_cap) {
-    LV_CUDA(cudaDeviceSynchronize());
-    if (ctx->d_fit) cudaFree(ctx->d_fit);
-    ctx->d_fit = nullptr;
-    ctx->fit_cap = 0;
-    if (cudaMalloc(&ctx->d_fit, need) != cudaSuccess) return LV_ENOMEM;
-    ctx->fit_cap = need;
-  }
-  unsigned char *base = static_cast<unsigned char *>(ctx->d_fit);
-  FitAcc *partial = reinterpret_cast<FitAcc *>(base);
-  FitAcc *totals = reinterpret_cast<FitAcc *>(base + o_tot);
-  FitOut *out = reinterpret_cast<FitOut *>(base + o_out);
-
-  TileArgs a{};
-  a.p = b->p;
-  a.c = b->c;
-  a.ph = b->phase;
-  a.off = b->offsets;
-  a.n_req = b->n_req;
-  a.n_batch = b->n_batch;
-  a.status = ctx->d_status;
-  a.mp.split[0] = inout[0].split[0];
-  a.mp.split[1] = inout[0].split[1];
-  a.fit.y = y;
-  a.fit.n_y = n_y;
-  a.fit.partial = partial;
-  ctx->last_grid = 0;
-  st = run_tiles(ctx, a, M_FEAT | M_FIT, stream);
+  FitAcc *totals = nullptr;
+  FitOut *out = nullptr;
+  lv_status st = fit_pass(ctx, b, y, n_y, inout[0].split, stream, &totals, &out);
   if (st != LV_OK) return st;
-  const int n_cta = (int)ctx->last_grid;
-  k_fit_reduce<<<n_ent, kFitRedThreads, 0, stream>>>(partial, n_cta, n_ent, totals);
-  LV_CUDA(cudaGetLastError());
   k_fit_solve<<<4 * kFitMaxY, 32, 0, stream>>>(totals, n_y, out);
   LV_CUDA(cudaGetLastError());
   FitOut h[4 * kFitMaxY];
-  int hs = 0;
   LV_CUDA(cudaMemcpyAsync(h, out, sizeof(FitOut) * 4 * (size_t)n_y, cudaMemcpyDeviceToHost, stream));
-  LV_CUDA(cudaMemcpyAsync(&hs, ctx->d_status, sizeof(int), cudaMemcpyDeviceToHost, stream));
-  LV_CUDA(cudaMemsetAsync(ctx->d_status, 0, sizeof(int), stream));
-  LV_CUDA(cudaStreamSynchronize(stream));
-  if (hs & kStatusData) return LV_EDATA;
-  if (hs & kStatusOverflow) return LV_EOVERFLOW;
-  if (hs & kStatusTimeout) return LV_ETIMEOUT;
+  st = fit_status(ctx, stream);
+  if (st != LV_OK) return st;
   for (int k = 0; k < n_y; ++k) {
     for (int g = 0; g < 4; ++g) {
       const FitOut &o = h[k * 4 + g];
@@ -870,6 +895,112 @@ lv_status lv_fit(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y,
       }
     }
   }
+  return LV_OK;
+}
+
+lv_status lv_fit_vtc(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t n_y, double *coef, int32_t *status,
+                     int64_t *count, void *stream_) {
+  if (!ctx || !coef || !status || n_y < 1 || n_y > kFitMaxY) return LV_EINVAL;
+  cudaStream_t stream = (cudaStream_t)stream_;
+  FitAcc *totals = nullptr;
+  FitOut *out = nullptr;
+  const int64_t split[2] = {0, 0};  // the groups do not matter: the line pools all four
+  lv_status st = fit_pass(ctx, b, y, n_y, split, stream, &totals, &out);
+  if (st != LV_OK) return st;
+  static_assert(sizeof(VtcOut) * kFitMaxY <= sizeof(FitOut) * 4 * kFitMaxY, "VTC output fits the solve area");
+  VtcOut *vo = reinterpret_cast<VtcOut *>(out);
+  k_vtc_solve<<<1, 32, 0, stream>>>(totals, n_y, vo);
+  LV_CUDA(cudaGetLastError());
+  VtcOut h[kFitMaxY];
+  LV_CUDA(cudaMemcpyAsync(h, vo, sizeof(VtcOut) * (size_t)n_y, cudaMemcpyDeviceToHost, stream));
+  st = fit_status(ctx, stream);
+  if (st != LV_OK) return st;
+  for (int k = 0; k < n_y; ++k) {
+    status[k] = h[k].status;
+    if (count) count[k] = h[k].n;
+    if (h[k].status == LV_OK) {
+      coef[2 * k] = h[k].beta;
+      coef[2 * k + 1] = h[k].a;
+    }
+  }
+  return LV_OK;
+}
+
+lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, lv_accuracy_report *rep,
+                      void *stream_) {
+  if (!ctx || !rep || n < 0 || (n > 0 && (!y || !T || !aligned(y, 8) || !aligned(T, 8)))) return LV_EINVAL;
+  const double nan = std::nan("");
+  rep->n = 0;
+  rep->r2_ssr = rep->r2_corr = rep->mean_rel = rep->p50 = rep->p90 = rep->p99 = nan;
+  if (n == 0) return LV_OK;
+  cudaStream_t stream = (cudaStream_t)stream_;
+  const int blocks = (int)std::min<int64_t>((n + kAccBlock - 1) / kAccBlock, (int64_t)ctx->sms * 8);
+  const size_t o_part = ((size_t)n * sizeof(uint64_t) + 255) & ~(size_t)255;
+  const size_t o_sum = (o_part + sizeof(double) * 5 * (size_t)blocks + 255) & ~(size_t)255;
+  const size_t o_pf = o_sum + 256;
+  const size_t o_hist = o_pf + 256;
+  const size_t need = o_hist + sizeof(unsigned int) * kAccTargets * kAccBins;
+  if (need > ctx->acc_cap) {
+    LV_CUDA(cudaDeviceSynchronize());
+    if (ctx->d_acc) cudaFree(ctx->d_acc);
+    ctx->d_acc = nullptr;
+    ctx->acc_cap = 0;
+    if (cudaMalloc(&ctx->d_acc, need) != cudaSuccess) return LV_ENOMEM;
+    ctx->acc_cap = need;
+  }
+  unsigned char *base = static_cast<unsigned char *>(ctx->d_acc);
+  uint64_t *relbits = reinterpret_cast<uint64_t *>(base);
+  double *part = reinterpret_cast<double *>(base + o_part);
+  double *sums = reinterpret_cast<double *>(base + o_sum);  // count, sum y, sum T, then the five moments
+  uint64_t *pf = reinterpret_cast<uint64_t *>(base + o_pf);
+  unsigned int *hist = reinterpret_cast<unsigned int *>(base + o_hist);
+  k_acc_sums<<<blocks, kAccBlock, 0, stream>>>(y, T, n, relbits, part);
+  LV_CUDA(cudaGetLastError());
+  k_acc_fold<<<1, 32, 0, stream>>>(part, blocks, 3, sums);
+  LV_CUDA(cudaGetLastError());
+  k_acc_moments<<<blocks, kAccBlock, 0, stream>>>(y, T, relbits, n, sums, part);
+  LV_CUDA(cudaGetLastError());
+  k_acc_fold<<<1, 32, 0, stream>>>(part, blocks, 5, sums + 3);
+  LV_CUDA(cudaGetLastError());
+  double h[8];
+  LV_CUDA(cudaMemcpyAsync(h, sums, sizeof(h), cudaMemcpyDeviceToHost, stream));
+  LV_CUDA(cudaStreamSynchronize(stream));
+  const double m = h[0];
+  rep->n = (int64_t)m;
+  if (m == 0) return LV_OK;
+  const double sxx = h[3], syy = h[4], sxy = h[5], ssr = h[6], srel = h[7];
+  rep->r2_ssr = sxx != 0 ? 1.0 - ssr / sxx : nan;
+  rep->r2_corr = (sxx != 0 && syy != 0) ? sxy * sxy / (sxx * syy) : nan;
+  rep->mean_rel = srel / m;
+  // exact nearest-rank percentiles: ranks ceil(q m / 100), one 8-bit digit per pass
+  const int64_t mi = (int64_t)m;
+  int64_t rank[kAccTargets] = {(50 * mi + 99) / 100, (90 * mi + 99) / 100, (99 * mi + 99) / 100};
+  uint64_t prefix[kAccTargets] = {0, 0, 0};
+  unsigned int hh[kAccTargets * kAccBins];
+  for (int pass = 0; pass < 8; ++pass) {
+    const int shift = 64 - 8 * pass;
+    LV_CUDA(cudaMemcpyAsync(pf, prefix, sizeof(prefix), cudaMemcpyHostToDevice, stream));
+    LV_CUDA(cudaMemsetAsync(hist, 0, sizeof(hh), stream));
+    k_acc_hist<<<blocks, kAccBlock, 0, stream>>>(relbits, n, pf, shift, hist);
+    LV_CUDA(cudaGetLastError());
+    LV_CUDA(cudaMemcpyAsync(hh, hist, sizeof(hh), cudaMemcpyDeviceToHost, stream));
+    LV_CUDA(cudaStreamSynchronize(stream));
+    for (int t = 0; t < kAccTargets; ++t) {
+      int64_t below = 0;
+      int d = 0;
+      for (; d < kAccBins - 1; ++d) {
+        if (below + hh[t * kAccBins + d] >= rank[t]) break;
+        below += hh[t * kAccBins + d];
+      }
+      rank[t] -= below;
+      prefix[t] = (prefix[t] << 8) | (uint64_t)d;
+    }
+  }
+  double pv[kAccTargets];
+  for (int t = 0; t < kAccTargets; ++t) std::memcpy(&pv[t], &prefix[t], sizeof(double));
+  rep->p50 = pv[0];
+  rep->p90 = pv[1];
+  rep->p99 = pv[2];
   return LV_OK;
 }
 

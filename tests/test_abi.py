@@ -47,6 +47,7 @@ def test_struct_layouts(lv):
     assert ctypes.sizeof(lv.lv_model) == 4 * 5 * 8 + 16
     assert ctypes.sizeof(lv.lv_batches) == 5 * 8 + 2 * 8 + 8
     assert ctypes.sizeof(lv.lv_fit_report) == 32 + 16 + 16 + 32 + 32
+    assert ctypes.sizeof(lv.lv_accuracy_report) == 8 + 6 * 8
 
 
 def test_arch_constants_host(lv, golden_dir):
@@ -72,6 +73,8 @@ def test_invalid_arguments_rejected_before_launch(lv):
     assert L.lv_ctx_status(None, None) == lv.LV_EINVAL
     assert L.lv_tenant_acc_create(None, 4, ctypes.byref(ctypes.c_void_p())) == lv.LV_EINVAL
     assert L.lv_arch_constants(None, None, None) == lv.LV_EINVAL
+    assert L.lv_accuracy(None, None, None, 0, None, None) == lv.LV_EINVAL
+    assert L.lv_fit_vtc(None, None, None, 1, None, None, None, None) == lv.LV_EINVAL
     assert lv.lv_status_string(lv.LV_EDATA) == "invalid input data"
     assert L.lv_tenant_acc_state_bytes(None) == 0
 

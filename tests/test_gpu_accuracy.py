@@ -1,0 +1,116 @@
+"""GPU parity of the token-count baseline fit (lv_fit_vtc) and of the accuracy
+metrics (lv_accuracy) against the oracle.
+
+The VTC line is held to the fit's bar, 1e-9 relative on each coefficient
+(the oracle solves exactly and rounds once).  Accuracy: the sample count and
+the three percentiles are exact (each is one of the relative errors, computed
+by the same correctly rounded subtraction and division on both sides); R^2
+and the mean relative error within 1e-12 (fixed-order fp64 sums against
+correctly rounded ones).
+"""
+
+import numpy as np
+import pytest
+
+import oracle
+import workloads
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def lv():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2608_08382_gb300
+    return paper_2608_08382_gb300
+
+
+@pytest.fixture(scope="module")
+def ctx(lv):
+    return lv.Context()
+
+
+def _dev(a):
+    import torch
+    return torch.as_tensor(np.ascontiguousarray(a, dtype=np.float64), device="cuda")
+
+
+@pytest.mark.parametrize("scale", [0.01, 0.1])
+def test_vtc_fit_matches_oracle(lv, ctx, scale):
+    w = workloads.config(2, scale=scale)
+    T, _ = oracle.attribute(w.offsets, w.p, w.c, w.phase, w.split, w.coef)
+    Y = np.stack([T * w.noise, T])
+    b = lv.batches_to_device(w.p, w.c, w.phase, w.offsets)
+    res = lv.lv_fit_vtc(ctx, b, _dev(Y))
+    feat, _ = oracle.batch_features(w.offsets, w.p, w.c, w.phase, w.split)
+    for k in range(2):
+        beta, a, st, m = oracle.vtc_fit(feat[0], feat[3], Y[k])
+        gb, ga, gst, gm = res[k]
+        assert (gst, gm) == (st, m)
+        assert abs(gb - beta) <= 1e-9 * abs(beta) and abs(ga - a) <= 1e-9 * abs(a)
+
+
+def test_vtc_fit_degenerate(lv, ctx):
+    # every batch with the same S1: singular; one batch: no data
+    off = np.array([0, 2, 4, 6], np.int64)
+    p = np.array([3, 4, 2, 5, 6, 1], np.int32)
+    c = np.arange(6, dtype=np.int32)
+    ph = np.ones(6, np.int32)
+    b = lv.batches_to_device(p, c, ph, off)
+    assert lv.lv_fit_vtc(ctx, b, _dev(np.array([[1.0, 2.0, 3.0]])))[0][2] == lv.LV_ESINGULAR
+    b1 = lv.batches_to_device(p[:2], c[:2], ph[:2], off[:2])
+    assert lv.lv_fit_vtc(ctx, b1, _dev(np.array([[1.0]])))[0][2] == lv.LV_ENODATA
+
+
+def _check_accuracy(g, o):
+    assert g["n"] == o["n"]
+    for key in ("p50", "p90", "p99"):
+        assert g[key] == o[key], key
+    for key in ("r2_ssr", "r2_corr", "mean_rel"):
+        if np.isnan(o[key]):
+            assert np.isnan(g[key])
+        else:
+            assert abs(g[key] - o[key]) <= 1e-12 * max(1.0, abs(o[key])), key
+
+
+def test_accuracy_models_vs_vtc_config2(lv, ctx):
+    """The paper's comparison on synthetic profiles: the fitted piecewise model
+    and the token-count line, each against the noisy latencies."""
+    import torch
+    w = workloads.config(2, scale=0.05)
+    T, _ = oracle.attribute(w.offsets, w.p, w.c, w.phase, w.split, w.coef)
+    y = T * w.noise
+    b = lv.batches_to_device(w.p, w.c, w.phase, w.offsets)
+    models = [lv.make_model(np.zeros((4, 5)), w.split)]
+    lv.lv_fit(ctx, b, _dev(y[None]), models)
+    Tm = torch.empty(w.n_batch, dtype=torch.float64, device="cuda")
+    lv.lv_attribute(ctx, models[0], b, Tm, None, None)
+    beta, a, st, _ = lv.lv_fit_vtc(ctx, b, _dev(y[None]))[0]
+    assert st == lv.LV_OK
+    vtc = lv.make_model(np.tile([beta, a, 0.0, 0.0, 0.0], (4, 1)), w.split)
+    Tv = torch.empty(w.n_batch, dtype=torch.float64, device="cuda")
+    lv.lv_attribute(ctx, vtc, b, Tv, None, None)
+    yd = _dev(y)
+    gm, gv = lv.lv_accuracy(ctx, yd, Tm), lv.lv_accuracy(ctx, yd, Tv)
+    _check_accuracy(gm, oracle.accuracy(y, Tm.cpu().numpy()))
+    _check_accuracy(gv, oracle.accuracy(y, Tv.cpu().numpy()))
+    assert gm["r2_ssr"] > gv["r2_ssr"] and gm["p90"] < gv["p90"]  # the roofline form fits better
+    assert lv.lv_accuracy(ctx, yd, Tm) == gm  # fixed-order sums: bit-identical repeats
+
+
+def test_accuracy_edge_cases(lv, ctx):
+    rng = np.random.default_rng(9)
+    for n in (1, 2, 3, 257, 100_003):
+        y = rng.uniform(0.5, 2.0, n)
+        y[rng.random(n) < 0.1] = 0.0  # not samples
+        T = y * (1 + rng.normal(0, 0.1, n))
+        _check_accuracy(lv.lv_accuracy(ctx, _dev(y), _dev(T)), oracle.accuracy(y, T))
+    # ties everywhere: many equal relative errors
+    y = np.ones(1000)
+    T = 1.0 + np.repeat(np.arange(10) / 16.0, 100)
+    _check_accuracy(lv.lv_accuracy(ctx, _dev(y), _dev(T)), oracle.accuracy(y, T))
+    # no sample at all
+    g = lv.lv_accuracy(ctx, _dev(np.zeros(5)), _dev(np.ones(5)))
+    assert g["n"] == 0 and np.isnan(g["p50"]) and np.isnan(g["r2_ssr"])
