@@ -9,13 +9,15 @@ arrays resident in HBM; they are ~2.2 GB, far larger than L2, so no flush is
 needed between steps.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--workload attr1|attr4|fit2|whatif3|admit3|step] [--scale X] [--no-cpu-baseline]
+                    [--workload attr1|attr4|fit2|whatif3|admit3|acc2|step] [--scale X] [--no-cpu-baseline]
 
 attr1 (the default) is the headline line.  attr4 is the skew stress, fit2 the
 coefficient fit over 2e6 profiled batches (one step = lv_fit of a noisy and a
 noiseless latency vector), whatif3 the what-if pairs (one step = lv_whatif over
 4096 pending x 1024 candidates), admit3 the same pairs with the admission
-epilogue (lv_whatif_admit), step the single-step scheduler mode (one
+epilogue (lv_whatif_admit), acc2 the paper's accuracy comparison on the
+fit workload (lv_accuracy of the fitted model and of the token-count line
+against the noisy latencies), step the single-step scheduler mode (one
 batch of 2048 requests per step, replayed from a CUDA graph; the line adds
 us_per_step); each prints a line of the same shape with its own metric and the
 roofline of its dominant kernel.
@@ -45,7 +47,8 @@ sys.path.insert(0, ROOT)
 METRIC = "attributed requests/sec on 1 GB300; achieved HBM GB/s vs ~8 TB/s peak"
 KERNEL_SOURCES = ["paper_2608_08382_gb300/csrc/lv_kernels.cuh", "paper_2608_08382_gb300/csrc/lv_fixed.cuh",
                   "paper_2608_08382_gb300/csrc/lv_api.cu", "paper_2608_08382_gb300/csrc/lv_fit.cuh",
-                  "paper_2608_08382_gb300/csrc/lv_whatif.cuh", "paper_2608_08382_gb300/csrc/lv_warp.cuh"]
+                  "paper_2608_08382_gb300/csrc/lv_whatif.cuh", "paper_2608_08382_gb300/csrc/lv_warp.cuh",
+                  "paper_2608_08382_gb300/csrc/lv_metrics.cuh"]
 
 
 def kernel_hash() -> str:
@@ -169,6 +172,7 @@ def barrier(world):
 METRIC_FIT = "profiled requests/sec through the coefficient fit on 1 GB300"
 METRIC_WHATIF = "what-if (pending request, candidate batch) pairs/sec on 1 GB300"
 METRIC_ADMIT = "what-if pairs/sec with SLO-aware admission (per-tenant budget, latency objective) on 1 GB300"
+METRIC_ACC = "profiled batches/sec through the accuracy comparison (fitted model and token-count line) on 1 GB300"
 METRIC_STEP = "attributed requests/sec, one 2048-request serving step per CUDA-graph replay on 1 GB300"
 
 WORKLOADS = {
@@ -182,6 +186,8 @@ WORKLOADS = {
                              "4,194,304 pairs"),
     "admit3": ("admit", 3, "qwen2.5-32b tp4 what-if with admission: 1024 candidate batches x 4096 pending requests "
                            "of 64 tenants, per-tenant budgets and a latency objective, 4,194,304 pairs"),
+    "acc2": ("acc", 2, "llama3.1-8b tp1 accuracy: 2e6 profiled batches, fitted piecewise model and token-count "
+                       "(VTC) line against the noisy latencies: both R^2 forms, mean and p50/p90/p99 relative error"),
     "step": ("step", 5, "qwen2.5-14b tp2 serving step: one batch of 2048 requests (4 chunked prefills), "
                         "256 Zipf(1.1) tenants, replayed from a CUDA graph"),
 }
@@ -285,7 +291,8 @@ def _setup_step(lv, ctx, w, stream):
     return dict(step=step, e2e_step=e2e_step, units=w.n_req, unit="requests/s", metric=METRIC_STEP,
                 h2d=sum(int(t.numel() * t.element_size()) for t in hp.values()),
                 d2h=8 * (w.n_req + w.n_batch + w.n_tenants), launches_per_step=5,
-                kernel="graph", time_mask=0, graph=True, flush=True,
+                kernel="graph", time_mask=0, graph=True, whole_step=True, flush=True,
+                timed="the whole CUDA-graph replay, CUDA events on the launching stream",
                 bytes_per_launch=24.0 * w.n_req + 16.0 * w.n_batch,
                 bytes_rule="24 B/request + 16 B/batch over the whole replay (memsets, k_partition, k_warps, k_jumbo, "
                            "k_tenant_fold, k_tenant_totals): a single batch is bound by launch latency, not HBM",
@@ -294,6 +301,47 @@ def _setup_step(lv, ctx, w, stream):
                               "outside the step's events",
                         "step": "CUDA-graph replay of lv_tenant_acc_reset + lv_attribute(T, shares, tenant pass) + "
                                 "lv_tenant_totals"})
+
+
+def _setup_acc(lv, ctx, w, stream):
+    """Step: lv_accuracy of the fitted model's and of the token-count line's batch latencies against the noisy
+    ones (the fits and the latencies are formed once, before timing)."""
+    import torch
+    b = lv.batches_to_device(w.p, w.c, w.phase, w.offsets)
+    T0 = torch.empty(w.n_batch, dtype=torch.float64, device="cuda")
+    lv.lv_attribute(ctx, lv.make_model(w.coef, w.split), b, T0, None, None, stream=stream)
+    y = (T0 * torch.as_tensor(w.noise, device="cuda")).contiguous()
+    models = [lv.make_model(np.zeros((4, 5)), w.split)]
+    lv.lv_fit(ctx, b, y[None], models, stream=stream)
+    beta, a, st, _ = lv.lv_fit_vtc(ctx, b, y[None], stream=stream)[0]
+    Tm = torch.empty_like(T0)
+    Tv = torch.empty_like(T0)
+    lv.lv_attribute(ctx, models[0], b, Tm, None, None, stream=stream)
+    lv.lv_attribute(ctx, lv.make_model(np.tile([beta, a, 0.0, 0.0, 0.0], (4, 1)), w.split), b, Tv, None, None,
+                    stream=stream)
+    out = {}
+
+    def step():
+        out["model"] = lv.lv_accuracy(ctx, y, Tm, stream=stream)
+        out["vtc"] = lv.lv_accuracy(ctx, y, Tv, stream=stream)
+
+    hy, hm, hv = y.cpu().pin_memory(), Tm.cpu().pin_memory(), Tv.cpu().pin_memory()
+
+    def e2e_step():
+        y.copy_(hy, non_blocking=True)
+        Tm.copy_(hm, non_blocking=True)
+        Tv.copy_(hv, non_blocking=True)
+        step()
+
+    return dict(step=step, e2e_step=e2e_step, units=w.n_batch, unit="batches/s", metric=METRIC_ACC,
+                h2d=3 * 8 * w.n_batch, d2h=2 * 56, launches_per_step=2 * 12, kernel="accuracy", time_mask=0,
+                whole_step=True, timed="the whole step (two synchronous lv_accuracy calls), CUDA events",
+                bytes_per_launch=2 * 16.0 * w.n_batch,
+                bytes_rule="16 B/batch (y, T) read once per model; the exact percentile select re-reads 8 B/batch "
+                           "of relative-error bits per 8-bit pass (8 passes), counted as overhead",
+                config={"n_batch": w.n_batch, "seed": w.seed,
+                        "step": "lv_accuracy(y, T_model) + lv_accuracy(y, T_vtc) (synchronous)",
+                        "result": out})
 
 
 def _setup_fit(lv, ctx, w, stream):
@@ -408,7 +456,7 @@ def run_ours(args, world, rank, local):
     ctx = lv.Context()
     stream = torch.cuda.current_stream()
     s = {"attr": _setup_attr, "fit": _setup_fit, "whatif": _setup_whatif, "step": _setup_step,
-         "admit": lambda *x: _setup_whatif(*x, admit=True)}[kind](lv, ctx, w, stream)
+         "admit": lambda *x: _setup_whatif(*x, admit=True), "acc": _setup_acc}[kind](lv, ctx, w, stream)
     step = s["step"]
 
     for _ in range(args.warmup):
@@ -470,13 +518,13 @@ def run_ours(args, world, rank, local):
     step_ms = ms_max / args.steps
     value = world * s["units"] / (step_ms / 1e3)
     kavg_ms = kms / max(klaunch, 1)
-    if s.get("graph"):
-        kavg_ms, klaunch = step_ms, args.steps  # the replay is the timed unit
+    if s.get("whole_step"):
+        kavg_ms, klaunch = step_ms, args.steps  # the whole step is the timed unit
     achieved = s["bytes_per_launch"] / (kavg_ms / 1e3) / 1e9
     peak, peak_kind = measured_peaks()
     traffic = ncu_traffic(s["kernel"], args.workload)
-    timed = ("k_warps + k_jumbo, one event pair per launch pair" if s["kernel"] == "k_warps" else
-             "the whole CUDA-graph replay, CUDA events on the launching stream" if s.get("graph") else s["kernel"])
+    timed = s.get("timed") or ("k_warps + k_jumbo, one event pair per launch pair" if s["kernel"] == "k_warps"
+                               else s["kernel"])
     config = {"workload": desc, **s["config"], "parallelism": f"replicas{world}"}
     config.setdefault("l2", "inputs far larger than the 129 MB L2, no flush")
     line = {
@@ -528,6 +576,20 @@ def _oracle_sample(kind, w):
             if kind == "admit":
                 oracle.admit(T, S, un, Lh, Bh, 0.05)
         return run, rows * c.n_batch, f"first {rows} of {w.n_pending} pending requests x all {c.n_batch} candidates"
+    if kind == "acc":
+        nb = max(1, w.n_batch // 10)
+        hi = int(w.offsets[nb])
+        off = w.offsets[:nb + 1]
+        T, _ = oracle.attribute(off, w.p[:hi], w.c[:hi], w.phase[:hi], w.split, w.coef)
+        y = T * w.noise[:nb]
+        feat, _ = oracle.batch_features(off, w.p[:hi], w.c[:hi], w.phase[:hi], w.split)
+        beta, a, _, _ = oracle.vtc_fit(feat[0], feat[3], y)
+        Tv = beta + a * feat[0].astype(np.float64)
+
+        def run():
+            oracle.accuracy(y, T)
+            oracle.accuracy(y, Tv)
+        return run, nb, f"first {nb} of {w.n_batch} batches: accuracy of the generating model and of the token-count line"
     if kind == "step":
         t = w.tenant
 
@@ -567,7 +629,7 @@ def cpu_baseline(kind, w, min_seconds=10.0):
         el = time.perf_counter() - t0
         if el >= min_seconds:
             break
-    unit = "pairs/s" if kind in ("whatif", "admit") else "requests/s"
+    unit = "pairs/s" if kind in ("whatif", "admit") else "batches/s" if kind == "acc" else "requests/s"
     return {"value": done / el, "unit": unit, "cores": 1, "kind": "oracle",
             "sample": f"{sample}; repeated for {el:.1f} s, single thread"}
 
@@ -584,9 +646,9 @@ def run_reference(args, world, rank):
         run()
     el = time.perf_counter() - t0
     value = units * args.steps / el
-    unit = "pairs/s" if kind in ("whatif", "admit") else "requests/s"
+    unit = "pairs/s" if kind in ("whatif", "admit") else "batches/s" if kind == "acc" else "requests/s"
     metric = {"attr": METRIC, "fit": METRIC_FIT, "whatif": METRIC_WHATIF, "admit": METRIC_ADMIT,
-              "step": METRIC_STEP}[kind]
+              "step": METRIC_STEP, "acc": METRIC_ACC}[kind]
     return {"impl": "reference", "metric": metric, "value": value, "unit": unit, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
