@@ -9,9 +9,11 @@ arrays resident in HBM; they are ~2.2 GB, far larger than L2, so no flush is
 needed between steps.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--workload attr1|attr4|fit2|whatif3|admit3|acc2|step] [--scale X] [--no-cpu-baseline]
+                    [--workload attr1|attr1f32|attr4|fit2|whatif3|admit3|acc2|step] [--scale X]
+                    [--no-cpu-baseline]
 
-attr1 (the default) is the headline line.  attr4 is the skew stress, fit2 the
+attr1 (the default) is the headline line.  attr1f32 is the same workload through
+the single-precision variant (float T and shares).  attr4 is the skew stress, fit2 the
 coefficient fit over 2e6 profiled batches (one step = lv_fit of a noisy and a
 noiseless latency vector), whatif3 the what-if pairs (one step = lv_whatif over
 4096 pending x 1024 candidates), admit3 the same pairs with the admission
@@ -178,6 +180,8 @@ METRIC_STEP = "attributed requests/sec, one 2048-request serving step per CUDA-g
 WORKLOADS = {
     "attr1": ("attr", 1, "qwen2.5-14b tp2 continuous batching: 1e6 batches U{16..256}, ~136M requests, "
                          "256 Zipf(1.1) tenants"),
+    "attr1f32": ("attr", 1, "qwen2.5-14b tp2 continuous batching, single-precision variant (lv_attribute_f32): "
+                            "1e6 batches U{16..256}, ~136M requests, 256 Zipf(1.1) tenants"),
     "attr4": ("attr", 4, "llama3.1-8b tp1 skew: 1e7 Pareto(1.5) batches <= 4096, ~25.8M requests, "
                          "65536 Zipf(1.2) tenants"),
     "fit2": ("fit", 2, "llama3.1-8b tp1 fit: 2e6 profiled batches U{1..256}, ~257M requests, noisy (sigma 0.03) "
@@ -207,24 +211,27 @@ def _workload(args):
     return kind, w, desc
 
 
-def _setup_attr(lv, ctx, w, stream):
-    """Step: lv_attribute (T, shares, fused tenant pass) + lv_tenant_totals over config 1 or 4."""
+def _setup_attr(lv, ctx, w, stream, f32=False):
+    """Step: lv_attribute (T, shares, fused tenant pass) + lv_tenant_totals over config 1 or 4 (f32: the
+    single-precision variant, lv_attribute_f32)."""
     import torch
     b = lv.batches_to_device(w.p, w.c, w.phase, w.offsets, w.tenant, w.n_tenants)
     model = lv.make_model(w.coef, w.split)
-    T = torch.empty(w.n_batch, dtype=torch.float64, device="cuda")
-    share = torch.empty(w.n_req, dtype=torch.float64, device="cuda")
+    fdt = torch.float32 if f32 else torch.float64
+    T = torch.empty(w.n_batch, dtype=fdt, device="cuda")
+    share = torch.empty(w.n_req, dtype=fdt, device="cuda")
     L = torch.empty(w.n_tenants, dtype=torch.float64, device="cuda")
     acc = lv.TenantAcc(ctx, w.n_tenants)
+    attribute = lv.lv_attribute_f32 if f32 else lv.lv_attribute
 
     def step():
-        lv.lv_attribute(ctx, model, b, T, share, acc, stream=stream)
+        attribute(ctx, model, b, T, share, acc, stream=stream)
         lv.lv_tenant_totals(ctx, acc, L, stream=stream)
 
     hp = {k: torch.from_numpy(np.ascontiguousarray(v)).pin_memory()
           for k, v in dict(p=w.p, c=w.c, phase=w.phase, tenant=w.tenant, offsets=w.offsets).items()}
-    h_share = torch.empty(w.n_req, dtype=torch.float64).pin_memory()
-    h_T = torch.empty(w.n_batch, dtype=torch.float64).pin_memory()
+    h_share = torch.empty(w.n_req, dtype=fdt).pin_memory()
+    h_T = torch.empty(w.n_batch, dtype=fdt).pin_memory()
     h_L = torch.empty(w.n_tenants, dtype=torch.float64).pin_memory()
 
     def e2e_step():
@@ -237,9 +244,13 @@ def _setup_attr(lv, ctx, w, stream):
 
     return dict(step=step, e2e_step=e2e_step, units=w.n_req, unit="requests/s", metric=METRIC,
                 h2d=sum(int(t.numel() * t.element_size()) for t in hp.values()),
-                d2h=8 * (w.n_req + w.n_batch + w.n_tenants), launches_per_step=5,
-                kernel="k_warps", time_mask=lv.LV_TIME_TILES, bytes_per_launch=24.0 * w.n_req + 16.0 * w.n_batch,
-                bytes_rule="24 B/request (p, c, phase, tenant read; share written) + 16 B/batch (offset read; T written)",
+                d2h=(4 if f32 else 8) * (w.n_req + w.n_batch) + 8 * w.n_tenants, launches_per_step=5,
+                kernel="k_warps", time_mask=lv.LV_TIME_TILES,
+                bytes_per_launch=(20.0 if f32 else 24.0) * w.n_req + (12.0 if f32 else 16.0) * w.n_batch,
+                bytes_rule=("20 B/request (p, c, phase, tenant read; fp32 share written) + 12 B/batch (offset read; "
+                            "fp32 T written)" if f32 else
+                            "24 B/request (p, c, phase, tenant read; share written) + 16 B/batch (offset read; T written)"),
+                dtype="f32" if f32 else "f64",
                 config={"n_batch": w.n_batch, "n_req": w.n_req, "n_tenants": w.n_tenants, "seed": w.seed,
                         "step": "lv_attribute(T, shares, tenant pass) + lv_tenant_totals"})
 
@@ -456,7 +467,8 @@ def run_ours(args, world, rank, local):
     ctx = lv.Context()
     stream = torch.cuda.current_stream()
     s = {"attr": _setup_attr, "fit": _setup_fit, "whatif": _setup_whatif, "step": _setup_step,
-         "admit": lambda *x: _setup_whatif(*x, admit=True), "acc": _setup_acc}[kind](lv, ctx, w, stream)
+         "admit": lambda *x: _setup_whatif(*x, admit=True), "acc": _setup_acc}[kind](lv, ctx, w, stream) \
+        if args.workload != "attr1f32" else _setup_attr(lv, ctx, w, stream, f32=True)
     step = s["step"]
 
     for _ in range(args.warmup):
@@ -538,7 +550,7 @@ def run_ours(args, world, rank, local):
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "f64",
+        "dtype": s.get("dtype", "f64"),
         "data": "synthetic",
         "config": config,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,

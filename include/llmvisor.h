@@ -192,6 +192,17 @@ lv_status lv_batch_latency(lv_ctx *ctx, const lv_model *model, const int64_t *ba
 lv_status lv_attribute(lv_ctx *ctx, const lv_model *model, const lv_batches *b, double *T, double *share,
                        lv_tenant_acc *acc, void *stream);
 
+/* Single-precision variant of lv_attribute: T and shares evaluated in fp32
+ * (coefficients rounded to float; T by Eq. 1 in four fused multiply-adds; a
+ * share as fl(beta/n) + fl(a4 n) + p (a1 + a3 p) + a2 c in fused multiply-adds)
+ * and written as float (device float[n_batch], float[n_req], either may be
+ * NULL).  Within 1e-5 relative of the exact results for this package's
+ * workloads (shares relative to max(|share|, T/n)).  With acc, the tenant totals
+ * are the exact sums of the fp32 shares (each rounded to 2^-72 s, as
+ * lv_attribute's).  Errors as lv_attribute; float outputs 4-byte aligned. */
+lv_status lv_attribute_f32(lv_ctx *ctx, const lv_model *model, const lv_batches *b, float *T, float *share,
+                           lv_tenant_acc *acc, void *stream);
+
 /* Per-tenant accumulator (Section 2: L_u).  Every fp64 share is rounded to a
  * multiple of 2^-72 s (exact for shares of at least 2^-20 s; the rounding error
  * is below 1.1e-22 s otherwise) and summed EXACTLY in a 128-bit integer per

@@ -27,7 +27,7 @@ LV_TIME_TILES, LV_TIME_PAIRS = 1, 2
 EXPORTED = [
     "lv_status_string", "lv_arch_constants", "lv_ctx_create", "lv_ctx_destroy", "lv_ctx_set_arith", "lv_ctx_status",
     "lv_ctx_set_timing", "lv_ctx_kernel_time",
-    "lv_features", "lv_batch_latency", "lv_attribute", "lv_tenant_acc_create", "lv_tenant_acc_destroy",
+    "lv_features", "lv_batch_latency", "lv_attribute", "lv_attribute_f32", "lv_tenant_acc_create", "lv_tenant_acc_destroy",
     "lv_tenant_acc_reset", "lv_tenant_accumulate", "lv_tenant_totals", "lv_tenant_acc_state_bytes",
     "lv_tenant_acc_export", "lv_tenant_acc_import", "lv_fit", "lv_fit_vtc", "lv_accuracy", "lv_whatif",
     "lv_whatif_admit", "lv_attribute_noalloc",
@@ -88,6 +88,7 @@ def _load():
         "lv_features": ([P, P, P, P, P, P, P, P], I32),
         "lv_batch_latency": ([P, P, P, P, I64, P, P], I32),
         "lv_attribute": ([P, P, P, P, P, P, P], I32),
+        "lv_attribute_f32": ([P, P, P, P, P, P, P], I32),
         "lv_tenant_acc_create": ([P, I32, P], I32),
         "lv_tenant_acc_destroy": ([P], None),
         "lv_tenant_acc_reset": ([P, P], I32),
@@ -267,6 +268,13 @@ def lv_attribute(ctx: Context, model: lv_model, b: Batches, T=None, share=None, 
     bs = b.struct()
     _check(_lib.lv_attribute(ctx.h, ctypes.byref(model), ctypes.byref(bs), _ptr(T), _ptr(share),
                              acc.h if acc is not None else None, _stream(stream)), "lv_attribute")
+
+
+def lv_attribute_f32(ctx: Context, model: lv_model, b: "Batches", T=None, share=None, acc: "TenantAcc | None" = None,
+                     stream=None):
+    bs = b.struct()
+    _check(_lib.lv_attribute_f32(ctx.h, ctypes.byref(model), ctypes.byref(bs), _ptr(T), _ptr(share),
+                                 acc.h if acc is not None else None, _stream(stream)), "lv_attribute_f32")
 
 
 class TenantAcc:

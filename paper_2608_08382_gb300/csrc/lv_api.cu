@@ -381,6 +381,8 @@ lv_status run_tiles(lv_ctx *ctx, TileArgs &a, int mode, cudaStream_t stream) {
     case M_ATTR | M_FIX: return launch_warps_mode<M_ATTR | M_FIX>(ctx, sms, a, stream, g);
     case M_ATTR | M_TEN: return launch_warps_mode<M_ATTR | M_TEN>(ctx, sms, a, stream, g);
     case M_ATTR | M_TEN | M_FIX: return launch_warps_mode<M_ATTR | M_TEN | M_FIX>(ctx, sms, a, stream, g);
+    case M_ATTR | M_F32: return launch_warps_mode<M_ATTR | M_F32>(ctx, sms, a, stream, g);
+    case M_ATTR | M_TEN | M_F32: return launch_warps_mode<M_ATTR | M_TEN | M_F32>(ctx, sms, a, stream, g);
     case M_FEAT: return launch_warps_mode<M_FEAT>(ctx, sms, a, stream, g);
     case M_FEAT | M_FIT: return launch_warps_mode<M_FEAT | M_FIT>(ctx, sms, a, stream, g);
     default: return LV_EINVAL;
@@ -753,6 +755,45 @@ lv_status lv_attribute(lv_ctx *ctx, const lv_model *model, const lv_batches *b, 
   a.status = ctx->d_status;
   a.mp = mp;
   int mode = M_ATTR | (mp.fixed ? M_FIX : 0);
+  if (acc) {
+    mode |= M_TEN;
+    a.ten_pend = acc->d_pend;
+    a.n_tenants = acc->n_tenants;
+    a.H = std::min<int32_t>(acc->n_tenants, kHotMax);
+  }
+  st = run_tiles(ctx, a, mode, stream);
+  if (st != LV_OK) return st;
+  st = record_event(ctx->ev_used, stream);
+  if (st != LV_OK) return st;
+  if (acc) return fold_tenants(ctx, acc, stream);
+  return LV_OK;
+}
+
+lv_status lv_attribute_f32(lv_ctx *ctx, const lv_model *model, const lv_batches *b, float *T, float *share,
+                           lv_tenant_acc *acc, void *stream_) {
+  if (!ctx || check_model(model) != LV_OK) return LV_EINVAL;
+  lv_status st = check_batches(b, acc != nullptr);
+  if (st != LV_OK) return st;
+  if ((T && !aligned(T, 4)) || (share && !aligned(share, 4))) return LV_EINVAL;
+  if (acc && (acc->ctx != ctx || acc->n_tenants != b->n_tenants)) return LV_EINVAL;
+  if (!T && !share && !acc) return LV_OK;
+  cudaStream_t stream = (cudaStream_t)stream_;
+  ModelP mp;
+  st = prepare_model(ctx, model, stream, &mp);
+  if (st != LV_OK) return st;
+  TileArgs a{};
+  a.p = b->p;
+  a.c = b->c;
+  a.ph = b->phase;
+  a.ten = acc ? b->tenant : nullptr;
+  a.off = b->offsets;
+  a.n_req = b->n_req;
+  a.n_batch = b->n_batch;
+  a.T32 = T;
+  a.share32 = share;
+  a.status = ctx->d_status;
+  a.mp = mp;
+  int mode = M_ATTR | M_F32;
   if (acc) {
     mode |= M_TEN;
     a.ten_pend = acc->d_pend;

@@ -167,6 +167,7 @@ struct TileArgs {
   int64_t n_tiles;
   int64_t D;             // merge positions per tile
   double *T, *share;
+  float *T32, *share32;  // fp32 variant (M_F32): T and shares as float, or null
   int64_t *bfeat;   // [5][n_batch] or null
   uint8_t *bseg;    // [n_batch] or null
   unsigned long long *ten_pend;  // [n_tenants][4] 32-bit limbs in 64-bit words, or null
@@ -303,6 +304,40 @@ __device__ __forceinline__ bool eq1_fast(const SegFix &f, const BatchAgg &g, dou
   int ex2;
   *T = round96((uint32_t)lo, (uint32_t)(lo >> 32), (uint32_t)hi, f.E, m, ex2);
   return true;
+}
+
+// Eq. 1 in single precision (the fp32 variant): coefficients rounded to float,
+// the sums converted, four fused multiply-adds.
+__device__ __forceinline__ float eq1_f32(const double *k, const BatchAgg &g) {
+  if (g.n == 0) return 0.0f;
+  float T = __double2float_rn(k[0]);
+  T = __fmaf_rn(__double2float_rn(k[1]), (float)g.s1, T);
+  T = __fmaf_rn(__double2float_rn(k[2]), (float)g.s2, T);
+  T = __fmaf_rn(__double2float_rn(k[3]), (float)g.s3, T);
+  T = __fmaf_rn(__double2float_rn(k[4]), (float)(g.n * g.n), T);
+  return T;
+}
+
+// Single-precision share coefficients of a segment and batch size n:
+// {K = fl(beta/n) + fl(a4 n), a1, a2, a3}.
+struct Share32 {
+  float K, a1, a2, a3;
+};
+
+__device__ __forceinline__ Share32 share32_const(const double *k, int64_t n) {
+  const float fn = (float)n;
+  Share32 r;
+  r.K = n > 0 ? __fadd_rn(__fdiv_rn(__double2float_rn(k[0]), fn), __fmul_rn(__double2float_rn(k[4]), fn)) : 0.0f;
+  r.a1 = __double2float_rn(k[1]);
+  r.a2 = __double2float_rn(k[2]);
+  r.a3 = __double2float_rn(k[3]);
+  return r;
+}
+
+// K + p (a1 + a3 p) + a2 c in fused multiply-adds.
+__device__ __forceinline__ float share_f32(const Share32 &q, int32_t p, int32_t c) {
+  const float fp = (float)p;
+  return __fmaf_rn(q.a2, (float)c, __fmaf_rn(__fmaf_rn(q.a3, fp, q.a1), fp, q.K));
 }
 
 // Per-batch share constant: q = fl(beta/n), a4n = fl(a4*n), kf = fix(fl(q+a4n)).
@@ -483,6 +518,7 @@ enum : int {
   M_FEAT = 8,    // write batch features / segment codes only
   M_FIX = 16,    // fixed-point arithmetic (else fp64)
   M_FIT = 32,    // accumulate the least-squares statistics (with M_FEAT's reduction)
+  M_F32 = 64,    // single-precision T and shares (into a.T32 / a.share32), with M_ATTR
 };
 
 // Per-segment integers the share path needs, kept in shared memory so that a
@@ -510,7 +546,8 @@ __device__ __forceinline__ void emit_batch(const TileArgs &a, int64_t gb, const 
     }
     if (a.bseg) a.bseg[gb] = (uint8_t)s;
   }
-  if ((MODE & M_ATTR) && a.T) {
+  if ((MODE & M_ATTR) && (MODE & M_F32) && a.T32) a.T32[gb] = eq1_f32(a.mp.coef[s], g);
+  if ((MODE & M_ATTR) && !(MODE & M_F32) && a.T) {
     double T;
     if (!(MODE & M_FIX))
       T = eq1_fp64(a.mp.coef[s], g);

@@ -205,6 +205,38 @@ __device__ __forceinline__ bool tenant_fast(const TileArgs &a, uint32_t *tt, int
   return true;
 }
 
+// Tenant contribution of an fp32 share (the fp32 variant): its exact value
+// m24 * 2^(e - 150) re-expressed with a 53-bit significand for tenant_fast;
+// zero adds nothing, the rest (negative, subnormal, out of range) the general
+// add of its exact double.
+__device__ __forceinline__ void tenant_f32(const TileArgs &a, uint32_t *tt, int32_t u, float s, int *bad) {
+  const uint32_t bits = __float_as_uint(s);
+  const uint32_t e = (bits >> 23) & 0xffu;
+  if (!(bits >> 31) && e != 0u && e != 0xffu) {
+    const uint64_t m = (uint64_t)((bits & 0x7fffffu) | 0x800000u) << 29;
+    if (tenant_fast(a, tt, u, m, (int)e - 150 - 29)) return;
+  }
+  if (s != 0.0f) tenant_add(a, tt, u, decompose((double)s), bad);
+}
+
+// Warp-strided fp32 shares of requests [r0, r1) of one batch (the fp32 variant:
+// every request inline, no deferral).
+template <int MODE>
+__device__ __forceinline__ void big_shares_f32(const TileArgs &a, uint32_t *tt, const Share32 &q, int64_t r0,
+                                               int64_t r1, int lane, int *bad) {
+  const int32_t *P = a.p + r0, *C = a.c + r0, *U = a.ten + r0;
+  float *S = a.share32 ? a.share32 + r0 : nullptr;
+  const int n = (int)(r1 - r0);
+  for (int q0 = lane; q0 < n; q0 += 32) {
+    int32_t p = P[q0], c = C[q0];
+    p = p < 0 ? 0 : p;
+    c = c < 0 ? 0 : c;
+    const float s = share_f32(q, p, c);
+    if (S) __stcs(S + q0, s);
+    if (MODE & M_TEN) tenant_f32(a, tt, U[q0], s, bad);
+  }
+}
+
 // One request's share, its store and its tenant contribution.
 template <int MODE>
 __device__ __forceinline__ void attribute_one(const TileArgs &a, uint32_t *tt, const SegS &sg, int s, bool slow,
@@ -487,7 +519,20 @@ __device__ __forceinline__ void small_rounds(const TileArgs &a, const WSmem &ws,
     }
     const Sums tot = shfl_sums(v, in ? P - start + pn - 1 : 0);
     if (in) mys = tot;
-    if (MODE & M_ATTR) {
+    if ((MODE & M_ATTR) && (MODE & M_F32)) {
+      Share32 mq{0.0f, 0.0f, 0.0f, 0.0f};
+      if (in) {
+        const BatchAgg g{mys.s1, mys.s2, mys.s3, pn, mys.ph > 0};
+        mq = share32_const(a.mp.coef[segment_of(a.mp, g)], pn);
+      }
+      const Share32 q{__shfl_sync(kFull, mq.K, j), __shfl_sync(kFull, mq.a1, j), __shfl_sync(kFull, mq.a2, j),
+                      __shfl_sync(kFull, mq.a3, j)};
+      if (act) {
+        const float s = share_f32(q, p, c);
+        if (a.share32) __stcs(a.share32 + r, s);
+        if (MODE & M_TEN) tenant_f32(a, tt, a.ten[r], s, bad);
+      }
+    } else if (MODE & M_ATTR) {
       i128 myk = mk128(0, 0);
       int mymeta = 0;
       if (in) {
@@ -725,7 +770,11 @@ __device__ __forceinline__ void process_group(const TileArgs &a, WSmem &ws, uint
     }
     const Sums tot = big_reduce(a, r0, r1, lane, bad);
     if (lane == j) gsum[j] = tot;
-    if (kAttr) {
+    if (kAttr && (MODE & M_F32)) {
+      const BatchAgg g{tot.s1, tot.s2, tot.s3, r1 - r0, tot.ph > 0};
+      const Share32 q = share32_const(a.mp.coef[segment_of(a.mp, g)], r1 - r0);
+      big_shares_f32<MODE>(a, tt, q, r0, r1, lane, bad);
+    } else if (kAttr) {
       const BatchAgg g{tot.s1, tot.s2, tot.s3, r1 - r0, tot.ph > 0};
       const int s = segment_of(a.mp, g);
       bool slow = false;
@@ -927,7 +976,17 @@ __global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_bas
       if (tid < 4 * NE && tid / NE == s && in_range)
         fit_owner_add(facc, tid % NE, a.fit.n_y, x, a.fit.y, a.n_batch, b, g.s1 != g.s3, &bad);
     }
-    if (MODE & M_ATTR) {
+    if ((MODE & M_ATTR) && (MODE & M_F32)) {
+      const Share32 q = share32_const(a.mp.coef[s], g.n);
+      for (int64_t i = r0 + tid; i < r1; i += kJBlock) {
+        int32_t p = a.p[i], c = a.c[i];
+        p = p < 0 ? 0 : p;
+        c = c < 0 ? 0 : c;
+        const float sh = share_f32(q, p, c);
+        if (a.share32) __stcs(a.share32 + i, sh);
+        if (kTen) tenant_f32(a, tt, a.ten[i], sh, &bad);
+      }
+    } else if (MODE & M_ATTR) {
       bool slow = false;
       const i128 kf = batch_const_w<MODE>(a, nullptr, s, g.n, &slow);
       const SegS sg = js.seg[s];
