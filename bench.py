@@ -578,7 +578,7 @@ def _oracle_sample(kind, w):
     oracle.build()
     if kind in ("whatif", "admit"):
         c = w.cand
-        rows = 64
+        rows = min(64, w.n_pending)
         pn, cn, phn = w.p_new[:rows], w.c_new[:rows], w.phase_new[:rows]
         rng = np.random.default_rng(w.seed)
         un, Lh, Bh = rng.integers(0, 64, rows), rng.uniform(0, 1e-3, 64), rng.uniform(0, 2e-3, 64)
