@@ -1,6 +1,6 @@
 """GPU parity of the single-precision variant (lv_attribute_f32) against the
-fp64 oracle: T, shares and tenant totals within 1e-5 relative (shares relative
-to max(|oracle share|, T_b / n)); the tenant totals are also the exact sums of
+fp64 oracle: T, shares and tenant totals within 1e-5 relative (plain relative
+error, every coefficient positive); the tenant totals are also the exact sums of
 the fp32 shares the call returned (each rounded to 2^-72 s)."""
 
 from fractions import Fraction
@@ -48,9 +48,7 @@ def test_f32_parity(lv, cfg, scale):
     nz = T_o != 0
     assert np.all(T[~nz] == 0)
     assert np.max(np.abs(T[nz] - T_o[nz]) / np.abs(T_o[nz])) <= TOL
-    sizes = np.diff(w.offsets)
-    den = np.maximum(np.abs(s_o), np.repeat(np.abs(T_o) / np.maximum(sizes, 1), sizes))
-    assert np.max(np.abs(S - s_o) / den) <= TOL
+    assert np.max(np.abs(S - s_o) / np.abs(s_o)) <= TOL
     L_o = oracle.tenant_totals(s_o, w.tenant, w.n_tenants)
     m = L_o != 0
     assert np.max(np.abs(L[m] - L_o[m]) / np.abs(L_o[m])) <= TOL

@@ -48,9 +48,7 @@ def _run(lv, ctx, off, p, c, ph, pn, cn, phn, coef, split, arith=0):
 def _check(off, p, c, ph, pn, cn, phn, coef, split, T, S):
     To, So = oracle.whatif(off, p, c, ph, pn, cn, phn, split, coef)
     assert np.max(np.abs(T - To) / np.abs(To)) <= TOL
-    n1 = np.diff(np.asarray(off))[None, :] + 1
-    den = np.maximum(np.abs(So), np.abs(To) / n1)
-    assert np.max(np.abs(S - So) / den) <= TOL
+    assert np.max(np.abs(S - So) / np.abs(So)) <= TOL
     return To, So
 
 

@@ -1,4 +1,4 @@
-"""The allocation-free attribution entry point agrees with lv_attribute.
+"""The allocation-free attribution entry point agrees with lv_attribute and the oracle.
 
 lv_attribute_noalloc exists for callers that must not allocate device memory
 while they run -- for instance a serving engine's scheduler that has already
@@ -14,6 +14,7 @@ import ctypes
 import numpy as np
 import pytest
 
+import oracle
 import workloads
 
 pytestmark = pytest.mark.gpu
@@ -70,6 +71,11 @@ def test_noalloc_matches_lv_attribute_twice(lv):
         assert np.all(Tg[~nz] == 0)
         assert np.max(np.abs(Tg[nz] - T_ref[nz]) / np.abs(T_ref[nz])) <= TOL
         assert np.max(np.abs(sg - s_ref) / np.abs(s_ref)) <= TOL
+        # and against the CPU oracle directly
+        T_o, s_o = oracle.attribute(w.offsets, w.p, w.c, w.phase, w.split, w.coef)
+        assert np.all(Tg[T_o == 0] == 0)
+        assert np.max(np.abs(Tg[T_o != 0] - T_o[T_o != 0]) / np.abs(T_o[T_o != 0])) <= TOL
+        assert np.max(np.abs(sg - s_o) / np.abs(s_o)) <= TOL
 
 
 def test_noalloc_rejects_beyond_its_fixed_scratch(lv):
