@@ -235,6 +235,28 @@ def test_negative_coefficient_cancellation(lv, ctx):
     _check_parity(w, T, share, L, guarded=True)
 
 
+def test_outputs_only_8_byte_aligned(lv, ctx):
+    """Share and T arrays need only 8-byte alignment: an output offset by one double gives the
+    same bits as an aligned one (the kernel falls back from its 16-byte stores)."""
+    import torch
+    w = workloads.config(0, scale=0.1)
+    b = _dev(lv, w)
+    model = lv.make_model(w.coef, w.split)
+    outs = []
+    for off in (0, 1):
+        T = torch.full((w.n_batch + off,), float("nan"), dtype=torch.float64, device="cuda")[off:]
+        S = torch.full((w.n_req + off,), float("nan"), dtype=torch.float64, device="cuda")[off:]
+        a = lv.TenantAcc(ctx, w.n_tenants)
+        lv.lv_attribute(ctx, model, b, T, S, a)
+        L = torch.empty(w.n_tenants, dtype=torch.float64, device="cuda")
+        lv.lv_tenant_totals(ctx, a, L)
+        assert ctx.status() == lv.LV_OK
+        outs.append((T.cpu().numpy(), S.cpu().numpy(), L.cpu().numpy()))
+    for x, y in zip(*outs):
+        assert np.array_equal(x.view(np.int64), y.view(np.int64))
+    _check_parity(w, *outs[1])
+
+
 def test_determinism(lv, ctx):
     w = workloads.config(4, scale=0.02)
     a = _run(lv, ctx, w)
