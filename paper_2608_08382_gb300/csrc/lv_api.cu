@@ -14,7 +14,7 @@
 #include "lv_fit.cuh"
 #include "lv_kernels.cuh"
 #include "lv_metrics.cuh"
-#include "lv_stream.cuh"
+#include "lv_warp.cuh"
 #include "lv_whatif.cuh"
 
 using namespace lv;
@@ -40,7 +40,7 @@ struct lv_ctx {
   void *d_fit = nullptr;      // fit partials + solve output
   size_t fit_cap = 0;
   int64_t last_grid = 0;      // CTAs of the most recent tile-kernel launch
-  std::vector<uint64_t> configured;  // modes whose stream-kernel attributes are set
+  std::vector<std::pair<uint64_t, int>> occ;  // (mode << 32 | dynamic smem) -> k_warps CTAs per SM
   void *d_wi = nullptr;       // what-if per-candidate / per-pending tables
   size_t wi_cap = 0;
   void *d_acc = nullptr;      // accuracy metrics: relative-error bits, partials, histograms
@@ -273,58 +273,54 @@ lv_status timing_end(cudaEvent_t stop, cudaStream_t stream) {
   return LV_OK;
 }
 
-// Warps per CTA of k_stream (one CTA per SM): attribution keeps a 3-chunk
-// ring per warp, the features and fit passes do not.
+// Dynamic shared memory of k_warps for a tenant table of H entries and n_y fit vectors.
 template <int MODE>
-constexpr int stream_warps() {
-  return 16;
+size_t warps_smem(int H, int n_y) {
+  return sizeof(WSmem) + ((MODE & M_TEN) ? ten_bytes(H) : 0) +
+         ((MODE & M_FIT) ? (size_t)kWarps * 4 * fit_entries(n_y) * sizeof(FitAcc) : 0) +
+         ((MODE & M_ATTR) ? (size_t)kWarps * sizeof(DeferList) : 0);
 }
 
 constexpr int kJumboCtasPerSm = 2;
 
-// Upper bound on the CTAs of one k_stream + k_jumbo pair (rows of fit partials).
-int64_t max_tile_ctas(int sms) { return (int64_t)sms * (1 + kJumboCtasPerSm); }
+// Upper bound on the CTAs of one k_warps + k_jumbo pair (rows of fit partials).
+int64_t max_tile_ctas(int sms) { return (int64_t)sms * (2048 / kWThreads + kJumboCtasPerSm); }
 
-// Sets k_stream's and k_jumbo's dynamic shared-memory limits for MODE (once
-// per process and mode: the attribute belongs to the function, not to a
-// context).
-template <int MODE>
-lv_status configure_mode() {
-  static std::mutex mu;
-  static bool done = false;
-  std::lock_guard<std::mutex> lock(mu);
-  if (done) return LV_OK;
-  constexpr int NW = stream_warps<MODE>();
-  LV_CUDA(cudaFuncSetAttribute(k_stream<MODE, NW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)stream_smem<MODE>(kHotMax, kFitMaxY, NW)));
-  LV_CUDA(cudaFuncSetAttribute(k_jumbo<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)(sizeof(JSmem) + ten_bytes(kHotMax))));
-  done = true;
-  return LV_OK;
-}
-
-// k_stream then k_jumbo for the partitioned batches in `a` (a.part, a.ctr,
+// k_warps then k_jumbo for the partitioned batches in `a` (a.part, a.ctr,
 // a.jumbo* set, counters zeroed on `stream`).  *ctas receives the number of
 // CTAs launched (fit partial rows).  ctx may be null (no timing).
 template <int MODE>
-lv_status launch_stream_mode(lv_ctx *ctx, int sms, TileArgs &a, cudaStream_t stream, int64_t *ctas) {
+lv_status launch_warps_mode(lv_ctx *ctx, int sms, TileArgs &a, cudaStream_t stream, int64_t *ctas) {
   *ctas = 0;
-  constexpr int NW = stream_warps<MODE>();
-  lv_status st = configure_mode<MODE>();
-  if (st != LV_OK) return st;
-  const size_t smem = stream_smem<MODE>(a.H, a.fit.n_y, NW);
+  const size_t smem = warps_smem<MODE>(a.H, a.fit.n_y);
   const size_t jsmem = sizeof(JSmem) + ((MODE & M_TEN) ? ten_bytes(a.H) : 0);
-  const int64_t grid = std::min<int64_t>((a.n_tiles + NW - 1) / NW, (int64_t)sms);
+  const uint64_t key = ((uint64_t)MODE << 32) | smem;
+  int per_sm = 0;
+  if (ctx) {
+    for (const auto &e : ctx->occ)
+      if (e.first == key) per_sm = e.second;
+  }
+  if (per_sm == 0) {
+    // kernel attributes and occupancy: once per (context, mode, shared-memory size)
+    LV_CUDA(cudaFuncSetAttribute(k_warps<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)warps_smem<MODE>(kHotMax, kFitMaxY)));
+    LV_CUDA(cudaFuncSetAttribute(k_jumbo<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)(sizeof(JSmem) + ten_bytes(kHotMax))));
+    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_warps<MODE>, kWThreads, smem));
+    if (per_sm < 1) per_sm = 1;
+    if (ctx) ctx->occ.emplace_back(key, per_sm);
+  }
+  const int64_t grid = std::min<int64_t>(a.n_tiles, (int64_t)sms * per_sm);
   if (grid <= 0) return LV_OK;
-  // k_jumbo: at most one CTA per batch that can exceed kSJ requests (none for
-  // small inputs, e.g. a single serving step of a couple of hundred requests)
-  const int64_t jgrid = std::min<int64_t>((int64_t)sms * kJumboCtasPerSm, a.n_req / (kSJ + 1));
+  // k_jumbo: at most one CTA per batch that can exceed kJumbo requests (none
+  // for small inputs, e.g. a single serving step of a few hundred requests)
+  const int64_t jgrid = std::min<int64_t>((int64_t)sms * kJumboCtasPerSm, a.n_req / (kJumbo + 1));
   cudaEvent_t stop = nullptr;
   if (ctx) {
-    st = timing_begin(ctx, LV_TIME_TILES, stream, &stop);
+    lv_status st = timing_begin(ctx, LV_TIME_TILES, stream, &stop);
     if (st != LV_OK) return st;
   }
-  k_stream<MODE, NW><<<(unsigned)grid, NW * 32, smem, stream>>>(a);
+  k_warps<MODE><<<(unsigned)grid, kWThreads, smem, stream>>>(a);
   LV_CUDA(cudaGetLastError());
   if (jgrid > 0) {
     k_jumbo<MODE><<<(unsigned)jgrid, kJBlock, jsmem, stream>>>(a, (int)grid);
@@ -350,16 +346,16 @@ lv_status ensure_sched(lv_ctx *ctx, int64_t jumbo_cap) {
   return LV_OK;
 }
 
-// Most batches of more than kSJ requests that valid offsets allow.
-int64_t jumbo_bound(int64_t n_req) { return n_req / (kSJ + 1) + 1; }
+// Most batches of more than kJumbo requests that valid offsets allow.
+int64_t jumbo_bound(int64_t n_req) { return n_req / (kJumbo + 1) + 1; }
 
 // Partition + warp and jumbo kernels for the given batches.
 lv_status run_tiles(lv_ctx *ctx, TileArgs &a, int mode, cudaStream_t stream) {
   ctx->last_grid = 0;
   const int64_t units = a.n_batch + a.n_req;
-  // larger tiles cost less stream start-up; keep at least six tiles per
-  // resident warp for the dynamic schedule's tail
-  const int64_t warps = (int64_t)ctx->sms * 24;
+  // larger tiles fill the per-lane batch groups better; keep at least six tiles
+  // per resident warp for the dynamic schedule's tail
+  const int64_t warps = (int64_t)ctx->sms * (2048 / kWThreads) * kWarps;
   a.D = units / (2 * kDW) >= 6 * warps ? 2 * kDW : kDW;
   a.n_tiles = (units + a.D - 1) / a.D;
   if (a.n_batch == 0) return LV_OK;
@@ -381,14 +377,14 @@ lv_status run_tiles(lv_ctx *ctx, TileArgs &a, int mode, cudaStream_t stream) {
   int64_t *g = &ctx->last_grid;
   const int sms = ctx->sms;
   switch (mode) {
-    case M_ATTR: return launch_stream_mode<M_ATTR>(ctx, sms, a, stream, g);
-    case M_ATTR | M_FIX: return launch_stream_mode<M_ATTR | M_FIX>(ctx, sms, a, stream, g);
-    case M_ATTR | M_TEN: return launch_stream_mode<M_ATTR | M_TEN>(ctx, sms, a, stream, g);
-    case M_ATTR | M_TEN | M_FIX: return launch_stream_mode<M_ATTR | M_TEN | M_FIX>(ctx, sms, a, stream, g);
-    case M_ATTR | M_F32: return launch_stream_mode<M_ATTR | M_F32>(ctx, sms, a, stream, g);
-    case M_ATTR | M_TEN | M_F32: return launch_stream_mode<M_ATTR | M_TEN | M_F32>(ctx, sms, a, stream, g);
-    case M_FEAT: return launch_stream_mode<M_FEAT>(ctx, sms, a, stream, g);
-    case M_FEAT | M_FIT: return launch_stream_mode<M_FEAT | M_FIT>(ctx, sms, a, stream, g);
+    case M_ATTR: return launch_warps_mode<M_ATTR>(ctx, sms, a, stream, g);
+    case M_ATTR | M_FIX: return launch_warps_mode<M_ATTR | M_FIX>(ctx, sms, a, stream, g);
+    case M_ATTR | M_TEN: return launch_warps_mode<M_ATTR | M_TEN>(ctx, sms, a, stream, g);
+    case M_ATTR | M_TEN | M_FIX: return launch_warps_mode<M_ATTR | M_TEN | M_FIX>(ctx, sms, a, stream, g);
+    case M_ATTR | M_F32: return launch_warps_mode<M_ATTR | M_F32>(ctx, sms, a, stream, g);
+    case M_ATTR | M_TEN | M_F32: return launch_warps_mode<M_ATTR | M_TEN | M_F32>(ctx, sms, a, stream, g);
+    case M_FEAT: return launch_warps_mode<M_FEAT>(ctx, sms, a, stream, g);
+    case M_FEAT | M_FIT: return launch_warps_mode<M_FEAT | M_FIT>(ctx, sms, a, stream, g);
     default: return LV_EINVAL;
   }
 }
@@ -1081,7 +1077,7 @@ constexpr size_t kNoAllocPartBytes = sizeof(TilePart) * (size_t)(kNoAllocMaxTile
 constexpr size_t kNoAllocTabOffset = (kNoAllocPartBytes + 255) & ~(size_t)255;
 constexpr size_t kNoAllocCtrOffset = (kNoAllocTabOffset + sizeof(KEntry) * 4 * (kKTableN + 1) + 255) & ~(size_t)255;
 constexpr size_t kNoAllocJumboOffset = kNoAllocCtrOffset + 256;
-constexpr int64_t kNoAllocJumboCap = kNoAllocMaxTiles * kDW / (kSJ + 1) + 1;
+constexpr int64_t kNoAllocJumboCap = kNoAllocMaxTiles * kDW / (kJumbo + 1) + 1;
 constexpr size_t kNoAllocBytes = kNoAllocJumboOffset + sizeof(int64_t) * (size_t)kNoAllocJumboCap;
 
 }  // namespace
@@ -1181,6 +1177,6 @@ extern "C" lv_status lv_attribute_noalloc(const lv_model *model, const lv_batche
   k_partition<<<(unsigned)pblocks, 256, 0, stream>>>(a.off, a.n_batch, a.n_req, a.n_tiles, kDW, part, status);
   LV_CUDA(cudaGetLastError());
   int64_t ctas = 0;
-  return mp.fixed ? launch_stream_mode<M_ATTR | M_FIX>(nullptr, sms, a, stream, &ctas)
-                  : launch_stream_mode<M_ATTR>(nullptr, sms, a, stream, &ctas);
+  return mp.fixed ? launch_warps_mode<M_ATTR | M_FIX>(nullptr, sms, a, stream, &ctas)
+                  : launch_warps_mode<M_ATTR>(nullptr, sms, a, stream, &ctas);
 }

@@ -1,18 +1,55 @@
-// Warp-level building blocks shared by the request-stream kernel
-// (lv_stream.cuh) and the block-per-batch kernel k_jumbo for batches too large
-// for the stream: the decode fast path of the fixed-point share, the tenant
-// adds, the general path for the requests the fast path leaves, the fit
-// statistics of a group of batches, and k_jumbo itself.
+// Warp-centric attribution kernels (sm_103a).
+//
+// Every step of the path is a stream over request arrays, so the kernels are
+// built to keep many independent warps busy with coalesced loads and no
+// block-wide barrier while tiles are processed.
+//
+// Work decomposition.  The merge of batch boundaries and requests is cut every
+// kDW positions (k_partition); a warp tile owns the batches whose start falls
+// in its window (whole batches, no data shared with neighbours).  Persistent
+// warps take tiles from a global counter and walk each tile 32 batches at a
+// time, batch b0 + j on lane j:
+//   - a batch of kBig..kJumbo requests is reduced by the whole warp with
+//     coalesced strided loads and a butterfly sum; its segment and per-request
+//     constant follow (uniform across the warp) and its shares come from a
+//     second strided pass while its requests are still in L1;
+//   - batches of fewer than kBig requests are packed into rounds of up to 32
+//     requests (whole batches per round, one request per lane), reduced with a
+//     segmented scan across lanes and attributed in a second sweep of the same
+//     rounds;
+//   - a batch of more than kJumbo requests is queued for k_jumbo, where a whole
+//     CTA takes it, so that no warp holds a disproportionate share of the work;
+//   - T, the batch features and the fit statistics of the 32 batches are then
+//     produced with one lane per batch.
+// All sums are exact integers, so results do not depend on this schedule.
 #pragma once
 
 #include "lv_kernels.cuh"
 
 namespace lv {
 
+constexpr int kWarps = 16;                 // warps per CTA of k_warps
+constexpr int kWThreads = 32 * kWarps;
 constexpr int kDW = 1024;                  // merge positions per warp tile (large inputs: 2 kDW)
+constexpr int kJumbo = 512;                // larger batches are attributed by k_jumbo
+constexpr int kBig = 32;                   // batches with at least this many requests are processed warp-strided
 constexpr int kJBlock = 512;               // threads per CTA of k_jumbo
 constexpr int kJWarps = kJBlock / 32;
 constexpr unsigned kFull = 0xffffffffu;
+
+static_assert(kJumbo <= kNK * 4, "jumbo threshold");
+
+// Shared memory of k_warps; the tenant table (4 x H words) and, in fit mode,
+// the per-warp fit accumulators ([kWarps][4 * NE]) follow it.
+struct WSmem {
+  alignas(16) i128 kfix[4][kNK + 1];     // K at 2^E for n <= kNK (fixed-point mode)
+  alignas(16) SegS seg[4];
+  alignas(16) uint8_t kslow[4][kNK + 4];  // 1: K outside the fixed-point range
+  alignas(16) uint8_t owner[kWarps][32];  // small-batch rounds: head slot -> lane
+  alignas(16) Sums gsum[kWarps][32];      // sums of the group's big batches (kept out of registers)
+  alignas(16) SegFix fx[4];               // Eq. 1 parameters (lanes of a warp read different segments)
+};
+static_assert(sizeof(WSmem) % 16 == 0, "tenant table follows WSmem");
 
 // Shared memory of k_jumbo (tenant table follows).
 struct JSmem {
@@ -30,6 +67,11 @@ __device__ __forceinline__ Sums add_sums(Sums a, const Sums &b) {
   return a;
 }
 
+__device__ __forceinline__ Sums shfl_sums(const Sums &v, int src) {
+  return Sums{__shfl_sync(kFull, v.s1, src), __shfl_sync(kFull, v.s2, src), __shfl_sync(kFull, v.s3, src),
+              __shfl_sync(kFull, v.ph, src)};
+}
+
 __device__ __forceinline__ Sums warp_sum(Sums v) {
 #pragma unroll
   for (int d = 16; d; d >>= 1) {
@@ -40,6 +82,37 @@ __device__ __forceinline__ Sums warp_sum(Sums v) {
   }
   return v;
 }
+
+// Warp sum of per-lane sums over at most 16 requests each (s1, s2 below 2^35,
+// ph at most 16; s3 modulo 2^64, as 64-bit adds take it), from 32-bit warp
+// reductions of 27-bit pieces: 32 of them sum below 2^32.
+__device__ __forceinline__ Sums warp_sum16(const Sums &v) {
+  constexpr uint32_t kM27 = (1u << 27) - 1u;
+  const uint64_t a = (uint64_t)v.s1, b = (uint64_t)v.s2, c = (uint64_t)v.s3;
+  const uint32_t a0 = __reduce_add_sync(kFull, (uint32_t)a & kM27), a1 = __reduce_add_sync(kFull, (uint32_t)(a >> 27));
+  const uint32_t b0 = __reduce_add_sync(kFull, (uint32_t)b & kM27), b1 = __reduce_add_sync(kFull, (uint32_t)(b >> 27));
+  const uint32_t c0 = __reduce_add_sync(kFull, (uint32_t)c & kM27);
+  const uint32_t c1 = __reduce_add_sync(kFull, (uint32_t)(c >> 27) & kM27);
+  const uint32_t c2 = __reduce_add_sync(kFull, (uint32_t)(c >> 54));
+  Sums r;
+  r.s1 = (int64_t)(((uint64_t)a1 << 27) + a0);
+  r.s2 = (int64_t)(((uint64_t)b1 << 27) + b0);
+  r.s3 = (int64_t)(((uint64_t)c2 << 54) + ((uint64_t)c1 << 27) + c0);
+  r.ph = (int32_t)__reduce_add_sync(kFull, (uint32_t)v.ph);
+  return r;
+}
+
+__device__ __forceinline__ int warp_excl_scan_int(int v, int lane) {
+  int x = v;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const int y = __shfl_up_sync(kFull, x, d);
+    if (lane >= d) x += y;
+  }
+  return x - v;
+}
+
+__device__ __forceinline__ void prefetch_l2(const void *p) { asm volatile("prefetch.global.L2 [%0];" ::"l"(p)); }
 
 // ---------------------------------------------------------------- decode fast path
 //
@@ -146,6 +219,24 @@ __device__ __forceinline__ void tenant_f32(const TileArgs &a, uint32_t *tt, int3
   if (s != 0.0f) tenant_add(a, tt, u, decompose((double)s), bad);
 }
 
+// Warp-strided fp32 shares of requests [r0, r1) of one batch (the fp32 variant:
+// every request inline, no deferral).
+template <int MODE>
+__device__ __forceinline__ void big_shares_f32(const TileArgs &a, uint32_t *tt, const Share32 &q, int64_t r0,
+                                               int64_t r1, int lane, int *bad) {
+  const int32_t *P = a.p + r0, *C = a.c + r0, *U = a.ten + r0;
+  float *S = a.share32 ? a.share32 + r0 : nullptr;
+  const int n = (int)(r1 - r0);
+  for (int q0 = lane; q0 < n; q0 += 32) {
+    int32_t p = P[q0], c = C[q0];
+    p = p < 0 ? 0 : p;
+    c = c < 0 ? 0 : c;
+    const float s = share_f32(q, p, c);
+    if (S) __stcs(S + q0, s);
+    if (MODE & M_TEN) tenant_f32(a, tt, U[q0], s, bad);
+  }
+}
+
 // One request's share, its store and its tenant contribution.
 template <int MODE>
 __device__ __forceinline__ void attribute_one(const TileArgs &a, uint32_t *tt, const SegS &sg, int s, bool slow,
@@ -160,11 +251,17 @@ __device__ __forceinline__ void attribute_one(const TileArgs &a, uint32_t *tt, c
   if (MODE & M_TEN) tenant_add(a, tt, u, r, bad);
 }
 
-// Per-request constant of a batch from the model's K table: fixed-point K,
-// or {fl(beta/n), fl(a4 n)} in fp64 mode.
+// Per-request constant of a batch: fixed-point K (from the shared table for
+// n <= kNK), or {fl(beta/n), fl(a4 n)} in fp64 mode.
 template <int MODE>
-__device__ __forceinline__ i128 batch_const_w(const TileArgs &a, int s, int64_t n, bool *slow) {
-  if (MODE & M_FIX) return batch_k(a.mp, s, n, slow).kf;
+__device__ __forceinline__ i128 batch_const_w(const TileArgs &a, const WSmem *ws, int s, int64_t n, bool *slow) {
+  if (MODE & M_FIX) {
+    if (ws && n >= 1 && n <= kNK) {
+      if (ws->kslow[s][n]) *slow = true;
+      return ws->kfix[s][n];
+    }
+    return batch_k(a.mp, s, n, slow).kf;
+  }
   bool dummy = false;
   const KEntry e = batch_k(a.mp, s, n, &dummy);
   return mk128((uint64_t)__double_as_longlong(e.q), (uint64_t)__double_as_longlong(e.a4n));
@@ -208,6 +305,273 @@ struct DeferList {
   int32_t p[kDeferCap], c[kDeferCap], u[kDeferCap];
 };
 
+// Attribute the first min(cnt, 32) entries, one per lane (the batch constant
+// looked up again), move the rest (at most 31 when cnt < kDeferCap) to the
+// front and return their number.  Out of line: once per 32 deferred requests;
+// bad data is flagged in the status word directly.
+template <int MODE>
+__device__ __noinline__ int defer_flush(const TileArgs &a, uint32_t *tt, const WSmem &ws, DeferList &L, int cnt,
+                                        int lane) {
+  const int take = cnt < 32 ? cnt : 32;
+  if (lane < take) {
+    const int m = L.meta[lane];
+    const int s = m & 3;
+    const int64_t n = m >> 4;
+    bool slow = false;
+    int bad = 0;
+    const i128 kf = batch_const_w<MODE>(a, &ws, s, n, &slow);
+    defer_one<MODE>(a, tt, ws.seg, s, slow, kf, n, L.q[lane], L.p[lane], L.c[lane], L.u[lane], &bad);
+    if (bad) flag(a.status, kStatusData);
+  }
+  const int rest = cnt - take;
+  int64_t q = 0;
+  int m = 0, p = 0, c = 0, u = 0;
+  __syncwarp();
+  if (lane < rest) {
+    q = L.q[take + lane];
+    m = L.meta[take + lane];
+    p = L.p[take + lane];
+    c = L.c[take + lane];
+    u = L.u[take + lane];
+  }
+  __syncwarp();
+  if (lane < rest) {
+    L.q[lane] = q;
+    L.meta[lane] = m;
+    L.p[lane] = p;
+    L.c[lane] = c;
+    L.u[lane] = u;
+  }
+  __syncwarp();
+  return rest;
+}
+
+// Append the request of every lane with `flag` (all lanes call); attribute 32
+// at once when the list holds that many.
+template <int MODE>
+__device__ __forceinline__ void defer_push(const TileArgs &a, uint32_t *tt, const WSmem &ws, DeferList &L, int &cnt,
+                                           bool flag, int64_t q, int meta, int32_t p, int32_t c, int32_t u, int lane) {
+  const uint32_t bm = __ballot_sync(kFull, flag);
+  if (!bm) return;
+  if (flag) {
+    const int slot = cnt + __popc(bm & ((1u << lane) - 1u));
+    L.q[slot] = q;
+    L.meta[slot] = meta;
+    L.p[slot] = p;
+    L.c[slot] = c;
+    L.u[slot] = u;
+  }
+  cnt += __popc(bm);
+  __syncwarp();
+  if (cnt >= 32) cnt = defer_flush<MODE>(a, tt, ws, L, cnt, lane);
+}
+
+// Warp-strided sums over requests [r0, r1) (at most kJumbo); uniform result on
+// every lane.  Indices are 32-bit offsets from the batch's first request.  With
+// a tenant pass the tenant ids are loaded (and checked) here as well, so that
+// the share pass finds the whole batch in L1.
+__device__ __forceinline__ Sums big_reduce(const TileArgs &a, int64_t r0, int64_t r1, int lane, int *bad) {
+  const int32_t *P = a.p + r0, *C = a.c + r0, *PH = a.ph + r0;
+  const int n = (int)(r1 - r0);
+  Sums acc{0, 0, 0, 0};
+  int32_t sgn = 0, phx = 0;  // sign bits of p and c; bits of phase beyond 0/1
+  for (int i = lane; i < n; i += 4 * 32) {
+    int32_t p[4], c[4], ph[4], u[4];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      const int q = i + 32 * t;
+      const bool in = q < n;
+      u[t] = (in && a.ten) ? a.ten[r0 + q] : 0;
+      p[t] = in ? P[q] : 0;
+      c[t] = in ? C[q] : 0;
+      ph[t] = in ? PH[q] : 0;
+    }
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      sgn |= p[t] | c[t];
+      if (a.ten && (unsigned)u[t] >= (unsigned)a.n_tenants) sgn |= 0x80000000;
+      phx |= ph[t] & ~1;
+      const int32_t pt = p[t] < 0 ? 0 : p[t], ct = c[t] < 0 ? 0 : c[t];
+      acc.s1 += pt;
+      acc.s2 += ct;
+      acc.s3 += (int64_t)pt * pt;
+      acc.ph += ph[t] != 0;
+    }
+  }
+  if (sgn < 0 || phx != 0) *bad = 1;  // clamped as check_req does
+  static_assert(kJumbo <= 4 * 4 * 32, "at most 16 requests per lane");
+  return warp_sum16(acc);
+}
+
+// Warp-strided shares of requests [r0, r1) of one batch (segment s, constant kf):
+// the general loop for fp64 mode, an out-of-range constant or a wide A2 (out
+// of line: the fast loop serves the common case).
+template <int MODE>
+__device__ __noinline__ void big_shares(const TileArgs &a, uint32_t *tt, const SegS &sg, int s, bool slow,
+                                           i128 kf, int64_t r0, int64_t r1, int lane) {
+  const int64_t n = r1 - r0;
+  int bad = 0;
+  for (int64_t i = r0 + lane; i < r1; i += 4 * 32) {
+    int32_t p[4], c[4], u[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int64_t q = i + 32 * k;
+      const bool in = q < r1;
+      p[k] = in ? a.p[q] : 0;
+      c[k] = in ? a.c[q] : 0;
+      u[k] = (in && (MODE & M_TEN)) ? a.ten[q] : 0;
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int64_t q = i + 32 * k;
+      if (q < r1) {
+        const int32_t pk = p[k] < 0 ? 0 : p[k], ck = c[k] < 0 ? 0 : c[k];
+        attribute_one<MODE>(a, tt, sg, s, slow, kf, n, q, pk, ck, u[k], &bad);
+      }
+    }
+  }
+  if (bad) flag(a.status, kStatusData);
+}
+
+// Warp-strided shares of a batch whose requests take the fast path
+// (fixed-point mode, in-range constant kf, A2 < 2^64).  The batch was just
+// reduced, tenant ids included, so its requests are in L1 and the loop takes
+// one request per lane per step; every lane runs every step, so the requests
+// the fast path does not cover go to the defer list as they appear.  ALLDEC:
+// every p = 1, p is not loaded.
+template <int MODE, bool ALLDEC>
+__device__ __forceinline__ void big_shares_fast(const TileArgs &a, uint32_t *tt, const WSmem &ws, DeferList &L,
+                                                int &cnt, int s, i128 kf, int64_t r0, int64_t r1, int lane) {
+  const SegS &sg = ws.seg[s];
+  const i128 K13 = add128(kf, sg.A13);
+  const uint32_t k0 = (uint32_t)K13.lo, k1 = (uint32_t)(K13.lo >> 32), k2 = (uint32_t)K13.hi,
+                 k3 = (uint32_t)(K13.hi >> 32);
+  const uint32_t a0 = (uint32_t)sg.A2.lo, a1 = (uint32_t)(sg.A2.lo >> 32);
+  const int E = sg.E;
+  const int32_t *P = a.p + r0, *C = a.c + r0, *U = a.ten + r0;
+  double *S = a.share ? a.share + r0 : nullptr;
+  const int n = (int)(r1 - r0);
+  const int meta = (n << 4) | s;
+  for (int q0 = 0; q0 < n; q0 += 32) {
+    const int q = q0 + lane;
+    bool done = true;
+    int32_t c0 = 0, u0 = 0, p0 = 1;
+    if (q < n) {
+      c0 = C[q];
+      u0 = (MODE & M_TEN) ? U[q] : 0;
+      p0 = ALLDEC ? 1 : P[q];
+      uint32_t v0, v1, v2, v3;
+      mad_k13(k0, k1, k2, k3, a0, a1, (uint32_t)(c0 < 0 ? 0 : c0), v0, v1, v2, v3);
+      uint64_t m;
+      int ex2;
+      const double d = round96(v0, v1, v2, E, m, ex2);
+      done = (ALLDEC || p0 == 1) && v3 == 0u && v2 != 0u;
+      if (MODE & M_TEN) {
+        if (done) done = tenant_fast(a, tt, u0, m, ex2);
+      }
+      if (done && S) __stcs(S + q, d);
+    }
+    defer_push<MODE>(a, tt, ws, L, cnt, !done, r0 + q, meta, p0, c0, u0, lane);
+  }
+}
+
+// Rounds over the small batches of a group (lanes with `small`): every round
+// takes the next batches whose requests fit in 32 slots, one request per lane.
+// A segmented scan gives each batch's sums to its lane (`mys`).  With
+// attribution the same round then forms those batches' constants on their
+// lanes and attributes the round's requests, whose fields are still in
+// registers: a batch lies within one round.  pn: the lane's request count (0
+// for other lanes); P: exclusive prefix of pn; base = o0 - P so that slot q of
+// the lane's batch is request base + q.  meta = n << 4 | fast << 3 | slow << 2
+// | segment.
+template <int MODE>
+__device__ __forceinline__ void small_rounds(const TileArgs &a, const WSmem &ws, uint32_t *tt, uint8_t *owner,
+                                             DeferList *dl, int &dcnt, bool small, int pn, int P, int64_t base,
+                                             Sums &mys, int lane, int *bad) {
+  uint32_t rem = __ballot_sync(kFull, small);
+  while (rem) {
+    const int start = __shfl_sync(kFull, P, __ffs(rem) - 1);
+    const bool in = ((rem >> lane) & 1u) && (P + pn <= start + 32);
+    const uint32_t rm = __ballot_sync(kFull, in);
+    rem &= ~rm;
+    if (in) owner[P - start] = (uint8_t)lane;
+    const uint32_t H = __reduce_or_sync(kFull, in ? (1u << (P - start)) : 0u);
+    __syncwarp();
+    const int len = __shfl_sync(kFull, P + pn, 31 - __clz(rm)) - start;
+    const bool act = lane < len;
+    const int hp = act ? 31 - __clz(H & ((2u << lane) - 1u)) : 0;  // head slot of this lane's batch
+    const int j = owner[hp];
+    const int64_t r = __shfl_sync(kFull, base, j) + start + lane;
+    Sums v{0, 0, 0, 0};
+    int32_t p = 0, c = 0, ph = 0;
+    if (act) {
+      p = a.p[r];
+      c = a.c[r];
+      ph = a.ph[r];
+      check_req(p, c, ph, bad);  // clamped: the share paths clamp the same way
+      v = Sums{p, c, (int64_t)p * p, ph};
+    }
+    const int maxn = __reduce_max_sync(kFull, in ? pn : 0);
+    for (int d = 1; d < maxn; d <<= 1) {
+      const Sums w{__shfl_up_sync(kFull, v.s1, d), __shfl_up_sync(kFull, v.s2, d),
+                   __shfl_up_sync(kFull, v.s3, d), __shfl_up_sync(kFull, v.ph, d)};
+      if (lane - d >= hp) v = add_sums(v, w);
+    }
+    const Sums tot = shfl_sums(v, in ? P - start + pn - 1 : 0);
+    if (in) mys = tot;
+    if ((MODE & M_ATTR) && (MODE & M_F32)) {
+      Share32 mq{0.0f, 0.0f, 0.0f, 0.0f};
+      if (in) {
+        const BatchAgg g{mys.s1, mys.s2, mys.s3, pn, mys.ph > 0};
+        mq = share32_const(a.mp.coef[segment_of(a.mp, g)], pn);
+      }
+      const Share32 q{__shfl_sync(kFull, mq.K, j), __shfl_sync(kFull, mq.a1, j), __shfl_sync(kFull, mq.a2, j),
+                      __shfl_sync(kFull, mq.a3, j)};
+      if (act) {
+        const float s = share_f32(q, p, c);
+        if (a.share32) __stcs(a.share32 + r, s);
+        if (MODE & M_TEN) tenant_f32(a, tt, a.ten[r], s, bad);
+      }
+    } else if (MODE & M_ATTR) {
+      i128 myk = mk128(0, 0);
+      int mymeta = 0;
+      if (in) {
+        const BatchAgg g{mys.s1, mys.s2, mys.s3, pn, mys.ph > 0};
+        const int s = segment_of(a.mp, g);
+        bool slow = false;
+        myk = batch_const_w<MODE>(a, &ws, s, pn, &slow);
+        const bool fast = (MODE & M_FIX) && !slow && ws.seg[s].a2_narrow;
+        mymeta = (pn << 4) | (fast ? 8 : 0) | (slow ? 4 : 0) | s;
+      }
+      const uint64_t klo = __shfl_sync(kFull, myk.lo, j), khi = __shfl_sync(kFull, myk.hi, j);
+      const int meta = __shfl_sync(kFull, mymeta, j);
+      bool done = true;
+      int32_t u = 0;
+      if (act) {
+        done = false;
+        u = (MODE & M_TEN) ? a.ten[r] : 0;
+        if (meta & 8) {
+          const SegS &sg = ws.seg[meta & 3];
+          const i128 K13 = add128(mk128(klo, khi), sg.A13);
+          uint32_t v0, v1, v2, v3;
+          mad_k13((uint32_t)K13.lo, (uint32_t)(K13.lo >> 32), (uint32_t)K13.hi, (uint32_t)(K13.hi >> 32),
+                  (uint32_t)sg.A2.lo, (uint32_t)(sg.A2.lo >> 32), (uint32_t)c, v0, v1, v2, v3);
+          uint64_t m;
+          int ex2;
+          const double d = round96(v0, v1, v2, sg.E, m, ex2);
+          done = p == 1 && v3 == 0u && v2 != 0u;
+          if (MODE & M_TEN) {
+            if (done) done = tenant_fast(a, tt, u, m, ex2);
+          }
+          if (done && a.share) __stcs(a.share + r, d);
+        }
+      }
+      defer_push<MODE>(a, tt, ws, *dl, dcnt, !done, r, meta, p, c, u, lane);
+    }
+    __syncwarp();  // owner[] is rewritten by the next round
+  }
+}
+
 // Fit statistics of the group's batches into this warp's accumulators
 // fw[group][entry].  Entry order: 15 Gram pairs (a <= b, row order), 5 X^T y
 // columns per y vector, one y'y per y vector, one flag.  Every entry adds
@@ -223,6 +587,8 @@ struct DeferList {
 // of per-request constants, which the fit does not use.
 constexpr int kFitRecWords = 6 + 6 * kFitMaxY;
 constexpr int kFitRecs = 4;
+static_assert(sizeof(uint64_t) * kWarps * kFitRecs * kFitRecWords <= sizeof(i128) * 4 * (kNK + 1),
+              "fit record slots fit in the per-request constant table");
 
 struct FitRole {
   int xa, b0, b1, b2;  // record words of x and of B's three words
@@ -356,6 +722,101 @@ __device__ __forceinline__ void fit_group(const TileArgs &a, FitAcc *fw, uint64_
   __syncwarp();  // the record slot is rewritten by the next group
 }
 
+// One group of up to 32 consecutive batches [g0, g0 + ng) of a tile.
+template <int MODE>
+__device__ __forceinline__ void process_group(const TileArgs &a, WSmem &ws, uint32_t *tt, uint8_t *owner,
+                                              DeferList *dl, int &dcnt, FitAcc *fw, uint64_t *frec, int64_t g0, int ng,
+                                              int lane, int *bad) {
+  constexpr bool kAttr = (MODE & M_ATTR) != 0;
+  const bool valid = lane < ng;
+  int64_t o0 = valid ? a.off[g0 + lane] : 0;
+  int n = 0;  // requests of this lane's batch; 0 for jumbo batches (k_jumbo's)
+  bool jumbo = false;
+  {
+    int64_t o1 = __shfl_down_sync(kFull, o0, 1);
+    if (valid && lane == ng - 1) o1 = a.off[g0 + lane + 1];
+    if (valid) {
+      const int64_t c0 = clampi(o0, 0, a.n_req), c1 = clampi(o1, c0, a.n_req);
+      if (c0 != o0 || c1 != o1) *bad = 1;
+      o0 = c0;
+      jumbo = c1 - c0 > kJumbo;
+      n = jumbo ? 0 : (int)(c1 - c0);
+    }
+  }
+  if (jumbo) {
+    const unsigned long long slot = atomicAdd(a.jumbo_n, 1ull);
+    if (slot < (unsigned long long)a.jumbo_cap)
+      a.jumbo[slot] = g0 + lane;
+    else
+      *bad = 1;
+  }
+  Sums mys{0, 0, 0, 0};
+  Sums *gsum = ws.gsum[threadIdx.x >> 5];
+
+  // ---- big batches: reduce, constant and shares one batch at a time
+  const uint32_t big0 = __ballot_sync(kFull, n >= kBig);
+  uint32_t big = big0;
+  while (big) {
+    const int j = __ffs(big) - 1;
+    big &= big - 1;
+    const int64_t r0 = __shfl_sync(kFull, o0, j), r1 = r0 + __shfl_sync(kFull, n, j);
+    {
+      // the next 256 requests (the batches after this one) into L2 while this
+      // batch is reduced and attributed: one line per lane, 8 per array.  Not
+      // bounded by the tile: measured faster than stopping at its end.
+      const int32_t *arr = lane < 8 ? a.p : lane < 16 ? a.c : lane < 24 ? a.ph : a.ten;
+      const int64_t pq = (r1 & ~(int64_t)31) + 32 * (lane & 7);
+      if (arr && pq < a.n_req) prefetch_l2(arr + pq);
+    }
+    const Sums tot = big_reduce(a, r0, r1, lane, bad);
+    if (lane == j) gsum[j] = tot;
+    if (kAttr && (MODE & M_F32)) {
+      const BatchAgg g{tot.s1, tot.s2, tot.s3, r1 - r0, tot.ph > 0};
+      const Share32 q = share32_const(a.mp.coef[segment_of(a.mp, g)], r1 - r0);
+      big_shares_f32<MODE>(a, tt, q, r0, r1, lane, bad);
+    } else if (kAttr) {
+      const BatchAgg g{tot.s1, tot.s2, tot.s3, r1 - r0, tot.ph > 0};
+      const int s = segment_of(a.mp, g);
+      bool slow = false;
+      const i128 kf = batch_const_w<MODE>(a, &ws, s, r1 - r0, &slow);
+      if ((MODE & M_FIX) && !slow && ws.seg[s].a2_narrow) {
+        if (tot.s1 == r1 - r0 && tot.s3 == r1 - r0)
+          big_shares_fast<MODE, true>(a, tt, ws, *dl, dcnt, s, kf, r0, r1, lane);
+        else
+          big_shares_fast<MODE, false>(a, tt, ws, *dl, dcnt, s, kf, r0, r1, lane);
+      } else {
+        big_shares<MODE>(a, tt, ws.seg[s], s, slow, kf, r0, r1, lane);
+      }
+    }
+  }
+
+  if ((big0 >> lane) & 1u) mys = gsum[lane];  // slot j is written and read by lane j only
+
+  // ---- small batches: packed rounds
+  const bool small = n > 0 && n < kBig;
+  if (__any_sync(kFull, small)) {
+    const int pn = small ? n : 0;
+    const int P = warp_excl_scan_int(pn, lane);
+    const int64_t base = o0 - P;
+    small_rounds<MODE>(a, ws, tt, owner, dl, dcnt, small, pn, P, base, mys, lane, bad);
+  }
+
+  // ---- per batch: T, features; fit statistics
+  int fseg = -1;
+  if (valid && !jumbo) {
+    const BatchAgg g{mys.s1, mys.s2, mys.s3, n, mys.ph > 0};
+    const int s = segment_of(a.mp, g);
+    emit_batch<MODE>(a, g0 + lane, g, s, ws.fx);
+    if (MODE & M_FIT) {
+      const bool in_range = g.s1 < kFitFeatMax && g.s2 < kFitFeatMax && g.s3 < kFitFeatMax &&
+                            (int64_t)n * n < kFitFeatMax;
+      if (!in_range) flag(a.status, kStatusOverflow);
+      if (n > 0 && in_range) fseg = s;
+    }
+  }
+  if (MODE & M_FIT) fit_group(a, fw, frec, g0, mys, n, fseg, lane, bad);
+}
+
 // Shared-memory tables of a CTA: per-segment share parameters and, in
 // fixed-point attribution, the per-request constants for n <= kNK.
 template <int MODE>
@@ -375,8 +836,96 @@ __device__ __forceinline__ void init_segs(const TileArgs &a, SegS *seg) {
   }
 }
 
-// Batches too large for the request stream, one CTA per batch (grid-stride
-// over the queue that k_stream filled).  Fit partials go to row fit_base + CTA.
+template <int MODE>
+__global__ void __launch_bounds__(kWThreads, 2) k_warps(const TileArgs a) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  WSmem &ws = *reinterpret_cast<WSmem *>(smem_raw);
+  uint32_t *tt = reinterpret_cast<uint32_t *>(smem_raw + sizeof(WSmem));
+  constexpr bool kTen = (MODE & M_TEN) != 0;
+  constexpr bool kFit = (MODE & M_FIT) != 0;
+  static_assert(!(kFit && (MODE & M_ATTR)), "fit records share the attribution constant table");
+  FitAcc *facc = reinterpret_cast<FitAcc *>(smem_raw + sizeof(WSmem) + (kTen ? ten_bytes(a.H) : 0));
+  DeferList *dlists = reinterpret_cast<DeferList *>(smem_raw + sizeof(WSmem) + (kTen ? ten_bytes(a.H) : 0) +
+                                                    (kFit ? (size_t)kWarps * 4 * fit_entries(a.fit.n_y) * sizeof(FitAcc) : 0));
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const int NE4 = kFit ? 4 * fit_entries(a.fit.n_y) : 0;
+  int bad = 0;
+
+  if (kTen)
+    for (int i = tid; i < 4 * ten_plane(a.H); i += kWThreads) tt[i] = 0;
+  if (kFit)
+    for (int i = tid; i < kWarps * NE4; i += kWThreads) facc[i] = FitAcc{{0, 0, 0, 0}};
+  if ((MODE & M_ATTR) && tid < 4) ws.fx[tid] = a.mp.fx[tid];
+  if (MODE & M_ATTR) {
+    init_segs<MODE>(a, ws.seg);
+    if (MODE & M_FIX) {
+      for (int i = tid; i < 4 * (kNK + 1); i += kWThreads) {
+        const int s = i / (kNK + 1), n = i % (kNK + 1);
+        i128 kf = mk128(0, 0);
+        bool ovf = false;
+        if (n >= 1 && n <= a.mp.nk) {
+          kf = a.mp.ktab[s * (a.mp.nk + 1) + n].kf;  // fix(fl(q + a4n)), built once per model
+          ovf = kf.hi == kKSlowHi;
+        }
+        ws.kfix[s][n] = kf;
+        ws.kslow[s][n] = ovf ? 1 : 0;
+      }
+    }
+  }
+  __syncthreads();
+
+  uint8_t *owner = ws.owner[wid];
+  FitAcc *fw = facc + wid * NE4;
+  DeferList *dl = dlists + wid;
+  uint64_t *frec = reinterpret_cast<uint64_t *>(&ws.kfix[0][0]) + wid * kFitRecs * kFitRecWords;  // fit mode only
+  int dcnt = 0;
+  unsigned long long t = 0;
+  if (lane == 0) t = atomicAdd(a.ctr, 1ull);
+  t = __shfl_sync(kFull, t, 0);
+  while (t < (unsigned long long)a.n_tiles) {
+    unsigned long long tn = 0;
+    if (lane == 0) tn = atomicAdd(a.ctr, 1ull);  // next tile, fetched early
+    const int64_t b0 = clampi(a.part[t].b, 0, a.n_batch);
+    int64_t b1 = clampi(a.part[t + 1].b, b0, a.n_batch);
+    if (b1 - b0 > a.D) {
+      b1 = b0 + a.D;
+      bad = 1;
+    }
+    for (int64_t g0 = b0; g0 < b1; g0 += 32)
+      process_group<MODE>(a, ws, tt, owner, dl, dcnt, fw, frec, g0, (int)(b1 - g0 < 32 ? b1 - g0 : 32), lane, &bad);
+    t = __shfl_sync(kFull, tn, 0);
+  }
+  if (MODE & M_ATTR) {
+    while (dcnt > 0) dcnt = defer_flush<MODE>(a, tt, ws, *dl, dcnt, lane);
+  }
+
+  if (bad) flag(a.status, kStatusData);
+  if (kTen || kFit) __syncthreads();
+  if (kTen) {
+    for (int u = tid; u < a.H; u += kWThreads) {
+      const i128 v = hot_value(tt, a.H, u);
+      if (v.lo | v.hi) pend_add(a.ten_pend, u, v);
+    }
+  }
+  if (kFit) {
+    // this CTA's partial: exact sum over its warps (flag entries ORed)
+    const int NE = fit_entries(a.fit.n_y);
+    for (int e = tid; e < NE4; e += kWThreads) {
+      FitAcc s{{0, 0, 0, 0}};
+      for (int w = 0; w < kWarps; ++w) {
+        const FitAcc &v = facc[w * NE4 + e];
+        if (e % NE == NE - 1)
+          s.w[0] |= v.w[0];
+        else
+          acc_add256(s.w, v.w[0], v.w[1], v.w[2], v.w[3]);
+      }
+      a.fit.partial[(int64_t)blockIdx.x * NE4 + e] = s;
+    }
+  }
+}
+
+// Batches of more than kJumbo requests, one CTA per batch (grid-stride over
+// the queue that k_warps filled).  Fit partials go to row fit_base + CTA.
 template <int MODE>
 __global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_base) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -439,7 +988,7 @@ __global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_bas
       }
     } else if (MODE & M_ATTR) {
       bool slow = false;
-      const i128 kf = batch_const_w<MODE>(a, s, g.n, &slow);
+      const i128 kf = batch_const_w<MODE>(a, nullptr, s, g.n, &slow);
       const SegS sg = js.seg[s];
       // decode requests through the same fast path as k_warps; the rest general
       const bool fast = (MODE & M_FIX) && !slow && sg.a2_narrow;
