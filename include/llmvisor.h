@@ -34,8 +34,8 @@
  *    clamp and record LV_EDATA in the context's sticky status word, which
  *    lv_ctx_status() reports.  CUDA failures return LV_ECUDA.
  *  - Alignment: request arrays (p, c, phase, tenant) and offsets must be
- *    16-byte aligned (they are read with bulk asynchronous copies), fp64 outputs
- *    8-byte aligned; otherwise LV_EINVAL.
+ *    16-byte aligned (so that kernels may read them with 16-byte vector loads),
+ *    fp64 outputs 8-byte aligned; otherwise LV_EINVAL.
  *  - One lv_ctx must not be used from two host threads at once.
  *  - CUDA graphs: lv_features, lv_batch_latency, lv_attribute,
  *    lv_tenant_acc_reset, lv_tenant_accumulate, lv_tenant_totals, lv_whatif
@@ -65,7 +65,7 @@ typedef int32_t lv_status;
 #define LV_ECUDA (-5)      /* a CUDA runtime call failed */
 #define LV_EDATA (-6)      /* invalid input data seen on the device (sticky) */
 #define LV_ENOMEM (-7)     /* device allocation failed */
-#define LV_ETIMEOUT (-8)   /* a bounded device-side wait gave up */
+#define LV_ETIMEOUT (-8)   /* reserved: no current kernel waits on the device, so no call returns it */
 
 /* Model architecture; integers only.  tp is the modelled tensor-parallel degree
  * (an arithmetic input: constants are per rank).  kv_bytes is the KV-cache
@@ -136,7 +136,8 @@ void lv_ctx_destroy(lv_ctx *ctx);
 /* Select LV_ARITH_AUTO (default) or LV_ARITH_FP64. */
 lv_status lv_ctx_set_arith(lv_ctx *ctx, int32_t mode);
 /* Synchronise `stream`, then return and clear the sticky device status
- * (LV_OK or LV_EDATA / LV_ETIMEOUT). */
+ * (LV_OK, or LV_EDATA when a kernel met invalid input data since the last
+ * query). */
 lv_status lv_ctx_status(lv_ctx *ctx, void *stream);
 /* Static description of a status code. */
 const char *lv_status_string(lv_status s);
@@ -304,14 +305,14 @@ lv_status lv_whatif_admit(lv_ctx *ctx, const lv_model *model, const lv_batches *
  * Computes exactly what lv_attribute computes for T and share (no tenant
  * accumulation), with default arithmetic, using instead of an lv_ctx a fixed
  * scratch area that lives in the library image as a static device array
- * (about 1.6 MB on every GPU that loads the library, held until the process
+ * (about 2.6 MB on every GPU that loads the library, held until the process
  * exits).  It calls no cudaMalloc, cudaFree or other allocating routine.
  *  - Limit: n_batch + n_req must not exceed 67,108,864 (65,536 tiles of 1,024
  *    batch boundaries and requests); larger inputs return LV_EINVAL before
  *    anything is launched.
  *  - status: optional DEVICE int32 (caller-owned).  It is set to 0 on the
- *    stream, then kernels OR in 1 for invalid input data and 2 for a device
- *    wait that timed out; read it after synchronising the stream.
+ *    stream, then kernels OR in 1 for invalid input data (other bits are
+ *    reserved); read it after synchronising the stream.
  *  - The first call on each device looks up the scratch array's device address
  *    (cudaGetSymbolAddress) and caches it; make that first call before any
  *    stream capture.

@@ -283,6 +283,19 @@ size_t warps_smem(int H, int n_y) {
 
 constexpr int kJumboCtasPerSm = 2;
 
+// Occupancy of k_warps<MODE> for launches without a context, by (mode << 32 |
+// dynamic shared memory); the kernel attributes are process-wide as well.
+template <int MODE>
+std::vector<std::pair<uint64_t, int>> &free_occ() {
+  static std::vector<std::pair<uint64_t, int>> v;
+  return v;
+}
+template <int MODE>
+std::mutex &free_occ_mu() {
+  static std::mutex m;
+  return m;
+}
+
 // Upper bound on the CTAs of one k_warps + k_jumbo pair (rows of fit partials).
 int64_t max_tile_ctas(int sms) { return (int64_t)sms * (2048 / kWThreads + kJumboCtasPerSm); }
 
@@ -299,6 +312,11 @@ lv_status launch_warps_mode(lv_ctx *ctx, int sms, TileArgs &a, cudaStream_t stre
   if (ctx) {
     for (const auto &e : ctx->occ)
       if (e.first == key) per_sm = e.second;
+  } else {
+    // context-free callers (lv_attribute_noalloc): a process-wide cache per mode
+    std::lock_guard<std::mutex> lock(free_occ_mu<MODE>());
+    for (const auto &e : free_occ<MODE>())
+      if (e.first == key) per_sm = e.second;
   }
   if (per_sm == 0) {
     // kernel attributes and occupancy: once per (context, mode, shared-memory size)
@@ -308,7 +326,12 @@ lv_status launch_warps_mode(lv_ctx *ctx, int sms, TileArgs &a, cudaStream_t stre
                                  (int)(sizeof(JSmem) + ten_bytes(kHotMax))));
     LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_warps<MODE>, kWThreads, smem));
     if (per_sm < 1) per_sm = 1;
-    if (ctx) ctx->occ.emplace_back(key, per_sm);
+    if (ctx) {
+      ctx->occ.emplace_back(key, per_sm);
+    } else {
+      std::lock_guard<std::mutex> lock(free_occ_mu<MODE>());
+      free_occ<MODE>().emplace_back(key, per_sm);
+    }
   }
   const int64_t grid = std::min<int64_t>(a.n_tiles, (int64_t)sms * per_sm);
   if (grid <= 0) return LV_OK;
@@ -455,7 +478,6 @@ lv_status fit_status(lv_ctx *ctx, cudaStream_t stream) {
   LV_CUDA(cudaStreamSynchronize(stream));
   if (hs & kStatusData) return LV_EDATA;
   if (hs & kStatusOverflow) return LV_EOVERFLOW;
-  if (hs & kStatusTimeout) return LV_ETIMEOUT;
   return LV_OK;
 }
 
@@ -546,7 +568,7 @@ const char *lv_status_string(lv_status s) {
     case LV_ECUDA: return "CUDA error";
     case LV_EDATA: return "invalid input data";
     case LV_ENOMEM: return "out of device memory";
-    case LV_ETIMEOUT: return "device wait timed out";
+    case LV_ETIMEOUT: return "reserved status (device wait timed out)";
     default: return "unknown status";
   }
 }
@@ -660,7 +682,6 @@ lv_status lv_ctx_status(lv_ctx *ctx, void *stream) {
   LV_CUDA(cudaMemcpy(&h, ctx->d_status, sizeof(int), cudaMemcpyDeviceToHost));
   LV_CUDA(cudaMemset(ctx->d_status, 0, sizeof(int)));
   if (h & kStatusData) return LV_EDATA;
-  if (h & kStatusTimeout) return LV_ETIMEOUT;
   return LV_OK;
 }
 
@@ -1079,6 +1100,8 @@ constexpr size_t kNoAllocCtrOffset = (kNoAllocTabOffset + sizeof(KEntry) * 4 * (
 constexpr size_t kNoAllocJumboOffset = kNoAllocCtrOffset + 256;
 constexpr int64_t kNoAllocJumboCap = kNoAllocMaxTiles * kDW / (kJumbo + 1) + 1;
 constexpr size_t kNoAllocBytes = kNoAllocJumboOffset + sizeof(int64_t) * (size_t)kNoAllocJumboCap;
+// the size stated in include/llmvisor.h ("about 2.6 MB")
+static_assert(kNoAllocBytes > 2500000 && kNoAllocBytes < 2700000, "no-alloc scratch size as documented");
 
 }  // namespace
 

@@ -17,8 +17,9 @@ constexpr int kNK = 256;                           // per-batch constants cached
 constexpr int64_t kPMaxFix = 1ll << 24;            // p beyond this uses the fp64 share path
 constexpr int kTenLsb = -72;                       // tenant totals: shares rounded to 2^-72 s, summed exactly
 
+// Bits of the sticky status word: invalid input data; a fit feature beyond
+// the exact range (bit 2 is reserved).
 constexpr int kStatusData = 1;
-constexpr int kStatusTimeout = 2;
 constexpr int kStatusOverflow = 4;
 
 struct SegFix {
