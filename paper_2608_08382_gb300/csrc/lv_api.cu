@@ -999,8 +999,7 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   const int blocks = (int)std::min<int64_t>((n + kAccBlock - 1) / kAccBlock, (int64_t)ctx->sms * 8);
   const size_t o_part = ((size_t)n * sizeof(uint64_t) + 255) & ~(size_t)255;
   const size_t o_sum = (o_part + sizeof(double) * 5 * (size_t)blocks + 255) & ~(size_t)255;
-  const size_t o_pf = o_sum + 256;
-  const size_t o_hist = o_pf + 256;
+  const size_t o_hist = o_sum + 256;  // sums (8 doubles), prefixes (3), ranks (3): 112 bytes
   const size_t need = o_hist + sizeof(unsigned int) * kAccTargets * kAccBins;
   if (need > ctx->acc_cap) {
     LV_CUDA(cudaDeviceSynchronize());
@@ -1014,7 +1013,8 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   uint64_t *relbits = reinterpret_cast<uint64_t *>(base);
   double *part = reinterpret_cast<double *>(base + o_part);
   double *sums = reinterpret_cast<double *>(base + o_sum);  // count, sum y, sum T, then the five moments
-  uint64_t *pf = reinterpret_cast<uint64_t *>(base + o_pf);
+  uint64_t *pf = reinterpret_cast<uint64_t *>(base + o_sum + 64);
+  int64_t *rk = reinterpret_cast<int64_t *>(base + o_sum + 88);
   unsigned int *hist = reinterpret_cast<unsigned int *>(base + o_hist);
   k_acc_sums<<<blocks, kAccBlock, 0, stream>>>(y, T, n, relbits, part);
   LV_CUDA(cudaGetLastError());
@@ -1024,7 +1024,15 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   LV_CUDA(cudaGetLastError());
   k_acc_fold<<<1, 32, 0, stream>>>(part, blocks, 5, sums + 3);
   LV_CUDA(cudaGetLastError());
-  double h[8];
+  // exact nearest-rank percentiles: one 8-bit digit per pass, picked on the device
+  LV_CUDA(cudaMemsetAsync(hist, 0, sizeof(unsigned int) * kAccTargets * kAccBins, stream));
+  for (int pass = 0; pass < 8; ++pass) {
+    k_acc_hist<<<blocks, kAccBlock, 0, stream>>>(relbits, n, pf, 64 - 8 * pass, hist);
+    LV_CUDA(cudaGetLastError());
+    k_acc_pick<<<1, 32, 0, stream>>>(hist, sums, pf, rk, pass);
+    LV_CUDA(cudaGetLastError());
+  }
+  double h[11];  // eight sums, then the three percentile bit patterns
   LV_CUDA(cudaMemcpyAsync(h, sums, sizeof(h), cudaMemcpyDeviceToHost, stream));
   LV_CUDA(cudaStreamSynchronize(stream));
   const double m = h[0];
@@ -1034,35 +1042,9 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   rep->r2_ssr = sxx != 0 ? 1.0 - ssr / sxx : nan;
   rep->r2_corr = (sxx != 0 && syy != 0) ? sxy * sxy / (sxx * syy) : nan;
   rep->mean_rel = srel / m;
-  // exact nearest-rank percentiles: ranks ceil(q m / 100), one 8-bit digit per pass
-  const int64_t mi = (int64_t)m;
-  int64_t rank[kAccTargets] = {(50 * mi + 99) / 100, (90 * mi + 99) / 100, (99 * mi + 99) / 100};
-  uint64_t prefix[kAccTargets] = {0, 0, 0};
-  unsigned int hh[kAccTargets * kAccBins];
-  for (int pass = 0; pass < 8; ++pass) {
-    const int shift = 64 - 8 * pass;
-    LV_CUDA(cudaMemcpyAsync(pf, prefix, sizeof(prefix), cudaMemcpyHostToDevice, stream));
-    LV_CUDA(cudaMemsetAsync(hist, 0, sizeof(hh), stream));
-    k_acc_hist<<<blocks, kAccBlock, 0, stream>>>(relbits, n, pf, shift, hist);
-    LV_CUDA(cudaGetLastError());
-    LV_CUDA(cudaMemcpyAsync(hh, hist, sizeof(hh), cudaMemcpyDeviceToHost, stream));
-    LV_CUDA(cudaStreamSynchronize(stream));
-    for (int t = 0; t < kAccTargets; ++t) {
-      int64_t below = 0;
-      int d = 0;
-      for (; d < kAccBins - 1; ++d) {
-        if (below + hh[t * kAccBins + d] >= rank[t]) break;
-        below += hh[t * kAccBins + d];
-      }
-      rank[t] -= below;
-      prefix[t] = (prefix[t] << 8) | (uint64_t)d;
-    }
-  }
-  double pv[kAccTargets];
-  for (int t = 0; t < kAccTargets; ++t) std::memcpy(&pv[t], &prefix[t], sizeof(double));
-  rep->p50 = pv[0];
-  rep->p90 = pv[1];
-  rep->p99 = pv[2];
+  rep->p50 = h[8];
+  rep->p90 = h[9];
+  rep->p99 = h[10];
   return LV_OK;
 }
 

@@ -9,8 +9,8 @@
 // tree per block, then the block partials in index order), so results repeat
 // bit for bit.  The percentiles are exact: rel is a non-negative double, so its
 // bit pattern orders like its value, and a most-significant-digit radix select
-// (8 bits per pass, one shared-memory histogram per block) finds the bit
-// pattern of the element of each target rank.
+// (8 bits per pass, one shared-memory histogram per block, the digit chosen on
+// the device) finds the bit pattern of the element of each target rank.
 #pragma once
 
 #include <cstdint>
@@ -133,6 +133,40 @@ __global__ void __launch_bounds__(kAccBlock) k_acc_hist(const uint64_t *__restri
     const unsigned int c = (&h[0][0])[i];
     if (c) atomicAdd(hist + i, c);
   }
+}
+
+// After a histogram pass: for each target, the digit whose bin holds its rank
+// (ranks ceil(q m / 100), q = 50, 90, 99, set from the sample count m at the
+// first pass), appended to its prefix; the histograms are cleared for the next
+// pass.  One warp: lane t < 3 takes target t.  All passes then run back to back
+// on the stream with no host round trip.
+__global__ void __launch_bounds__(32) k_acc_pick(unsigned int *__restrict__ hist, const double *__restrict__ sums,
+                                                 uint64_t *__restrict__ prefix, int64_t *__restrict__ rank, int pass) {
+  const int t = threadIdx.x;
+  if (t < kAccTargets) {
+    int64_t r;
+    uint64_t pf;
+    if (pass == 0) {
+      const int64_t m = (int64_t)sums[0];
+      const int64_t q = t == 0 ? 50 : t == 1 ? 90 : 99;
+      r = (q * m + 99) / 100;
+      pf = 0;
+    } else {
+      r = rank[t];
+      pf = prefix[t];
+    }
+    int64_t below = 0;
+    int d = 0;
+    for (; d < kAccBins - 1; ++d) {
+      const unsigned int c = hist[t * kAccBins + d];
+      if (below + c >= r) break;
+      below += c;
+    }
+    rank[t] = r - below;
+    prefix[t] = (pf << 8) | (uint64_t)d;
+  }
+  __syncwarp();
+  for (int i = t; i < kAccTargets * kAccBins; i += 32) hist[i] = 0u;
 }
 
 // ---------------------------------------------------------------- token-count baseline
