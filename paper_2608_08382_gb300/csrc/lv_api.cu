@@ -412,6 +412,24 @@ lv_status run_tiles(lv_ctx *ctx, TileArgs &a, int mode, cudaStream_t stream) {
   }
 }
 
+// The single-CTA path for small inputs (k_small); state: the tenant
+// accumulator's exact state, or null.
+lv_status run_small(lv_ctx *ctx, TileArgs &a, int mode, i128 *state, cudaStream_t stream) {
+  const size_t smem = sizeof(SmallSmem) + ((mode & M_TEN) ? ten_bytes(a.H) : 0);
+  cudaEvent_t stop = nullptr;
+  lv_status st = timing_begin(ctx, LV_TIME_TILES, stream, &stop);
+  if (st != LV_OK) return st;
+  switch (mode) {
+    case M_ATTR: k_small<M_ATTR><<<1, kSmallThreads, smem, stream>>>(a, state); break;
+    case M_ATTR | M_FIX: k_small<M_ATTR | M_FIX><<<1, kSmallThreads, smem, stream>>>(a, state); break;
+    case M_ATTR | M_TEN: k_small<M_ATTR | M_TEN><<<1, kSmallThreads, smem, stream>>>(a, state); break;
+    case M_ATTR | M_TEN | M_FIX: k_small<M_ATTR | M_TEN | M_FIX><<<1, kSmallThreads, smem, stream>>>(a, state); break;
+    default: return LV_EINVAL;
+  }
+  LV_CUDA(cudaGetLastError());
+  return timing_end(stop, stream);
+}
+
 lv_status fold_tenants(lv_ctx *ctx, lv_tenant_acc *acc, cudaStream_t stream) {
   const int n = acc->n_tenants;
   k_tenant_fold<<<(n + 255) / 256, 256, 0, stream>>>(acc->d_pend, acc->d_state, n, ctx->d_status);
@@ -781,6 +799,15 @@ lv_status lv_attribute(lv_ctx *ctx, const lv_model *model, const lv_batches *b, 
     a.ten_pend = acc->d_pend;
     a.n_tenants = acc->n_tenants;
     a.H = std::min<int32_t>(acc->n_tenants, kHotMax);
+  }
+  if (b->n_req <= kSmallMaxReq && b->n_batch <= kSmallMaxBatch && b->n_batch > 0) {
+    // one serving step: a single CTA, no partition, scheduling counters or fold
+    st = run_small(ctx, a, mode, acc ? acc->d_state : nullptr, stream);
+    if (st != LV_OK) return st;
+    st = record_event(ctx->ev_used, stream);
+    if (st != LV_OK) return st;
+    if (acc && acc->n_tenants > kHotMax) return fold_tenants(ctx, acc, stream);
+    return LV_OK;
   }
   st = run_tiles(ctx, a, mode, stream);
   if (st != LV_OK) return st;

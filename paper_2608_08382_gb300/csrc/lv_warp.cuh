@@ -1032,4 +1032,92 @@ __global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_bas
   }
 }
 
+// ---------------------------------------------------------------- small inputs
+
+// A serving scheduler attributes one step's batch (a few thousand requests) at
+// a time, where launch latency, not bandwidth, bounds the call.  For such
+// inputs lv_attribute runs this single CTA instead of the partition, tile,
+// jumbo and fold kernels: it takes the batches one after another, each with a
+// block-wide reduction, forms T and every share, and adds its shared-memory
+// tenant table straight into the exact per-tenant state (tenant ids from H up
+// still go to the pending limbs, which the caller folds).
+constexpr int kSmallThreads = 1024;
+constexpr int kSmallWarps = kSmallThreads / 32;
+constexpr int64_t kSmallMaxReq = 8192;
+constexpr int64_t kSmallMaxBatch = 16;
+
+struct SmallSmem {
+  alignas(16) SegS seg[4];
+  alignas(16) Sums red[kSmallWarps];
+  alignas(16) Sums tot;
+};
+static_assert(sizeof(SmallSmem) % 16 == 0, "tenant table follows SmallSmem");
+
+template <int MODE>
+__global__ void __launch_bounds__(kSmallThreads) k_small(const TileArgs a, i128 *state) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  SmallSmem &ss = *reinterpret_cast<SmallSmem *>(smem_raw);
+  uint32_t *tt = reinterpret_cast<uint32_t *>(smem_raw + sizeof(SmallSmem));
+  constexpr bool kTen = (MODE & M_TEN) != 0;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  int bad = 0;
+  if (kTen)
+    for (int i = tid; i < 4 * ten_plane(a.H); i += kSmallThreads) tt[i] = 0;
+  init_segs<MODE>(a, ss.seg);
+  __syncthreads();
+  int64_t prev = 0;
+  for (int64_t b = 0; b < a.n_batch; ++b) {
+    const int64_t o0 = a.off[b], o1 = a.off[b + 1];
+    const int64_t r0 = clampi(o0, prev, a.n_req), r1 = clampi(o1, r0, a.n_req);
+    if (r0 != o0 || r1 != o1 || (b == 0 && o0 != 0) || (b == a.n_batch - 1 && o1 != a.n_req)) bad = 1;
+    prev = r1;
+    Sums acc{0, 0, 0, 0};
+    for (int64_t i = r0 + tid; i < r1; i += kSmallThreads) {
+      int32_t p = a.p[i], c = a.c[i], ph = a.ph[i];
+      check_req(p, c, ph, &bad);
+      acc.s1 += p;
+      acc.s2 += c;
+      acc.s3 += (int64_t)p * p;
+      acc.ph += ph;
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) ss.red[wid] = acc;
+    __syncthreads();
+    if (tid == 0) {
+      Sums t{0, 0, 0, 0};
+      for (int w = 0; w < kSmallWarps; ++w) t = add_sums(t, ss.red[w]);
+      ss.tot = t;
+    }
+    __syncthreads();
+    const Sums tot = ss.tot;
+    const BatchAgg g{tot.s1, tot.s2, tot.s3, r1 - r0, tot.ph > 0};
+    const int s = segment_of(a.mp, g);
+    if (tid == 0) emit_batch<MODE>(a, b, g, s, a.mp.fx);
+    if (r1 > r0) {
+      bool slow = false;
+      const i128 kf = batch_const_w<MODE>(a, nullptr, s, g.n, &slow);
+      const SegS sg = ss.seg[s];
+      for (int64_t i = r0 + tid; i < r1; i += kSmallThreads) {
+        int32_t p = a.p[i], c = a.c[i];
+        p = p < 0 ? 0 : p;
+        c = c < 0 ? 0 : c;
+        attribute_one<MODE>(a, tt, sg, s, slow, kf, g.n, i, p, c, kTen ? a.ten[i] : 0, &bad);
+      }
+    }
+    __syncthreads();  // ss.red / ss.tot are rewritten for the next batch
+  }
+  if (bad) flag(a.status, kStatusData);
+  if (kTen) {
+    // the table into the exact state (this CTA is the only writer here)
+    for (int u = tid; u < a.H; u += kSmallThreads) {
+      const i128 v = hot_value(tt, a.H, u);
+      if (!(v.lo | v.hi)) continue;
+      const i128 old = state[u];
+      const i128 nw = add128(old, v);
+      if (is_neg128(old) == is_neg128(v) && is_neg128(nw) != is_neg128(old)) flag(a.status, kStatusData);
+      state[u] = nw;
+    }
+  }
+}
+
 }  // namespace lv

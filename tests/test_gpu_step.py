@@ -3,8 +3,9 @@ graph of lv_tenant_acc_reset + lv_attribute + lv_tenant_totals, captured once
 and replayed.
 
 Every replay must give the eager call's T, shares and tenant totals bit for
-bit, and those the oracle's within the attribution tolerance (1e-12 relative;
-shares relative to max(|oracle share|, T_b / n)).
+bit, and those the oracle's within the attribution tolerance (1e-12 relative).
+Inputs of at most 8,192 requests in at most 16 batches take a single-CTA
+kernel; its cases are checked against the oracle here as well.
 """
 
 import numpy as np
@@ -82,3 +83,65 @@ def test_graph_replay_matches_eager_and_oracle(lv, n_req, n_prefill):
     m = L_o != 0
     assert np.all(L[~m] == 0)
     assert np.max(np.abs(L[m] - L_o[m]) / np.abs(L_o[m])) <= TOL
+
+
+@pytest.mark.parametrize("sizes,nt,arith", [
+    ([300, 0, 17, 2048, 1, 0, 900, 5], 256, 0),          # several batches, two empty
+    ([4096, 4096], 3000, 0),                             # up to 8192 requests, tenants beyond the shared table
+    ([7, 64, 1000, 3, 3, 3, 3, 3, 3, 3, 3, 3, 3, 3, 3, 3], 40, 1),  # 16 batches, the fp64 arithmetic mode
+])
+def test_small_inputs_against_oracle(lv, sizes, nt, arith):
+    """lv_attribute on a serving step's worth of requests (at most 8,192 in at most 16 batches)
+    runs a single-CTA kernel: T, shares and tenant totals against the oracle over two calls
+    into one accumulator, each total equal to the exact sum of the returned shares."""
+    import torch
+    from fractions import Fraction
+    rng = np.random.default_rng(sum(sizes) + nt)
+    off = np.zeros(len(sizes) + 1, np.int64)
+    np.cumsum(sizes, out=off[1:])
+    n = int(off[-1])
+    ph = (rng.random(n) < 0.05).astype(np.int32)
+    p = np.where(ph == 1, rng.integers(1, 2000, n), 1).astype(np.int32)
+    c = np.where(ph == 1, 0, rng.integers(1, 32768, n)).astype(np.int32)
+    t = rng.integers(0, nt, n).astype(np.int32)
+    coef, _ = workloads.draw_coefficients(np.random.default_rng(3), "qwen2.5-14b")
+    split = np.array([256, 256], np.int64)
+    ctx = lv.Context()
+    ctx.set_arith(arith)
+    b = lv.batches_to_device(p, c, ph, off, t, nt)
+    model = lv.make_model(coef, split)
+    acc = lv.TenantAcc(ctx, nt)
+    T = torch.full((len(sizes),), float("nan"), dtype=torch.float64, device="cuda")
+    S = torch.full((n,), float("nan"), dtype=torch.float64, device="cuda")
+    for _ in range(2):
+        lv.lv_attribute(ctx, model, b, T, S, acc)
+    L = torch.empty(nt, dtype=torch.float64, device="cuda")
+    lv.lv_tenant_totals(ctx, acc, L)
+    assert ctx.status() == lv.LV_OK
+    T_o, s_o = oracle.attribute(off, p, c, ph, split, coef)
+    Tg, Sg, Lg = T.cpu().numpy(), S.cpu().numpy(), L.cpu().numpy()
+    assert np.all(Tg[T_o == 0] == 0)
+    assert np.max(np.abs(Tg[T_o != 0] - T_o[T_o != 0]) / np.abs(T_o[T_o != 0])) <= TOL
+    assert np.max(np.abs(Sg - s_o) / np.abs(s_o)) <= TOL
+    if arith == 1:
+        assert np.array_equal(Tg, T_o) and np.array_equal(Sg, s_o)
+    L_o = oracle.TenantSums(nt).add(s_o, t).add(s_o, t).totals()
+    m = L_o != 0
+    assert np.all(Lg[~m] == 0)
+    assert np.max(np.abs(Lg[m] - L_o[m]) / np.abs(L_o[m])) <= TOL
+    for u in list(np.unique(t)[:20]) + [int(t.max())]:
+        tot = 2 * sum(round(Fraction(v) * 2**72) for v in Sg[t == u].tolist())
+        assert Lg[u] == float(Fraction(tot, 2**72))
+
+
+def test_small_input_data_error(lv):
+    """A negative token count in a small input records LV_EDATA (clamped, no fault)."""
+    import torch
+    w = workloads.step_config(n_req=512, n_prefill=2)
+    w.p[17] = -3
+    ctx = lv.Context()
+    b = lv.batches_to_device(w.p, w.c, w.phase, w.offsets, w.tenant, w.n_tenants)
+    S = torch.empty(w.n_req, dtype=torch.float64, device="cuda")
+    lv.lv_attribute(ctx, lv.make_model(w.coef, w.split), b, None, S, None)
+    assert ctx.status() == lv.LV_EDATA
+    assert ctx.status() == lv.LV_OK
