@@ -437,3 +437,38 @@ def test_full_size_parity(lv, ctx, k):
     T, share, L, st = _run(lv, ctx, w)
     assert st == lv.LV_OK
     _check_parity(w, T, share, L)
+
+
+def test_chunked_calls_equal_one_call(lv, ctx):
+    """Batch ranges submitted one call at a time (rebased offsets, views into the same arrays,
+    one tenant accumulator) give the one-call T, shares and tenant totals bit for bit: every
+    sum is exact, so the split cannot change a result."""
+    import torch
+    w = workloads.config(1, scale=0.005)
+    b = _dev(lv, w)
+    model = lv.make_model(w.coef, w.split)
+    outs = []
+    for k in (1, 5):
+        T = torch.full((w.n_batch,), float("nan"), dtype=torch.float64, device="cuda")
+        S = torch.full((w.n_req,), float("nan"), dtype=torch.float64, device="cuda")
+        acc = lv.TenantAcc(ctx, w.n_tenants)
+        cuts = [0]
+        for j in range(1, k):
+            c = w.n_batch * j // k
+            while w.offsets[c] % 4:
+                c += 1
+            cuts.append(c)
+        cuts.append(w.n_batch)
+        for b0, b1 in zip(cuts[:-1], cuts[1:]):
+            lo, hi = int(w.offsets[b0]), int(w.offsets[b1])
+            off = torch.as_tensor(w.offsets[b0:b1 + 1] - w.offsets[b0], device="cuda")
+            bj = lv.Batches(p=b.p[lo:hi], c=b.c[lo:hi], phase=b.phase[lo:hi], offsets=off, tenant=b.tenant[lo:hi],
+                            n_tenants=w.n_tenants)
+            lv.lv_attribute(ctx, model, bj, T[b0:b1], S[lo:hi], acc)
+        L = torch.empty(w.n_tenants, dtype=torch.float64, device="cuda")
+        lv.lv_tenant_totals(ctx, acc, L)
+        assert ctx.status() == lv.LV_OK
+        outs.append((T.cpu().numpy(), S.cpu().numpy(), L.cpu().numpy()))
+    for x, y in zip(*outs):
+        assert np.array_equal(x.view(np.int64), y.view(np.int64))
+    _check_parity(w, *outs[1])
