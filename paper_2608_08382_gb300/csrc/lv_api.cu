@@ -1025,42 +1025,41 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   if (n == 0) return LV_OK;
   cudaStream_t stream = (cudaStream_t)stream_;
   const int blocks = (int)std::min<int64_t>((n + kAccBlock - 1) / kAccBlock, (int64_t)ctx->sms * 8);
-  const size_t o_part = ((size_t)n * sizeof(uint64_t) + 255) & ~(size_t)255;
-  const size_t o_sum = (o_part + sizeof(double) * 5 * (size_t)blocks + 255) & ~(size_t)255;
-  const size_t o_hist = o_sum + 256;  // sums (8 doubles), prefixes (3), ranks (3): 112 bytes
-  const size_t need = o_hist + sizeof(unsigned int) * kAccTargets * kAccBins;
+  // a fixed head (tickets, sums, prefixes, ranks, histograms: zeroed once at
+  // allocation, and every pass leaves the tickets and histograms at zero), then
+  // the relative errors' bit patterns and the block partials
+  constexpr size_t o_hist = 256, o_rel = 4096;
+  static_assert(o_hist + sizeof(unsigned int) * kAccTargets * kAccBins <= o_rel, "accuracy scratch head");
+  const size_t o_part = o_rel + (((size_t)n * sizeof(uint64_t) + 255) & ~(size_t)255);
+  const size_t need = o_part + sizeof(double) * 5 * (size_t)blocks;
   if (need > ctx->acc_cap) {
     LV_CUDA(cudaDeviceSynchronize());
     if (ctx->d_acc) cudaFree(ctx->d_acc);
     ctx->d_acc = nullptr;
     ctx->acc_cap = 0;
     if (cudaMalloc(&ctx->d_acc, need) != cudaSuccess) return LV_ENOMEM;
+    if (cudaMemset(ctx->d_acc, 0, o_rel) != cudaSuccess) return LV_ECUDA;
     ctx->acc_cap = need;
   }
   unsigned char *base = static_cast<unsigned char *>(ctx->d_acc);
-  uint64_t *relbits = reinterpret_cast<uint64_t *>(base);
-  double *part = reinterpret_cast<double *>(base + o_part);
-  double *sums = reinterpret_cast<double *>(base + o_sum);  // count, sum y, sum T, then the five moments
-  uint64_t *pf = reinterpret_cast<uint64_t *>(base + o_sum + 64);
-  int64_t *rk = reinterpret_cast<int64_t *>(base + o_sum + 88);
+  unsigned int *ticket = reinterpret_cast<unsigned int *>(base);                  // 3
+  double *sums = reinterpret_cast<double *>(base + 64);  // count, sum y, sum T, then the five moments
+  uint64_t *pf = reinterpret_cast<uint64_t *>(base + 128);                       // 3
+  int64_t *rk = reinterpret_cast<int64_t *>(base + 152);                         // 3
   unsigned int *hist = reinterpret_cast<unsigned int *>(base + o_hist);
-  k_acc_sums<<<blocks, kAccBlock, 0, stream>>>(y, T, n, relbits, part);
+  uint64_t *relbits = reinterpret_cast<uint64_t *>(base + o_rel);
+  double *part = reinterpret_cast<double *>(base + o_part);
+  k_acc_sums<<<blocks, kAccBlock, 0, stream>>>(y, T, n, relbits, part, sums, ticket);
   LV_CUDA(cudaGetLastError());
-  k_acc_fold<<<1, 32, 0, stream>>>(part, blocks, 3, sums);
-  LV_CUDA(cudaGetLastError());
-  k_acc_moments<<<blocks, kAccBlock, 0, stream>>>(y, T, relbits, n, sums, part);
-  LV_CUDA(cudaGetLastError());
-  k_acc_fold<<<1, 32, 0, stream>>>(part, blocks, 5, sums + 3);
+  k_acc_moments<<<blocks, kAccBlock, 0, stream>>>(y, T, relbits, n, sums, part, ticket + 1);
   LV_CUDA(cudaGetLastError());
   // exact nearest-rank percentiles: one 8-bit digit per pass, picked on the device
-  LV_CUDA(cudaMemsetAsync(hist, 0, sizeof(unsigned int) * kAccTargets * kAccBins, stream));
   for (int pass = 0; pass < 8; ++pass) {
-    k_acc_hist<<<blocks, kAccBlock, 0, stream>>>(relbits, n, pf, 64 - 8 * pass, hist);
-    LV_CUDA(cudaGetLastError());
-    k_acc_pick<<<1, 32, 0, stream>>>(hist, sums, pf, rk, pass);
+    k_acc_hist<<<blocks, kAccBlock, 0, stream>>>(relbits, n, pf, 64 - 8 * pass, hist, sums, rk, ticket + 2);
     LV_CUDA(cudaGetLastError());
   }
-  double h[11];  // eight sums, then the three percentile bit patterns
+  double h[11];  // eight sums, then the three percentile bit patterns (sums and prefixes are adjacent)
+  static_assert(64 + 8 * sizeof(double) == 128, "prefixes follow the sums");
   LV_CUDA(cudaMemcpyAsync(h, sums, sizeof(h), cudaMemcpyDeviceToHost, stream));
   LV_CUDA(cudaStreamSynchronize(stream));
   const double m = h[0];

@@ -36,11 +36,38 @@ __device__ __forceinline__ double block_sum_fixed(double v, double *red) {
   return s;  // thread 0
 }
 
+// True in the block that finishes last (its partial and every other block's
+// are visible to it then).  The ticket is reset for the next launch; blocks
+// never wait on one another.
+__device__ __forceinline__ bool last_block(unsigned int *ticket) {
+  __shared__ bool last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+    if (last) *ticket = 0u;
+  }
+  __syncthreads();
+  if (last) __threadfence();
+  return last;
+}
+
+// `k` interleaved values summed over `blocks` partials, in index order.
+__device__ __forceinline__ void fold_partials(const double *part, int blocks, int k, double *out) {
+  if (threadIdx.x < k) {
+    double s = 0.0;
+    for (int b = 0; b < blocks; ++b) s += part[(int64_t)b * k + threadIdx.x];
+    out[threadIdx.x] = s;
+  }
+}
+
 // Pass 1: per-block count, sum y, sum T over y > 0; rel's bit patterns stored
-// (all ones for y <= 0, which the select never counts).
+// (all ones for y <= 0, which the select never counts).  The last block folds
+// the partials into tot[0..2].
 __global__ void __launch_bounds__(kAccBlock) k_acc_sums(const double *__restrict__ y, const double *__restrict__ T,
                                                         int64_t n, uint64_t *__restrict__ relbits,
-                                                        double *__restrict__ part) {
+                                                        double *__restrict__ part, double *__restrict__ tot,
+                                                        unsigned int *ticket) {
   __shared__ double red[kAccBlock / 32];
   double c = 0.0, sy = 0.0, st = 0.0;
   const int64_t stride = (int64_t)gridDim.x * kAccBlock;
@@ -61,23 +88,15 @@ __global__ void __launch_bounds__(kAccBlock) k_acc_sums(const double *__restrict
     part[3 * blockIdx.x + 1] = b;
     part[3 * blockIdx.x + 2] = d;
   }
+  if (last_block(ticket)) fold_partials(part, gridDim.x, 3, tot);
 }
 
-// Sums `k` interleaved values over `blocks` partials, in index order (one block).
-__global__ void __launch_bounds__(32) k_acc_fold(const double *__restrict__ part, int blocks, int k,
-                                                 double *__restrict__ out) {
-  if (threadIdx.x < k) {
-    double s = 0.0;
-    for (int b = 0; b < blocks; ++b) s += part[(int64_t)b * k + threadIdx.x];
-    out[threadIdx.x] = s;
-  }
-}
-
-// Pass 2: centred moments with the means from pass 1 (tot = {count, sum y, sum T}).
+// Pass 2: centred moments with the means from pass 1 (tot = {count, sum y,
+// sum T}); the last block folds them into tot[3..7].
 __global__ void __launch_bounds__(kAccBlock) k_acc_moments(const double *__restrict__ y, const double *__restrict__ T,
                                                            const uint64_t *__restrict__ relbits, int64_t n,
-                                                           const double *__restrict__ tot,
-                                                           double *__restrict__ part) {
+                                                           double *__restrict__ tot, double *__restrict__ part,
+                                                           unsigned int *ticket) {
   __shared__ double red[kAccBlock / 32];
   const double m = tot[0];
   const double my = m > 0 ? tot[1] / m : 0.0, mt = m > 0 ? tot[2] / m : 0.0;
@@ -104,13 +123,50 @@ __global__ void __launch_bounds__(kAccBlock) k_acc_moments(const double *__restr
     p[3] = v3;
     p[4] = v4;
   }
+  if (last_block(ticket)) fold_partials(part, gridDim.x, 5, tot + 3);
+}
+
+// After a histogram pass: for each target, the digit whose bin holds its rank
+// (ranks ceil(q m / 100), q = 50, 90, 99, set from the sample count m at the
+// first pass), appended to its prefix; the histograms are cleared for the next
+// pass.  One warp: lane t < 3 takes target t.  All passes run back to back on
+// the stream with no host round trip.
+__device__ __forceinline__ void acc_pick(unsigned int *__restrict__ hist, const double *__restrict__ sums,
+                                         uint64_t *__restrict__ prefix, int64_t *__restrict__ rank, int pass) {
+  const int t = threadIdx.x;
+  if (t < kAccTargets) {
+    int64_t r;
+    uint64_t pf;
+    if (pass == 0) {
+      const int64_t m = (int64_t)sums[0];
+      const int64_t q = t == 0 ? 50 : t == 1 ? 90 : 99;
+      r = (q * m + 99) / 100;
+      pf = 0;
+    } else {
+      r = rank[t];
+      pf = prefix[t];
+    }
+    int64_t below = 0;
+    int d = 0;
+    for (; d < kAccBins - 1; ++d) {
+      const unsigned int c = hist[t * kAccBins + d];
+      if (below + c >= r) break;
+      below += c;
+    }
+    rank[t] = r - below;
+    prefix[t] = (pf << 8) | (uint64_t)d;
+  }
+  __syncwarp();
+  for (int i = t; i < kAccTargets * kAccBins; i += 32) hist[i] = 0u;
 }
 
 // One radix-select pass: for each target t whose top `shift`..63 bits are
-// prefix[t] (shift = 64 - 8 * passes done), count the next 8-bit digit.
+// prefix[t] (shift = 64 - 8 * passes done), count the next 8-bit digit; the
+// last block picks each target's digit and clears the histograms.
 __global__ void __launch_bounds__(kAccBlock) k_acc_hist(const uint64_t *__restrict__ relbits, int64_t n,
-                                                        const uint64_t *__restrict__ prefix, int shift,
-                                                        unsigned int *__restrict__ hist) {
+                                                        uint64_t *__restrict__ prefix, int shift,
+                                                        unsigned int *__restrict__ hist, const double *__restrict__ sums,
+                                                        int64_t *__restrict__ rank, unsigned int *ticket) {
   __shared__ unsigned int h[kAccTargets][kAccBins];
   for (int i = threadIdx.x; i < kAccTargets * kAccBins; i += kAccBlock) (&h[0][0])[i] = 0u;
   __syncthreads();
@@ -133,6 +189,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc_hist(const uint64_t *__restri
     const unsigned int c = (&h[0][0])[i];
     if (c) atomicAdd(hist + i, c);
   }
+  if (last_block(ticket) && threadIdx.x < 32) acc_pick(hist, sums, prefix, rank, (64 - shift) / 8);
 }
 
 // After a histogram pass: for each target, the digit whose bin holds its rank
