@@ -1043,13 +1043,15 @@ __global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_bas
 // still go to the pending limbs, which the caller folds).
 constexpr int kSmallThreads = 1024;
 constexpr int kSmallWarps = kSmallThreads / 32;
-constexpr int64_t kSmallMaxReq = 8192;
+constexpr int64_t kSmallMaxReq = 4096;
 constexpr int64_t kSmallMaxBatch = 16;
 
 struct SmallSmem {
   alignas(16) SegS seg[4];
   alignas(16) Sums red[kSmallWarps];
-  alignas(16) Sums tot;
+  alignas(16) i128 kf;  // the current batch's per-request constant
+  int s, slow;
+  alignas(16) int64_t off[kSmallMaxBatch + 1];
 };
 static_assert(sizeof(SmallSmem) % 16 == 0, "tenant table follows SmallSmem");
 
@@ -1059,63 +1061,85 @@ __global__ void __launch_bounds__(kSmallThreads) k_small(const TileArgs a, i128 
   SmallSmem &ss = *reinterpret_cast<SmallSmem *>(smem_raw);
   uint32_t *tt = reinterpret_cast<uint32_t *>(smem_raw + sizeof(SmallSmem));
   constexpr bool kTen = (MODE & M_TEN) != 0;
+  constexpr int kPer = (int)(kSmallMaxReq / kSmallThreads);  // requests per thread
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
   int bad = 0;
+  // every global read up front, independent of one another: this thread's
+  // requests (i = tid + k * kSmallThreads; every request lies in some batch of
+  // valid offsets), the offsets, and the state of the tenants it will fold
+  int32_t p[kPer], c[kPer], ph[kPer], u[kPer];
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) {
+    const int64_t i = tid + (int64_t)k * kSmallThreads;
+    const bool in = i < a.n_req;
+    p[k] = in ? a.p[i] : 0;
+    c[k] = in ? a.c[i] : 0;
+    ph[k] = in ? a.ph[i] : 0;
+    u[k] = (kTen && in) ? a.ten[i] : 0;
+  }
+  if (tid <= a.n_batch) ss.off[tid] = a.off[tid];
+  i128 st0 = mk128(0, 0);
+  if (kTen && tid < a.H) st0 = state[tid];
   if (kTen)
     for (int i = tid; i < 4 * ten_plane(a.H); i += kSmallThreads) tt[i] = 0;
   init_segs<MODE>(a, ss.seg);
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) check_req(p[k], c[k], ph[k], &bad);
   __syncthreads();
   int64_t prev = 0;
   for (int64_t b = 0; b < a.n_batch; ++b) {
-    const int64_t o0 = a.off[b], o1 = a.off[b + 1];
+    const int64_t o0 = ss.off[b], o1 = ss.off[b + 1];
     const int64_t r0 = clampi(o0, prev, a.n_req), r1 = clampi(o1, r0, a.n_req);
     if (r0 != o0 || r1 != o1 || (b == 0 && o0 != 0) || (b == a.n_batch - 1 && o1 != a.n_req)) bad = 1;
     prev = r1;
     Sums acc{0, 0, 0, 0};
-    for (int64_t i = r0 + tid; i < r1; i += kSmallThreads) {
-      int32_t p = a.p[i], c = a.c[i], ph = a.ph[i];
-      check_req(p, c, ph, &bad);
-      acc.s1 += p;
-      acc.s2 += c;
-      acc.s3 += (int64_t)p * p;
-      acc.ph += ph;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      const int64_t i = tid + (int64_t)k * kSmallThreads;
+      if (i >= r0 && i < r1) {
+        acc.s1 += p[k];
+        acc.s2 += c[k];
+        acc.s3 += (int64_t)p[k] * p[k];
+        acc.ph += ph[k];
+      }
     }
     acc = warp_sum(acc);
     if (lane == 0) ss.red[wid] = acc;
     __syncthreads();
     if (tid == 0) {
+      // the batch's sums, segment, T and per-request constant, formed once
       Sums t{0, 0, 0, 0};
       for (int w = 0; w < kSmallWarps; ++w) t = add_sums(t, ss.red[w]);
-      ss.tot = t;
+      const BatchAgg g{t.s1, t.s2, t.s3, r1 - r0, t.ph > 0};
+      const int s = segment_of(a.mp, g);
+      emit_batch<MODE>(a, b, g, s, a.mp.fx);
+      bool slow = false;
+      ss.kf = r1 > r0 ? batch_const_w<MODE>(a, nullptr, s, g.n, &slow) : mk128(0, 0);
+      ss.s = s;
+      ss.slow = slow ? 1 : 0;
     }
     __syncthreads();
-    const Sums tot = ss.tot;
-    const BatchAgg g{tot.s1, tot.s2, tot.s3, r1 - r0, tot.ph > 0};
-    const int s = segment_of(a.mp, g);
-    if (tid == 0) emit_batch<MODE>(a, b, g, s, a.mp.fx);
-    if (r1 > r0) {
-      bool slow = false;
-      const i128 kf = batch_const_w<MODE>(a, nullptr, s, g.n, &slow);
-      const SegS sg = ss.seg[s];
-      for (int64_t i = r0 + tid; i < r1; i += kSmallThreads) {
-        int32_t p = a.p[i], c = a.c[i];
-        p = p < 0 ? 0 : p;
-        c = c < 0 ? 0 : c;
-        attribute_one<MODE>(a, tt, sg, s, slow, kf, g.n, i, p, c, kTen ? a.ten[i] : 0, &bad);
-      }
+    const int s = ss.s;
+    const bool slow = ss.slow != 0;
+    const i128 kf = ss.kf;
+    const SegS sg = ss.seg[s];
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      const int64_t i = tid + (int64_t)k * kSmallThreads;
+      if (i >= r0 && i < r1) attribute_one<MODE>(a, tt, sg, s, slow, kf, r1 - r0, i, p[k], c[k], u[k], &bad);
     }
-    __syncthreads();  // ss.red / ss.tot are rewritten for the next batch
+    __syncthreads();  // ss is rewritten for the next batch
   }
   if (bad) flag(a.status, kStatusData);
   if (kTen) {
     // the table into the exact state (this CTA is the only writer here)
-    for (int u = tid; u < a.H; u += kSmallThreads) {
-      const i128 v = hot_value(tt, a.H, u);
+    for (int v0 = tid; v0 < a.H; v0 += kSmallThreads) {
+      const i128 v = hot_value(tt, a.H, v0);
       if (!(v.lo | v.hi)) continue;
-      const i128 old = state[u];
+      const i128 old = v0 == tid ? st0 : state[v0];
       const i128 nw = add128(old, v);
       if (is_neg128(old) == is_neg128(v) && is_neg128(nw) != is_neg128(old)) flag(a.status, kStatusData);
-      state[u] = nw;
+      state[v0] = nw;
     }
   }
 }

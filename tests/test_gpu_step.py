@@ -4,7 +4,7 @@ and replayed.
 
 Every replay must give the eager call's T, shares and tenant totals bit for
 bit, and those the oracle's within the attribution tolerance (1e-12 relative).
-Inputs of at most 8,192 requests in at most 16 batches take a single-CTA
+Inputs of at most 4,096 requests in at most 16 batches take a single-CTA
 kernel; its cases are checked against the oracle here as well.
 """
 
@@ -87,11 +87,11 @@ def test_graph_replay_matches_eager_and_oracle(lv, n_req, n_prefill):
 
 @pytest.mark.parametrize("sizes,nt,arith", [
     ([300, 0, 17, 2048, 1, 0, 900, 5], 256, 0),          # several batches, two empty
-    ([4096, 4096], 3000, 0),                             # up to 8192 requests, tenants beyond the shared table
+    ([2048, 2048], 3000, 0),                             # 4096 requests (the limit), tenants beyond the shared table
     ([7, 64, 1000, 3, 3, 3, 3, 3, 3, 3, 3, 3, 3, 3, 3, 3], 40, 1),  # 16 batches, the fp64 arithmetic mode
 ])
 def test_small_inputs_against_oracle(lv, sizes, nt, arith):
-    """lv_attribute on a serving step's worth of requests (at most 8,192 in at most 16 batches)
+    """lv_attribute on a serving step's worth of requests (at most 4,096 in at most 16 batches)
     runs a single-CTA kernel: T, shares and tenant totals against the oracle over two calls
     into one accumulator, each total equal to the exact sum of the returned shares."""
     import torch
