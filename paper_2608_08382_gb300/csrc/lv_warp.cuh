@@ -125,23 +125,17 @@ __device__ __forceinline__ void prefetch_l2(const void *p) { asm volatile("prefe
 // steps with K + p (A1 + A3 p) in place of K13 (prefill_const) where that is
 // exact, and the general path, exact for every case, otherwise.
 
-// v = k + (a1:a0) * c, four 32-bit words, exact (the sum stays below 2^128).
+// v = k + (a1:a0) * c, four 32-bit words, exact (the sum stays below 2^128):
+// carry-propagating multiply-adds, low word first.
 __device__ __forceinline__ void mad_k13(uint32_t k0, uint32_t k1, uint32_t k2, uint32_t k3, uint32_t a0, uint32_t a1,
                                         uint32_t c, uint32_t &v0, uint32_t &v1, uint32_t &v2, uint32_t &v3) {
-  asm("{\n\t"
-      ".reg .u32 l0, h0, l1, h1;\n\t"
-      "mul.lo.u32 l0, %4, %6;\n\t"
-      "mul.hi.u32 h0, %4, %6;\n\t"
-      "mul.lo.u32 l1, %5, %6;\n\t"
-      "mul.hi.u32 h1, %5, %6;\n\t"
-      "add.cc.u32 %0, %7, l0;\n\t"
-      "addc.cc.u32 %1, %8, h0;\n\t"
+  asm("mad.lo.cc.u32 %0, %4, %6, %7;\n\t"
+      "madc.hi.cc.u32 %1, %4, %6, %8;\n\t"
       "addc.cc.u32 %2, %9, 0;\n\t"
       "addc.u32 %3, %10, 0;\n\t"
-      "add.cc.u32 %1, %1, l1;\n\t"
-      "addc.cc.u32 %2, %2, h1;\n\t"
-      "addc.u32 %3, %3, 0;\n\t"
-      "}"
+      "mad.lo.cc.u32 %1, %5, %6, %1;\n\t"
+      "madc.hi.cc.u32 %2, %5, %6, %2;\n\t"
+      "addc.u32 %3, %3, 0;"
       : "=r"(v0), "=r"(v1), "=r"(v2), "=r"(v3)
       : "r"(a0), "r"(a1), "r"(c), "r"(k0), "r"(k1), "r"(k2), "r"(k3));
 }
