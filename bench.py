@@ -631,67 +631,6 @@ def run_ours(args, world, rank, local):
     return line
 
 
-def _oracle_sample(kind, w):
-    """A bounded piece of the workload for the oracle and the function that processes it once.
-
-    Returns (run, units per run, description)."""
-    import oracle
-    oracle.build()
-    if kind in ("whatif", "admit"):
-        c = w.cand
-        rows = min(64, w.n_pending)
-        pn, cn, phn = w.p_new[:rows], w.c_new[:rows], w.phase_new[:rows]
-        rng = np.random.default_rng(w.seed)
-        un, Lh, Bh = rng.integers(0, 64, rows), rng.uniform(0, 1e-3, 64), rng.uniform(0, 2e-3, 64)
-
-        def run():
-            T, S = oracle.whatif(c.offsets, c.p, c.c, c.phase, pn, cn, phn, w.split, w.coef)
-            if kind == "admit":
-                oracle.admit(T, S, un, Lh, Bh, 0.05)
-        return run, rows * c.n_batch, f"first {rows} of {w.n_pending} pending requests x all {c.n_batch} candidates"
-    if kind == "acc":
-        nb = max(1, w.n_batch // 10)
-        hi = int(w.offsets[nb])
-        off = w.offsets[:nb + 1]
-        T, _ = oracle.attribute(off, w.p[:hi], w.c[:hi], w.phase[:hi], w.split, w.coef)
-        y = T * w.noise[:nb]
-        feat, _ = oracle.batch_features(off, w.p[:hi], w.c[:hi], w.phase[:hi], w.split)
-        beta, a, _, _ = oracle.vtc_fit(feat[0], feat[3], y)
-        Tv = beta + a * feat[0].astype(np.float64)
-
-        def run():
-            oracle.accuracy(y, T)
-            oracle.accuracy(y, Tv)
-        return run, nb, f"first {nb} of {w.n_batch} batches: accuracy of the generating model and of the token-count line"
-    if kind == "step":
-        t = w.tenant
-
-        def run():
-            _, s = oracle.attribute(w.offsets, w.p, w.c, w.phase, w.split, w.coef)
-            oracle.tenant_totals(s, t, w.n_tenants)
-        return run, w.n_req, f"the whole batch ({w.n_req} requests), attribution + tenant totals"
-    frac = 10 if kind == "attr" else 200
-    nb = max(1, w.n_batch // frac)
-    hi = int(w.offsets[nb])
-    off = w.offsets[:nb + 1]
-    p, c, ph = w.p[:hi], w.c[:hi], w.phase[:hi]
-    if kind == "attr":
-        t = w.tenant[:hi]
-
-        def run():
-            _, s = oracle.attribute(off, p, c, ph, w.split, w.coef)
-            oracle.tenant_totals(s, t, w.n_tenants)
-        return run, hi, f"first {nb} of {w.n_batch} batches ({hi} requests), attribution + tenant totals"
-    T, _ = oracle.attribute(off, p, c, ph, w.split, w.coef)
-    Y = np.stack([T * w.noise[:nb], T])
-
-    def run():
-        feat, seg = oracle.batch_features(off, p, c, ph, w.split)
-        for y in Y:
-            oracle.fit(feat, seg, y)
-    return run, hi, f"first {nb} of {w.n_batch} batches ({hi} requests), batch sums + exact fit of 2 latency vectors"
-
-
 def cpu_model() -> str:
     """The host CPU's model name (lscpu), or the machine type if lscpu has none."""
     try:
@@ -743,11 +682,11 @@ def _oracle_jobs(kind, w, k):
     return jobs, (int(w.offsets[nb]) if kind != "acc" else nb), f"first {nb} of {w.n_batch} batches, {what}"
 
 
-def _oracle_worker(job, seconds):
-    """Runs one piece of the oracle sample repeatedly for about `seconds`; returns (passes, elapsed, totals)."""
+def _oracle_prepare(job):
+    """The oracle's work on one piece of the sample, as a function of no arguments (inputs formed beforehand, as
+    the GPU bench forms them before its timed region); attribution returns the piece's tenant totals."""
     import oracle
     kind = job["kind"]
-    totals = None
     if kind in ("attr", "step"):
         def run():
             _, s = oracle.attribute(job["off"], job["p"], job["c"], job["ph"], job["split"], job["coef"])
@@ -780,6 +719,13 @@ def _oracle_worker(job, seconds):
             feat, seg = oracle.batch_features(job["off"], job["p"], job["c"], job["ph"], job["split"])
             for y in Y:
                 oracle.fit(feat, seg, y)
+    return run
+
+
+def _oracle_worker(job, seconds):
+    """Runs one piece of the oracle sample repeatedly for about `seconds`; returns (passes, elapsed, totals)."""
+    run = _oracle_prepare(job)
+    totals = None
     passes, t0 = 0, time.perf_counter()
     while True:
         totals = run()
@@ -788,6 +734,49 @@ def _oracle_worker(job, seconds):
         if el >= seconds:
             break
     return passes, el, totals
+
+
+# ---- the sample's pieces in one shared-memory block, for a persistent pool of oracle workers
+
+_SHM = {}
+_PREPARED = {}
+
+
+def _shm_put(jobs):
+    """Copies every array of the jobs into one shared-memory block; returns (block, per-job layouts)."""
+    from multiprocessing import shared_memory
+    total = sum(np.ascontiguousarray(v).nbytes for j in jobs for v in j.values() if isinstance(v, np.ndarray))
+    shm = shared_memory.SharedMemory(create=True, size=max(total, 8))
+    buf = np.ndarray((max(total, 8),), np.uint8, shm.buf)
+    layouts, pos = [], 0
+    for j in jobs:
+        lay = {}
+        for k, v in j.items():
+            if isinstance(v, np.ndarray):
+                a = np.ascontiguousarray(v)
+                buf[pos:pos + a.nbytes] = a.reshape(-1).view(np.uint8)
+                lay[k] = ("arr", pos, a.dtype.str, a.shape)
+                pos += a.nbytes
+            else:
+                lay[k] = ("val", v)
+        layouts.append(lay)
+    return shm, layouts
+
+
+def _oracle_pass(name, index, lay):
+    """One pass of piece `index` of the sample (a pool task; the piece is attached and prepared once per
+    worker); returns the seconds the pass took."""
+    from multiprocessing import shared_memory
+    key = (name, index)
+    if key not in _PREPARED:
+        if name not in _SHM:
+            _SHM[name] = shared_memory.SharedMemory(name=name)
+        buf = _SHM[name].buf
+        job = {k: (np.ndarray(v[3], np.dtype(v[2]), buf, v[1]) if v[0] == "arr" else v[1]) for k, v in lay.items()}
+        _PREPARED[key] = _oracle_prepare(job)
+    t0 = time.perf_counter()
+    _PREPARED[key]()
+    return time.perf_counter() - t0
 
 
 def cpu_baseline(kind, w, min_seconds=10.0):
@@ -828,26 +817,47 @@ def cpu_baseline(kind, w, min_seconds=10.0):
 
 
 def run_reference(args, world, rank):
+    """The oracle as it stands on every host core: one step is one pass over a bounded sample of the workload,
+    cut into one contiguous piece per core and run by a persistent pool of spawned worker processes that read
+    the pieces from shared memory."""
     if rank != 0:
         return None
+    import concurrent.futures as cf
+    import multiprocessing as mp
+
+    import oracle
+    oracle.build()
     kind, w, desc = _workload(args)
-    run, units, sample = _oracle_sample(kind, w)
-    for _ in range(args.warmup):
-        run()
-    t0 = time.perf_counter()
-    for _ in range(args.steps):
-        run()
-    el = time.perf_counter() - t0
+    cores = len(os.sched_getaffinity(0))
+    jobs, units, sample = _oracle_jobs(kind, w, cores)
+    shm, lays = _shm_put(jobs)
+    try:
+        with cf.ProcessPoolExecutor(max_workers=len(jobs), mp_context=mp.get_context("spawn")) as pool:
+            def step():
+                futs = [pool.submit(_oracle_pass, shm.name, i, lay) for i, lay in enumerate(lays)]
+                for f in futs:
+                    f.result(timeout=600)
+            for _ in range(max(args.warmup, 1)):  # the first pass attaches and prepares every piece
+                step()
+            t0 = time.perf_counter()
+            for _ in range(args.steps):
+                step()
+            el = time.perf_counter() - t0
+    finally:
+        shm.close()
+        shm.unlink()
     value = units * args.steps / el
     unit = "pairs/s" if kind in ("whatif", "admit") else "batches/s" if kind == "acc" else "requests/s"
     metric = {"attr": METRIC, "fit": METRIC_FIT, "whatif": METRIC_WHATIF, "admit": METRIC_ADMIT,
               "step": METRIC_STEP, "acc": METRIC_ACC}[kind]
+    how = (f"{sample} per step, cut into {len(jobs)} contiguous pieces run by {len(jobs)} spawned worker "
+           f"processes (one per host core)")
     return {"impl": "reference", "metric": metric, "value": value, "unit": unit, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": desc, "parallelism": "host", "sample": sample},
-            "cpu_baseline": {"value": value, "unit": unit, "cores": 1, "kind": "oracle",
-                             "sample": f"{sample} per step, single thread"},
+            "config": {"workload": desc, "parallelism": f"host, {len(jobs)} processes", "sample": sample},
+            "cpu_baseline": {"value": value, "unit": unit, "cores": len(jobs), "kind": "oracle",
+                             "cpu_model": cpu_model(), "sample": how},
             "e2e": {"value": value, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
