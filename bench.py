@@ -396,12 +396,15 @@ def _setup_acc(lv, ctx, w, stream):
         step()
 
     return dict(step=step, e2e_step=e2e_step, units=w.n_batch, unit="batches/s", metric=METRIC_ACC,
-                h2d=3 * 8 * w.n_batch, d2h=2 * 56, launches_per_step=2 * 12, kernel="accuracy", time_mask=0,
+                h2d=3 * 8 * w.n_batch, d2h=2 * 88, launches_per_step=2 * 10, kernel="accuracy", time_mask=0,
                 whole_step=True, timed="the whole step (two synchronous lv_accuracy calls), CUDA events",
-                bytes_per_launch=2 * 16.0 * w.n_batch,
-                bytes_rule="16 B/batch (y, T) read once per model; the exact percentile select re-reads 8 B/batch "
-                           "of relative-error bits per 8-bit pass (8 passes), counted as overhead",
+                bytes_per_launch=2 * 16.0 * w.n_batch, flush=True,
+                bytes_rule="16 B/batch (y, T) read once per model; the range pass's second read of y and T, the "
+                           "8 B/batch of relative-error bits written, and their re-reads by the select passes "
+                           "(11-bit digits, up to 6) are counted as overhead",
                 config={"n_batch": w.n_batch, "seed": w.seed,
+                        "l2": "working set below L2 size: a 512 MB buffer is overwritten before every timed step, "
+                              "outside the step's events",
                         "step": "lv_accuracy(y, T_model) + lv_accuracy(y, T_vtc) (synchronous)",
                         "result": out})
 

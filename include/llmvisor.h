@@ -261,9 +261,15 @@ lv_status lv_fit_vtc(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t 
 /* Accuracy of predicted batch latencies T against measured y (both device
  * double[n]; Section 3.2, Tables 1-2), over the batches with y > 0: both forms
  * of R^2, the mean relative error and its nearest-rank p50/p90/p99 (the
- * ceil(q m / 100)-th smallest of the m relative errors, exact).  Sums are fp64
- * in a fixed order, so results repeat bit for bit.  rep: host.  With no sample
- * every value is NaN and n = 0; an R^2 whose denominator is 0 is NaN.
+ * ceil(q m / 100)-th smallest of the m relative errors, exact; each error is
+ * fl(fl(T - y) / y), as fp64 arithmetic gives it).  When every sample's y and
+ * non-zero T lie on one grid 2^(E - 78), E the largest binary exponent among
+ * them, and -160 <= E <= 224, the sums are exact integers and R^2 is rounded
+ * once from them; otherwise (a non-finite value, magnitudes too far apart or
+ * extreme) they are fp64 in a fixed order.  The mean relative error is a
+ * fixed-point sum on a grid 2^-100 below the largest error.  Either way results
+ * repeat bit for bit.  n < 2^32 (LV_EINVAL otherwise).  rep: host.  With no
+ * sample every value is NaN and n = 0; an R^2 whose denominator is 0 is NaN.
  * Synchronous. */
 lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, lv_accuracy_report *rep,
                       void *stream);

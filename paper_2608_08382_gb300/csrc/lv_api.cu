@@ -3,6 +3,7 @@
 #include <cuda_runtime.h>
 
 #include <cmath>
+#include <cstddef>
 #include <mutex>
 #include <cstdint>
 #include <cstdlib>
@@ -1018,20 +1019,29 @@ lv_status lv_fit_vtc(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t 
 
 lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, lv_accuracy_report *rep,
                       void *stream_) {
-  if (!ctx || !rep || n < 0 || (n > 0 && (!y || !T || !aligned(y, 8) || !aligned(T, 8)))) return LV_EINVAL;
+  if (!ctx || !rep || n < 0 || n >= ((int64_t)1 << 32) ||
+      (n > 0 && (!y || !T || !aligned(y, 8) || !aligned(T, 8))))
+    return LV_EINVAL;
   const double nan = std::nan("");
   rep->n = 0;
   rep->r2_ssr = rep->r2_corr = rep->mean_rel = rep->p50 = rep->p90 = rep->p99 = nan;
   if (n == 0) return LV_OK;
   cudaStream_t stream = (cudaStream_t)stream_;
   const int blocks = (int)std::min<int64_t>((n + kAccBlock - 1) / kAccBlock, (int64_t)ctx->sms * 8);
-  // a fixed head (tickets, sums, prefixes, ranks, histograms: zeroed once at
-  // allocation, and every pass leaves the tickets and histograms at zero), then
-  // the relative errors' bit patterns and the block partials
-  constexpr size_t o_hist = 256, o_rel = 4096;
-  static_assert(o_hist + sizeof(unsigned int) * kAccTargets * kAccBins <= o_rel, "accuracy scratch head");
+  const int sblocks = (int)std::min<int64_t>((n + kSelBlock - 1) / kSelBlock, (int64_t)ctx->sms * 2);
+  // a fixed head (tickets, range, sums, select state, rel extremes,
+  // histograms: zeroed once at allocation, and every call leaves the tickets,
+  // accumulators and histograms at zero), then the relative errors' bit
+  // patterns and the block partials
+  constexpr size_t o_range = 32, o_sums = 64, o_sel = 128, o_ra = 192, o_hist = 256, o_rel = 32768;
+  static_assert(sizeof(AccRange) <= o_sums - o_range && sizeof(SelState) <= o_ra - o_sel &&
+                    sizeof(RelAcc) <= o_hist - o_ra,
+                "accuracy scratch head");
+  static_assert(o_sel == o_sums + 8 * sizeof(double) && offsetof(SelState, pf) == 0,
+                "the prefixes follow the sums");
+  static_assert(o_hist + sizeof(unsigned int) * kAccTargets * kSelBins <= o_rel, "accuracy histograms");
   const size_t o_part = o_rel + (((size_t)n * sizeof(uint64_t) + 255) & ~(size_t)255);
-  const size_t need = o_part + sizeof(double) * 5 * (size_t)blocks;
+  const size_t need = o_part + sizeof(uint64_t) * kAccPart * (size_t)std::max(blocks, sblocks);
   if (need > ctx->acc_cap) {
     LV_CUDA(cudaDeviceSynchronize());
     if (ctx->d_acc) cudaFree(ctx->d_acc);
@@ -1042,29 +1052,37 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
     ctx->acc_cap = need;
   }
   unsigned char *base = static_cast<unsigned char *>(ctx->d_acc);
-  unsigned int *ticket = reinterpret_cast<unsigned int *>(base);                  // 3
-  double *sums = reinterpret_cast<double *>(base + 64);  // count, sum y, sum T, then the five moments
-  uint64_t *pf = reinterpret_cast<uint64_t *>(base + 128);                       // 3
-  int64_t *rk = reinterpret_cast<int64_t *>(base + 152);                         // 3
+  unsigned int *ticket = reinterpret_cast<unsigned int *>(base);  // range, exact, sums, moments, select
+  AccRange *rg = reinterpret_cast<AccRange *>(base + o_range);
+  double *sums = reinterpret_cast<double *>(base + o_sums);  // m, sum y, sum T, sxx, syy, sxy, ssr, sum rel
+  SelState *sel = reinterpret_cast<SelState *>(base + o_sel);
+  RelAcc *ra = reinterpret_cast<RelAcc *>(base + o_ra);
   unsigned int *hist = reinterpret_cast<unsigned int *>(base + o_hist);
   uint64_t *relbits = reinterpret_cast<uint64_t *>(base + o_rel);
-  double *part = reinterpret_cast<double *>(base + o_part);
-  k_acc_sums<<<blocks, kAccBlock, 0, stream>>>(y, T, n, relbits, part, sums, ticket);
+  uint64_t *part = reinterpret_cast<uint64_t *>(base + o_part);
+  k_acc_range<<<blocks, kAccBlock, 0, stream>>>(y, T, n, rg, ticket);
   LV_CUDA(cudaGetLastError());
-  k_acc_moments<<<blocks, kAccBlock, 0, stream>>>(y, T, relbits, n, sums, part, ticket + 1);
+  // exactly one of the two paths does work; the other returns at once
+  k_acc_exact<<<blocks, kAccBlock, 0, stream>>>(y, T, n, rg, relbits, part, sums, ra, sel, ticket + 1);
   LV_CUDA(cudaGetLastError());
-  // exact nearest-rank percentiles: one 8-bit digit per pass, picked on the device
-  for (int pass = 0; pass < 8; ++pass) {
-    k_acc_hist<<<blocks, kAccBlock, 0, stream>>>(relbits, n, pf, 64 - 8 * pass, hist, sums, rk, ticket + 2);
+  double *dpart = reinterpret_cast<double *>(part);
+  k_acc_sums<<<blocks, kAccBlock, 0, stream>>>(y, T, n, rg, relbits, dpart, sums, ra, sel, ticket + 2);
+  LV_CUDA(cudaGetLastError());
+  k_acc_moments<<<blocks, kAccBlock, 0, stream>>>(y, T, n, rg, sums, dpart, ticket + 3);
+  LV_CUDA(cudaGetLastError());
+  // exact nearest-rank percentiles (and the sum of rel), picked on the device
+  for (int pass = 0; pass < kSelPasses; ++pass) {
+    k_acc_select<<<sblocks, kSelBlock, 0, stream>>>(relbits, n, sel, hist, part, sums, ticket + 4, pass);
     LV_CUDA(cudaGetLastError());
   }
-  double h[11];  // eight sums, then the three percentile bit patterns (sums and prefixes are adjacent)
-  static_assert(64 + 8 * sizeof(double) == 128, "prefixes follow the sums");
+  double h[11];  // eight sums, then the three percentile bit patterns
   LV_CUDA(cudaMemcpyAsync(h, sums, sizeof(h), cudaMemcpyDeviceToHost, stream));
   LV_CUDA(cudaStreamSynchronize(stream));
   const double m = h[0];
   rep->n = (int64_t)m;
   if (m == 0) return LV_OK;
+  // sxx, syy, sxy, ssr: plain sums (fp64 path) or the same times m 2^(2S)
+  // (exact path); both R^2 are ratios, so the common factor cancels
   const double sxx = h[3], syy = h[4], sxy = h[5], ssr = h[6], srel = h[7];
   rep->r2_ssr = sxx != 0 ? 1.0 - ssr / sxx : nan;
   rep->r2_corr = (sxx != 0 && syy != 0) ? sxy * sxy / (sxx * syy) : nan;

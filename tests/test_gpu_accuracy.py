@@ -4,9 +4,12 @@ metrics (lv_accuracy) against the oracle.
 The VTC line is held to the fit's bar, 1e-9 relative on each coefficient
 (the oracle solves exactly and rounds once).  Accuracy: the sample count and
 the three percentiles are exact (each is one of the relative errors, computed
-by the same correctly rounded subtraction and division on both sides); R^2
-and the mean relative error within 1e-12 (fixed-order fp64 sums against
-correctly rounded ones).
+by the same correctly rounded subtraction and division on both sides; on
+the GPU's exact path that division is done in integers); R^2 and the mean
+relative error within 1e-12 (exact integer or fixed-order fp64 sums against
+the oracle's correctly rounded fp64 ones).  Inputs cover both of the
+library's paths: values on one 79-bit grid (the exact integer path) and
+magnitudes too far apart, non-finite or extreme ones (the fp64 path).
 """
 
 import numpy as np
@@ -114,3 +117,95 @@ def test_accuracy_edge_cases(lv, ctx):
     # no sample at all
     g = lv.lv_accuracy(ctx, _dev(np.zeros(5)), _dev(np.ones(5)))
     assert g["n"] == 0 and np.isnan(g["p50"]) and np.isnan(g["r2_ssr"])
+
+
+def test_accuracy_division_single_samples(lv, ctx):
+    """n = 1: every percentile and the mean are the one relative error, so each
+    call checks one correctly rounded fl(fl(T - y) / y) bit for bit, over
+    differences that need rounding (exponents up to 26 apart), tiny ones (T
+    within a few ulps of y), negative and zero T, and power-of-two y."""
+    rng = np.random.default_rng(21)
+    cases = []
+    for k in range(400):
+        y = float(rng.uniform(0.5, 2.0)) * 2.0 ** int(rng.integers(-12, 12))
+        kind = k % 8
+        if kind == 0:
+            T = y * (1 + rng.normal(0, 0.1))
+        elif kind == 1:
+            T = y + float(rng.integers(-6, 7)) * np.spacing(y)
+        elif kind == 2:
+            T = -y * float(rng.uniform(0, 3))
+        elif kind == 3:
+            T = float(rng.uniform(0.5, 2.0)) * 2.0 ** int(rng.integers(-14, 14))
+        elif kind == 4:
+            T = 0.0
+        elif kind == 5:
+            y = 2.0 ** int(rng.integers(-20, 20))
+            T = y * float(rng.uniform(0, 4))
+        elif kind == 6:
+            T = y * (1 + float(rng.integers(1, 2 ** 20)) * 2.0 ** -52)
+        else:
+            T = y * 2.0 ** 25 * float(rng.uniform(1, 2))  # far apart: the difference is rounded
+        cases.append((y, T))
+    for y, T in cases:
+        g = lv.lv_accuracy(ctx, _dev([y]), _dev([T]))
+        o = oracle.accuracy(np.array([y]), np.array([T]))
+        assert g["n"] == 1
+        assert g["p50"] == o["p50"] and g["p99"] == o["p99"], (y, T)
+        assert g["mean_rel"] == o["mean_rel"], (y, T)
+
+
+_PATH_CASES = ["integers", "negative_T", "wide_range", "large", "huge", "tiny", "nonfinite_T", "few_values",
+               "zero_T"]
+
+
+@pytest.mark.parametrize("case", _PATH_CASES)
+def test_accuracy_paths(lv, ctx, case):
+    """Both paths against the oracle: values on one grid (integers with zero
+    low bits, negative or zero predictions, magnitudes near 1e60 or 1e-40) take
+    the exact integer path; magnitudes 2^60 apart, non-finite predictions and
+    values near 1e100 take the fp64 path."""
+    rng = np.random.default_rng(100 + _PATH_CASES.index(case))
+    n = 200_003
+    y = rng.uniform(0.5, 2.0, n) * 1e-3
+    T = y * (1 + rng.normal(0, 0.2, n))
+    if case == "integers":
+        y = rng.integers(1, 2 ** 40, n).astype(np.float64)
+        T = np.round(y * (1 + rng.normal(0, 0.1, n)))
+    elif case == "negative_T":
+        T = -T
+    elif case == "wide_range":
+        y = y * 2.0 ** rng.integers(-30, 30, n)
+        T = y * (1 + rng.normal(0, 0.2, n))
+    elif case == "large":
+        y, T = y * 1e63, T * 1e63
+    elif case == "huge":
+        y, T = y * 1e63, T * 1e63
+        y[:10], T[:10] = y[:10] * 1e40, T[:10] * 1e40
+    elif case == "tiny":
+        y, T = y * 1e-37, T * 1e-37
+    elif case == "nonfinite_T":
+        T[5] = np.inf
+    elif case == "few_values":
+        y = np.ones(n)
+        T = 1.0 + rng.integers(0, 7, n) / 8.0
+    elif case == "zero_T":
+        T[rng.random(n) < 0.3] = 0.0
+    y[rng.random(n) < 0.05] = 0.0
+    if case == "nonfinite_T":
+        y[5] = 1e-3  # a sample whose prediction is infinite
+    g = lv.lv_accuracy(ctx, _dev(y), _dev(T))
+    if case == "nonfinite_T":
+        # the oracle's correctly rounded sums reject inf - inf; the order
+        # statistics below the top are those of the same data with the
+        # infinite prediction replaced by one larger than every other
+        Tf = T.copy()
+        Tf[5] = 1e300
+        o = oracle.accuracy(y, Tf)
+        assert g["n"] == o["n"] and g["p50"] == o["p50"] and g["p90"] == o["p90"]
+        assert np.isinf(g["mean_rel"])
+        return
+    o = oracle.accuracy(y, T)
+    _check_accuracy(g, o)
+    again = lv.lv_accuracy(ctx, _dev(y), _dev(T))  # repeats bit for bit (NaN where NaN)
+    assert all(again[k] == g[k] or (np.isnan(again[k]) and np.isnan(g[k])) for k in g)
