@@ -46,6 +46,7 @@ struct lv_ctx {
   size_t wi_cap = 0;
   void *d_acc = nullptr;      // accuracy metrics: relative-error bits, partials, histograms
   size_t acc_cap = 0;
+  int acc_occ[5] = {0, 0, 0, 0, 0};  // CTAs per SM: range, exact, sel0, selB, sel1 (0: not yet queried)
   int timing = 0;  // LV_TIME_* mask
   std::vector<cudaEvent_t> tev;  // start/stop pairs
   size_t tev_used = 0;
@@ -1027,21 +1028,37 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   rep->r2_ssr = rep->r2_corr = rep->mean_rel = rep->p50 = rep->p90 = rep->p99 = nan;
   if (n == 0) return LV_OK;
   cudaStream_t stream = (cudaStream_t)stream_;
-  const int blocks = (int)std::min<int64_t>((n + kAccBlock - 1) / kAccBlock, (int64_t)ctx->sms * 8);
-  const int sblocks = (int)std::min<int64_t>((n + kSelBlock - 1) / kSelBlock, (int64_t)ctx->sms * 2);
-  // a fixed head (tickets, range, sums, select state, rel extremes,
-  // histograms: zeroed once at allocation, and every call leaves the tickets,
-  // accumulators and histograms at zero), then the relative errors' bit
-  // patterns and the block partials
-  constexpr size_t o_range = 32, o_sums = 64, o_sel = 128, o_ra = 192, o_hist = 256, o_rel = 32768;
-  static_assert(sizeof(AccRange) <= o_sums - o_range && sizeof(SelState) <= o_ra - o_sel &&
-                    sizeof(RelAcc) <= o_hist - o_ra,
+  if (ctx->acc_occ[0] == 0) {
+    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ[0], k_acc_range, kAccBlock, 0));
+    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ[1], k_acc_exact, kAccBlock, 0));
+    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ[2], k_acc_sel0, kSelBlock, 0));
+    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ[3], k_acc_selB, kSelBlock, 0));
+    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ[4], k_acc_sel1, kSelBlock, 0));
+    LV_CUDA(cudaFuncSetAttribute(k_acc_sel2, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)(kSelSmemList * sizeof(uint64_t))));
+  }
+  // every pass is one wave (at most the blocks that fit at once), looping over
+  // its share; the select passes take eight patterns per thread and step
+  const auto wave = [&](int k, int64_t want) {
+    return (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)ctx->sms * std::max(ctx->acc_occ[k], 1)));
+  };
+  const int64_t want = (n + kAccBlock - 1) / kAccBlock, swant = (n + 8 * kSelBlock - 1) / (8 * kSelBlock);
+  const int rblocks = wave(0, want), xblocks = wave(1, want), fblocks = (int)std::min<int64_t>(want, ctx->sms * 4);
+  const int sblocks0 = wave(2, swant), sblocksB = wave(3, swant), sblocks1 = wave(4, swant);
+  const int sblocks = std::max(sblocks0, std::max(sblocksB, sblocks1));
+  // a fixed head (tickets, path, sums, select state, the digit histograms: zeroed once at allocation, and every call leaves the tickets,
+  // cursors and histograms at zero), then the
+  // relative errors' bit patterns, the candidate lists and the block partials
+  constexpr size_t o_range = 32, o_sums = 64, o_sel = 128, o_hist = 512, o_rel = 32768;
+  static_assert(sizeof(AccRange) <= o_sums - o_range && sizeof(SelState) <= o_hist - o_sel,
                 "accuracy scratch head");
   static_assert(o_sel == o_sums + 8 * sizeof(double) && offsetof(SelState, pf) == 0,
                 "the prefixes follow the sums");
   static_assert(o_hist + sizeof(unsigned int) * kAccTargets * kSelBins <= o_rel, "accuracy histograms");
-  const size_t o_part = o_rel + (((size_t)n * sizeof(uint64_t) + 255) & ~(size_t)255);
-  const size_t need = o_part + sizeof(uint64_t) * kAccPart * (size_t)std::max(blocks, sblocks);
+  const size_t rel_bytes = ((size_t)n * sizeof(uint64_t) + 255) & ~(size_t)255;
+  const size_t o_cand = o_rel + rel_bytes, o_part = o_cand + rel_bytes;
+  const size_t need =
+      o_part + sizeof(uint64_t) * kAccPart * (size_t)std::max(std::max(rblocks, xblocks), std::max(fblocks, sblocks));
   if (need > ctx->acc_cap) {
     LV_CUDA(cudaDeviceSynchronize());
     if (ctx->d_acc) cudaFree(ctx->d_acc);
@@ -1052,29 +1069,35 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
     ctx->acc_cap = need;
   }
   unsigned char *base = static_cast<unsigned char *>(ctx->d_acc);
-  unsigned int *ticket = reinterpret_cast<unsigned int *>(base);  // range, exact, sums, moments, select
+  unsigned int *ticket = reinterpret_cast<unsigned int *>(base);  // range, exact, sums, moments, two digits
   AccRange *rg = reinterpret_cast<AccRange *>(base + o_range);
   double *sums = reinterpret_cast<double *>(base + o_sums);  // m, sum y, sum T, sxx, syy, sxy, ssr, sum rel
   SelState *sel = reinterpret_cast<SelState *>(base + o_sel);
-  RelAcc *ra = reinterpret_cast<RelAcc *>(base + o_ra);
   unsigned int *hist = reinterpret_cast<unsigned int *>(base + o_hist);
   uint64_t *relbits = reinterpret_cast<uint64_t *>(base + o_rel);
+  uint64_t *cand = reinterpret_cast<uint64_t *>(base + o_cand);
   uint64_t *part = reinterpret_cast<uint64_t *>(base + o_part);
-  k_acc_range<<<blocks, kAccBlock, 0, stream>>>(y, T, n, rg, ticket);
+  k_acc_range<<<rblocks, kAccBlock, 0, stream>>>(y, T, n, rg, part, ticket);
   LV_CUDA(cudaGetLastError());
   // exactly one of the two paths does work; the other returns at once
-  k_acc_exact<<<blocks, kAccBlock, 0, stream>>>(y, T, n, rg, relbits, part, sums, ra, sel, ticket + 1);
+  k_acc_exact<<<xblocks, kAccBlock, 0, stream>>>(y, T, n, rg, relbits, part, sums, sel, ticket + 1);
   LV_CUDA(cudaGetLastError());
   double *dpart = reinterpret_cast<double *>(part);
-  k_acc_sums<<<blocks, kAccBlock, 0, stream>>>(y, T, n, rg, relbits, dpart, sums, ra, sel, ticket + 2);
+  k_acc_sums<<<fblocks, kAccBlock, 0, stream>>>(y, T, n, rg, relbits, dpart, sums, sel, ticket + 2);
   LV_CUDA(cudaGetLastError());
-  k_acc_moments<<<blocks, kAccBlock, 0, stream>>>(y, T, n, rg, sums, dpart, ticket + 3);
+  k_acc_moments<<<fblocks, kAccBlock, 0, stream>>>(y, T, n, rg, sums, dpart, ticket + 3);
   LV_CUDA(cudaGetLastError());
-  // exact nearest-rank percentiles (and the sum of rel), picked on the device
-  for (int pass = 0; pass < kSelPasses; ++pass) {
-    k_acc_select<<<sblocks, kSelBlock, 0, stream>>>(relbits, n, sel, hist, part, sums, ticket + 4, pass);
-    LV_CUDA(cudaGetLastError());
-  }
+  // exact nearest-rank percentiles (and the sum of rel): two digits over the
+  // samples, gather each target's remaining candidates, settle the rest per
+  // target
+  k_acc_sel0<<<sblocks0, kSelBlock, 0, stream>>>(relbits, n, sel, hist, part, sums, ticket + 4);
+  LV_CUDA(cudaGetLastError());
+  k_acc_selB<<<sblocksB, kSelBlock, 0, stream>>>(relbits, n, sel, hist, ticket + 5);
+  LV_CUDA(cudaGetLastError());
+  k_acc_sel1<<<sblocks1, kSelBlock, 0, stream>>>(relbits, n, sel, cand);
+  LV_CUDA(cudaGetLastError());
+  k_acc_sel2<<<kAccTargets, kSelFinish, kSelSmemList * sizeof(uint64_t), stream>>>(cand, sel);
+  LV_CUDA(cudaGetLastError());
   double h[11];  // eight sums, then the three percentile bit patterns
   LV_CUDA(cudaMemcpyAsync(h, sums, sizeof(h), cudaMemcpyDeviceToHost, stream));
   LV_CUDA(cudaStreamSynchronize(stream));

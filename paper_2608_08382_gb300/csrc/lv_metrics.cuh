@@ -9,29 +9,36 @@
 //
 // GB300 issues fp64 at 1/64 of the fp32 rate, so the common case runs on the
 // integer pipes, exactly:
-//   k_acc_range    the largest binary exponent Emax among the samples' y and
-//                  non-zero T, and the exponent of the lowest set bit among
-//                  them.  When every such value lies on the grid 2^(Emax - 78)
-//                  and Emax is moderate, the exact path below is taken.
-//   k_acc_exact    per sample the integers Y = y 2^S and T 2^S (S = 78 - Emax,
-//                  both below 2^79 in magnitude) and D = Y - T; the exact sums
+//   k_acc_range    the largest and smallest binary exponents Emax, Emin among
+//                  the samples' y and non-zero T.  When Emax is finite and
+//                  moderate the exact path below is taken: on the grid
+//                  2^(Emax - 62) in 64-bit integers when Emax - Emin <= 10 (every
+//                  value then lies on it), else on 2^(Emax - 78) in 128-bit
+//                  integers, handing over to the fp64 path when a value turns
+//                  out not to lie on that grid.
+//   k_acc_exact    per sample the integers Y = y 2^S and T 2^S (below 2^63 or
+//                  2^79 in magnitude) and D = Y - T; the exact sums
 //                  of Y, T, Y^2, T^2 and D^2, from which
 //                    m sxx = m sum Y^2 - (sum Y)^2,   m syy = m sum T^2 - (sum T)^2,
 //                    2 m sxy = m (sum Y^2 + sum T^2 - sum D^2) - 2 sum Y sum T,
 //                    m ssr = m sum D^2
 //                  follow exactly (all on the grid 2^(-2S), which both R^2
 //                  cancel); and rel by exact integer division.
-//   k_acc_sums,    otherwise (a non-finite sample value, magnitudes too far
-//   k_acc_moments  apart, or extreme ones): the same quantities in fp64, means
-//                  first, then centred moments, each in a fixed order.
-//   k_acc_select   the percentiles, exact: rel is a non-negative double, so
-//                  its bit pattern orders like its value, and a
-//                  most-significant-digit radix select (11-bit digits below the
-//                  prefix that every sample shares, one shared-memory histogram
-//                  per distinct prefix, the digit picked on the device) finds
-//                  the bit pattern of the element of each target rank.  The
-//                  first pass also sums rel in fixed point anchored at the
-//                  largest rel (terms below 2^-100 of it truncated).
+//   k_acc_sums,    otherwise (a non-finite sample value, extreme magnitudes,
+//   k_acc_moments  or a value off the grid): the same quantities in fp64,
+//                  means first, then centred moments, each in a fixed order.
+//   k_acc_sel0,    the percentiles, exact: rel is a non-negative double, so
+//   k_acc_selB,    its bit pattern orders like its value, and a
+//   k_acc_sel1,    most-significant-digit radix select finds the bit pattern of
+//   k_acc_sel2     the element of each target rank.  The first digit (11 bits
+//                  below the prefix every sample shares) is histogrammed over
+//                  all samples, which also sums rel in fixed point anchored at
+//                  the largest rel (terms below 2^-100 of it truncated); the
+//                  next digit over the samples in a target's bin (typically
+//                  well under 1% of them); the samples in each target's
+//                  second-digit bin (typically a handful) are gathered into a
+//                  candidate list, and one block per target settles the
+//                  remaining digits on its list.
 // Blocks never wait on one another: each fold runs in the block that finishes
 // last (an atomic ticket, reset for the next launch), and every kernel of a
 // call runs back to back on the stream with no host round trip.
@@ -52,26 +59,23 @@ constexpr int kAccPart = 16;    // words per block partial (any pass)
 constexpr int kSelBits = 11;    // radix digit
 constexpr int kSelBins = 1 << kSelBits;
 constexpr int kSelBlock = 512;
-constexpr int kSelPasses = (63 + kSelBits - 1) / kSelBits;  // a sample's sign bit is 0
+constexpr int kSelFinish = 1024;     // threads of a finishing block (one per target)
+constexpr int kSelSmemList = 20480;  // candidates a finishing block holds in shared memory
 constexpr int kAccGrid = 78;  // S = kAccGrid - Emax puts every |v 2^S| below 2^79
 // Range of Emax for the exact path: within it the definition's own fp64
 // arithmetic (squared deviations, their products in r2_corr) neither overflows
 // nor underflows for values on the grid, so the exact results are what fp64
 // evaluation approximates.
 constexpr int kAccEmaxLo = -160, kAccEmaxHi = 224;
-constexpr int kAccLkeyBias = 2100;  // lowest-set-bit exponents stored as kAccLkeyBias - e > 0
 constexpr uint64_t kFracMask = (1ull << 52) - 1, kHiddenBit = 1ull << 52;
 
-// Exponent range and exactness of one call (accumulators zero at allocation
-// and reset by the block that reads them; the result words are rewritten by
-// every call).
+// Path of one call, rewritten by every call: set by the range pass, except
+// `inexact`, which the exact pass sets when a value is off its grid.
 struct AccRange {
-  int emax;   // max biased exponent of the samples' y and non-zero T
-  int lkey;   // max of kAccLkeyBias - (exponent of the lowest set bit)
-  int bad;    // a sample's y or T is not finite
-  int exact;  // result: the exact path applies
-  int S;      // result: grid exponent, S = kAccGrid - Emax
-  int pad[3];
+  int exact;    // the exact path applies
+  int narrow;   // ... on the 63-bit grid (every exponent within 10 of the largest)
+  int S;        // grid exponent: 62 - Emax (narrow) or 78 - Emax
+  int inexact;  // a value fell off the grid
 };
 
 // Select state: the three prefixes first (they become the percentiles' bit
@@ -82,12 +86,14 @@ struct SelState {
   uint64_t relmax;          // largest rel (its bit pattern)
   int shift;                // bits below the settled prefixes; 0 when done
   int pad;
-};
-
-// Largest and smallest rel over the samples: max(bits) and max(~bits), so that
-// zero is the identity of both (reset by the block that reads them).
-struct RelAcc {
-  unsigned long long max, nmax;
+  // candidate lists after the first digit: target t's samples sit in list
+  // slot[t] (targets with the same prefix share one), at cbase[slot] in the
+  // candidate buffer, ccnt[t] of them; ccur[] are the append cursors
+  int64_t cbase[kAccTargets];
+  int64_t ccnt[kAccTargets];
+  unsigned long long ccur[kAccTargets];
+  int slot[kAccTargets];
+  int pad2;
 };
 
 // y > 0 on the bit pattern: sign clear, not zero, not NaN (+inf counts).
@@ -127,6 +133,28 @@ __device__ __forceinline__ double block_sum_fixed(double v, double *red) {
   return s;
 }
 
+// Block maxima of two words, valid in thread 0; `red` holds two words per
+// warp.
+__device__ __forceinline__ void block_max2(unsigned long long &a, unsigned long long &b, unsigned long long *red) {
+#pragma unroll
+  for (int d = 16; d; d >>= 1) {
+    a = max(a, __shfl_xor_sync(0xffffffffu, a, d));
+    b = max(b, __shfl_xor_sync(0xffffffffu, b, d));
+  }
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  __syncthreads();
+  if (lane == 0) {
+    red[2 * wid] = a;
+    red[2 * wid + 1] = b;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0)
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) {
+      a = max(a, red[2 * w]);
+      b = max(b, red[2 * w + 1]);
+    }
+}
+
 // `k` interleaved doubles summed over `blocks` partials with the whole block:
 // thread j takes partials j, j + blockDim, ... in order, then the block sum in
 // its fixed order; out[0..k) is written by thread 0.
@@ -139,57 +167,60 @@ __device__ __forceinline__ void fold_partials(const double *part, int blocks, in
   }
 }
 
-__device__ __forceinline__ int block_max_int(int v, int *red) {
-  v = (int)__reduce_max_sync(0xffffffffu, (unsigned)v);
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  __syncthreads();
-  if (lane == 0) red[wid] = v;
-  __syncthreads();
-  int s = 0;
-  if (threadIdx.x == 0)
-    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s = max(s, red[w]);
-  return s;  // thread 0
-}
-
-__device__ __forceinline__ void range_note(uint64_t b, int &emax, int &lkey, int &bad) {
-  const int be = (int)((b >> 52) & 0x7FF);
-  if (be == 0x7FF) {
-    bad = 1;
-    return;
-  }
-  const uint64_t M = (b & kFracMask) | (be ? kHiddenBit : 0ull);
-  const int eb = be ? be : 1;
-  emax = max(emax, eb);
-  lkey = max(lkey, kAccLkeyBias - (eb - 1075 + __ffsll((long long)M) - 1));
-}
-
-// Exponent range of the samples' y and non-zero T, and with it the path.
+// Largest magnitude (high word of the largest sample y or |T|) and smallest
+// exponent over the samples' y and non-zero T, and with them the path: exact
+// when the values are finite, n < 2^32 (the integer widths hold any count
+// below it) and Emax lies in [kAccEmaxLo, kAccEmaxHi]; narrow (64-bit
+// integers) when in addition every exponent is within 10 of Emax.  On the wide
+// grid the exact pass checks that every value lies on it.  (A NaN y counts
+// here, sending the call to the fp64 path, which leaves it out.)  Block maxima
+// go to the partials; the last block folds them.
 __global__ void __launch_bounds__(kAccBlock) k_acc_range(const double *__restrict__ y, const double *__restrict__ T,
                                                          int64_t n, AccRange *__restrict__ rg,
-                                                         unsigned int *ticket) {
-  __shared__ int red[kAccBlock / 32];
-  int emax = 0, lkey = 0, bad = 0;
+                                                         uint64_t *__restrict__ part, unsigned int *ticket) {
+  __shared__ unsigned long long red[kAccBlock / 32 * 2];
+  unsigned int top = 0u, nmin = 0u;  // nmin: max of 2047 - biased exponent
   const int64_t stride = (int64_t)gridDim.x * kAccBlock;
-  for (int64_t i = blockIdx.x * (int64_t)kAccBlock + threadIdx.x; i < n; i += stride) {
-    const uint64_t yb = (uint64_t)__double_as_longlong(__ldg(y + i));
-    if (!acc_is_sample(yb)) continue;
-    const uint64_t tb = (uint64_t)__double_as_longlong(__ldg(T + i));
-    range_note(yb, emax, lkey, bad);
-    if (tb << 1) range_note(tb, emax, lkey, bad);
+  for (int64_t i0 = blockIdx.x * (int64_t)kAccBlock + threadIdx.x; i0 < n; i0 += 4 * stride) {
+    uint2 yv[4], tv[4];  // four elements' loads in flight (a pattern of 0 is not a sample)
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int64_t i = i0 + k * stride;
+      yv[k] = i < n ? __ldg(reinterpret_cast<const uint2 *>(y) + i) : make_uint2(0u, 0u);
+      tv[k] = i < n ? __ldg(reinterpret_cast<const uint2 *>(T) + i) : make_uint2(0u, 0u);
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const unsigned int yh = yv[k].y, th = tv[k].y & 0x7FFFFFFFu;
+      if ((int)yh > 0 || (yh == 0u && yv[k].x != 0u)) {
+        top = max(top, max(yh, th));
+        nmin = max(nmin, 2047u - (yh >> 20));
+        if (th | tv[k].x) nmin = max(nmin, 2047u - (th >> 20));
+      }
+    }
   }
-  const int e = block_max_int(emax, red), k = block_max_int(lkey, red), b = block_max_int(bad, red);
-  if (threadIdx.x == 0 && e > 0) {
-    atomicMax(&rg->emax, e);
-    atomicMax(&rg->lkey, k);
-    if (b) atomicOr(&rg->bad, 1);
+  unsigned long long a = top, b = nmin;
+  block_max2(a, b, red);
+  if (threadIdx.x == 0) {
+    part[(int64_t)kAccPart * blockIdx.x] = a;
+    part[(int64_t)kAccPart * blockIdx.x + 1] = b;
   }
-  if (last_block(ticket) && threadIdx.x == 0) {
-    const int eb = __ldcg(&rg->emax), lk = __ldcg(&rg->lkey), bd = __ldcg(&rg->bad);
-    const int E = eb - 1023, lmin = kAccLkeyBias - lk;
-    rg->exact = !bd && n < (int64_t)1 << 32 &&
-                (eb == 0 || (E >= kAccEmaxLo && E <= kAccEmaxHi && lmin >= E - kAccGrid));
-    rg->S = kAccGrid - E;
-    rg->emax = rg->lkey = rg->bad = 0;
+  if (!last_block(ticket)) return;
+  a = 0ull;
+  b = 0ull;
+  for (int k = threadIdx.x; k < (int)gridDim.x; k += kAccBlock) {
+    a = max(a, (unsigned long long)__ldcg(part + (int64_t)kAccPart * k));
+    b = max(b, (unsigned long long)__ldcg(part + (int64_t)kAccPart * k + 1));
+  }
+  block_max2(a, b, red);
+  if (threadIdx.x == 0) {
+    const int E = (int)(a >> 20) - 1023;  // no sample: -1023, and nothing to sum
+    const int Emin = 2047 - (int)b - 1023;
+    const bool ex = a < 0x7FF00000ull && n < (int64_t)1 << 32 && (b == 0 || (E >= kAccEmaxLo && E <= kAccEmaxHi));
+    rg->exact = ex;
+    rg->narrow = ex && E - Emin <= 10;
+    rg->S = (E - Emin <= 10 ? 62 : kAccGrid) - E;
+    rg->inexact = 0;
   }
 }
 
@@ -201,69 +232,68 @@ __device__ __forceinline__ float rcp_approx(float x) {
   return r;
 }
 
-// A quotient digit from its estimate: one below the estimate's integer part
-// (never above the true digit when the estimate is within one half of it).
-__device__ __forceinline__ uint32_t acc_digit(float e) { return e >= 1.0f ? __float2uint_rz(e) - 1u : 0u; }
+// x as a float, truncated to 24 bits (relative error below 2^-23), by bit
+// arithmetic on the integer pipe.
+__device__ __forceinline__ float acc_u64_to_f32(uint64_t x) {
+  const int lz = __clzll((long long)x);
+  const uint64_t nx = x << (lz & 63);
+  const uint32_t bits = ((uint32_t)(190 - lz) << 23) + (uint32_t)(nx >> 40) - 0x800000u;
+  return x ? __uint_as_float(bits) : 0.0f;
+}
+
+// floor(e) for 0 <= e < 2^23: adding 2^23 rounded downward leaves it in the
+// low mantissa bits.
+__device__ __forceinline__ uint32_t acc_floor(float e) {
+  return __float_as_uint(__fadd_rd(e, 8388608.0f)) - 0x4B000000u;
+}
+
+// q B exactly (q < 2^32, B < 2^64), from two 32 x 32 -> 64-bit products.
+__device__ __forceinline__ u128 acc_mul32x64(uint32_t q, uint64_t B) {
+  return ((u128)((uint64_t)q * (uint32_t)(B >> 32)) << 32) + (uint64_t)q * (uint32_t)B;
+}
+
+// One schoolbook quotient digit: q = floor(R / Bs) given an estimate within
+// one of the true digit, R reduced by q Bs.  The remainder after the estimate
+// lies in [-Bs, 2 Bs); one conditional add and one conditional subtract settle
+// it.  |R| < 2^127 throughout, so the top bit is the sign.
+__device__ __forceinline__ uint32_t acc_settle(u128 &R, u128 Bs, u128 qBs, uint32_t q) {
+  R -= qBs;
+  const bool neg = (uint64_t)(R >> 64) >> 63;
+  R += neg ? Bs : (u128)0;
+  q -= neg ? 1u : 0u;
+  const bool ge = R >= Bs;
+  R -= ge ? Bs : (u128)0;
+  return q + (ge ? 1u : 0u);
+}
 
 // floor(Ma 2^54 / B) for 2^52 <= Ma, B < 2^53 (so the quotient lies in
 // [2^53, 2^55)), and whether the remainder is non-zero.  Schoolbook division
 // with three digits of 20, 20 and 15 bits: each digit is estimated from a
-// single-precision reciprocal of B's top 24 bits (relative error below 2^-21
-// all told, so with digits below 2^20 the estimate is within one half of the
-// true digit) and settled exactly on the integer remainder, which the digit
-// taken one low leaves non-negative and at most two steps away.
+// single-precision reciprocal of B's top 24 bits and the remainder's top bits
+// (relative error below 2^-20.4 all told, so with digits below 2^20 the
+// estimate's floor is within one of the true digit) and settled exactly on the
+// integer remainder.
 __device__ __forceinline__ uint64_t acc_div54(uint64_t Ma, uint64_t B, bool &rem_nz) {
-  const float inv = rcp_approx((float)(uint32_t)(B >> 29));  // B >> 29 in [2^23, 2^24): exact in float
+  // B >> 29 lies in [2^23, 2^24): its float is exponent 150 and the low 23 bits
+  const float inv = rcp_approx(__uint_as_float((150u << 23) | ((uint32_t)(B >> 29) & 0x7FFFFFu)));
   u128 R = (u128)Ma << 54;
-  const u128 B35 = (u128)B << 35, B15 = (u128)B << 15;
-  uint32_t q1 = acc_digit(__fmul_rn(__ull2float_rn((uint64_t)(R >> 64)), inv));
-  R -= ((u128)q1 * B) << 35;
-  for (int k = 0; k < 3 && R >= B35; ++k) {
-    R -= B35;
-    ++q1;
-  }
-  uint32_t q2 = acc_digit(__fmul_rn(__fmul_rn(__ull2float_rn((uint64_t)(R >> 40)), inv), 0.0625f));
-  R -= ((u128)q2 * B) << 15;
-  for (int k = 0; k < 3 && R >= B15; ++k) {
-    R -= B15;
-    ++q2;
-  }
-  uint32_t q3 = acc_digit(__fmul_rn(__fmul_rn(__ull2float_rn((uint64_t)(R >> 20)), inv), 1.0f / 512.0f));
-  R -= (u128)q3 * B;
-  for (int k = 0; k < 3 && R >= (u128)B; ++k) {
-    R -= B;
-    ++q3;
-  }
+  const u128 B35 = (u128)B << 35, B15 = (u128)B << 15, B0 = (u128)B;
+  uint32_t q1 = acc_floor(__fmul_rn(acc_u64_to_f32(Ma >> 10), inv));
+  q1 = acc_settle(R, B35, acc_mul32x64(q1, B) << 35, q1);
+  uint32_t q2 = acc_floor(__fmul_rn(__fmul_rn(acc_u64_to_f32((uint64_t)(R >> 40)), inv), 0.0625f));
+  q2 = acc_settle(R, B15, acc_mul32x64(q2, B) << 15, q2);
+  uint32_t q3 = acc_floor(__fmul_rn(__fmul_rn(acc_u64_to_f32((uint64_t)(R >> 20)), inv), 1.0f / 512.0f));
+  q3 = acc_settle(R, B0, acc_mul32x64(q3, B), q3);
   rem_nz = R != 0;
   return ((uint64_t)q1 << 35) + ((uint64_t)q2 << 15) + q3;
 }
 
-// Bit pattern of fl(fl(|D|) / y), where |D| (below 2^80) is |T - y| on the
-// grid and y = My 2^ky on the same grid: the difference rounded to 53 bits
-// (nearest, ties to even), then the quotient rounded the same way.  Every
-// quotient lies in [2^-81, 2^81], a normal double.
-__device__ __forceinline__ uint64_t acc_rel_bits(u128 Dm, uint64_t My, int ky) {
-  if (Dm == 0) return 0ull;
-  const uint64_t dh = (uint64_t)(Dm >> 64), dl = (uint64_t)Dm;
-  const int lead = dh ? 127 - __clzll((long long)dh) : 63 - __clzll((long long)dl);
-  uint64_t Ma;
-  int ka;
-  if (lead <= 52) {
-    Ma = dl << (52 - lead);
-    ka = lead - 52;
-  } else {
-    int s = lead - 52;  // 1..27: the dropped bits lie in the low word
-    Ma = (uint64_t)(Dm >> s);
-    const uint64_t low = dl & ((1ull << s) - 1), half = 1ull << (s - 1);
-    Ma += (low > half || (low == half && (Ma & 1ull))) ? 1ull : 0ull;
-    if (Ma >> 53) {
-      Ma >>= 1;
-      ++s;
-    }
-    ka = s;
-  }
+// fl(Ma 2^ka / (My 2^ky)) as a bit pattern, for 2^52 <= Ma, My < 2^53: the
+// quotient rounded to nearest (ties to even).  Every quotient here lies in
+// [2^-81, 2^81], a normal double.
+__device__ __forceinline__ uint64_t acc_quot_bits(uint64_t Ma, int ka, uint64_t My, int ky) {
   bool rem;
-  const uint64_t Q = acc_div54(Ma, My, rem);  // rel = (Q + frac) 2^(ka - ky - 54)
+  const uint64_t Q = acc_div54(Ma, My, rem);  // quotient = (Q + frac) 2^(ka - ky - 54)
   int e = ka - ky - 54;
   uint64_t mant, rb;
   bool st;
@@ -286,6 +316,48 @@ __device__ __forceinline__ uint64_t acc_rel_bits(u128 Dm, uint64_t My, int ky) {
   return ((uint64_t)(e + 1075) << 52) | (mant & kFracMask);
 }
 
+// Bit pattern of fl(fl(|D|) / y), where |D| (below 2^80) is |T - y| on the
+// grid and y = My 2^ky on the same grid: the difference rounded to 53 bits
+// (nearest, ties to even), then the quotient rounded the same way.
+__device__ __forceinline__ uint64_t acc_rel_bits(u128 Dm, uint64_t My, int ky) {
+  if (Dm == 0) return 0ull;
+  const uint64_t dh = (uint64_t)(Dm >> 64), dl = (uint64_t)Dm;
+  const int lead = dh ? 127 - __clzll((long long)dh) : 63 - __clzll((long long)dl);
+  int ka = lead - 52;
+  uint64_t Ma;
+  if (ka <= 0) {
+    Ma = dl << -ka;
+  } else {
+    // drop ka (1..27) bits, all in the low word, rounding to nearest even
+    Ma = (dl >> ka) | (dh << (64 - ka));
+    const uint64_t low = dl & ((1ull << ka) - 1), half = 1ull << (ka - 1);
+    Ma += (low > half || (low == half && (Ma & 1ull))) ? 1ull : 0ull;
+    const uint64_t carry = Ma >> 53;
+    Ma >>= carry;
+    ka += (int)carry;
+  }
+  return acc_quot_bits(Ma, ka, My, ky);
+}
+
+// The same for |D| below 2^64.
+__device__ __forceinline__ uint64_t acc_rel_bits64(uint64_t d, uint64_t My, int ky) {
+  if (d == 0) return 0ull;
+  int ka = 63 - __clzll((long long)d) - 52;
+  uint64_t Ma;
+  if (ka <= 0) {
+    Ma = d << -ka;
+  } else {
+    // drop ka (1..11) bits, rounding to nearest even
+    Ma = d >> ka;
+    const uint64_t low = d & ((1ull << ka) - 1), half = 1ull << (ka - 1);
+    Ma += (low > half || (low == half && (Ma & 1ull))) ? 1ull : 0ull;
+    const uint64_t carry = Ma >> 53;
+    Ma >>= carry;
+    ka += (int)carry;
+  }
+  return acc_quot_bits(Ma, ka, My, ky);
+}
+
 __device__ __forceinline__ void add128w(uint64_t *a, u128 x) {
   const u128 s = (((u128)a[1] << 64) | a[0]) + x;
   a[0] = (uint64_t)s;
@@ -306,6 +378,11 @@ __device__ __forceinline__ void add_sq(uint64_t *a, u128 X) {
   const u128 p = (u128)xl * xl, q = (u128)xl * (xh << 1);
   const u128 mid = (p >> 64) + (uint64_t)q;
   add192w(a, (uint64_t)p, (uint64_t)mid, (uint64_t)(q >> 64) + xh * xh + (uint64_t)(mid >> 64));
+}
+
+// a += x^2 for x < 2^64 (a: 192 bits).
+__device__ __forceinline__ void add_sq64(uint64_t *a, uint64_t x) {
+  add192w(a, x * x, __umul64hi(x, x), 0ull);
 }
 
 // The exact sums: [0] count, [1..2] sum Y, [3..4] sum T (two's complement),
@@ -339,18 +416,29 @@ __device__ __forceinline__ void acc_block_combine(uint64_t *w, uint64_t *red) {
     for (int v = 1; v < (int)(blockDim.x >> 5); ++v) acc_combine(w, red + v * kAccWords);
 }
 
-// One sample on the grid 2^-S (the range pass guarantees both values are
-// normal and on it): the sums and rel's bit pattern.
-__device__ __forceinline__ uint64_t acc_exact_sample(uint64_t yb, uint64_t tb, int S, uint64_t *w) {
+// M 2^k as an integer for k <= 26; `lost` is set when k < 0 drops set bits
+// (the value is not on the grid).
+__device__ __forceinline__ u128 acc_grid(uint64_t M, int k, bool &lost) {
+  const int r = min(-k, 63);
+  lost |= k < 0 && (-k > 52 || (M & ((1ull << r) - 1)) != 0ull);
+  const uint64_t lo = k >= 0 ? M << k : M >> r;
+  const uint64_t hi = k > 0 ? M >> (64 - k) : 0ull;
+  return ((u128)hi << 64) | lo;
+}
+
+// One sample on the grid 2^-S: the sums and rel's bit pattern.  `lost` is set
+// when y or T is not on the grid (the results are then discarded).
+__device__ __forceinline__ uint64_t acc_exact_sample(uint64_t yb, uint64_t tb, int S, uint64_t *w, bool &lost) {
+  const int bey = (int)(yb >> 52);
   const uint64_t My = (yb & kFracMask) | kHiddenBit;
-  const int ky = (int)(yb >> 52) - 1075 + S;  // y = My 2^ky on the grid, ky <= 26
-  const u128 Y = ky >= 0 ? (u128)My << ky : (u128)(My >> min(-ky, 63));
+  const int ky = max(bey, 1) - 1075 + S;  // y = My 2^ky on the grid, ky <= 26
+  lost |= bey == 0;                       // subnormal: far below any grid in use
+  const u128 Y = acc_grid(My, ky, lost);
   u128 Tm = 0;
   const bool tneg = (tb >> 63) != 0;
   if (tb << 1) {
-    const uint64_t Mt = (tb & kFracMask) | kHiddenBit;
-    const int kt = (int)((tb >> 52) & 0x7FF) - 1075 + S;
-    Tm = kt >= 0 ? (u128)Mt << kt : (u128)(Mt >> min(-kt, 63));
+    const int bet = (int)((tb >> 52) & 0x7FF);
+    Tm = acc_grid((tb & kFracMask) | (bet ? kHiddenBit : 0ull), max(bet, 1) - 1075 + S, lost);
   }
   w[0] += 1;
   add128w(w + 1, Y);
@@ -360,6 +448,26 @@ __device__ __forceinline__ uint64_t acc_exact_sample(uint64_t yb, uint64_t tb, i
   add_sq(w + 8, Tm);
   add_sq(w + 11, Dm);
   return acc_rel_bits(Dm, My, ky);
+}
+
+// One sample on the 63-bit grid 2^-S (every exponent within 10 of the
+// largest, so each value is an integer below 2^63 there): the sums and rel's
+// bit pattern.
+__device__ __forceinline__ uint64_t acc_exact_sample64(uint64_t yb, uint64_t tb, int S, uint64_t *w) {
+  const uint64_t My = (yb & kFracMask) | kHiddenBit;
+  const int ky = (int)(yb >> 52) - 1075 + S;  // 0..10
+  const uint64_t Y = My << ky;
+  uint64_t Tm = 0ull;
+  const bool tneg = (tb >> 63) != 0;
+  if (tb << 1) Tm = ((tb & kFracMask) | kHiddenBit) << ((int)((tb >> 52) & 0x7FF) - 1075 + S);
+  w[0] += 1;
+  add128w(w + 1, Y);
+  add128w(w + 3, tneg ? (u128)0 - Tm : (u128)Tm);
+  const uint64_t Dm = tneg ? Y + Tm : (Y >= Tm ? Y - Tm : Tm - Y);
+  add_sq64(w + 5, Y);
+  add_sq64(w + 8, Tm);
+  add_sq64(w + 11, Dm);
+  return acc_rel_bits64(Dm, My, ky);
 }
 
 // 64 x 192 -> 256-bit product.
@@ -384,13 +492,53 @@ __device__ __forceinline__ void sub256(uint64_t *a, const uint64_t *b) {
   acc_add256(a, 1, 0, 0, 0);
 }
 
+// The signed 256-bit two's-complement integer w, times 2^e2, as the nearest
+// double (ties to even), by integer operations only; `ok` is cleared when the
+// result would leave the normal range (the caller then takes a slower route).
+__device__ __forceinline__ double acc_i256_to_double(const uint64_t *wi, int e2, bool &ok) {
+  uint64_t w0 = wi[0], w1 = wi[1], w2 = wi[2], w3 = wi[3];
+  const bool neg = (w3 >> 63) != 0;
+  if (neg) {
+    w0 = ~w0;
+    w1 = ~w1;
+    w2 = ~w2;
+    w3 = ~w3;
+    u128 s = (u128)w0 + 1;
+    w0 = (uint64_t)s;
+    s = (u128)w1 + (uint64_t)(s >> 64);
+    w1 = (uint64_t)s;
+    s = (u128)w2 + (uint64_t)(s >> 64);
+    w2 = (uint64_t)s;
+    w3 += (uint64_t)(s >> 64);
+  }
+  const int t = w3 ? 3 : w2 ? 2 : w1 ? 1 : 0;
+  const uint64_t a = t == 3 ? w3 : t == 2 ? w2 : t == 1 ? w1 : w0;
+  if (a == 0) return 0.0;
+  const uint64_t b = t == 3 ? w2 : t == 2 ? w1 : t == 1 ? w0 : 0ull;
+  const bool rest = (t == 3 ? (w1 | w0) : t == 2 ? w0 : 0ull) != 0ull;
+  const int lz = __clzll((long long)a);
+  const uint64_t top = lz ? (a << lz) | (b >> (64 - lz)) : a;  // leading one at bit 63
+  const bool below = (lz ? (b << lz) : b) != 0ull || rest;
+  uint64_t mant = top >> 11;
+  const uint64_t rb = (top >> 10) & 1ull;
+  const bool st = (top & 0x3FFull) != 0ull || below;
+  mant += rb & ((st ? 1ull : 0ull) | (mant & 1ull));
+  int ex = 64 * t + 63 - lz + e2;  // exponent of the leading bit
+  if (mant >> 53) {
+    mant >>= 1;
+    ++ex;
+  }
+  if (ex < -1022 || ex > 1023) {
+    ok = false;
+    return 0.0;
+  }
+  return __longlong_as_double((long long)(((uint64_t)neg << 63) | ((uint64_t)(ex + 1023) << 52) | (mant & kFracMask)));
+}
+
 // Select state for a new call: the prefix every sample shares (the common
-// leading bits of the smallest and largest rel) and the target ranks
-// ceil(q m / 100), q = 50, 90, 99.  Resets the rel accumulators.
-__device__ __forceinline__ void acc_publish_select(RelAcc *ra, SelState *sel, int64_t m) {
-  const uint64_t hi = __ldcg(&ra->max), lo = ~(uint64_t)__ldcg(&ra->nmax);
-  ra->max = 0ull;
-  ra->nmax = 0ull;
+// leading bits of the smallest and largest rel, lo and hi) and the target
+// ranks ceil(q m / 100), q = 50, 90, 99.
+__device__ __forceinline__ void acc_publish_select(uint64_t hi, uint64_t lo, SelState *sel, int64_t m) {
   sel->relmax = hi;
   const int cp = m == 0 || hi == lo ? 64 : __clzll((long long)(hi ^ lo));
   sel->shift = m == 0 ? 0 : 64 - cp;
@@ -402,64 +550,85 @@ __device__ __forceinline__ void acc_publish_select(RelAcc *ra, SelState *sel, in
   }
 }
 
+// Largest rel and largest ~rel (so zero is the identity of both).
 __device__ __forceinline__ void acc_note_rel(uint64_t rb, unsigned long long &rmax, unsigned long long &rnmax) {
   rmax = max(rmax, (unsigned long long)rb);
   rnmax = max(rnmax, (unsigned long long)~rb);
 }
 
-__device__ __forceinline__ void acc_flush_rel(unsigned long long rmax, unsigned long long rnmax, RelAcc *ra) {
+template <bool kNarrow>
+__device__ __forceinline__ void acc_exact_loop(const double *__restrict__ y, const double *__restrict__ T, int64_t n,
+                                               int S, uint64_t *__restrict__ relbits, uint64_t *w,
+                                               unsigned long long &rmax, unsigned long long &rnmax, bool &lost) {
+  const int64_t stride = (int64_t)gridDim.x * kAccBlock;
+  for (int64_t i0 = blockIdx.x * (int64_t)kAccBlock + threadIdx.x; i0 < n; i0 += 2 * stride) {
+    uint64_t yb[2], tb[2];  // two elements' loads in flight (a pattern of 0 is not a sample)
 #pragma unroll
-  for (int d = 16; d; d >>= 1) {
-    rmax = max(rmax, __shfl_xor_sync(0xffffffffu, rmax, d));
-    rnmax = max(rnmax, __shfl_xor_sync(0xffffffffu, rnmax, d));
-  }
-  if ((threadIdx.x & 31) == 0 && (rmax | rnmax)) {
-    atomicMax(&ra->max, rmax);
-    atomicMax(&ra->nmax, rnmax);
+    for (int k = 0; k < 2; ++k) {
+      const int64_t i = i0 + k * stride;
+      yb[k] = i < n ? (uint64_t)__double_as_longlong(__ldg(y + i)) : 0ull;
+      tb[k] = i < n ? (uint64_t)__double_as_longlong(__ldg(T + i)) : 0ull;
+    }
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const int64_t i = i0 + k * stride;
+      uint64_t rb = ~0ull;  // not a sample
+      if (acc_is_sample(yb[k])) {
+        rb = kNarrow ? acc_exact_sample64(yb[k], tb[k], S, w) : acc_exact_sample(yb[k], tb[k], S, w, lost);
+        acc_note_rel(rb, rmax, rnmax);
+      }
+      if (i < n) relbits[i] = rb;
+    }
   }
 }
 
 // Exact path: the sums and every rel in one pass over y and T; the last block
 // folds the block partials and writes sums[0] = m and, scaled by m 2^(2S),
 // sums[3..6] = sxx, syy, sxy, ssr.  Returns at once when the range pass chose
-// the fp64 path.
+// the fp64 path; flags rg->inexact (and the fp64 path then redoes the call)
+// when a value is not on the grid.
 __global__ void __launch_bounds__(kAccBlock) k_acc_exact(const double *__restrict__ y, const double *__restrict__ T,
-                                                         int64_t n, const AccRange *__restrict__ rg,
+                                                         int64_t n, AccRange *__restrict__ rg,
                                                          uint64_t *__restrict__ relbits, uint64_t *__restrict__ part,
-                                                         double *__restrict__ sums, RelAcc *__restrict__ ra,
-                                                         SelState *__restrict__ sel, unsigned int *ticket) {
+                                                         double *__restrict__ sums, SelState *__restrict__ sel,
+                                                         unsigned int *ticket) {
   __shared__ uint64_t red[kAccBlock / 32 * kAccWords];
+  __shared__ unsigned long long red2[kAccBlock / 32 * 2];
   if (!rg->exact) return;
   const int S = rg->S;
   uint64_t w[kAccWords];
 #pragma unroll
   for (int j = 0; j < kAccWords; ++j) w[j] = 0ull;
   unsigned long long rmax = 0ull, rnmax = 0ull;
-  const int64_t stride = (int64_t)gridDim.x * kAccBlock;
-  for (int64_t i = blockIdx.x * (int64_t)kAccBlock + threadIdx.x; i < n; i += stride) {
-    const uint64_t yb = (uint64_t)__double_as_longlong(__ldg(y + i));
-    const uint64_t tb = (uint64_t)__double_as_longlong(__ldg(T + i));
-    uint64_t rb = ~0ull;  // not a sample
-    if (acc_is_sample(yb)) {
-      rb = acc_exact_sample(yb, tb, S, w);
-      acc_note_rel(rb, rmax, rnmax);
-    }
-    relbits[i] = rb;
-  }
-  acc_flush_rel(rmax, rnmax, ra);
+  bool lost = false;
+  if (rg->narrow)
+    acc_exact_loop<true>(y, T, n, S, relbits, w, rmax, rnmax, lost);
+  else
+    acc_exact_loop<false>(y, T, n, S, relbits, w, rmax, rnmax, lost);
+  if (__syncthreads_or(lost) && threadIdx.x == 0) atomicOr(&rg->inexact, 1);
+  block_max2(rmax, rnmax, red2);
   acc_block_combine(w, red);
-  if (threadIdx.x == 0)
+  if (threadIdx.x == 0) {
+    uint64_t *p = part + (int64_t)blockIdx.x * kAccPart;
 #pragma unroll
-    for (int j = 0; j < kAccWords; ++j) part[(int64_t)blockIdx.x * kAccPart + j] = w[j];
+    for (int j = 0; j < kAccWords; ++j) p[j] = w[j];
+    p[kAccWords] = rmax;
+    p[kAccWords + 1] = rnmax;
+  }
   if (!last_block(ticket)) return;
 #pragma unroll
   for (int j = 0; j < kAccWords; ++j) w[j] = 0ull;
+  rmax = rnmax = 0ull;
   for (int b = threadIdx.x; b < (int)gridDim.x; b += kAccBlock) {
+    const uint64_t *p = part + (int64_t)b * kAccPart;
     uint64_t o[kAccWords];
 #pragma unroll
-    for (int j = 0; j < kAccWords; ++j) o[j] = __ldcg(part + (int64_t)b * kAccPart + j);
+    for (int j = 0; j < kAccWords; ++j) o[j] = __ldcg(p + j);
     acc_combine(w, o);
+    rmax = max(rmax, (unsigned long long)__ldcg(p + kAccWords));
+    rnmax = max(rnmax, (unsigned long long)__ldcg(p + kAccWords + 1));
   }
+  block_max2(rmax, rnmax, red2);
   acc_block_combine(w, red);
   if (threadIdx.x != 0) return;
   const uint64_t m = w[0];
@@ -503,12 +672,13 @@ __global__ void __launch_bounds__(kAccBlock) k_acc_exact(const double *__restric
   else
     sub256(sxy, tmp);
   mul64x192(m, w + 11, ssr);
+  bool ok = true;  // every value here is below 2^227 in magnitude
   sums[0] = (double)m;
-  sums[3] = int256_to_dd(sxx, 0).hi;
-  sums[4] = int256_to_dd(syy, 0).hi;
-  sums[5] = 0.5 * int256_to_dd(sxy, 0).hi;
-  sums[6] = int256_to_dd(ssr, 0).hi;
-  acc_publish_select(ra, sel, (int64_t)m);
+  sums[3] = acc_i256_to_double(sxx, 0, ok);
+  sums[4] = acc_i256_to_double(syy, 0, ok);
+  sums[5] = acc_i256_to_double(sxy, -1, ok);
+  sums[6] = acc_i256_to_double(ssr, 0, ok);
+  acc_publish_select(rmax, ~(uint64_t)rnmax, sel, (int64_t)m);
 }
 
 // ---------------------------------------------------------------- fp64 path
@@ -516,14 +686,15 @@ __global__ void __launch_bounds__(kAccBlock) k_acc_exact(const double *__restric
 // Pass 1: per-block count, sum y, sum T over the samples; rel's bit patterns
 // stored (all ones for a batch that is not a sample, which the select never
 // counts).  The last block folds the partials into sums[0..2] and sets up the
-// select.  Returns at once when the range pass chose the exact path.
+// select.  Returns at once when the exact path did the call.
 __global__ void __launch_bounds__(kAccBlock) k_acc_sums(const double *__restrict__ y, const double *__restrict__ T,
                                                         int64_t n, const AccRange *__restrict__ rg,
                                                         uint64_t *__restrict__ relbits, double *__restrict__ part,
-                                                        double *__restrict__ sums, RelAcc *__restrict__ ra,
-                                                        SelState *__restrict__ sel, unsigned int *ticket) {
+                                                        double *__restrict__ sums, SelState *__restrict__ sel,
+                                                        unsigned int *ticket) {
   __shared__ double red[kAccBlock / 32];
-  if (rg->exact) return;
+  __shared__ unsigned long long red2[kAccBlock / 32 * 2];
+  if (rg->exact && !rg->inexact) return;
   double c = 0.0, sy = 0.0, st = 0.0;
   unsigned long long rmax = 0ull, rnmax = 0ull;
   const int64_t stride = (int64_t)gridDim.x * kAccBlock;
@@ -539,17 +710,26 @@ __global__ void __launch_bounds__(kAccBlock) k_acc_sums(const double *__restrict
     }
     relbits[i] = bits;
   }
-  acc_flush_rel(rmax, rnmax, ra);
+  block_max2(rmax, rnmax, red2);
   const double a = block_sum_fixed(c, red), b = block_sum_fixed(sy, red), d = block_sum_fixed(st, red);
   if (threadIdx.x == 0) {
     double *p = part + (int64_t)kAccPart * blockIdx.x;
     p[0] = a;
     p[1] = b;
     p[2] = d;
+    p[3] = __longlong_as_double((long long)rmax);  // bit patterns, folded as integers
+    p[4] = __longlong_as_double((long long)rnmax);
   }
   if (!last_block(ticket)) return;
   fold_partials(part, gridDim.x, 3, red, sums);
-  if (threadIdx.x == 0) acc_publish_select(ra, sel, (int64_t)sums[0]);
+  rmax = rnmax = 0ull;
+  for (int k = threadIdx.x; k < (int)gridDim.x; k += kAccBlock) {
+    const double *p = part + (int64_t)kAccPart * k;
+    rmax = max(rmax, (unsigned long long)__double_as_longlong(__ldcg(p + 3)));
+    rnmax = max(rnmax, (unsigned long long)__double_as_longlong(__ldcg(p + 4)));
+  }
+  block_max2(rmax, rnmax, red2);
+  if (threadIdx.x == 0) acc_publish_select(rmax, ~(uint64_t)rnmax, sel, (int64_t)sums[0]);
 }
 
 // Pass 2: centred moments with the means from pass 1 (sums = {count, sum y,
@@ -559,7 +739,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc_moments(const double *__restr
                                                            double *__restrict__ sums, double *__restrict__ part,
                                                            unsigned int *ticket) {
   __shared__ double red[kAccBlock / 32];
-  if (rg->exact) return;
+  if (rg->exact && !rg->inexact) return;
   const double m = sums[0];
   const double my = m > 0 ? sums[1] / m : 0.0, mt = m > 0 ? sums[2] / m : 0.0;
   double sxx = 0.0, syy = 0.0, sxy = 0.0, ssr = 0.0;
@@ -598,163 +778,428 @@ __device__ __forceinline__ u128 acc_rel_fixed(uint64_t v, int bemax) {
   return sv >= 0 ? (u128)M << sv : sv > -64 ? (u128)(M >> -sv) : (u128)0;
 }
 
-// The three targets' next digit, one warp per target: lane l sums bins
-// [64 l, 64 l + 64) of the target's histogram, a warp scan finds the lane
-// whose range holds the remaining rank, then the same over that lane's bins
-// two at a time.
-__device__ __forceinline__ void acc_pick(const unsigned int *__restrict__ hs, SelState *sel, int t, uint64_t pf,
-                                         int w) {
+
+// One warp: the bin of a kSelBins-bin histogram that holds rank r (1-based),
+// the count below that bin and the bin's own count, valid in every lane.  Lane
+// l sums bins [64 l, 64 l + 64), a warp scan finds the lane whose range holds
+// r, then the same over that lane's bins two at a time.  kGlobal: the
+// histogram is in global memory, written by other blocks' atomics.
+template <bool kGlobal>
+__device__ __forceinline__ void acc_scan_pick(const unsigned int *h, int64_t r, int &bin, int64_t &below,
+                                              int64_t &cnt) {
+  static_assert(kSelBins == 64 * 32, "64 bins per lane");
   const int lane = threadIdx.x & 31;
-  const int64_t r = sel->rk[t];
-  const uint4 *h4 = reinterpret_cast<const uint4 *>(hs + 64 * lane);
-  uint64_t s = 0;
+  int64_t s = 0;
 #pragma unroll
   for (int j = 0; j < 16; ++j) {
-    const uint4 q = __ldcg(h4 + j);
-    s += (uint64_t)q.x + q.y + q.z + q.w;
+    const uint4 *p = reinterpret_cast<const uint4 *>(h + 64 * lane + 4 * j);
+    const uint4 q = kGlobal ? __ldcg(p) : *p;
+    s += (int64_t)q.x + q.y + q.z + q.w;
   }
-  uint64_t inc = s;
+  int64_t inc = s;
 #pragma unroll
   for (int d = 1; d < 32; d <<= 1) {
-    const uint64_t o = __shfl_up_sync(0xffffffffu, inc, d);
+    const int64_t o = __shfl_up_sync(0xffffffffu, inc, d);
     if (lane >= d) inc += o;
   }
-  unsigned ball = __ballot_sync(0xffffffffu, (int64_t)inc >= r);
+  unsigned ball = __ballot_sync(0xffffffffu, inc >= r);
   const int L = ball ? __ffs(ball) - 1 : 31;
-  const uint64_t below = __shfl_sync(0xffffffffu, inc - s, L);
-  const uint2 pr = __ldcg(reinterpret_cast<const uint2 *>(hs + 64 * L) + lane);
-  const uint64_t ps = (uint64_t)pr.x + pr.y;
-  uint64_t inc2 = ps;
+  const int64_t bl = __shfl_sync(0xffffffffu, inc - s, L);
+  const uint2 *p2 = reinterpret_cast<const uint2 *>(h + 64 * L + 2 * lane);
+  const uint2 pr = kGlobal ? __ldcg(p2) : *p2;
+  const int64_t ps = (int64_t)pr.x + pr.y;
+  int64_t inc2 = ps;
 #pragma unroll
   for (int d = 1; d < 32; d <<= 1) {
-    const uint64_t o = __shfl_up_sync(0xffffffffu, inc2, d);
+    const int64_t o = __shfl_up_sync(0xffffffffu, inc2, d);
     if (lane >= d) inc2 += o;
   }
-  ball = __ballot_sync(0xffffffffu, (int64_t)(below + inc2) >= r);
+  ball = __ballot_sync(0xffffffffu, bl + inc2 >= r);
   const int L2 = ball ? __ffs(ball) - 1 : 31;
-  if (lane == L2) {
-    const uint64_t b0 = below + inc2 - ps;
-    const bool first = (int64_t)(b0 + pr.x) >= r;
-    const int bin = 64 * L + 2 * lane + (first ? 0 : 1);
-    sel->rk[t] = r - (int64_t)(first ? b0 : b0 + pr.x);
-    sel->pf[t] = (pf << w) | (uint64_t)bin;
-  }
+  const int64_t b0 = bl + inc2 - ps;
+  const bool first = b0 + pr.x >= r;
+  bin = __shfl_sync(0xffffffffu, 64 * L + 2 * lane + (first ? 0 : 1), L2);
+  below = __shfl_sync(0xffffffffu, first ? b0 : b0 + (int64_t)pr.x, L2);
+  cnt = __shfl_sync(0xffffffffu, (int64_t)(first ? pr.x : pr.y), L2);
 }
 
-// One radix-select pass.  Every sample whose bits above `shift` equal a
-// target's prefix adds one to that prefix's histogram at its next digit (the
-// kSelBits bits below `shift`, fewer at the end); targets with the same
-// prefix share one histogram, and prefixes of one length are either equal or
-// disjoint, so a sample counts at most once.  The last block picks each
-// target's digit and clears the histograms.  Pass 0 also sums rel in fixed
-// point into sums[7] (the largest rel itself when it is inf or NaN, which is
-// what an exact sum gives then).  Later passes return at once once every
-// digit is settled.
-__global__ void __launch_bounds__(kSelBlock) k_acc_select(const uint64_t *__restrict__ relbits, int64_t n,
-                                                          SelState *__restrict__ sel, unsigned int *__restrict__ hist,
-                                                          uint64_t *__restrict__ part, double *__restrict__ sums,
-                                                          unsigned int *ticket, int pass) {
-  __shared__ unsigned int h[kAccTargets * kSelBins];
+// Select, first digit: every sample adds one to the histogram of its first
+// digit below the shared prefix (all samples share it, so no compare), and
+// its rel to the fixed-point sum.  The last block writes sums[7] (the largest
+// rel itself when that is inf or NaN, which is what an exact sum gives then),
+// picks each target's digit, and lays out the candidate lists: targets in the
+// same bin share one.  With no digit left (every rel equal) the prefixes are
+// already the answers.
+__global__ void __launch_bounds__(kSelBlock) k_acc_sel0(const uint64_t *__restrict__ relbits, int64_t n,
+                                                        SelState *__restrict__ sel, unsigned int *__restrict__ hist,
+                                                        uint64_t *__restrict__ part, double *__restrict__ sums,
+                                                        unsigned int *ticket) {
+  __shared__ unsigned int h[kSelBins];
   __shared__ uint64_t red[kSelBlock / 32 * 3];
   const int shift = sel->shift;
   const uint64_t relmax = sel->relmax;
   const bool digit = shift > 0;
-  const bool rsum = pass == 0 && relmax < 0x7FF0000000000000ull;
-  if (!digit && pass != 0) return;
-  const uint64_t pf0 = sel->pf[0], pf1 = sel->pf[1], pf2 = sel->pf[2];
+  const bool rsum = relmax < 0x7FF0000000000000ull;
   const int w = min(kSelBits, shift), lo = shift - w;
   const uint64_t dmask = (1ull << w) - 1;
-  if (digit) {
-    for (int i = threadIdx.x; i < kAccTargets * kSelBins; i += kSelBlock) h[i] = 0u;
-    __syncthreads();
-  }
+  for (int i = threadIdx.x; i < kSelBins; i += kSelBlock) h[i] = 0u;
+  __syncthreads();
   const int bemax = max((int)(relmax >> 52), 1);
-  uint64_t s0 = 0, s1 = 0, s2 = 0;  // sum of rel on its grid, 192 bits
-  const int64_t stride = (int64_t)gridDim.x * kSelBlock;
-  for (int64_t i = blockIdx.x * (int64_t)kSelBlock + threadIdx.x; i < n; i += stride) {
-    const uint64_t v = __ldcg(relbits + i);
-    if (v == ~0ull) continue;  // not a sample
-    if (digit) {
-      const uint64_t key = v >> shift;
-      const int s = key == pf0 ? 0 : key == pf1 ? 1 : key == pf2 ? 2 : -1;
-      if (s >= 0) atomicAdd(&h[s * kSelBins + (int)((v >> lo) & dmask)], 1u);
-    }
+  uint64_t acc[3] = {0, 0, 0};  // sum of rel on its grid, 192 bits
+  auto visit = [&](uint64_t v) {
+    if (v == ~0ull) return;  // not a sample
+    if (digit) atomicAdd(&h[(int)((v >> lo) & dmask)], 1u);
     if (rsum) {
-      uint64_t a[3] = {s0, s1, s2};
       const u128 x = acc_rel_fixed(v, bemax);
-      add192w(a, (uint64_t)x, (uint64_t)(x >> 64), 0);
-      s0 = a[0];
-      s1 = a[1];
-      s2 = a[2];
+      add192w(acc, (uint64_t)x, (uint64_t)(x >> 64), 0);
+    }
+  };
+  // eight consecutive patterns per thread (four 16-byte loads in flight), then the tail
+  const int64_t n8 = n >> 3;
+  const int64_t g = blockIdx.x * (int64_t)kSelBlock + threadIdx.x, stride = (int64_t)gridDim.x * kSelBlock;
+  const ulonglong2 *r2 = reinterpret_cast<const ulonglong2 *>(relbits);
+  for (int64_t c = g; c < n8; c += stride) {
+    ulonglong2 q[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) q[k] = __ldcg(r2 + 4 * c + k);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      visit(q[k].x);
+      visit(q[k].y);
     }
   }
-  if (digit) {
-    __syncthreads();
-    for (int i = threadIdx.x; i < kAccTargets * kSelBins; i += kSelBlock) {
+  if (g < n - 8 * n8) visit(__ldcg(relbits + 8 * n8 + g));
+  __syncthreads();
+  if (digit)
+    for (int i = threadIdx.x; i < kSelBins; i += kSelBlock) {
       const unsigned int c = h[i];
       if (c) atomicAdd(hist + i, c);
     }
-  }
-  if (pass == 0) {
-    uint64_t a[3] = {s0, s1, s2};
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
 #pragma unroll
-    for (int d = 16; d; d >>= 1) {
-      const uint64_t o0 = __shfl_xor_sync(0xffffffffu, a[0], d), o1 = __shfl_xor_sync(0xffffffffu, a[1], d),
-                     o2 = __shfl_xor_sync(0xffffffffu, a[2], d);
-      add192w(a, o0, o1, o2);
-    }
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    if (lane == 0) {
-      red[3 * wid] = a[0];
-      red[3 * wid + 1] = a[1];
-      red[3 * wid + 2] = a[2];
-    }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      for (int v = 1; v < kSelBlock / 32; ++v) add192w(a, red[3 * v], red[3 * v + 1], red[3 * v + 2]);
-      uint64_t *p = part + (int64_t)kAccPart * blockIdx.x;
-      p[0] = a[0];
-      p[1] = a[1];
-      p[2] = a[2];
-    }
+  for (int d = 16; d; d >>= 1) {
+    const uint64_t o0 = __shfl_xor_sync(0xffffffffu, acc[0], d), o1 = __shfl_xor_sync(0xffffffffu, acc[1], d),
+                   o2 = __shfl_xor_sync(0xffffffffu, acc[2], d);
+    add192w(acc, o0, o1, o2);
+  }
+  if (lane == 0) {
+    red[3 * wid] = acc[0];
+    red[3 * wid + 1] = acc[1];
+    red[3 * wid + 2] = acc[2];
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int v = 1; v < kSelBlock / 32; ++v) add192w(acc, red[3 * v], red[3 * v + 1], red[3 * v + 2]);
+    uint64_t *p = part + (int64_t)kAccPart * blockIdx.x;
+    p[0] = acc[0];
+    p[1] = acc[1];
+    p[2] = acc[2];
   }
   if (!last_block(ticket)) return;
-  if (pass == 0) {
-    uint64_t a[3] = {0, 0, 0};
-    for (int b = threadIdx.x; b < (int)gridDim.x; b += kSelBlock) {
-      const uint64_t *p = part + (int64_t)kAccPart * b;
-      add192w(a, __ldcg(p), __ldcg(p + 1), __ldcg(p + 2));
-    }
+  uint64_t a[3] = {0, 0, 0};
+  for (int b = threadIdx.x; b < (int)gridDim.x; b += kSelBlock) {
+    const uint64_t *p = part + (int64_t)kAccPart * b;
+    add192w(a, __ldcg(p), __ldcg(p + 1), __ldcg(p + 2));
+  }
 #pragma unroll
-    for (int d = 16; d; d >>= 1) {
-      const uint64_t o0 = __shfl_xor_sync(0xffffffffu, a[0], d), o1 = __shfl_xor_sync(0xffffffffu, a[1], d),
-                     o2 = __shfl_xor_sync(0xffffffffu, a[2], d);
-      add192w(a, o0, o1, o2);
-    }
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    __syncthreads();
-    if (lane == 0) {
-      red[3 * wid] = a[0];
-      red[3 * wid + 1] = a[1];
-      red[3 * wid + 2] = a[2];
-    }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      for (int v = 1; v < kSelBlock / 32; ++v) add192w(a, red[3 * v], red[3 * v + 1], red[3 * v + 2]);
-      const uint64_t wv[4] = {a[0], a[1], a[2], 0ull};
-      sums[7] = rsum ? ldexp(int256_to_dd(wv, 0).hi, bemax - 1123) : __longlong_as_double((long long)relmax);
-    }
+  for (int d = 16; d; d >>= 1) {
+    const uint64_t o0 = __shfl_xor_sync(0xffffffffu, a[0], d), o1 = __shfl_xor_sync(0xffffffffu, a[1], d),
+                   o2 = __shfl_xor_sync(0xffffffffu, a[2], d);
+    add192w(a, o0, o1, o2);
+  }
+  __syncthreads();
+  if (lane == 0) {
+    red[3 * wid] = a[0];
+    red[3 * wid + 1] = a[1];
+    red[3 * wid + 2] = a[2];
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int v = 1; v < kSelBlock / 32; ++v) add192w(a, red[3 * v], red[3 * v + 1], red[3 * v + 2]);
+    const uint64_t wv[4] = {a[0], a[1], a[2], 0ull};
+    bool ok = true;
+    double sr = rsum ? acc_i256_to_double(wv, bemax - 1123, ok) : __longlong_as_double((long long)relmax);
+    if (!ok) sr = ldexp(int256_to_dd(wv, 0).hi, bemax - 1123);  // sums below 2^-1022 or above 2^1023
+    sums[7] = sr;
   }
   if (!digit) return;
-  const int wid = threadIdx.x >> 5;
+  __shared__ uint64_t npf[kAccTargets];
+  __shared__ int64_t nrk[kAccTargets];
+  __syncthreads();
+  for (int i = threadIdx.x; i < kSelBins; i += kSelBlock) h[i] = __ldcg(hist + i);  // the grid's histogram
+  __syncthreads();
+  if (wid < kAccTargets) {
+    int bin;
+    int64_t below, cnt;
+    const int64_t r = sel->rk[wid];
+    acc_scan_pick<false>(h, r, bin, below, cnt);
+    if (lane == 0) {
+      npf[wid] = (sel->pf[wid] << w) | (uint64_t)bin;
+      nrk[wid] = r - below;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x < kAccTargets) {
+    sel->pf[threadIdx.x] = npf[threadIdx.x];
+    sel->rk[threadIdx.x] = nrk[threadIdx.x];
+  }
+  if (threadIdx.x == 0) sel->shift = lo;
+  for (int i = threadIdx.x; i < kSelBins; i += kSelBlock) hist[i] = 0u;
+}
+
+// Select, second digit: a sample whose bits above `shift` equal a target's
+// prefix adds one, in global memory, to that prefix's histogram at its next
+// digit (few samples do: those in a first-digit bin that holds a target).
+// Prefixes of one length are equal or disjoint, so a sample counts at most
+// once; targets with the same prefix share a histogram.  The last block picks
+// each target's digit and lays out the candidate lists for the gather:
+// targets whose bins coincide share one, of that bin's count.
+__global__ void __launch_bounds__(kSelBlock) k_acc_selB(const uint64_t *__restrict__ relbits, int64_t n,
+                                                        SelState *__restrict__ sel, unsigned int *__restrict__ hist,
+                                                        unsigned int *ticket) {
+  __shared__ unsigned int h[kAccTargets * kSelBins];
+  __shared__ uint64_t npf[kAccTargets];
+  __shared__ int64_t nrk[kAccTargets], ncnt[kAccTargets];
+  const int shift = sel->shift;
+  if (shift <= 0) return;
+  const uint64_t pf0 = sel->pf[0], pf1 = sel->pf[1], pf2 = sel->pf[2];
+  const int w = min(kSelBits, shift), lo = shift - w;
+  const uint64_t dmask = (1ull << w) - 1;
+  auto visit = [&](uint64_t v) {
+    if (v == ~0ull) return;  // not a sample
+    const uint64_t key = v >> shift;
+    const int s = key == pf0 ? 0 : key == pf1 ? 1 : key == pf2 ? 2 : -1;
+    if (s >= 0) atomicAdd(hist + s * kSelBins + (int)((v >> lo) & dmask), 1u);
+  };
+  const int64_t n8 = n >> 3;
+  const int64_t g = blockIdx.x * (int64_t)kSelBlock + threadIdx.x, stride = (int64_t)gridDim.x * kSelBlock;
+  const ulonglong2 *r2 = reinterpret_cast<const ulonglong2 *>(relbits);
+  for (int64_t c = g; c < n8; c += stride) {
+    ulonglong2 q[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) q[k] = __ldcg(r2 + 4 * c + k);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      visit(q[k].x);
+      visit(q[k].y);
+    }
+  }
+  if (g < n - 8 * n8) visit(__ldcg(relbits + 8 * n8 + g));
+  if (!last_block(ticket)) return;
+  for (int i = threadIdx.x; i < kAccTargets * kSelBins; i += kSelBlock) h[i] = __ldcg(hist + i);
+  __syncthreads();
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   if (wid < kAccTargets) {
     const uint64_t pf = wid == 0 ? pf0 : wid == 1 ? pf1 : pf2;
     const int slot = pf == pf0 ? 0 : pf == pf1 ? 1 : 2;
-    acc_pick(hist + slot * kSelBins, sel, wid, pf, w);
+    const int64_t r = sel->rk[wid];
+    int bin;
+    int64_t below, cnt;
+    acc_scan_pick<false>(h + slot * kSelBins, r, bin, below, cnt);
+    if (lane == 0) {
+      npf[wid] = (pf << w) | (uint64_t)bin;
+      nrk[wid] = r - below;
+      ncnt[wid] = cnt;
+    }
   }
   __syncthreads();
+  if (threadIdx.x == 0) {
+    // candidate lists: targets whose bins coincide share one, of that bin's count
+    int sl[kAccTargets];
+    int64_t base = 0;
+    for (int t = 0; t < kAccTargets; ++t) {
+      sl[t] = t;
+      for (int u = t - 1; u >= 0; --u)
+        if (npf[u] == npf[t]) sl[t] = sl[u];
+      sel->pf[t] = npf[t];
+      sel->rk[t] = nrk[t];
+      sel->ccnt[t] = ncnt[t];
+      sel->slot[t] = sl[t];
+      if (sl[t] == t) {
+        sel->cbase[t] = base;
+        base += ncnt[t];
+      }
+    }
+    sel->shift = lo;
+  }
   for (int i = threadIdx.x; i < kAccTargets * kSelBins; i += kSelBlock) hist[i] = 0u;
-  if (threadIdx.x == 0) sel->shift = lo;
+}
+
+// Select, gather: each sample whose bits above `shift` equal a target's
+// prefix is appended to that prefix's candidate list (a sample joins at most
+// one list, and each list's length is its bin's count).  A block counts its
+// samples per list, reserves its ranges with one atomic per list, and writes
+// them; the order within a list does not matter.
+__global__ void __launch_bounds__(kSelBlock) k_acc_sel1(const uint64_t *__restrict__ relbits, int64_t n,
+                                                        SelState *__restrict__ sel, uint64_t *__restrict__ cand) {
+  __shared__ int wofs[kSelBlock / 32][kAccTargets];
+  __shared__ unsigned long long bbase[kAccTargets];
+  const int shift = sel->shift;
+  if (shift <= 0) return;
+  const uint64_t pf0 = sel->pf[0], pf1 = sel->pf[1], pf2 = sel->pf[2];
+  const int64_t base0 = sel->cbase[0], base1 = sel->cbase[1], base2 = sel->cbase[2];
+  const int64_t cnt0 = sel->ccnt[0], cnt1 = sel->ccnt[1], cnt2 = sel->ccnt[2];
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const int64_t nc = (n + 7) >> 3;  // chunks of eight patterns, the last one padded
+  for (int64_t cb = blockIdx.x * (int64_t)kSelBlock; cb < nc; cb += (int64_t)gridDim.x * kSelBlock) {
+    const int64_t c = cb + threadIdx.x;
+    uint64_t v[8];
+    const bool full = 8 * c + 8 <= n;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      ulonglong2 q;
+      if (full) {
+        q = __ldcg(reinterpret_cast<const ulonglong2 *>(relbits) + 4 * c + k);
+      } else {
+        const int64_t i = 8 * c + 2 * k;
+        q.x = i < n ? __ldcg(relbits + i) : ~0ull;
+        q.y = i + 1 < n ? __ldcg(relbits + i + 1) : ~0ull;
+      }
+      v[2 * k] = q.x;
+      v[2 * k + 1] = q.y;
+    }
+    uint32_t sl = 0;  // two bits per pattern: its list, 3 for none
+    int own[kAccTargets] = {0, 0, 0};
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      uint32_t s = 3u;
+      if (v[k] != ~0ull) {
+        const uint64_t key = v[k] >> shift;
+        s = key == pf0 ? 0u : key == pf1 ? 1u : key == pf2 ? 2u : 3u;
+      }
+      sl |= s << (2 * k);
+#pragma unroll
+      for (int j = 0; j < kAccTargets; ++j) own[j] += s == (uint32_t)j ? 1 : 0;
+    }
+    int before[kAccTargets];  // this thread's offset within its warp, per list
+#pragma unroll
+    for (int j = 0; j < kAccTargets; ++j) {
+      int inc = own[j];
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const int o = __shfl_up_sync(0xffffffffu, inc, d);
+        if (lane >= d) inc += o;
+      }
+      before[j] = inc - own[j];
+      if (lane == 31) wofs[wid][j] = inc;
+    }
+    __syncthreads();
+    if (threadIdx.x < kAccTargets) {
+      const int j = threadIdx.x;
+      int run = 0;
+      for (int u = 0; u < kSelBlock / 32; ++u) {
+        const int t = wofs[u][j];
+        wofs[u][j] = run;
+        run += t;
+      }
+      bbase[j] = run ? atomicAdd(&sel->ccur[j], (unsigned long long)run) : 0ull;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+#pragma unroll
+      for (int j = 0; j < kAccTargets; ++j)
+        if (((sl >> (2 * k)) & 3u) == (uint32_t)j) {
+          const int64_t pos = (int64_t)bbase[j] + wofs[wid][j] + before[j];
+          before[j] += 1;
+          const int64_t cj = j == 0 ? cnt0 : j == 1 ? cnt1 : cnt2, bj = j == 0 ? base0 : j == 1 ? base1 : base2;
+          if (pos < cj) cand[bj + pos] = v[k];
+        }
+    __syncthreads();
+  }
+}
+
+// Select, finish: one block per target finds its rank in its candidate list,
+// writes the percentile's bit pattern and resets its append cursor.  A list
+// of at most one pattern per thread is ranked directly; a longer one is
+// settled digit by digit (from the common prefix of its smallest and largest
+// pattern on, one shared-memory histogram per digit), from shared memory when
+// it fits there (kSelSmemList patterns), else from global memory.
+__global__ void __launch_bounds__(kSelFinish) k_acc_sel2(const uint64_t *__restrict__ cand,
+                                                         SelState *__restrict__ sel) {
+  extern __shared__ uint64_t lst[];  // kSelSmemList patterns (dynamic)
+  __shared__ unsigned int h[kSelBins];
+  __shared__ unsigned long long mm[2];
+  __shared__ int64_t pick[2];
+  const int t = blockIdx.x;
+  if (sel->shift <= 0) return;
+  const uint64_t *list = cand + sel->cbase[sel->slot[t]];
+  const int64_t c = sel->ccnt[t];
+  int64_t r = sel->rk[t];
+  if (c <= 0) return;  // cannot happen: a bin that holds a rank is not empty
+  if (c <= kSelFinish) {
+    // a short list: the candidate with fewer than r smaller ones and at least
+    // r not larger is the answer (every thread that finds it holds the same value)
+    if (threadIdx.x < c) lst[threadIdx.x] = __ldcg(list + threadIdx.x);
+    __syncthreads();
+    if (threadIdx.x < c) {
+      const uint64_t v = lst[threadIdx.x];
+      int64_t less = 0, leq = 0;
+      for (int j = 0; j < (int)c; ++j) {
+        const uint64_t u = lst[j];
+        less += u < v ? 1 : 0;
+        leq += u <= v ? 1 : 0;
+      }
+      if (less < r && r <= leq) sel->pf[t] = v;
+    }
+    if (threadIdx.x == 0) sel->ccur[t] = 0ull;
+    return;
+  }
+  const bool inshared = c <= kSelSmemList;
+  if (threadIdx.x == 0) {
+    mm[0] = 0ull;
+    mm[1] = 0ull;
+  }
+  unsigned long long mx = 0ull, nmn = 0ull;
+  for (int64_t i = threadIdx.x; i < c; i += kSelFinish) {
+    const unsigned long long v = __ldcg(list + i);
+    if (inshared) lst[i] = v;
+    mx = max(mx, v);
+    nmn = max(nmn, ~v);
+  }
+#pragma unroll
+  for (int d = 16; d; d >>= 1) {
+    mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, d));
+    nmn = max(nmn, __shfl_xor_sync(0xffffffffu, nmn, d));
+  }
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) {
+    atomicMax(&mm[0], mx);
+    atomicMax(&mm[1], nmn);
+  }
+  __syncthreads();
+  const uint64_t hi = mm[0], lo0 = ~(uint64_t)mm[1];
+  int cur = hi == lo0 ? 0 : 64 - __clzll((long long)(hi ^ lo0));
+  uint64_t prefix = cur == 0 ? hi : hi >> cur;
+  while (cur > 0) {
+    const int w = min(kSelBits, cur), lo = cur - w;
+    const uint64_t dmask = (1ull << w) - 1;
+    for (int i = threadIdx.x; i < kSelBins; i += kSelFinish) h[i] = 0u;
+    __syncthreads();
+    for (int64_t i = threadIdx.x; i < c; i += kSelFinish) {
+      const uint64_t v = inshared ? lst[i] : __ldcg(list + i);
+      if ((v >> cur) == prefix) atomicAdd(&h[(int)((v >> lo) & dmask)], 1u);
+    }
+    __syncthreads();
+    if (threadIdx.x < 32) {
+      int bin;
+      int64_t below, cnt;
+      acc_scan_pick<false>(h, r, bin, below, cnt);
+      if (threadIdx.x == 0) {
+        pick[0] = bin;
+        pick[1] = below;
+      }
+    }
+    __syncthreads();
+    r -= pick[1];
+    prefix = (prefix << w) | (uint64_t)pick[0];
+    cur = lo;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    sel->pf[t] = prefix;
+    sel->ccur[t] = 0ull;
+  }
 }
 
 // ---------------------------------------------------------------- token-count baseline

@@ -209,3 +209,19 @@ def test_accuracy_paths(lv, ctx, case):
     _check_accuracy(g, o)
     again = lv.lv_accuracy(ctx, _dev(y), _dev(T))  # repeats bit for bit (NaN where NaN)
     assert all(again[k] == g[k] or (np.isnan(again[k]) and np.isnan(g[k])) for k in g)
+
+
+@pytest.mark.parametrize("n", [4_000, 30_000, 200_000])
+def test_accuracy_select_list_sizes(lv, ctx, n):
+    """Relative errors in two clusters: 70% in [0.5, 0.5 + 2^-14), the rest in
+    [0.52, 0.53).  Every sample shares the sign, exponent and top mantissa
+    bits, so the first select digit puts the first cluster into four bins of
+    about n / 6 each, and p50 (inside the first cluster) is settled from a
+    candidate list that is short (n = 4k, ranked directly), mid-sized (30k,
+    held in shared memory) or long (200k, read from global memory)."""
+    rng = np.random.default_rng(n)
+    y = rng.uniform(0.5, 2.0, n)
+    first = rng.random(n) < 0.7
+    rel = np.where(first, 0.5 + rng.uniform(0.0, 2.0 ** -14, n), rng.uniform(0.52, 0.53, n))
+    T = y * (1.0 + rel)
+    _check_accuracy(lv.lv_accuracy(ctx, _dev(y), _dev(T)), oracle.accuracy(y, T))
