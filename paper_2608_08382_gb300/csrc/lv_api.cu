@@ -46,7 +46,7 @@ struct lv_ctx {
   size_t wi_cap = 0;
   void *d_acc = nullptr;      // accuracy metrics: relative-error bits, partials, histograms
   size_t acc_cap = 0;
-  int acc_occ[5] = {0, 0, 0, 0, 0};  // CTAs per SM: range, exact, sel0, selB, sel1 (0: not yet queried)
+  int acc_occ = 0;            // CTAs per SM of the accuracy kernel (0: not yet queried)
   int timing = 0;  // LV_TIME_* mask
   std::vector<cudaEvent_t> tev;  // start/stop pairs
   size_t tev_used = 0;
@@ -1028,37 +1028,27 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   rep->r2_ssr = rep->r2_corr = rep->mean_rel = rep->p50 = rep->p90 = rep->p99 = nan;
   if (n == 0) return LV_OK;
   cudaStream_t stream = (cudaStream_t)stream_;
-  if (ctx->acc_occ[0] == 0) {
-    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ[0], k_acc_range, kAccBlock, 0));
-    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ[1], k_acc_exact, kAccBlock, 0));
-    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ[2], k_acc_sel0, kSelBlock, 0));
-    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ[3], k_acc_selB, kSelBlock, 0));
-    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ[4], k_acc_sel1, kSelBlock, 0));
-    LV_CUDA(cudaFuncSetAttribute(k_acc_sel2, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)(kSelSmemList * sizeof(uint64_t))));
+  if (ctx->acc_occ == 0) {
+    LV_CUDA(cudaFuncSetAttribute(k_acc, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 (int)cudaSharedmemCarveoutMaxShared));
+    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ, k_acc, kAccBlock, 0));
+    if (ctx->acc_occ <= 0) return LV_ECUDA;
   }
-  // every pass is one wave (at most the blocks that fit at once), looping over
-  // its share; the select passes take eight patterns per thread and step
-  const auto wave = [&](int k, int64_t want) {
-    return (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)ctx->sms * std::max(ctx->acc_occ[k], 1)));
-  };
-  const int64_t want = (n + kAccBlock - 1) / kAccBlock, swant = (n + 8 * kSelBlock - 1) / (8 * kSelBlock);
-  const int rblocks = wave(0, want), xblocks = wave(1, want), fblocks = (int)std::min<int64_t>(want, ctx->sms * 4);
-  const int sblocks0 = wave(2, swant), sblocksB = wave(3, swant), sblocks1 = wave(4, swant);
-  const int sblocks = std::max(sblocks0, std::max(sblocksB, sblocks1));
-  // a fixed head (tickets, path, sums, select state, the digit histograms: zeroed once at allocation, and every call leaves the tickets,
-  // cursors and histograms at zero), then the
-  // relative errors' bit patterns, the candidate lists and the block partials
-  constexpr size_t o_range = 32, o_sums = 64, o_sel = 128, o_hist = 512, o_rel = 32768;
-  static_assert(sizeof(AccRange) <= o_sums - o_range && sizeof(SelState) <= o_hist - o_sel,
+  // a cooperative launch: at most the blocks that fit at once, each looping over its share
+  const int blocks = (int)std::max<int64_t>(
+      1, std::min<int64_t>((n + kAccBlock - 1) / kAccBlock, (int64_t)ctx->sms * ctx->acc_occ));
+  // a fixed head (barrier, list cursors, results, digit histograms: zeroed
+  // once at allocation, and every call leaves the barrier, cursors and
+  // histograms at zero), then the relative errors' bit patterns, the
+  // candidate lists and the block partials
+  constexpr size_t o_bar = 0, o_ccur = 64, o_out = 128, o_hist1 = 256, o_hist2 = o_hist1 + 8 * kSelBins,
+                   o_rel = 45056;
+  static_assert(o_ccur + 2 * kAccTargets * sizeof(unsigned long long) <= o_out &&
+                    o_out + 12 * sizeof(double) <= o_hist1 && o_hist2 + 4 * kAccTargets * kSelBins <= o_rel,
                 "accuracy scratch head");
-  static_assert(o_sel == o_sums + 8 * sizeof(double) && offsetof(SelState, pf) == 0,
-                "the prefixes follow the sums");
-  static_assert(o_hist + sizeof(unsigned int) * kAccTargets * kSelBins <= o_rel, "accuracy histograms");
   const size_t rel_bytes = ((size_t)n * sizeof(uint64_t) + 255) & ~(size_t)255;
-  const size_t o_cand = o_rel + rel_bytes, o_part = o_cand + rel_bytes;
-  const size_t need =
-      o_part + sizeof(uint64_t) * kAccPart * (size_t)std::max(std::max(rblocks, xblocks), std::max(fblocks, sblocks));
+  const size_t o_cand = o_rel + rel_bytes, o_cand2 = o_cand + rel_bytes, o_part = o_cand2 + rel_bytes;
+  const size_t need = o_part + sizeof(uint64_t) * kAccPartW * (size_t)blocks;
   if (need > ctx->acc_cap) {
     LV_CUDA(cudaDeviceSynchronize());
     if (ctx->d_acc) cudaFree(ctx->d_acc);
@@ -1069,38 +1059,33 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
     ctx->acc_cap = need;
   }
   unsigned char *base = static_cast<unsigned char *>(ctx->d_acc);
-  unsigned int *ticket = reinterpret_cast<unsigned int *>(base);  // range, exact, sums, moments, two digits
-  AccRange *rg = reinterpret_cast<AccRange *>(base + o_range);
-  double *sums = reinterpret_cast<double *>(base + o_sums);  // m, sum y, sum T, sxx, syy, sxy, ssr, sum rel
-  SelState *sel = reinterpret_cast<SelState *>(base + o_sel);
-  unsigned int *hist = reinterpret_cast<unsigned int *>(base + o_hist);
-  uint64_t *relbits = reinterpret_cast<uint64_t *>(base + o_rel);
-  uint64_t *cand = reinterpret_cast<uint64_t *>(base + o_cand);
-  uint64_t *part = reinterpret_cast<uint64_t *>(base + o_part);
-  k_acc_range<<<rblocks, kAccBlock, 0, stream>>>(y, T, n, rg, part, ticket);
-  LV_CUDA(cudaGetLastError());
-  // exactly one of the two paths does work; the other returns at once
-  k_acc_exact<<<xblocks, kAccBlock, 0, stream>>>(y, T, n, rg, relbits, part, sums, sel, ticket + 1);
-  LV_CUDA(cudaGetLastError());
-  double *dpart = reinterpret_cast<double *>(part);
-  k_acc_sums<<<fblocks, kAccBlock, 0, stream>>>(y, T, n, rg, relbits, dpart, sums, sel, ticket + 2);
-  LV_CUDA(cudaGetLastError());
-  k_acc_moments<<<fblocks, kAccBlock, 0, stream>>>(y, T, n, rg, sums, dpart, ticket + 3);
-  LV_CUDA(cudaGetLastError());
-  // exact nearest-rank percentiles (and the sum of rel): two digits over the
-  // samples, gather each target's remaining candidates, settle the rest per
-  // target
-  k_acc_sel0<<<sblocks0, kSelBlock, 0, stream>>>(relbits, n, sel, hist, part, sums, ticket + 4);
-  LV_CUDA(cudaGetLastError());
-  k_acc_selB<<<sblocksB, kSelBlock, 0, stream>>>(relbits, n, sel, hist, ticket + 5);
-  LV_CUDA(cudaGetLastError());
-  k_acc_sel1<<<sblocks1, kSelBlock, 0, stream>>>(relbits, n, sel, cand);
-  LV_CUDA(cudaGetLastError());
-  k_acc_sel2<<<kAccTargets, kSelFinish, kSelSmemList * sizeof(uint64_t), stream>>>(cand, sel);
-  LV_CUDA(cudaGetLastError());
-  double h[11];  // eight sums, then the three percentile bit patterns
-  LV_CUDA(cudaMemcpyAsync(h, sums, sizeof(h), cudaMemcpyDeviceToHost, stream));
+  AccArgs a;
+  a.y = y;
+  a.T = T;
+  a.n = n;
+  a.relbits = reinterpret_cast<uint64_t *>(base + o_rel);
+  a.cand = reinterpret_cast<uint64_t *>(base + o_cand);
+  a.cand2 = reinterpret_cast<uint64_t *>(base + o_cand2);
+  a.part = reinterpret_cast<uint64_t *>(base + o_part);
+  a.out = reinterpret_cast<double *>(base + o_out);
+  a.hist1 = reinterpret_cast<unsigned int *>(base + o_hist1);
+  a.hist2 = reinterpret_cast<unsigned int *>(base + o_hist2);
+  a.ccur = reinterpret_cast<unsigned long long *>(base + o_ccur);
+  a.bar = reinterpret_cast<unsigned int *>(base + o_bar);
+  void *args[] = {&a};
+  LV_CUDA(cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(k_acc), dim3(blocks), dim3(kAccBlock), args, 0,
+                                      stream));
+  double h[12];  // eight sums, the three percentile bit patterns, the barrier's error word
+  LV_CUDA(cudaMemcpyAsync(h, a.out, sizeof(h), cudaMemcpyDeviceToHost, stream));
   LV_CUDA(cudaStreamSynchronize(stream));
+  int err;
+  std::memcpy(&err, &h[11], sizeof(err));
+  if (err) {
+    // a block waited out the barrier: reset the barrier and the error word for the next call
+    LV_CUDA(cudaMemset(base + o_bar, 0, 8));
+    LV_CUDA(cudaMemset(base + o_out + 11 * sizeof(double), 0, sizeof(double)));
+    return LV_ETIMEOUT;
+  }
   const double m = h[0];
   rep->n = (int64_t)m;
   if (m == 0) return LV_OK;

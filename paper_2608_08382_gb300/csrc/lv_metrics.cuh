@@ -7,41 +7,36 @@
 //             double, as fp64 arithmetic gives them), its mean and its
 //             nearest-rank p50, p90, p99 (the ceil(q m / 100)-th smallest).
 //
-// GB300 issues fp64 at 1/64 of the fp32 rate, so the common case runs on the
-// integer pipes, exactly:
-//   k_acc_range    the largest and smallest binary exponents Emax, Emin among
-//                  the samples' y and non-zero T.  When Emax is finite and
-//                  moderate the exact path below is taken: on the grid
-//                  2^(Emax - 62) in 64-bit integers when Emax - Emin <= 10 (every
-//                  value then lies on it), else on 2^(Emax - 78) in 128-bit
-//                  integers, handing over to the fp64 path when a value turns
-//                  out not to lie on that grid.
-//   k_acc_exact    per sample the integers Y = y 2^S and T 2^S (below 2^63 or
-//                  2^79 in magnitude) and D = Y - T; the exact sums
-//                  of Y, T, Y^2, T^2 and D^2, from which
-//                    m sxx = m sum Y^2 - (sum Y)^2,   m syy = m sum T^2 - (sum T)^2,
-//                    2 m sxy = m (sum Y^2 + sum T^2 - sum D^2) - 2 sum Y sum T,
-//                    m ssr = m sum D^2
-//                  follow exactly (all on the grid 2^(-2S), which both R^2
-//                  cancel); and rel by exact integer division.
-//   k_acc_sums,    otherwise (a non-finite sample value, extreme magnitudes,
-//   k_acc_moments  or a value off the grid): the same quantities in fp64,
-//                  means first, then centred moments, each in a fixed order.
-//   k_acc_sel0,    the percentiles, exact: rel is a non-negative double, so
-//   k_acc_selB,    its bit pattern orders like its value, and a
-//   k_acc_sel1,    most-significant-digit radix select finds the bit pattern of
-//   k_acc_sel2     the element of each target rank.  The first digit (11 bits
-//                  below the prefix every sample shares) is histogrammed over
-//                  all samples, which also sums rel in fixed point anchored at
-//                  the largest rel (terms below 2^-100 of it truncated); the
-//                  next digit over the samples in a target's bin (typically
-//                  well under 1% of them); the samples in each target's
-//                  second-digit bin (typically a handful) are gathered into a
-//                  candidate list, and one block per target settles the
-//                  remaining digits on its list.
-// Blocks never wait on one another: each fold runs in the block that finishes
-// last (an atomic ticket, reset for the next launch), and every kernel of a
-// call runs back to back on the stream with no host round trip.
+// One cooperative kernel computes all of it; its phases are separated by a
+// grid-wide barrier, and after each barrier every block folds the small
+// per-block partials it needs itself (in a fixed order, so all blocks agree):
+//   range   the largest and smallest binary exponents Emax, Emin among the
+//           samples' y and non-zero T.  GB300 issues fp64 at 1/64 of the fp32
+//           rate, so when Emax is finite and moderate the sums are formed
+//           exactly on the integer pipes: on the grid 2^(Emax - 62) in 64-bit
+//           integers when Emax - Emin <= 10 (every value then lies on it), else
+//           on 2^(Emax - 78) in 128-bit integers.
+//   exact   per sample the integers Y = y 2^S and T 2^S and D = Y - T; the
+//           exact sums of Y, T, Y^2, T^2 and D^2, from which
+//             m sxx = m sum Y^2 - (sum Y)^2,   m syy = m sum T^2 - (sum T)^2,
+//             2 m sxy = m (sum Y^2 + sum T^2 - sum D^2) - 2 sum Y sum T,
+//             m ssr = m sum D^2
+//           follow exactly (all on the grid 2^(-2S), which both R^2 cancel);
+//           and rel by exact integer division.  A value off the wide grid
+//           sends the call to the fp64 phases.
+//   fp64    otherwise (a non-finite sample value, extreme magnitudes, a value
+//           off the grid): the same quantities in fp64, means first, then
+//           centred moments, each in a fixed order.
+//   select  the percentiles, exact: rel is a non-negative double, so its bit
+//           pattern orders like its value, and a most-significant-digit radix
+//           select finds the bit pattern of the element of each target rank.
+//           The first digit (the pattern's exponent and top mantissa bits) is
+//           histogrammed by the pass that forms rel; a second pass takes the
+//           next 11 bits of the samples in a target's first-digit bin
+//           (typically a small fraction) and copies those samples into a
+//           candidate list per target; one block per target then picks the
+//           second digit and finds the rank among the list's matching samples.
+//           The mean of rel is an fp64 sum in a fixed order.
 #pragma once
 
 #include <cstdint>
@@ -54,14 +49,11 @@ typedef unsigned __int128 u128;
 
 constexpr int kAccBlock = 256;
 constexpr int kAccTargets = 3;  // p50, p90, p99
-constexpr int kAccWords = 14;   // per-block partial of the exact sums
-constexpr int kAccPart = 16;    // words per block partial (any pass)
+constexpr int kAccWords = 14;   // the exact sums of one block
 constexpr int kSelBits = 11;    // radix digit
 constexpr int kSelBins = 1 << kSelBits;
-constexpr int kSelBlock = 512;
-constexpr int kSelFinish = 1024;     // threads of a finishing block (one per target)
-constexpr int kSelSmemList = 20480;  // candidates a finishing block holds in shared memory
-constexpr int kAccGrid = 78;  // S = kAccGrid - Emax puts every |v 2^S| below 2^79
+constexpr int kAccBuf = kSelBins / 2;  // a block's buffered candidates per list
+constexpr int kAccGrid = 78;  // wide grid: S = kAccGrid - Emax puts every |v 2^S| below 2^79
 // Range of Emax for the exact path: within it the definition's own fp64
 // arithmetic (squared deviations, their products in r2_corr) neither overflows
 // nor underflows for values on the grid, so the exact results are what fp64
@@ -69,31 +61,28 @@ constexpr int kAccGrid = 78;  // S = kAccGrid - Emax puts every |v 2^S| below 2^
 constexpr int kAccEmaxLo = -160, kAccEmaxHi = 224;
 constexpr uint64_t kFracMask = (1ull << 52) - 1, kHiddenBit = 1ull << 52;
 
-// Path of one call, rewritten by every call: set by the range pass, except
-// `inexact`, which the exact pass sets when a value is off its grid.
-struct AccRange {
-  int exact;    // the exact path applies
-  int narrow;   // ... on the 63-bit grid (every exponent within 10 of the largest)
-  int S;        // grid exponent: 62 - Emax (narrow) or 78 - Emax
-  int inexact;  // a value fell off the grid
-};
+// One block's partial, kAccPartW words: sample count, off-grid flag, rel sum
+// (fp64), the range maxima, the exact sums, the fp64 sums (count, sum y,
+// sum T) and the fp64 centred moments.
+constexpr int kAccPartW = 32;
+constexpr int kPC = 0, kPL = 1, kPQ = 2, kPR = 4, kPX = 8, kPS = 22, kPM = 25;
+static_assert(kPX + kAccWords <= kPS && kPS + 3 <= kPM && kPM + 4 <= kAccPartW, "partial layout");
 
-// Select state: the three prefixes first (they become the percentiles' bit
-// patterns and sit right after the eight sums, so one copy reads both).
-struct SelState {
-  uint64_t pf[kAccTargets];
-  int64_t rk[kAccTargets];  // rank still to find below each prefix
-  uint64_t relmax;          // largest rel (its bit pattern)
-  int shift;                // bits below the settled prefixes; 0 when done
-  int pad;
-  // candidate lists after the first digit: target t's samples sit in list
-  // slot[t] (targets with the same prefix share one), at cbase[slot] in the
-  // candidate buffer, ccnt[t] of them; ccur[] are the append cursors
-  int64_t cbase[kAccTargets];
-  int64_t ccnt[kAccTargets];
-  unsigned long long ccur[kAccTargets];
-  int slot[kAccTargets];
-  int pad2;
+// Device arguments of one call.  `out` holds the eight sums (m, -, -, sxx,
+// syy, sxy, ssr, sum rel), the three percentiles' bit patterns and the
+// barrier's error word, so one copy reads them all.
+struct AccArgs {
+  const double *y, *T;
+  int64_t n;
+  uint64_t *relbits;          // n rel bit patterns (all ones: not a sample)
+  uint64_t *cand;             // first-digit candidate lists, n patterns
+  uint64_t *cand2;            // final candidate lists, n patterns
+  uint64_t *part;             // kAccPartW words per block
+  double *out;                // 8 doubles, 3 patterns, error word
+  unsigned int *hist1;        // 2 * kSelBins: first digit, exact pass then fp64 pass
+  unsigned int *hist2;        // kAccTargets * kSelBins: the second digit
+  unsigned long long *ccur;   // 2 * kAccTargets list cursors (first-digit lists, final lists)
+  unsigned int *bar;          // grid barrier: arrivals, generation (zero between calls)
 };
 
 // y > 0 on the bit pattern: sign clear, not zero, not NaN (+inf counts).
@@ -101,20 +90,36 @@ __device__ __forceinline__ bool acc_is_sample(uint64_t b) {
   return (int64_t)b > 0 && b <= 0x7FF0000000000000ull;
 }
 
-// True in the block that finishes last (its partial and every other block's
-// are visible to it then).  The ticket is reset for the next launch; blocks
-// never wait on one another.
-__device__ __forceinline__ bool last_block(unsigned int *ticket) {
-  __shared__ bool last;
-  __threadfence();
+// Grid-wide barrier of a cooperative launch (every block resident).  Thread 0
+// of each block arrives on bar[0]; the last arrival resets it and advances
+// the generation bar[1]; the others wait for the generation to move, for at
+// most about a second, after which they set the error word and go on.
+// Returns false once the error word is set (every block then leaves).
+__device__ __forceinline__ bool grid_barrier(unsigned int *bar, int *err) {
+  __shared__ int ok;
   __syncthreads();
   if (threadIdx.x == 0) {
-    last = atomicAdd(ticket, 1u) == gridDim.x - 1;
-    if (last) *ticket = 0u;
+    volatile unsigned int *gen = bar + 1;
+    const unsigned int g = *gen;  // read before arriving: it cannot move until this block arrives
+    __threadfence();
+    if (atomicAdd(bar, 1u) == gridDim.x - 1) {
+      atomicExch(bar, 0u);
+      __threadfence();
+      atomicAdd(bar + 1, 1u);
+    } else {
+      for (long long k = 0; *gen == g; ++k) {
+        if (k > (1ll << 24)) {
+          atomicExch(err, 1);
+          break;
+        }
+        __nanosleep(32);
+      }
+    }
+    __threadfence();
+    ok = *(volatile int *)err == 0;
   }
   __syncthreads();
-  if (last) __threadfence();
-  return last;
+  return ok;
 }
 
 // Sum of `v` over the block in a fixed order (shuffle tree, then the warps in
@@ -155,73 +160,10 @@ __device__ __forceinline__ void block_max2(unsigned long long &a, unsigned long 
     }
 }
 
-// `k` interleaved doubles summed over `blocks` partials with the whole block:
-// thread j takes partials j, j + blockDim, ... in order, then the block sum in
-// its fixed order; out[0..k) is written by thread 0.
-__device__ __forceinline__ void fold_partials(const double *part, int blocks, int k, double *red, double *out) {
-  for (int c = 0; c < k; ++c) {
-    double s = 0.0;
-    for (int b = threadIdx.x; b < blocks; b += blockDim.x) s += __ldcg(part + (int64_t)b * kAccPart + c);
-    s = block_sum_fixed(s, red);
-    if (threadIdx.x == 0) out[c] = s;
-  }
-}
-
-// Largest magnitude (high word of the largest sample y or |T|) and smallest
-// exponent over the samples' y and non-zero T, and with them the path: exact
-// when the values are finite, n < 2^32 (the integer widths hold any count
-// below it) and Emax lies in [kAccEmaxLo, kAccEmaxHi]; narrow (64-bit
-// integers) when in addition every exponent is within 10 of Emax.  On the wide
-// grid the exact pass checks that every value lies on it.  (A NaN y counts
-// here, sending the call to the fp64 path, which leaves it out.)  Block maxima
-// go to the partials; the last block folds them.
-__global__ void __launch_bounds__(kAccBlock) k_acc_range(const double *__restrict__ y, const double *__restrict__ T,
-                                                         int64_t n, AccRange *__restrict__ rg,
-                                                         uint64_t *__restrict__ part, unsigned int *ticket) {
-  __shared__ unsigned long long red[kAccBlock / 32 * 2];
-  unsigned int top = 0u, nmin = 0u;  // nmin: max of 2047 - biased exponent
-  const int64_t stride = (int64_t)gridDim.x * kAccBlock;
-  for (int64_t i0 = blockIdx.x * (int64_t)kAccBlock + threadIdx.x; i0 < n; i0 += 4 * stride) {
-    uint2 yv[4], tv[4];  // four elements' loads in flight (a pattern of 0 is not a sample)
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int64_t i = i0 + k * stride;
-      yv[k] = i < n ? __ldg(reinterpret_cast<const uint2 *>(y) + i) : make_uint2(0u, 0u);
-      tv[k] = i < n ? __ldg(reinterpret_cast<const uint2 *>(T) + i) : make_uint2(0u, 0u);
-    }
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const unsigned int yh = yv[k].y, th = tv[k].y & 0x7FFFFFFFu;
-      if ((int)yh > 0 || (yh == 0u && yv[k].x != 0u)) {
-        top = max(top, max(yh, th));
-        nmin = max(nmin, 2047u - (yh >> 20));
-        if (th | tv[k].x) nmin = max(nmin, 2047u - (th >> 20));
-      }
-    }
-  }
-  unsigned long long a = top, b = nmin;
-  block_max2(a, b, red);
-  if (threadIdx.x == 0) {
-    part[(int64_t)kAccPart * blockIdx.x] = a;
-    part[(int64_t)kAccPart * blockIdx.x + 1] = b;
-  }
-  if (!last_block(ticket)) return;
-  a = 0ull;
-  b = 0ull;
-  for (int k = threadIdx.x; k < (int)gridDim.x; k += kAccBlock) {
-    a = max(a, (unsigned long long)__ldcg(part + (int64_t)kAccPart * k));
-    b = max(b, (unsigned long long)__ldcg(part + (int64_t)kAccPart * k + 1));
-  }
-  block_max2(a, b, red);
-  if (threadIdx.x == 0) {
-    const int E = (int)(a >> 20) - 1023;  // no sample: -1023, and nothing to sum
-    const int Emin = 2047 - (int)b - 1023;
-    const bool ex = a < 0x7FF00000ull && n < (int64_t)1 << 32 && (b == 0 || (E >= kAccEmaxLo && E <= kAccEmaxHi));
-    rg->exact = ex;
-    rg->narrow = ex && E - Emin <= 10;
-    rg->S = (E - Emin <= 10 ? 62 : kAccGrid) - E;
-    rg->inexact = 0;
-  }
+// Largest rel and largest ~rel (so zero is the identity of both).
+__device__ __forceinline__ void acc_note_rel(uint64_t rb, unsigned long long &rmax, unsigned long long &rnmax) {
+  rmax = max(rmax, (unsigned long long)rb);
+  rnmax = max(rnmax, (unsigned long long)~rb);
 }
 
 // ---------------------------------------------------------------- exact path
@@ -470,6 +412,8 @@ __device__ __forceinline__ uint64_t acc_exact_sample64(uint64_t yb, uint64_t tb,
   return acc_rel_bits64(Dm, My, ky);
 }
 
+// ---------------------------------------------------------------- wide integers
+
 // 64 x 192 -> 256-bit product.
 __device__ __forceinline__ void mul64x192(uint64_t m, const uint64_t *b, uint64_t *w) {
   w[0] = w[1] = w[2] = w[3] = 0;
@@ -535,238 +479,8 @@ __device__ __forceinline__ double acc_i256_to_double(const uint64_t *wi, int e2,
   return __longlong_as_double((long long)(((uint64_t)neg << 63) | ((uint64_t)(ex + 1023) << 52) | (mant & kFracMask)));
 }
 
-// Select state for a new call: the prefix every sample shares (the common
-// leading bits of the smallest and largest rel, lo and hi) and the target
-// ranks ceil(q m / 100), q = 50, 90, 99.
-__device__ __forceinline__ void acc_publish_select(uint64_t hi, uint64_t lo, SelState *sel, int64_t m) {
-  sel->relmax = hi;
-  const int cp = m == 0 || hi == lo ? 64 : __clzll((long long)(hi ^ lo));
-  sel->shift = m == 0 ? 0 : 64 - cp;
-  const uint64_t pf = cp == 64 ? hi : hi >> (64 - cp);
-  for (int t = 0; t < kAccTargets; ++t) {
-    const int64_t q = t == 0 ? 50 : t == 1 ? 90 : 99;
-    sel->pf[t] = pf;
-    sel->rk[t] = (q * m + 99) / 100;
-  }
-}
 
-// Largest rel and largest ~rel (so zero is the identity of both).
-__device__ __forceinline__ void acc_note_rel(uint64_t rb, unsigned long long &rmax, unsigned long long &rnmax) {
-  rmax = max(rmax, (unsigned long long)rb);
-  rnmax = max(rnmax, (unsigned long long)~rb);
-}
-
-template <bool kNarrow>
-__device__ __forceinline__ void acc_exact_loop(const double *__restrict__ y, const double *__restrict__ T, int64_t n,
-                                               int S, uint64_t *__restrict__ relbits, uint64_t *w,
-                                               unsigned long long &rmax, unsigned long long &rnmax, bool &lost) {
-  const int64_t stride = (int64_t)gridDim.x * kAccBlock;
-  for (int64_t i0 = blockIdx.x * (int64_t)kAccBlock + threadIdx.x; i0 < n; i0 += 2 * stride) {
-    uint64_t yb[2], tb[2];  // two elements' loads in flight (a pattern of 0 is not a sample)
-#pragma unroll
-    for (int k = 0; k < 2; ++k) {
-      const int64_t i = i0 + k * stride;
-      yb[k] = i < n ? (uint64_t)__double_as_longlong(__ldg(y + i)) : 0ull;
-      tb[k] = i < n ? (uint64_t)__double_as_longlong(__ldg(T + i)) : 0ull;
-    }
-#pragma unroll
-    for (int k = 0; k < 2; ++k) {
-      const int64_t i = i0 + k * stride;
-      uint64_t rb = ~0ull;  // not a sample
-      if (acc_is_sample(yb[k])) {
-        rb = kNarrow ? acc_exact_sample64(yb[k], tb[k], S, w) : acc_exact_sample(yb[k], tb[k], S, w, lost);
-        acc_note_rel(rb, rmax, rnmax);
-      }
-      if (i < n) relbits[i] = rb;
-    }
-  }
-}
-
-// Exact path: the sums and every rel in one pass over y and T; the last block
-// folds the block partials and writes sums[0] = m and, scaled by m 2^(2S),
-// sums[3..6] = sxx, syy, sxy, ssr.  Returns at once when the range pass chose
-// the fp64 path; flags rg->inexact (and the fp64 path then redoes the call)
-// when a value is not on the grid.
-__global__ void __launch_bounds__(kAccBlock) k_acc_exact(const double *__restrict__ y, const double *__restrict__ T,
-                                                         int64_t n, AccRange *__restrict__ rg,
-                                                         uint64_t *__restrict__ relbits, uint64_t *__restrict__ part,
-                                                         double *__restrict__ sums, SelState *__restrict__ sel,
-                                                         unsigned int *ticket) {
-  __shared__ uint64_t red[kAccBlock / 32 * kAccWords];
-  __shared__ unsigned long long red2[kAccBlock / 32 * 2];
-  if (!rg->exact) return;
-  const int S = rg->S;
-  uint64_t w[kAccWords];
-#pragma unroll
-  for (int j = 0; j < kAccWords; ++j) w[j] = 0ull;
-  unsigned long long rmax = 0ull, rnmax = 0ull;
-  bool lost = false;
-  if (rg->narrow)
-    acc_exact_loop<true>(y, T, n, S, relbits, w, rmax, rnmax, lost);
-  else
-    acc_exact_loop<false>(y, T, n, S, relbits, w, rmax, rnmax, lost);
-  if (__syncthreads_or(lost) && threadIdx.x == 0) atomicOr(&rg->inexact, 1);
-  block_max2(rmax, rnmax, red2);
-  acc_block_combine(w, red);
-  if (threadIdx.x == 0) {
-    uint64_t *p = part + (int64_t)blockIdx.x * kAccPart;
-#pragma unroll
-    for (int j = 0; j < kAccWords; ++j) p[j] = w[j];
-    p[kAccWords] = rmax;
-    p[kAccWords + 1] = rnmax;
-  }
-  if (!last_block(ticket)) return;
-#pragma unroll
-  for (int j = 0; j < kAccWords; ++j) w[j] = 0ull;
-  rmax = rnmax = 0ull;
-  for (int b = threadIdx.x; b < (int)gridDim.x; b += kAccBlock) {
-    const uint64_t *p = part + (int64_t)b * kAccPart;
-    uint64_t o[kAccWords];
-#pragma unroll
-    for (int j = 0; j < kAccWords; ++j) o[j] = __ldcg(p + j);
-    acc_combine(w, o);
-    rmax = max(rmax, (unsigned long long)__ldcg(p + kAccWords));
-    rnmax = max(rnmax, (unsigned long long)__ldcg(p + kAccWords + 1));
-  }
-  block_max2(rmax, rnmax, red2);
-  acc_block_combine(w, red);
-  if (threadIdx.x != 0) return;
-  const uint64_t m = w[0];
-  // |sum T| and its sign
-  const bool tneg = (int64_t)w[4] < 0;
-  const u128 st = ((u128)w[4] << 64) | w[3], sa = tneg ? (u128)0 - st : st;
-  const uint64_t s0 = (uint64_t)sa, s1 = (uint64_t)(sa >> 64);
-  uint64_t sxx[4], syy[4], sxy[4], ssr[4], tmp[4];
-  mul64x192(m, w + 5, sxx);
-  mul128x128(w[1], w[2], w[1], w[2], tmp);
-  sub256(sxx, tmp);
-  mul64x192(m, w + 8, syy);
-  mul128x128(s0, s1, s0, s1, tmp);
-  sub256(syy, tmp);
-  // 2 m sxy = m (sum Y^2 + sum T^2 - sum D^2) - 2 sum Y sum T; the 192-bit
-  // bracket may be negative (two's complement), hence the split below
-  uint64_t g[3] = {w[5], w[6], w[7]};
-  add192w(g, w[8], w[9], w[10]);
-  add192w(g, ~w[11], ~w[12], ~w[13]);
-  add192w(g, 1, 0, 0);
-  const bool gneg = (int64_t)g[2] < 0;
-  if (gneg) {
-    g[0] = ~g[0];
-    g[1] = ~g[1];
-    g[2] = ~g[2];
-    add192w(g, 1, 0, 0);
-  }
-  mul64x192(m, g, sxy);
-  if (gneg) {
-    uint64_t z[4] = {0, 0, 0, 0};
-    sub256(z, sxy);
-    sxy[0] = z[0];
-    sxy[1] = z[1];
-    sxy[2] = z[2];
-    sxy[3] = z[3];
-  }
-  mul128x128(w[1], w[2], s0, s1, tmp);
-  acc_add256(tmp, tmp[0], tmp[1], tmp[2], tmp[3]);  // 2 sum Y |sum T|
-  if (tneg)
-    acc_add256(sxy, tmp[0], tmp[1], tmp[2], tmp[3]);
-  else
-    sub256(sxy, tmp);
-  mul64x192(m, w + 11, ssr);
-  bool ok = true;  // every value here is below 2^227 in magnitude
-  sums[0] = (double)m;
-  sums[3] = acc_i256_to_double(sxx, 0, ok);
-  sums[4] = acc_i256_to_double(syy, 0, ok);
-  sums[5] = acc_i256_to_double(sxy, -1, ok);
-  sums[6] = acc_i256_to_double(ssr, 0, ok);
-  acc_publish_select(rmax, ~(uint64_t)rnmax, sel, (int64_t)m);
-}
-
-// ---------------------------------------------------------------- fp64 path
-
-// Pass 1: per-block count, sum y, sum T over the samples; rel's bit patterns
-// stored (all ones for a batch that is not a sample, which the select never
-// counts).  The last block folds the partials into sums[0..2] and sets up the
-// select.  Returns at once when the exact path did the call.
-__global__ void __launch_bounds__(kAccBlock) k_acc_sums(const double *__restrict__ y, const double *__restrict__ T,
-                                                        int64_t n, const AccRange *__restrict__ rg,
-                                                        uint64_t *__restrict__ relbits, double *__restrict__ part,
-                                                        double *__restrict__ sums, SelState *__restrict__ sel,
-                                                        unsigned int *ticket) {
-  __shared__ double red[kAccBlock / 32];
-  __shared__ unsigned long long red2[kAccBlock / 32 * 2];
-  if (rg->exact && !rg->inexact) return;
-  double c = 0.0, sy = 0.0, st = 0.0;
-  unsigned long long rmax = 0ull, rnmax = 0ull;
-  const int64_t stride = (int64_t)gridDim.x * kAccBlock;
-  for (int64_t i = blockIdx.x * (int64_t)kAccBlock + threadIdx.x; i < n; i += stride) {
-    const double yv = y[i], tv = T[i];
-    uint64_t bits = ~0ull;
-    if (yv > 0.0) {
-      c += 1.0;
-      sy += yv;
-      st += tv;
-      bits = (uint64_t)__double_as_longlong(__ddiv_rn(fabs(__dsub_rn(tv, yv)), yv));
-      acc_note_rel(bits, rmax, rnmax);
-    }
-    relbits[i] = bits;
-  }
-  block_max2(rmax, rnmax, red2);
-  const double a = block_sum_fixed(c, red), b = block_sum_fixed(sy, red), d = block_sum_fixed(st, red);
-  if (threadIdx.x == 0) {
-    double *p = part + (int64_t)kAccPart * blockIdx.x;
-    p[0] = a;
-    p[1] = b;
-    p[2] = d;
-    p[3] = __longlong_as_double((long long)rmax);  // bit patterns, folded as integers
-    p[4] = __longlong_as_double((long long)rnmax);
-  }
-  if (!last_block(ticket)) return;
-  fold_partials(part, gridDim.x, 3, red, sums);
-  rmax = rnmax = 0ull;
-  for (int k = threadIdx.x; k < (int)gridDim.x; k += kAccBlock) {
-    const double *p = part + (int64_t)kAccPart * k;
-    rmax = max(rmax, (unsigned long long)__double_as_longlong(__ldcg(p + 3)));
-    rnmax = max(rnmax, (unsigned long long)__double_as_longlong(__ldcg(p + 4)));
-  }
-  block_max2(rmax, rnmax, red2);
-  if (threadIdx.x == 0) acc_publish_select(rmax, ~(uint64_t)rnmax, sel, (int64_t)sums[0]);
-}
-
-// Pass 2: centred moments with the means from pass 1 (sums = {count, sum y,
-// sum T}); the last block folds them into sums[3..6] = sxx, syy, sxy, ssr.
-__global__ void __launch_bounds__(kAccBlock) k_acc_moments(const double *__restrict__ y, const double *__restrict__ T,
-                                                           int64_t n, const AccRange *__restrict__ rg,
-                                                           double *__restrict__ sums, double *__restrict__ part,
-                                                           unsigned int *ticket) {
-  __shared__ double red[kAccBlock / 32];
-  if (rg->exact && !rg->inexact) return;
-  const double m = sums[0];
-  const double my = m > 0 ? sums[1] / m : 0.0, mt = m > 0 ? sums[2] / m : 0.0;
-  double sxx = 0.0, syy = 0.0, sxy = 0.0, ssr = 0.0;
-  const int64_t stride = (int64_t)gridDim.x * kAccBlock;
-  for (int64_t i = blockIdx.x * (int64_t)kAccBlock + threadIdx.x; i < n; i += stride) {
-    const double yv = y[i], tv = T[i];
-    if (yv > 0.0) {
-      const double dy = yv - my, dt = tv - mt, e = yv - tv;
-      sxx += dy * dy;
-      syy += dt * dt;
-      sxy += dy * dt;
-      ssr += e * e;
-    }
-  }
-  const double v0 = block_sum_fixed(sxx, red), v1 = block_sum_fixed(syy, red), v2 = block_sum_fixed(sxy, red),
-               v3 = block_sum_fixed(ssr, red);
-  if (threadIdx.x == 0) {
-    double *p = part + (int64_t)kAccPart * blockIdx.x;
-    p[0] = v0;
-    p[1] = v1;
-    p[2] = v2;
-    p[3] = v3;
-  }
-  if (last_block(ticket)) fold_partials(part, gridDim.x, 4, red, sums + 3);
-}
-
-// ---------------------------------------------------------------- percentiles
+// ---------------------------------------------------------------- select helpers
 
 // rel (bit pattern v, finite, non-negative) on the grid 2^(bemax - 1123),
 // bemax the largest rel's biased exponent: below 2^101, truncated under the
@@ -823,368 +537,160 @@ __device__ __forceinline__ void acc_scan_pick(const unsigned int *h, int64_t r, 
   cnt = __shfl_sync(0xffffffffu, (int64_t)(first ? pr.x : pr.y), L2);
 }
 
-// Select, first digit: every sample adds one to the histogram of its first
-// digit below the shared prefix (all samples share it, so no compare), and
-// its rel to the fixed-point sum.  The last block writes sums[7] (the largest
-// rel itself when that is inf or NaN, which is what an exact sum gives then),
-// picks each target's digit, and lays out the candidate lists: targets in the
-// same bin share one.  With no digit left (every rel equal) the prefixes are
-// already the answers.
-__global__ void __launch_bounds__(kSelBlock) k_acc_sel0(const uint64_t *__restrict__ relbits, int64_t n,
-                                                        SelState *__restrict__ sel, unsigned int *__restrict__ hist,
-                                                        uint64_t *__restrict__ part, double *__restrict__ sums,
-                                                        unsigned int *ticket) {
-  __shared__ unsigned int h[kSelBins];
-  __shared__ uint64_t red[kSelBlock / 32 * 3];
-  const int shift = sel->shift;
-  const uint64_t relmax = sel->relmax;
-  const bool digit = shift > 0;
-  const bool rsum = relmax < 0x7FF0000000000000ull;
-  const int w = min(kSelBits, shift), lo = shift - w;
-  const uint64_t dmask = (1ull << w) - 1;
-  for (int i = threadIdx.x; i < kSelBins; i += kSelBlock) h[i] = 0u;
-  __syncthreads();
-  const int bemax = max((int)(relmax >> 52), 1);
-  uint64_t acc[3] = {0, 0, 0};  // sum of rel on its grid, 192 bits
-  auto visit = [&](uint64_t v) {
-    if (v == ~0ull) return;  // not a sample
-    if (digit) atomicAdd(&h[(int)((v >> lo) & dmask)], 1u);
-    if (rsum) {
-      const u128 x = acc_rel_fixed(v, bemax);
-      add192w(acc, (uint64_t)x, (uint64_t)(x >> 64), 0);
+
+// ---------------------------------------------------------------- phases
+
+// First select digit: the top 12 + kbits bits of rel's pattern (exponent and
+// kbits mantissa bits).  On the exact paths rel is 0 or lies in [2^elo,
+// 2^(elo + octaves)), so the digit is offset to start there, with bin 0 for
+// rel = 0; on the fp64 path it is the exponent field itself (bin 0 holds 0
+// and the subnormals, bin 2047 inf and NaN).
+struct AccKey {
+  int kbits;  // mantissa bits in the digit
+  int elo;    // lowest exponent of a non-zero rel (exact paths)
+  int exact;  // offset layout with a zero bin
+};
+
+__device__ __forceinline__ int acc_key1(uint64_t rb, const AccKey &K) {
+  if (!K.exact) return (int)(rb >> 52);
+  if (rb == 0) return 0;
+  const int64_t k = (int64_t)(rb >> (52 - K.kbits)) - ((int64_t)(1023 + K.elo) << K.kbits) + 1;
+  return (int)min(max(k, (int64_t)1), (int64_t)kSelBins - 1);  // within range by construction
+}
+
+// Block-local view of the select, identical in every block (each derives it
+// from the same global data in the same order).
+struct AccSel {
+  uint64_t pf[kAccTargets];   // prefix after the first digit; ~0 once a target is settled at 0
+  int64_t rk[kAccTargets];    // rank still to find below it
+  int64_t cnt[kAccTargets];   // samples in its first-digit bin (its list's length)
+  int64_t base[kAccTargets];  // list offset of its slot
+  int slot[kAccTargets];      // list shared by targets whose prefixes coincide
+  int shift;                  // bits below the first digit
+  int64_t m;                  // samples
+};
+
+// Exact pass over this block's share of y and T on the narrow or wide grid:
+// the sums into w, rel's patterns into relbits, rel's first digit into the
+// block histogram h1 and rel into srel (fp64, in the thread's fixed order);
+// `lost` when a value is off the wide grid.
+template <bool kNarrow>
+__device__ __forceinline__ void acc_exact_loop(const double *__restrict__ y, const double *__restrict__ T, int64_t n,
+                                               int S, uint64_t *__restrict__ relbits, uint64_t *w, unsigned int *h1,
+                                               const AccKey &K, double &srel, bool &lost) {
+  const int64_t stride = (int64_t)gridDim.x * kAccBlock;
+  for (int64_t i0 = blockIdx.x * (int64_t)kAccBlock + threadIdx.x; i0 < n; i0 += 2 * stride) {
+    uint64_t yb[2], tb[2];  // two elements' loads in flight (a pattern of 0 is not a sample)
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const int64_t i = i0 + k * stride;
+      yb[k] = i < n ? (uint64_t)__double_as_longlong(__ldg(y + i)) : 0ull;
+      tb[k] = i < n ? (uint64_t)__double_as_longlong(__ldg(T + i)) : 0ull;
     }
-  };
-  // eight consecutive patterns per thread (four 16-byte loads in flight), then the tail
-  const int64_t n8 = n >> 3;
-  const int64_t g = blockIdx.x * (int64_t)kSelBlock + threadIdx.x, stride = (int64_t)gridDim.x * kSelBlock;
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const int64_t i = i0 + k * stride;
+      uint64_t rb = ~0ull;  // not a sample
+      if (acc_is_sample(yb[k])) {
+        rb = kNarrow ? acc_exact_sample64(yb[k], tb[k], S, w) : acc_exact_sample(yb[k], tb[k], S, w, lost);
+        atomicAdd(&h1[acc_key1(rb, K)], 1u);
+        srel += __longlong_as_double((long long)rb);
+      }
+      if (i < n) relbits[i] = rb;
+    }
+  }
+}
+
+// Visit this block's share of the rel patterns in warp tiles of 256 (load k
+// of a warp reads 512 contiguous bytes; four loads in flight), then the tail.
+// Every lane of a warp runs the same number of iterations and visits, so the
+// visitor may use warp collectives.
+template <class F>
+__device__ __forceinline__ void acc_for_rel(const uint64_t *__restrict__ relbits, int64_t n, F &&visit) {
+  const int lane = threadIdx.x & 31;
+  const int64_t tiles = n >> 8, gw = blockIdx.x * (int64_t)(kAccBlock / 32) + (threadIdx.x >> 5);
+  const int64_t wstride = (int64_t)gridDim.x * (kAccBlock / 32);
   const ulonglong2 *r2 = reinterpret_cast<const ulonglong2 *>(relbits);
-  for (int64_t c = g; c < n8; c += stride) {
+  for (int64_t t = gw; t < tiles; t += wstride) {
     ulonglong2 q[4];
 #pragma unroll
-    for (int k = 0; k < 4; ++k) q[k] = __ldcg(r2 + 4 * c + k);
+    for (int k = 0; k < 4; ++k) q[k] = __ldcg(r2 + 128 * t + 32 * k + lane);
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
       visit(q[k].x);
       visit(q[k].y);
     }
   }
-  if (g < n - 8 * n8) visit(__ldcg(relbits + 8 * n8 + g));
-  __syncthreads();
-  if (digit)
-    for (int i = threadIdx.x; i < kSelBins; i += kSelBlock) {
-      const unsigned int c = h[i];
-      if (c) atomicAdd(hist + i, c);
-    }
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-#pragma unroll
-  for (int d = 16; d; d >>= 1) {
-    const uint64_t o0 = __shfl_xor_sync(0xffffffffu, acc[0], d), o1 = __shfl_xor_sync(0xffffffffu, acc[1], d),
-                   o2 = __shfl_xor_sync(0xffffffffu, acc[2], d);
-    add192w(acc, o0, o1, o2);
-  }
-  if (lane == 0) {
-    red[3 * wid] = acc[0];
-    red[3 * wid + 1] = acc[1];
-    red[3 * wid + 2] = acc[2];
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    for (int v = 1; v < kSelBlock / 32; ++v) add192w(acc, red[3 * v], red[3 * v + 1], red[3 * v + 2]);
-    uint64_t *p = part + (int64_t)kAccPart * blockIdx.x;
-    p[0] = acc[0];
-    p[1] = acc[1];
-    p[2] = acc[2];
-  }
-  if (!last_block(ticket)) return;
-  uint64_t a[3] = {0, 0, 0};
-  for (int b = threadIdx.x; b < (int)gridDim.x; b += kSelBlock) {
-    const uint64_t *p = part + (int64_t)kAccPart * b;
-    add192w(a, __ldcg(p), __ldcg(p + 1), __ldcg(p + 2));
-  }
-#pragma unroll
-  for (int d = 16; d; d >>= 1) {
-    const uint64_t o0 = __shfl_xor_sync(0xffffffffu, a[0], d), o1 = __shfl_xor_sync(0xffffffffu, a[1], d),
-                   o2 = __shfl_xor_sync(0xffffffffu, a[2], d);
-    add192w(a, o0, o1, o2);
-  }
-  __syncthreads();
-  if (lane == 0) {
-    red[3 * wid] = a[0];
-    red[3 * wid + 1] = a[1];
-    red[3 * wid + 2] = a[2];
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    for (int v = 1; v < kSelBlock / 32; ++v) add192w(a, red[3 * v], red[3 * v + 1], red[3 * v + 2]);
-    const uint64_t wv[4] = {a[0], a[1], a[2], 0ull};
-    bool ok = true;
-    double sr = rsum ? acc_i256_to_double(wv, bemax - 1123, ok) : __longlong_as_double((long long)relmax);
-    if (!ok) sr = ldexp(int256_to_dd(wv, 0).hi, bemax - 1123);  // sums below 2^-1022 or above 2^1023
-    sums[7] = sr;
-  }
-  if (!digit) return;
-  __shared__ uint64_t npf[kAccTargets];
-  __shared__ int64_t nrk[kAccTargets];
-  __syncthreads();
-  for (int i = threadIdx.x; i < kSelBins; i += kSelBlock) h[i] = __ldcg(hist + i);  // the grid's histogram
-  __syncthreads();
-  if (wid < kAccTargets) {
-    int bin;
-    int64_t below, cnt;
-    const int64_t r = sel->rk[wid];
-    acc_scan_pick<false>(h, r, bin, below, cnt);
-    if (lane == 0) {
-      npf[wid] = (sel->pf[wid] << w) | (uint64_t)bin;
-      nrk[wid] = r - below;
-    }
-  }
-  __syncthreads();
-  if (threadIdx.x < kAccTargets) {
-    sel->pf[threadIdx.x] = npf[threadIdx.x];
-    sel->rk[threadIdx.x] = nrk[threadIdx.x];
-  }
-  if (threadIdx.x == 0) sel->shift = lo;
-  for (int i = threadIdx.x; i < kSelBins; i += kSelBlock) hist[i] = 0u;
+  // the tail (fewer than 256): the first warp of each block takes a slice
+  const int64_t rest = n - 256 * tiles;
+  if (threadIdx.x < 32)
+    for (int64_t i = blockIdx.x * 32; i < rest; i += (int64_t)gridDim.x * 32)
+      visit(i + lane < rest ? __ldcg(relbits + 256 * tiles + i + lane) : ~0ull);
 }
 
-// Select, second digit: a sample whose bits above `shift` equal a target's
-// prefix adds one, in global memory, to that prefix's histogram at its next
-// digit (few samples do: those in a first-digit bin that holds a target).
-// Prefixes of one length are equal or disjoint, so a sample counts at most
-// once; targets with the same prefix share a histogram.  The last block picks
-// each target's digit and lays out the candidate lists for the gather:
-// targets whose bins coincide share one, of that bin's count.
-__global__ void __launch_bounds__(kSelBlock) k_acc_selB(const uint64_t *__restrict__ relbits, int64_t n,
-                                                        SelState *__restrict__ sel, unsigned int *__restrict__ hist,
-                                                        unsigned int *ticket) {
-  __shared__ unsigned int h[kAccTargets * kSelBins];
-  __shared__ uint64_t npf[kAccTargets];
-  __shared__ int64_t nrk[kAccTargets], ncnt[kAccTargets];
-  const int shift = sel->shift;
-  if (shift <= 0) return;
-  const uint64_t pf0 = sel->pf[0], pf1 = sel->pf[1], pf2 = sel->pf[2];
-  const int w = min(kSelBits, shift), lo = shift - w;
-  const uint64_t dmask = (1ull << w) - 1;
-  auto visit = [&](uint64_t v) {
-    if (v == ~0ull) return;  // not a sample
-    const uint64_t key = v >> shift;
-    const int s = key == pf0 ? 0 : key == pf1 ? 1 : key == pf2 ? 2 : -1;
-    if (s >= 0) atomicAdd(hist + s * kSelBins + (int)((v >> lo) & dmask), 1u);
-  };
-  const int64_t n8 = n >> 3;
-  const int64_t g = blockIdx.x * (int64_t)kSelBlock + threadIdx.x, stride = (int64_t)gridDim.x * kSelBlock;
-  const ulonglong2 *r2 = reinterpret_cast<const ulonglong2 *>(relbits);
-  for (int64_t c = g; c < n8; c += stride) {
-    ulonglong2 q[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k) q[k] = __ldcg(r2 + 4 * c + k);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      visit(q[k].x);
-      visit(q[k].y);
-    }
-  }
-  if (g < n - 8 * n8) visit(__ldcg(relbits + 8 * n8 + g));
-  if (!last_block(ticket)) return;
-  for (int i = threadIdx.x; i < kAccTargets * kSelBins; i += kSelBlock) h[i] = __ldcg(hist + i);
-  __syncthreads();
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  if (wid < kAccTargets) {
-    const uint64_t pf = wid == 0 ? pf0 : wid == 1 ? pf1 : pf2;
-    const int slot = pf == pf0 ? 0 : pf == pf1 ? 1 : 2;
-    const int64_t r = sel->rk[wid];
-    int bin;
-    int64_t below, cnt;
-    acc_scan_pick<false>(h + slot * kSelBins, r, bin, below, cnt);
-    if (lane == 0) {
-      npf[wid] = (pf << w) | (uint64_t)bin;
-      nrk[wid] = r - below;
-      ncnt[wid] = cnt;
-    }
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    // candidate lists: targets whose bins coincide share one, of that bin's count
-    int sl[kAccTargets];
-    int64_t base = 0;
-    for (int t = 0; t < kAccTargets; ++t) {
-      sl[t] = t;
-      for (int u = t - 1; u >= 0; --u)
-        if (npf[u] == npf[t]) sl[t] = sl[u];
-      sel->pf[t] = npf[t];
-      sel->rk[t] = nrk[t];
-      sel->ccnt[t] = ncnt[t];
-      sel->slot[t] = sl[t];
-      if (sl[t] == t) {
-        sel->cbase[t] = base;
-        base += ncnt[t];
-      }
-    }
-    sel->shift = lo;
-  }
-  for (int i = threadIdx.x; i < kAccTargets * kSelBins; i += kSelBlock) hist[i] = 0u;
+// Pick the digit of a histogram in shared memory (kSelBins bins) that holds
+// rank r: bin, count below it, its count.  One warp; valid in every lane.
+__device__ __forceinline__ void acc_pick1(const unsigned int *h, int64_t r, int &bin, int64_t &below, int64_t &cnt) {
+  acc_scan_pick<false>(h, r, bin, below, cnt);
 }
 
-// Select, gather: each sample whose bits above `shift` equal a target's
-// prefix is appended to that prefix's candidate list (a sample joins at most
-// one list, and each list's length is its bin's count).  A block counts its
-// samples per list, reserves its ranges with one atomic per list, and writes
-// them; the order within a list does not matter.
-__global__ void __launch_bounds__(kSelBlock) k_acc_sel1(const uint64_t *__restrict__ relbits, int64_t n,
-                                                        SelState *__restrict__ sel, uint64_t *__restrict__ cand) {
-  __shared__ int wofs[kSelBlock / 32][kAccTargets];
-  __shared__ unsigned long long bbase[kAccTargets];
-  const int shift = sel->shift;
-  if (shift <= 0) return;
-  const uint64_t pf0 = sel->pf[0], pf1 = sel->pf[1], pf2 = sel->pf[2];
-  const int64_t base0 = sel->cbase[0], base1 = sel->cbase[1], base2 = sel->cbase[2];
-  const int64_t cnt0 = sel->ccnt[0], cnt1 = sel->ccnt[1], cnt2 = sel->ccnt[2];
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  const int64_t nc = (n + 7) >> 3;  // chunks of eight patterns, the last one padded
-  for (int64_t cb = blockIdx.x * (int64_t)kSelBlock; cb < nc; cb += (int64_t)gridDim.x * kSelBlock) {
-    const int64_t c = cb + threadIdx.x;
-    uint64_t v[8];
-    const bool full = 8 * c + 8 <= n;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      ulonglong2 q;
-      if (full) {
-        q = __ldcg(reinterpret_cast<const ulonglong2 *>(relbits) + 4 * c + k);
-      } else {
-        const int64_t i = 8 * c + 2 * k;
-        q.x = i < n ? __ldcg(relbits + i) : ~0ull;
-        q.y = i + 1 < n ? __ldcg(relbits + i + 1) : ~0ull;
-      }
-      v[2 * k] = q.x;
-      v[2 * k + 1] = q.y;
-    }
-    uint32_t sl = 0;  // two bits per pattern: its list, 3 for none
-    int own[kAccTargets] = {0, 0, 0};
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      uint32_t s = 3u;
-      if (v[k] != ~0ull) {
-        const uint64_t key = v[k] >> shift;
-        s = key == pf0 ? 0u : key == pf1 ? 1u : key == pf2 ? 2u : 3u;
-      }
-      sl |= s << (2 * k);
-#pragma unroll
-      for (int j = 0; j < kAccTargets; ++j) own[j] += s == (uint32_t)j ? 1 : 0;
-    }
-    int before[kAccTargets];  // this thread's offset within its warp, per list
-#pragma unroll
-    for (int j = 0; j < kAccTargets; ++j) {
-      int inc = own[j];
-#pragma unroll
-      for (int d = 1; d < 32; d <<= 1) {
-        const int o = __shfl_up_sync(0xffffffffu, inc, d);
-        if (lane >= d) inc += o;
-      }
-      before[j] = inc - own[j];
-      if (lane == 31) wofs[wid][j] = inc;
-    }
-    __syncthreads();
-    if (threadIdx.x < kAccTargets) {
-      const int j = threadIdx.x;
-      int run = 0;
-      for (int u = 0; u < kSelBlock / 32; ++u) {
-        const int t = wofs[u][j];
-        wofs[u][j] = run;
-        run += t;
-      }
-      bbase[j] = run ? atomicAdd(&sel->ccur[j], (unsigned long long)run) : 0ull;
-    }
-    __syncthreads();
-#pragma unroll
-    for (int k = 0; k < 8; ++k)
-#pragma unroll
-      for (int j = 0; j < kAccTargets; ++j)
-        if (((sl >> (2 * k)) & 3u) == (uint32_t)j) {
-          const int64_t pos = (int64_t)bbase[j] + wofs[wid][j] + before[j];
-          before[j] += 1;
-          const int64_t cj = j == 0 ? cnt0 : j == 1 ? cnt1 : cnt2, bj = j == 0 ? base0 : j == 1 ? base1 : base2;
-          if (pos < cj) cand[bj + pos] = v[k];
-        }
-    __syncthreads();
-  }
-}
-
-// Select, finish: one block per target finds its rank in its candidate list,
-// writes the percentile's bit pattern and resets its append cursor.  A list
-// of at most one pattern per thread is ranked directly; a longer one is
-// settled digit by digit (from the common prefix of its smallest and largest
-// pattern on, one shared-memory histogram per digit), from shared memory when
-// it fits there (kSelSmemList patterns), else from global memory.
-__global__ void __launch_bounds__(kSelFinish) k_acc_sel2(const uint64_t *__restrict__ cand,
-                                                         SelState *__restrict__ sel) {
-  extern __shared__ uint64_t lst[];  // kSelSmemList patterns (dynamic)
-  __shared__ unsigned int h[kSelBins];
-  __shared__ unsigned long long mm[2];
+// The r-th smallest (1-based) of the samples in `list` (c patterns) whose
+// bits above `cur` equal `prefix`, by one block.  When they number at most
+// kShort they are gathered into shared memory (`sh`) and ranked directly:
+// the candidate with fewer than r smaller ones and at least r not larger;
+// otherwise the remaining digits are settled from global memory, with `sh`
+// as the digit histogram.
+__device__ uint64_t acc_finish(const uint64_t *__restrict__ list, int64_t c, uint64_t prefix, int cur, int64_t r,
+                               int64_t want, unsigned int *sh) {
+  __shared__ uint64_t res;
+  __shared__ int nsel;
   __shared__ int64_t pick[2];
-  const int t = blockIdx.x;
-  if (sel->shift <= 0) return;
-  const uint64_t *list = cand + sel->cbase[sel->slot[t]];
-  const int64_t c = sel->ccnt[t];
-  int64_t r = sel->rk[t];
-  if (c <= 0) return;  // cannot happen: a bin that holds a rank is not empty
-  if (c <= kSelFinish) {
-    // a short list: the candidate with fewer than r smaller ones and at least
-    // r not larger is the answer (every thread that finds it holds the same value)
-    if (threadIdx.x < c) lst[threadIdx.x] = __ldcg(list + threadIdx.x);
+  constexpr int kShort = kAccTargets * kSelBins / 2;
+  if (want <= kShort) {
+    uint64_t *ls = reinterpret_cast<uint64_t *>(sh);
+    if (threadIdx.x == 0) {
+      nsel = 0;
+      res = 0ull;
+    }
     __syncthreads();
-    if (threadIdx.x < c) {
-      const uint64_t v = lst[threadIdx.x];
+    for (int64_t i = threadIdx.x; i < c; i += kAccBlock) {
+      const uint64_t v = __ldcg(list + i);
+      if ((v >> cur) == prefix) {
+        const int p = atomicAdd(&nsel, 1);
+        if (p < kShort) ls[p] = v;
+      }
+    }
+    __syncthreads();
+    const int k = min(nsel, kShort);
+    for (int i = threadIdx.x; i < k; i += kAccBlock) {
+      const uint64_t v = ls[i];
       int64_t less = 0, leq = 0;
-      for (int j = 0; j < (int)c; ++j) {
-        const uint64_t u = lst[j];
+      for (int j = 0; j < k; ++j) {
+        const uint64_t u = ls[j];
         less += u < v ? 1 : 0;
         leq += u <= v ? 1 : 0;
       }
-      if (less < r && r <= leq) sel->pf[t] = v;
+      if (less < r && r <= leq) res = v;  // every finder holds the same value
     }
-    if (threadIdx.x == 0) sel->ccur[t] = 0ull;
-    return;
+    __syncthreads();
+    const uint64_t out = res;
+    __syncthreads();
+    return out;
   }
-  const bool inshared = c <= kSelSmemList;
-  if (threadIdx.x == 0) {
-    mm[0] = 0ull;
-    mm[1] = 0ull;
-  }
-  unsigned long long mx = 0ull, nmn = 0ull;
-  for (int64_t i = threadIdx.x; i < c; i += kSelFinish) {
-    const unsigned long long v = __ldcg(list + i);
-    if (inshared) lst[i] = v;
-    mx = max(mx, v);
-    nmn = max(nmn, ~v);
-  }
-#pragma unroll
-  for (int d = 16; d; d >>= 1) {
-    mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, d));
-    nmn = max(nmn, __shfl_xor_sync(0xffffffffu, nmn, d));
-  }
-  __syncthreads();
-  if ((threadIdx.x & 31) == 0) {
-    atomicMax(&mm[0], mx);
-    atomicMax(&mm[1], nmn);
-  }
-  __syncthreads();
-  const uint64_t hi = mm[0], lo0 = ~(uint64_t)mm[1];
-  int cur = hi == lo0 ? 0 : 64 - __clzll((long long)(hi ^ lo0));
-  uint64_t prefix = cur == 0 ? hi : hi >> cur;
   while (cur > 0) {
     const int w = min(kSelBits, cur), lo = cur - w;
     const uint64_t dmask = (1ull << w) - 1;
-    for (int i = threadIdx.x; i < kSelBins; i += kSelFinish) h[i] = 0u;
+    for (int i = threadIdx.x; i < kSelBins; i += kAccBlock) sh[i] = 0u;
     __syncthreads();
-    for (int64_t i = threadIdx.x; i < c; i += kSelFinish) {
-      const uint64_t v = inshared ? lst[i] : __ldcg(list + i);
-      if ((v >> cur) == prefix) atomicAdd(&h[(int)((v >> lo) & dmask)], 1u);
+    for (int64_t i = threadIdx.x; i < c; i += kAccBlock) {
+      const uint64_t v = __ldcg(list + i);
+      if ((v >> cur) == prefix) atomicAdd(&sh[(int)((v >> lo) & dmask)], 1u);
     }
     __syncthreads();
     if (threadIdx.x < 32) {
       int bin;
       int64_t below, cnt;
-      acc_scan_pick<false>(h, r, bin, below, cnt);
+      acc_scan_pick<false>(sh, r, bin, below, cnt);
       if (threadIdx.x == 0) {
         pick[0] = bin;
         pick[1] = below;
@@ -1196,9 +702,464 @@ __global__ void __launch_bounds__(kSelFinish) k_acc_sel2(const uint64_t *__restr
     cur = lo;
     __syncthreads();
   }
-  if (threadIdx.x == 0) {
-    sel->pf[t] = prefix;
-    sel->ccur[t] = 0ull;
+  return prefix;
+}
+
+// Sum of a double over the block's partials word `off` of every block, in a
+// fixed order (thread j takes blocks j, j + blockDim, ...; then the block
+// sum); valid in thread 0.
+__device__ __forceinline__ double acc_fold_double(const uint64_t *part, int off, double *redd) {
+  double s = 0.0;
+  for (int b = threadIdx.x; b < (int)gridDim.x; b += kAccBlock)
+    s += __longlong_as_double((long long)__ldcg(part + (int64_t)b * kAccPartW + off));
+  return block_sum_fixed(s, redd);
+}
+
+// Exact totals to sums: fold the blocks' exact partials and write out[0] = m
+// and, scaled by m 2^(2S), out[3..6] = sxx, syy, sxy, ssr.  One block.
+__device__ __forceinline__ void acc_exact_totals(const AccArgs &a, uint64_t *redw) {
+  uint64_t w[kAccWords];
+#pragma unroll
+  for (int j = 0; j < kAccWords; ++j) w[j] = 0ull;
+  for (int b = threadIdx.x; b < (int)gridDim.x; b += kAccBlock) {
+    const uint64_t *p = a.part + (int64_t)b * kAccPartW + kPX;
+    uint64_t o[kAccWords];
+#pragma unroll
+    for (int j = 0; j < kAccWords; ++j) o[j] = __ldcg(p + j);
+    acc_combine(w, o);
+  }
+  acc_block_combine(w, redw);
+  if (threadIdx.x != 0) return;
+  const uint64_t m = w[0];
+  // |sum T| and its sign
+  const bool tneg = (int64_t)w[4] < 0;
+  const u128 st = ((u128)w[4] << 64) | w[3], sa = tneg ? (u128)0 - st : st;
+  const uint64_t s0 = (uint64_t)sa, s1 = (uint64_t)(sa >> 64);
+  uint64_t sxx[4], syy[4], sxy[4], ssr[4], tmp[4];
+  mul64x192(m, w + 5, sxx);
+  mul128x128(w[1], w[2], w[1], w[2], tmp);
+  sub256(sxx, tmp);
+  mul64x192(m, w + 8, syy);
+  mul128x128(s0, s1, s0, s1, tmp);
+  sub256(syy, tmp);
+  // 2 m sxy = m (sum Y^2 + sum T^2 - sum D^2) - 2 sum Y sum T; the 192-bit
+  // bracket may be negative (two's complement), hence the split below
+  uint64_t g[3] = {w[5], w[6], w[7]};
+  add192w(g, w[8], w[9], w[10]);
+  add192w(g, ~w[11], ~w[12], ~w[13]);
+  add192w(g, 1, 0, 0);
+  const bool gneg = (int64_t)g[2] < 0;
+  if (gneg) {
+    g[0] = ~g[0];
+    g[1] = ~g[1];
+    g[2] = ~g[2];
+    add192w(g, 1, 0, 0);
+  }
+  mul64x192(m, g, sxy);
+  if (gneg) {
+    uint64_t z[4] = {0, 0, 0, 0};
+    sub256(z, sxy);
+    sxy[0] = z[0];
+    sxy[1] = z[1];
+    sxy[2] = z[2];
+    sxy[3] = z[3];
+  }
+  mul128x128(w[1], w[2], s0, s1, tmp);
+  acc_add256(tmp, tmp[0], tmp[1], tmp[2], tmp[3]);  // 2 sum Y |sum T|
+  if (tneg)
+    acc_add256(sxy, tmp[0], tmp[1], tmp[2], tmp[3]);
+  else
+    sub256(sxy, tmp);
+  mul64x192(m, w + 11, ssr);
+  bool ok = true;  // every value here is below 2^227 in magnitude
+  a.out[0] = (double)m;
+  a.out[3] = acc_i256_to_double(sxx, 0, ok);
+  a.out[4] = acc_i256_to_double(syy, 0, ok);
+  a.out[5] = acc_i256_to_double(sxy, -1, ok);
+  a.out[6] = acc_i256_to_double(ssr, 0, ok);
+}
+
+// The whole accuracy computation of one call; a cooperative launch of at
+// most as many blocks as fit at once.
+__global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
+  __shared__ __align__(16) unsigned int sh[kAccTargets * kSelBins];  // per-phase scratch
+  __shared__ unsigned long long red2[kAccBlock / 32 * 2];
+  __shared__ double redd[kAccBlock / 32];
+  __shared__ uint64_t redw[kAccBlock / 32 * kAccWords];
+  __shared__ AccSel L, F;  // after the first digit; after the second
+  __shared__ AccKey K;
+  __shared__ int bcnt[kAccTargets];
+  __shared__ unsigned long long bbase[kAccTargets];
+  __shared__ int path[3];  // exact, narrow, S
+  __shared__ double mean[2];
+  int *err = reinterpret_cast<int *>(a.out + 11);
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, nb = gridDim.x;
+  const int64_t n = a.n, stride = (int64_t)nb * kAccBlock, g0 = blockIdx.x * (int64_t)kAccBlock + tid;
+  uint64_t *mine = a.part + (int64_t)blockIdx.x * kAccPartW;
+  const uint64_t *all = a.part;
+
+  // ---- range: the largest magnitude (high word of the largest sample y or
+  // |T|) and smallest exponent over the samples' y and non-zero T.  (A NaN y
+  // counts here, sending the call to the fp64 phases, which leave it out.)
+  // The histograms and list cursors of the previous call are cleared here.
+  for (int64_t i = g0; i < 2 * kSelBins; i += stride) a.hist1[i] = 0u;
+  for (int64_t i = g0; i < kAccTargets * kSelBins; i += stride) a.hist2[i] = 0u;
+  if (g0 < 2 * kAccTargets) a.ccur[g0] = 0ull;
+  {
+    unsigned int top = 0u, nmin = 0u;  // nmin: max of 2047 - biased exponent
+    for (int64_t i0 = g0; i0 < n; i0 += 4 * stride) {
+      uint2 yv[4], tv[4];  // four elements' loads in flight (a pattern of 0 is not a sample)
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int64_t i = i0 + k * stride;
+        yv[k] = i < n ? __ldg(reinterpret_cast<const uint2 *>(a.y) + i) : make_uint2(0u, 0u);
+        tv[k] = i < n ? __ldg(reinterpret_cast<const uint2 *>(a.T) + i) : make_uint2(0u, 0u);
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const unsigned int yh = yv[k].y, th = tv[k].y & 0x7FFFFFFFu;
+        if ((int)yh > 0 || (yh == 0u && yv[k].x != 0u)) {
+          top = max(top, max(yh, th));
+          nmin = max(nmin, 2047u - (yh >> 20));
+          if (th | tv[k].x) nmin = max(nmin, 2047u - (th >> 20));
+        }
+      }
+    }
+    unsigned long long x = top, z = nmin;
+    block_max2(x, z, red2);
+    if (tid == 0) {
+      mine[kPR] = x;
+      mine[kPR + 1] = z;
+    }
+  }
+  if (!grid_barrier(a.bar, err)) return;
+  // the path: exact when the values are finite, n < 2^32 (the integer widths
+  // hold any count below it) and Emax is in [kAccEmaxLo, kAccEmaxHi]; narrow
+  // (64-bit integers) when every exponent is within 10 of Emax
+  {
+    unsigned long long x = 0ull, z = 0ull;
+    for (int b = tid; b < nb; b += kAccBlock) {
+      x = max(x, (unsigned long long)__ldcg(all + (int64_t)b * kAccPartW + kPR));
+      z = max(z, (unsigned long long)__ldcg(all + (int64_t)b * kAccPartW + kPR + 1));
+    }
+    block_max2(x, z, red2);
+    if (tid == 0) {
+      const int E = (int)(x >> 20) - 1023, Emin = 2047 - (int)z - 1023;  // no sample: nothing to sum
+      const bool ex = x < 0x7FF00000ull && n < ((int64_t)1 << 32) && (z == 0 || (E >= kAccEmaxLo && E <= kAccEmaxHi));
+      path[0] = ex;
+      path[1] = ex && E - Emin <= 10;
+      path[2] = (E - Emin <= 10 ? 62 : kAccGrid) - E;
+      // rel's exponents on the exact paths: [-63, 12] on the narrow grid
+      // (|D| < 2^64 and y >= 2^52 grid units, a non-zero |D| at least one),
+      // [-79, 80] on the wide one (|D| < 2^80, y at least one unit, below 2^79)
+      K.exact = 1;
+      K.kbits = path[1] ? 4 : 3;
+      K.elo = path[1] ? -63 : -79;
+    }
+    for (int i = tid; i < kSelBins; i += kAccBlock) sh[i] = 0u;
+    __syncthreads();
+  }
+
+  // ---- exact: sums, rel and its first digit on the grid
+  bool fp64 = path[0] == 0;
+  if (!fp64) {
+    uint64_t w[kAccWords];
+#pragma unroll
+    for (int j = 0; j < kAccWords; ++j) w[j] = 0ull;
+    double srel = 0.0;
+    bool lost = false;
+    if (path[1])
+      acc_exact_loop<true>(a.y, a.T, n, path[2], a.relbits, w, sh, K, srel, lost);
+    else
+      acc_exact_loop<false>(a.y, a.T, n, path[2], a.relbits, w, sh, K, srel, lost);
+    const int anylost = __syncthreads_or(lost);
+    for (int i = tid; i < kSelBins; i += kAccBlock) {
+      const unsigned int c = sh[i];
+      if (c) atomicAdd(a.hist1 + i, c);
+    }
+    srel = block_sum_fixed(srel, redd);
+    acc_block_combine(w, redw);
+    if (tid == 0) {
+      mine[kPC] = w[0];
+      mine[kPL] = (uint64_t)anylost;
+      mine[kPQ] = (uint64_t)__double_as_longlong(srel);
+#pragma unroll
+      for (int j = 0; j < kAccWords; ++j) mine[kPX + j] = w[j];
+    }
+    if (!grid_barrier(a.bar, err)) return;
+    int off = 0;
+    for (int b = tid; b < nb; b += kAccBlock) off |= (int)__ldcg(all + (int64_t)b * kAccPartW + kPL);
+    fp64 = __syncthreads_or(off) != 0;  // a value off the wide grid: redo the call in fp64
+  }
+
+  // ---- fp64: rel and its first digit, means, then centred moments, each in
+  // a fixed order
+  if (fp64) {
+    if (tid == 0) {
+      K.exact = 0;
+      K.kbits = 0;
+      K.elo = 0;
+    }
+    for (int i = tid; i < kSelBins; i += kAccBlock) sh[i] = 0u;
+    __syncthreads();
+    double c = 0.0, sy = 0.0, st = 0.0, srel = 0.0;
+    uint64_t cnt = 0;
+    for (int64_t i = g0; i < n; i += stride) {
+      const double yv = a.y[i], tv = a.T[i];
+      uint64_t bits = ~0ull;
+      if (yv > 0.0) {
+        c += 1.0;
+        ++cnt;
+        sy += yv;
+        st += tv;
+        bits = (uint64_t)__double_as_longlong(__ddiv_rn(fabs(__dsub_rn(tv, yv)), yv));
+        atomicAdd(&sh[(int)(bits >> 52)], 1u);
+        srel += __longlong_as_double((long long)bits);
+      }
+      a.relbits[i] = bits;
+    }
+    __syncthreads();
+    for (int i = tid; i < kSelBins; i += kAccBlock) {
+      const unsigned int h = sh[i];
+      if (h) atomicAdd(a.hist1 + kSelBins + i, h);
+    }
+    const double A = block_sum_fixed(c, redd), B = block_sum_fixed(sy, redd), C = block_sum_fixed(st, redd);
+    srel = block_sum_fixed(srel, redd);
+#pragma unroll
+    for (int d = 16; d; d >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, d);
+    __syncthreads();
+    if (lane == 0) redw[wid] = cnt;
+    __syncthreads();
+    if (tid == 0) {
+      uint64_t tc = 0;
+      for (int v = 0; v < kAccBlock / 32; ++v) tc += redw[v];
+      double *p = reinterpret_cast<double *>(mine);
+      mine[kPC] = tc;
+      mine[kPQ] = (uint64_t)__double_as_longlong(srel);
+      p[kPS] = A;
+      p[kPS + 1] = B;
+      p[kPS + 2] = C;
+    }
+    if (!grid_barrier(a.bar, err)) return;
+    const double s0 = acc_fold_double(all, kPS, redd), s1 = acc_fold_double(all, kPS + 1, redd),
+                 s2 = acc_fold_double(all, kPS + 2, redd);
+    if (tid == 0) {
+      mean[0] = s0 > 0 ? s1 / s0 : 0.0;
+      mean[1] = s0 > 0 ? s2 / s0 : 0.0;
+    }
+    __syncthreads();
+    const double my = mean[0], mt = mean[1];
+    double sxx = 0.0, syy = 0.0, sxy = 0.0, ssr = 0.0;
+    for (int64_t i = g0; i < n; i += stride) {
+      const double yv = a.y[i], tv = a.T[i];
+      if (yv > 0.0) {
+        const double dy = yv - my, dt = tv - mt, e = yv - tv;
+        sxx += dy * dy;
+        syy += dt * dt;
+        sxy += dy * dt;
+        ssr += e * e;
+      }
+    }
+    const double v0 = block_sum_fixed(sxx, redd), v1 = block_sum_fixed(syy, redd), v2 = block_sum_fixed(sxy, redd),
+                 v3 = block_sum_fixed(ssr, redd);
+    if (tid == 0) {
+      double *p = reinterpret_cast<double *>(mine);
+      p[kPM] = v0;
+      p[kPM + 1] = v1;
+      p[kPM + 2] = v2;
+      p[kPM + 3] = v3;
+    }
+    if (!grid_barrier(a.bar, err)) return;
+  }
+
+  // ---- first digit: sample count, then each target's bin (every block)
+  {
+    unsigned long long cnt = 0ull;
+    for (int b = tid; b < nb; b += kAccBlock) cnt += __ldcg(all + (int64_t)b * kAccPartW + kPC);
+#pragma unroll
+    for (int d = 16; d; d >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, d);
+    const unsigned int *h1 = a.hist1 + (fp64 ? kSelBins : 0);
+    for (int i = tid; i < kSelBins; i += kAccBlock) sh[i] = __ldcg(h1 + i);
+    __syncthreads();
+    if (lane == 0) redw[wid] = cnt;
+    __syncthreads();
+    if (tid == 0) {
+      int64_t m = 0;
+      for (int v = 0; v < kAccBlock / 32; ++v) m += (int64_t)redw[v];
+      L.m = m;
+      L.shift = 52 - K.kbits;
+      for (int t = 0; t < kAccTargets; ++t) {
+        const int64_t q = t == 0 ? 50 : t == 1 ? 90 : 99;
+        L.rk[t] = (q * m + 99) / 100;
+      }
+    }
+    __syncthreads();
+    int bin = 0;
+    int64_t below = 0, c1 = 0;
+    if (wid < kAccTargets && L.m > 0) acc_pick1(sh, L.rk[wid], bin, below, c1);
+    if (wid < kAccTargets && lane == 0) {
+      if (L.m == 0 || (K.exact && bin == 0)) {
+        L.pf[wid] = ~0ull;  // settled: rel = 0 (or no sample)
+        L.cnt[wid] = 0;
+      } else {
+        L.pf[wid] = K.exact ? (uint64_t)(bin - 1) + ((uint64_t)(1023 + K.elo) << K.kbits) : (uint64_t)bin;
+        L.rk[wid] -= below;
+        L.cnt[wid] = c1;
+      }
+    }
+    __syncthreads();
+    if (tid == 0) {
+      // candidate lists: targets in the same bin share one, of that bin's count
+      int64_t base = 0;
+      for (int t = 0; t < kAccTargets; ++t) {
+        int s = t;
+        for (int u = t - 1; u >= 0; --u)
+          if (L.pf[u] == L.pf[t]) s = L.slot[u];
+        L.slot[t] = s;
+        L.base[t] = s == t ? base : L.base[s];
+        if (s == t) base += L.cnt[t];
+      }
+    }
+    __syncthreads();
+  }
+
+  // ---- second digit and candidate lists: each sample in a target's bin adds
+  // one to that bin's histogram of its next 11 bits and joins the bin's list
+  // (a sample joins at most one).  A block gathers its samples per list in
+  // shared memory and reserves each list's range with one atomic; samples
+  // beyond a buffer's capacity are appended one warp's worth at a time.
+  {
+    const int shift = L.shift, lo = shift - kSelBits;
+    const uint64_t pf0 = L.pf[0], pf1 = L.pf[1], pf2 = L.pf[2];
+    uint64_t *buf = reinterpret_cast<uint64_t *>(sh);  // kAccTargets lists of kAccBuf patterns
+    if (tid < kAccTargets) bcnt[tid] = 0;
+    __syncthreads();
+    const unsigned below_me = (1u << lane) - 1u;
+    auto spill = [&](uint64_t v, int s) {  // every lane of the warp calls it together
+#pragma unroll
+      for (int j = 0; j < kAccTargets; ++j) {
+        const unsigned mk = __ballot_sync(0xffffffffu, s == j);
+        if (mk == 0u) continue;
+        const int leader = __ffs(mk) - 1;
+        unsigned long long b = 0ull;
+        if (lane == leader) b = atomicAdd(a.ccur + j, (unsigned long long)__popc(mk));
+        b = __shfl_sync(0xffffffffu, b, leader);
+        const int64_t pos = (int64_t)b + __popc(mk & below_me);
+        if (s == j && pos < L.cnt[j]) a.cand[L.base[j] + pos] = v;
+      }
+    };
+    acc_for_rel(a.relbits, n, [&](uint64_t v) {
+      int s = -1;
+      if (v != ~0ull) {
+        const uint64_t key = v >> shift;
+        s = key == pf0 ? 0 : key == pf1 ? 1 : key == pf2 ? 2 : -1;
+      }
+      int over = -1;
+      if (s >= 0) {
+        atomicAdd(a.hist2 + s * kSelBins + (int)((v >> lo) & (uint64_t)(kSelBins - 1)), 1u);
+        const int p = atomicAdd(&bcnt[s], 1);
+        if (p < kAccBuf)
+          buf[s * kAccBuf + p] = v;
+        else
+          over = s;
+      }
+      if (__any_sync(0xffffffffu, over >= 0)) spill(v, over);
+    });
+    __syncthreads();
+    if (tid < kAccTargets) {
+      const int k = min(bcnt[tid], kAccBuf);
+      bbase[tid] = k ? atomicAdd(a.ccur + tid, (unsigned long long)k) : 0ull;
+    }
+    __syncthreads();
+    for (int j = 0; j < kAccTargets; ++j) {
+      const int k = min(bcnt[j], kAccBuf);
+      for (int i = tid; i < k; i += kAccBlock) {
+        const int64_t pos = (int64_t)bbase[j] + i;
+        if (pos < L.cnt[j]) a.cand[L.base[j] + pos] = buf[j * kAccBuf + i];
+      }
+    }
+  }
+  if (!grid_barrier(a.bar, err)) return;
+
+  // ---- each target's second digit (every block), then every block copies
+  // its slice of each list's samples in the chosen bin to the target's final
+  // list (targets whose prefixes coincide share one)
+  {
+    for (int i = tid; i < kAccTargets * kSelBins; i += kAccBlock) sh[i] = __ldcg(a.hist2 + i);
+    __syncthreads();
+    int bin = 0;
+    int64_t below = 0, c2 = 0;
+    if (wid < kAccTargets && L.pf[wid] != ~0ull) acc_pick1(sh + L.slot[wid] * kSelBins, L.rk[wid], bin, below, c2);
+    if (wid < kAccTargets && lane == 0 && L.pf[wid] != ~0ull) {
+      F.pf[wid] = (L.pf[wid] << kSelBits) | (uint64_t)bin;
+      F.rk[wid] = L.rk[wid] - below;
+      F.cnt[wid] = c2;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      int64_t base = 0;
+      for (int t = 0; t < kAccTargets; ++t) {
+        F.slot[t] = t;
+        if (L.pf[t] == ~0ull) {
+          F.pf[t] = ~0ull;
+          F.cnt[t] = 0;
+        }
+        for (int u = t - 1; u >= 0; --u)
+          if (F.pf[u] == F.pf[t]) F.slot[t] = F.slot[u];
+        F.base[t] = F.slot[t] == t ? base : F.base[F.slot[t]];
+        if (F.slot[t] == t) base += F.cnt[t];
+      }
+    }
+    __syncthreads();
+    const int cur = L.shift - kSelBits;
+    const unsigned below_me = (1u << lane) - 1u;
+    for (int t = 0; t < kAccTargets; ++t) {
+      if (F.slot[t] != t || F.pf[t] == ~0ull) continue;  // the same list for every block
+      const uint64_t *list = a.cand + L.base[t];
+      const int64_t c = L.cnt[t], per = (c + nb - 1) / nb, lo = per * blockIdx.x, hi = min(c, lo + per);
+      const uint64_t want = F.pf[t];
+      for (int64_t i0 = lo; i0 < hi; i0 += kAccBlock) {  // the same trip count in every thread
+        const int64_t i = i0 + tid;
+        const uint64_t v = i < hi ? __ldcg(list + i) : ~0ull;
+        const bool hit = i < hi && (v >> cur) == want;
+        const unsigned mk = __ballot_sync(0xffffffffu, hit);
+        if (mk == 0u) continue;
+        const int leader = __ffs(mk) - 1;
+        unsigned long long b = 0ull;
+        if (lane == leader) b = atomicAdd(a.ccur + kAccTargets + t, (unsigned long long)__popc(mk));
+        b = __shfl_sync(0xffffffffu, b, leader);
+        const int64_t pos = (int64_t)b + __popc(mk & below_me);
+        if (hit && pos < F.cnt[t]) a.cand2[F.base[t] + pos] = v;
+      }
+    }
+  }
+  if (!grid_barrier(a.bar, err)) return;
+
+  // ---- finish: block t ranks target t's final list; another block forms
+  // the totals
+  uint64_t *pct = reinterpret_cast<uint64_t *>(a.out + 8);
+  for (int t = blockIdx.x; t < kAccTargets; t += nb) {
+    uint64_t r = 0ull;
+    if (F.pf[t] != ~0ull) {
+      const int s = F.slot[t];
+      r = acc_finish(a.cand2 + F.base[s], F.cnt[s], F.pf[t], L.shift - kSelBits, F.rk[t], F.cnt[s], sh);
+    }
+    if (tid == 0) pct[t] = r;
+    __syncthreads();
+  }
+  if (blockIdx.x == (kAccTargets % nb)) {
+    if (!fp64) {
+      acc_exact_totals(a, redw);
+    } else {
+      double v[4];
+      for (int j = 0; j < 4; ++j) v[j] = acc_fold_double(all, kPM + j, redd);
+      if (tid == 0) {
+        a.out[0] = (double)L.m;
+        for (int j = 0; j < 4; ++j) a.out[3 + j] = v[j];
+      }
+    }
+    const double sr = acc_fold_double(all, kPQ, redd);
+    if (tid == 0) a.out[7] = sr;
   }
 }
 
