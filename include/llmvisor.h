@@ -65,7 +65,7 @@ typedef int32_t lv_status;
 #define LV_ECUDA (-5)      /* a CUDA runtime call failed */
 #define LV_EDATA (-6)      /* invalid input data seen on the device (sticky) */
 #define LV_ENOMEM (-7)     /* device allocation failed */
-#define LV_ETIMEOUT (-8)   /* reserved: no current kernel waits on the device, so no call returns it */
+#define LV_ETIMEOUT (-8)   /* a grid-wide barrier inside a kernel waited out its bound (lv_accuracy) */
 
 /* Model architecture; integers only.  tp is the modelled tensor-parallel degree
  * (an arithmetic input: constants are per rank).  kv_bytes is the KV-cache
@@ -266,11 +266,12 @@ lv_status lv_fit_vtc(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t 
  * non-zero T lie on one grid 2^(E - 78), E the largest binary exponent among
  * them, and -160 <= E <= 224, the sums are exact integers and R^2 is rounded
  * once from them; otherwise (a non-finite value, magnitudes too far apart or
- * extreme) they are fp64 in a fixed order.  The mean relative error is a
- * fixed-point sum on a grid 2^-100 below the largest error.  Either way results
- * repeat bit for bit.  n < 2^32 (LV_EINVAL otherwise).  rep: host.  With no
- * sample every value is NaN and n = 0; an R^2 whose denominator is 0 is NaN.
- * Synchronous. */
+ * extreme) they are fp64 in a fixed order.  The mean relative error is an
+ * fp64 sum in a fixed order.  Either way results repeat bit for bit.  n < 2^32
+ * (LV_EINVAL otherwise).  One cooperative kernel launch: its blocks meet at
+ * grid-wide barriers whose waits are bounded (about a second), after which the
+ * call returns LV_ETIMEOUT.  rep: host.  With no sample every value is NaN and
+ * n = 0; an R^2 whose denominator is 0 is NaN.  Synchronous. */
 lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, lv_accuracy_report *rep,
                       void *stream);
 

@@ -47,6 +47,8 @@ struct lv_ctx {
   void *d_acc = nullptr;      // accuracy metrics: relative-error bits, partials, histograms
   size_t acc_cap = 0;
   int acc_occ = 0;            // CTAs per SM of the accuracy kernel (0: not yet queried)
+  double *h_acc = nullptr;    // accuracy results: pinned host memory the kernel writes (mapped)
+  double *hd_acc = nullptr;   // its device address
   int timing = 0;  // LV_TIME_* mask
   std::vector<cudaEvent_t> tev;  // start/stop pairs
   size_t tev_used = 0;
@@ -589,7 +591,7 @@ const char *lv_status_string(lv_status s) {
     case LV_ECUDA: return "CUDA error";
     case LV_EDATA: return "invalid input data";
     case LV_ENOMEM: return "out of device memory";
-    case LV_ETIMEOUT: return "reserved status (device wait timed out)";
+    case LV_ETIMEOUT: return "a device-side barrier wait timed out";
     default: return "unknown status";
   }
 }
@@ -662,6 +664,7 @@ void lv_ctx_destroy(lv_ctx *ctx) {
   if (ctx->d_fit) cudaFree(ctx->d_fit);
   if (ctx->d_wi) cudaFree(ctx->d_wi);
   if (ctx->d_acc) cudaFree(ctx->d_acc);
+  if (ctx->h_acc) cudaFreeHost(ctx->h_acc);
   if (ctx->ev_built) cudaEventDestroy(ctx->ev_built);
   if (ctx->ev_used) cudaEventDestroy(ctx->ev_used);
   for (cudaEvent_t e : ctx->tev) cudaEventDestroy(e);
@@ -1028,6 +1031,16 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   rep->r2_ssr = rep->r2_corr = rep->mean_rel = rep->p50 = rep->p90 = rep->p99 = nan;
   if (n == 0) return LV_OK;
   cudaStream_t stream = (cudaStream_t)stream_;
+  if (!ctx->h_acc) {
+    void *h = nullptr, *d = nullptr;
+    if (cudaHostAlloc(&h, 16 * sizeof(double), cudaHostAllocMapped) != cudaSuccess) return LV_ENOMEM;
+    if (cudaHostGetDevicePointer(&d, h, 0) != cudaSuccess) {
+      cudaFreeHost(h);
+      return LV_ECUDA;
+    }
+    ctx->h_acc = static_cast<double *>(h);
+    ctx->hd_acc = static_cast<double *>(d);
+  }
   if (ctx->acc_occ == 0) {
     LV_CUDA(cudaFuncSetAttribute(k_acc, cudaFuncAttributePreferredSharedMemoryCarveout,
                                  (int)cudaSharedmemCarveoutMaxShared));
@@ -1067,23 +1080,22 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   a.cand = reinterpret_cast<uint64_t *>(base + o_cand);
   a.cand2 = reinterpret_cast<uint64_t *>(base + o_cand2);
   a.part = reinterpret_cast<uint64_t *>(base + o_part);
-  a.out = reinterpret_cast<double *>(base + o_out);
+  a.res = ctx->hd_acc;
+  a.err = reinterpret_cast<int *>(base + o_out);
   a.hist1 = reinterpret_cast<unsigned int *>(base + o_hist1);
   a.hist2 = reinterpret_cast<unsigned int *>(base + o_hist2);
   a.ccur = reinterpret_cast<unsigned long long *>(base + o_ccur);
   a.bar = reinterpret_cast<unsigned int *>(base + o_bar);
+  volatile double *h = ctx->h_acc;  // eight sums, three percentile bit patterns, error word
+  *reinterpret_cast<volatile int *>(ctx->h_acc + 11) = 0;
   void *args[] = {&a};
   LV_CUDA(cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(k_acc), dim3(blocks), dim3(kAccBlock), args, 0,
                                       stream));
-  double h[12];  // eight sums, the three percentile bit patterns, the barrier's error word
-  LV_CUDA(cudaMemcpyAsync(h, a.out, sizeof(h), cudaMemcpyDeviceToHost, stream));
   LV_CUDA(cudaStreamSynchronize(stream));
-  int err;
-  std::memcpy(&err, &h[11], sizeof(err));
-  if (err) {
-    // a block waited out the barrier: reset the barrier and the error word for the next call
+  if (*reinterpret_cast<volatile int *>(ctx->h_acc + 11)) {
+    // a block waited out a barrier: reset the barrier and its error word for the next call
     LV_CUDA(cudaMemset(base + o_bar, 0, 8));
-    LV_CUDA(cudaMemset(base + o_out + 11 * sizeof(double), 0, sizeof(double)));
+    LV_CUDA(cudaMemset(base + o_out, 0, sizeof(int)));
     return LV_ETIMEOUT;
   }
   const double m = h[0];

@@ -68,9 +68,9 @@ constexpr int kAccPartW = 32;
 constexpr int kPC = 0, kPL = 1, kPQ = 2, kPR = 4, kPX = 8, kPS = 22, kPM = 25;
 static_assert(kPX + kAccWords <= kPS && kPS + 3 <= kPM && kPM + 4 <= kAccPartW, "partial layout");
 
-// Device arguments of one call.  `out` holds the eight sums (m, -, -, sxx,
-// syy, sxy, ssr, sum rel), the three percentiles' bit patterns and the
-// barrier's error word, so one copy reads them all.
+// Device arguments of one call.  `res` receives the eight sums (m, -, -,
+// sxx, syy, sxy, ssr, sum rel), the three percentiles' bit patterns and an
+// error word, in host memory the device writes directly.
 struct AccArgs {
   const double *y, *T;
   int64_t n;
@@ -78,7 +78,8 @@ struct AccArgs {
   uint64_t *cand;             // first-digit candidate lists, n patterns
   uint64_t *cand2;            // final candidate lists, n patterns
   uint64_t *part;             // kAccPartW words per block
-  double *out;                // 8 doubles, 3 patterns, error word
+  double *res;                // results (host memory, mapped): 8 sums, 3 patterns, error word
+  int *err;                   // the barrier's error word (device memory)
   unsigned int *hist1;        // 2 * kSelBins: first digit, exact pass then fp64 pass
   unsigned int *hist2;        // kAccTargets * kSelBins: the second digit
   unsigned long long *ccur;   // 2 * kAccTargets list cursors (first-digit lists, final lists)
@@ -120,6 +121,11 @@ __device__ __forceinline__ bool grid_barrier(unsigned int *bar, int *err) {
   }
   __syncthreads();
   return ok;
+}
+
+// A block leaving after a barrier timed out: mark the call failed.
+__device__ __forceinline__ void acc_left(const AccArgs &a) {
+  if (threadIdx.x == 0) *reinterpret_cast<volatile int *>(a.res + 11) = 1;
 }
 
 // Sum of `v` over the block in a fixed order (shuffle tree, then the warps in
@@ -174,60 +180,49 @@ __device__ __forceinline__ float rcp_approx(float x) {
   return r;
 }
 
-// x as a float, truncated to 24 bits (relative error below 2^-23), by bit
-// arithmetic on the integer pipe.
-__device__ __forceinline__ float acc_u64_to_f32(uint64_t x) {
-  const int lz = __clzll((long long)x);
-  const uint64_t nx = x << (lz & 63);
-  const uint32_t bits = ((uint32_t)(190 - lz) << 23) + (uint32_t)(nx >> 40) - 0x800000u;
-  return x ? __uint_as_float(bits) : 0.0f;
-}
-
-// floor(e) for 0 <= e < 2^23: adding 2^23 rounded downward leaves it in the
-// low mantissa bits.
-__device__ __forceinline__ uint32_t acc_floor(float e) {
-  return __float_as_uint(__fadd_rd(e, 8388608.0f)) - 0x4B000000u;
-}
-
-// q B exactly (q < 2^32, B < 2^64), from two 32 x 32 -> 64-bit products.
-__device__ __forceinline__ u128 acc_mul32x64(uint32_t q, uint64_t B) {
-  return ((u128)((uint64_t)q * (uint32_t)(B >> 32)) << 32) + (uint64_t)q * (uint32_t)B;
-}
-
-// One schoolbook quotient digit: q = floor(R / Bs) given an estimate within
-// one of the true digit, R reduced by q Bs.  The remainder after the estimate
-// lies in [-Bs, 2 Bs); one conditional add and one conditional subtract settle
-// it.  |R| < 2^127 throughout, so the top bit is the sign.
-__device__ __forceinline__ uint32_t acc_settle(u128 &R, u128 Bs, u128 qBs, uint32_t q) {
-  R -= qBs;
-  const bool neg = (uint64_t)(R >> 64) >> 63;
-  R += neg ? Bs : (u128)0;
-  q -= neg ? 1u : 0u;
-  const bool ge = R >= Bs;
-  R -= ge ? Bs : (u128)0;
-  return q + (ge ? 1u : 0u);
-}
-
 // floor(Ma 2^54 / B) for 2^52 <= Ma, B < 2^53 (so the quotient lies in
-// [2^53, 2^55)), and whether the remainder is non-zero.  Schoolbook division
-// with three digits of 20, 20 and 15 bits: each digit is estimated from a
-// single-precision reciprocal of B's top 24 bits and the remainder's top bits
-// (relative error below 2^-20.4 all told, so with digits below 2^20 the
-// estimate's floor is within one of the true digit) and settled exactly on the
-// integer remainder.
+// [2^53, 2^55)), and whether the remainder is non-zero.  Through a 64-bit
+// reciprocal V ~ 2^116 / B: a single-precision reciprocal of B's top 24 bits
+// (relative error about 2^-21) refined by two Newton-Raphson steps
+// V += V (2^116 - B V) / 2^116, each squaring the error, to within a few units
+// of 2^116 / B; then the quotient estimate Ma V / 2^62, which lies at most one
+// below the true quotient, settled on the exact remainder Ma 2^54 - Q B
+// (below 2^64 in magnitude, so formed modulo 2^64).  The products run on the
+// multiply-add pipe.
 __device__ __forceinline__ uint64_t acc_div54(uint64_t Ma, uint64_t B, bool &rem_nz) {
   // B >> 29 lies in [2^23, 2^24): its float is exponent 150 and the low 23 bits
-  const float inv = rcp_approx(__uint_as_float((150u << 23) | ((uint32_t)(B >> 29) & 0x7FFFFFu)));
-  u128 R = (u128)Ma << 54;
-  const u128 B35 = (u128)B << 35, B15 = (u128)B << 15, B0 = (u128)B;
-  uint32_t q1 = acc_floor(__fmul_rn(acc_u64_to_f32(Ma >> 10), inv));
-  q1 = acc_settle(R, B35, acc_mul32x64(q1, B) << 35, q1);
-  uint32_t q2 = acc_floor(__fmul_rn(__fmul_rn(acc_u64_to_f32((uint64_t)(R >> 40)), inv), 0.0625f));
-  q2 = acc_settle(R, B15, acc_mul32x64(q2, B) << 15, q2);
-  uint32_t q3 = acc_floor(__fmul_rn(__fmul_rn(acc_u64_to_f32((uint64_t)(R >> 20)), inv), 1.0f / 512.0f));
-  q3 = acc_settle(R, B0, acc_mul32x64(q3, B), q3);
+  const uint32_t fb = __float_as_uint(rcp_approx(__uint_as_float((150u << 23) | ((uint32_t)(B >> 29) & 0x7FFFFFu))));
+  const int sh = (int)(fb >> 23) - 63;  // the reciprocal lies in (2^-24, 2^-23]: 40 or 41
+  const uint64_t mf = (uint64_t)((fb & 0x7FFFFFu) | 0x800000u);
+  uint64_t V = sh >= 41 ? ~0ull : mf << sh;  // 2^-23 exactly would give 2^64
+  {
+    const __int128 E = (__int128)(((u128)1 << 116) - (u128)B * V);  // |E| < 2^96
+    const int64_t Ep = (int64_t)(E >> 52);
+    const uint64_t c = __umul64hi(V, (uint64_t)(Ep < 0 ? -Ep : Ep));
+    V = Ep < 0 ? V - c : V + c;
+  }
+  {
+    const __int128 E = (__int128)(((u128)1 << 116) - (u128)B * V);  // |E| < 2^75
+    const int64_t Ep = (int64_t)(E >> 12);
+    const uint64_t c = __umul64hi(V, (uint64_t)(Ep < 0 ? -Ep : Ep)) >> 40;
+    V = Ep < 0 ? V - c : V + c;
+  }
+  uint64_t Q = (__umul64hi(Ma, V) << 2) | ((Ma * V) >> 62);
+  uint64_t R = (Ma << 54) - Q * B;
+  if ((int64_t)R < 0) {  // not reached when the bounds above hold
+    R += B;
+    --Q;
+  }
+  if (R >= B) {
+    R -= B;
+    ++Q;
+  }
+  if (R >= B) {  // not reached when the bounds above hold
+    R -= B;
+    ++Q;
+  }
   rem_nz = R != 0;
-  return ((uint64_t)q1 << 35) + ((uint64_t)q2 << 15) + q3;
+  return Q;
 }
 
 // fl(Ma 2^ka / (My 2^ky)) as a bit pattern, for 2^52 <= Ma, My < 2^53: the
@@ -715,9 +710,11 @@ __device__ __forceinline__ double acc_fold_double(const uint64_t *part, int off,
   return block_sum_fixed(s, redd);
 }
 
-// Exact totals to sums: fold the blocks' exact partials and write out[0] = m
-// and, scaled by m 2^(2S), out[3..6] = sxx, syy, sxy, ssr.  One block.
+// Exact totals to sums: fold the blocks' exact partials and write res[0] = m
+// and, scaled by m 2^(2S), res[3..6] = sxx, syy, sxy, ssr (one each on
+// threads 0..3).  One block.
 __device__ __forceinline__ void acc_exact_totals(const AccArgs &a, uint64_t *redw) {
+  __shared__ uint64_t tw[kAccWords];
   uint64_t w[kAccWords];
 #pragma unroll
   for (int j = 0; j < kAccWords; ++j) w[j] = 0ull;
@@ -729,54 +726,63 @@ __device__ __forceinline__ void acc_exact_totals(const AccArgs &a, uint64_t *red
     acc_combine(w, o);
   }
   acc_block_combine(w, redw);
-  if (threadIdx.x != 0) return;
+  if (threadIdx.x == 0)
+#pragma unroll
+    for (int j = 0; j < kAccWords; ++j) tw[j] = w[j];
+  __syncthreads();
+  const int q = threadIdx.x;
+  if (q >= 4) return;
+#pragma unroll
+  for (int j = 0; j < kAccWords; ++j) w[j] = tw[j];
   const uint64_t m = w[0];
   // |sum T| and its sign
   const bool tneg = (int64_t)w[4] < 0;
   const u128 st = ((u128)w[4] << 64) | w[3], sa = tneg ? (u128)0 - st : st;
   const uint64_t s0 = (uint64_t)sa, s1 = (uint64_t)(sa >> 64);
-  uint64_t sxx[4], syy[4], sxy[4], ssr[4], tmp[4];
-  mul64x192(m, w + 5, sxx);
-  mul128x128(w[1], w[2], w[1], w[2], tmp);
-  sub256(sxx, tmp);
-  mul64x192(m, w + 8, syy);
-  mul128x128(s0, s1, s0, s1, tmp);
-  sub256(syy, tmp);
-  // 2 m sxy = m (sum Y^2 + sum T^2 - sum D^2) - 2 sum Y sum T; the 192-bit
-  // bracket may be negative (two's complement), hence the split below
-  uint64_t g[3] = {w[5], w[6], w[7]};
-  add192w(g, w[8], w[9], w[10]);
-  add192w(g, ~w[11], ~w[12], ~w[13]);
-  add192w(g, 1, 0, 0);
-  const bool gneg = (int64_t)g[2] < 0;
-  if (gneg) {
-    g[0] = ~g[0];
-    g[1] = ~g[1];
-    g[2] = ~g[2];
+  uint64_t v[4], tmp[4];
+  if (q == 0) {  // m sum Y^2 - (sum Y)^2
+    mul64x192(m, w + 5, v);
+    mul128x128(w[1], w[2], w[1], w[2], tmp);
+    sub256(v, tmp);
+  } else if (q == 1) {  // m sum T^2 - (sum T)^2
+    mul64x192(m, w + 8, v);
+    mul128x128(s0, s1, s0, s1, tmp);
+    sub256(v, tmp);
+  } else if (q == 2) {
+    // 2 m sxy = m (sum Y^2 + sum T^2 - sum D^2) - 2 sum Y sum T; the 192-bit
+    // bracket may be negative (two's complement), hence the split below
+    uint64_t g[3] = {w[5], w[6], w[7]};
+    add192w(g, w[8], w[9], w[10]);
+    add192w(g, ~w[11], ~w[12], ~w[13]);
     add192w(g, 1, 0, 0);
+    const bool gneg = (int64_t)g[2] < 0;
+    if (gneg) {
+      g[0] = ~g[0];
+      g[1] = ~g[1];
+      g[2] = ~g[2];
+      add192w(g, 1, 0, 0);
+    }
+    mul64x192(m, g, v);
+    if (gneg) {
+      uint64_t z[4] = {0, 0, 0, 0};
+      sub256(z, v);
+      v[0] = z[0];
+      v[1] = z[1];
+      v[2] = z[2];
+      v[3] = z[3];
+    }
+    mul128x128(w[1], w[2], s0, s1, tmp);
+    acc_add256(tmp, tmp[0], tmp[1], tmp[2], tmp[3]);  // 2 sum Y |sum T|
+    if (tneg)
+      acc_add256(v, tmp[0], tmp[1], tmp[2], tmp[3]);
+    else
+      sub256(v, tmp);
+  } else {  // m sum D^2
+    mul64x192(m, w + 11, v);
   }
-  mul64x192(m, g, sxy);
-  if (gneg) {
-    uint64_t z[4] = {0, 0, 0, 0};
-    sub256(z, sxy);
-    sxy[0] = z[0];
-    sxy[1] = z[1];
-    sxy[2] = z[2];
-    sxy[3] = z[3];
-  }
-  mul128x128(w[1], w[2], s0, s1, tmp);
-  acc_add256(tmp, tmp[0], tmp[1], tmp[2], tmp[3]);  // 2 sum Y |sum T|
-  if (tneg)
-    acc_add256(sxy, tmp[0], tmp[1], tmp[2], tmp[3]);
-  else
-    sub256(sxy, tmp);
-  mul64x192(m, w + 11, ssr);
   bool ok = true;  // every value here is below 2^227 in magnitude
-  a.out[0] = (double)m;
-  a.out[3] = acc_i256_to_double(sxx, 0, ok);
-  a.out[4] = acc_i256_to_double(syy, 0, ok);
-  a.out[5] = acc_i256_to_double(sxy, -1, ok);
-  a.out[6] = acc_i256_to_double(ssr, 0, ok);
+  a.res[3 + q] = acc_i256_to_double(v, q == 2 ? -1 : 0, ok);
+  if (q == 0) a.res[0] = (double)m;
 }
 
 // The whole accuracy computation of one call; a cooperative launch of at
@@ -792,7 +798,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
   __shared__ unsigned long long bbase[kAccTargets];
   __shared__ int path[3];  // exact, narrow, S
   __shared__ double mean[2];
-  int *err = reinterpret_cast<int *>(a.out + 11);
+  int *err = reinterpret_cast<int *>(a.err);
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, nb = gridDim.x;
   const int64_t n = a.n, stride = (int64_t)nb * kAccBlock, g0 = blockIdx.x * (int64_t)kAccBlock + tid;
   uint64_t *mine = a.part + (int64_t)blockIdx.x * kAccPartW;
@@ -832,7 +838,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
       mine[kPR + 1] = z;
     }
   }
-  if (!grid_barrier(a.bar, err)) return;
+  if (!grid_barrier(a.bar, err)) return acc_left(a);
   // the path: exact when the values are finite, n < 2^32 (the integer widths
   // hold any count below it) and Emax is in [kAccEmaxLo, kAccEmaxHi]; narrow
   // (64-bit integers) when every exponent is within 10 of Emax
@@ -886,7 +892,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
 #pragma unroll
       for (int j = 0; j < kAccWords; ++j) mine[kPX + j] = w[j];
     }
-    if (!grid_barrier(a.bar, err)) return;
+    if (!grid_barrier(a.bar, err)) return acc_left(a);
     int off = 0;
     for (int b = tid; b < nb; b += kAccBlock) off |= (int)__ldcg(all + (int64_t)b * kAccPartW + kPL);
     fp64 = __syncthreads_or(off) != 0;  // a value off the wide grid: redo the call in fp64
@@ -940,7 +946,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
       p[kPS + 1] = B;
       p[kPS + 2] = C;
     }
-    if (!grid_barrier(a.bar, err)) return;
+    if (!grid_barrier(a.bar, err)) return acc_left(a);
     const double s0 = acc_fold_double(all, kPS, redd), s1 = acc_fold_double(all, kPS + 1, redd),
                  s2 = acc_fold_double(all, kPS + 2, redd);
     if (tid == 0) {
@@ -969,7 +975,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
       p[kPM + 2] = v2;
       p[kPM + 3] = v3;
     }
-    if (!grid_barrier(a.bar, err)) return;
+    if (!grid_barrier(a.bar, err)) return acc_left(a);
   }
 
   // ---- first digit: sample count, then each target's bin (every block)
@@ -1079,7 +1085,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
       }
     }
   }
-  if (!grid_barrier(a.bar, err)) return;
+  if (!grid_barrier(a.bar, err)) return acc_left(a);
 
   // ---- each target's second digit (every block), then every block copies
   // its slice of each list's samples in the chosen bin to the target's final
@@ -1133,11 +1139,11 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
       }
     }
   }
-  if (!grid_barrier(a.bar, err)) return;
+  if (!grid_barrier(a.bar, err)) return acc_left(a);
 
   // ---- finish: block t ranks target t's final list; another block forms
   // the totals
-  uint64_t *pct = reinterpret_cast<uint64_t *>(a.out + 8);
+  uint64_t *pct = reinterpret_cast<uint64_t *>(a.res + 8);
   for (int t = blockIdx.x; t < kAccTargets; t += nb) {
     uint64_t r = 0ull;
     if (F.pf[t] != ~0ull) {
@@ -1154,12 +1160,15 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
       double v[4];
       for (int j = 0; j < 4; ++j) v[j] = acc_fold_double(all, kPM + j, redd);
       if (tid == 0) {
-        a.out[0] = (double)L.m;
-        for (int j = 0; j < 4; ++j) a.out[3 + j] = v[j];
+        a.res[0] = (double)L.m;
+        for (int j = 0; j < 4; ++j) a.res[3 + j] = v[j];
       }
     }
+  }
+  if (blockIdx.x == ((kAccTargets + 1) % nb)) {
+    __syncthreads();
     const double sr = acc_fold_double(all, kPQ, redd);
-    if (tid == 0) a.out[7] = sr;
+    if (tid == 0) a.res[7] = sr;
   }
 }
 
