@@ -1042,8 +1042,6 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
     ctx->hd_acc = static_cast<double *>(d);
   }
   if (ctx->acc_occ == 0) {
-    LV_CUDA(cudaFuncSetAttribute(k_acc, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                 (int)cudaSharedmemCarveoutMaxShared));
     LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ, k_acc, kAccBlock, 0));
     if (ctx->acc_occ <= 0) return LV_ECUDA;
   }

@@ -53,6 +53,7 @@ constexpr int kAccWords = 14;   // the exact sums of one block
 constexpr int kSelBits = 11;    // radix digit
 constexpr int kSelBins = 1 << kSelBits;
 constexpr int kAccBuf = kSelBins / 2;  // a block's buffered candidates per list
+constexpr int64_t kAccDirect = 1 << 15;  // first-digit lists a finishing block filters itself
 constexpr int kAccGrid = 78;  // wide grid: S = kAccGrid - Emax puts every |v 2^S| below 2^79
 // Range of Emax for the exact path: within it the definition's own fp64
 // arithmetic (squared deviations, their products in r2_corr) neither overflows
@@ -648,12 +649,16 @@ __device__ uint64_t acc_finish(const uint64_t *__restrict__ list, int64_t c, uin
       res = 0ull;
     }
     __syncthreads();
-    for (int64_t i = threadIdx.x; i < c; i += kAccBlock) {
-      const uint64_t v = __ldcg(list + i);
-      if ((v >> cur) == prefix) {
-        const int p = atomicAdd(&nsel, 1);
-        if (p < kShort) ls[p] = v;
-      }
+    for (int64_t i0 = threadIdx.x; i0 < c; i0 += 4 * kAccBlock) {
+      uint64_t v[4];  // four loads in flight
+#pragma unroll
+      for (int k = 0; k < 4; ++k) v[k] = i0 + k * kAccBlock < c ? __ldcg(list + i0 + k * kAccBlock) : ~0ull;
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        if (i0 + k * kAccBlock < c && (v[k] >> cur) == prefix) {
+          const int p = atomicAdd(&nsel, 1);
+          if (p < kShort) ls[p] = v[k];
+        }
     }
     __syncthreads();
     const int k = min(nsel, kShort);
@@ -1089,8 +1094,11 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
 
   // ---- each target's second digit (every block), then every block copies
   // its slice of each list's samples in the chosen bin to the target's final
-  // list (targets whose prefixes coincide share one)
-  {
+  // list (targets whose prefixes coincide share one).  Skipped when every
+  // first-digit list is short: the finishing blocks then filter their lists
+  // themselves.
+  const bool direct = max(L.cnt[0], max(L.cnt[1], L.cnt[2])) <= kAccDirect;
+  if (!direct) {
     for (int i = tid; i < kAccTargets * kSelBins; i += kAccBlock) sh[i] = __ldcg(a.hist2 + i);
     __syncthreads();
     int bin = 0;
@@ -1138,17 +1146,35 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
         if (hit && pos < F.cnt[t]) a.cand2[F.base[t] + pos] = v;
       }
     }
+    if (!grid_barrier(a.bar, err)) return acc_left(a);
   }
-  if (!grid_barrier(a.bar, err)) return acc_left(a);
 
-  // ---- finish: block t ranks target t's final list; another block forms
-  // the totals
+  // ---- finish: block t ranks target t among its list's samples in the
+  // chosen second-digit bin (its final list, or its first-digit list filtered
+  // here); other blocks form the totals
   uint64_t *pct = reinterpret_cast<uint64_t *>(a.res + 8);
   for (int t = blockIdx.x; t < kAccTargets; t += nb) {
     uint64_t r = 0ull;
-    if (F.pf[t] != ~0ull) {
-      const int s = F.slot[t];
-      r = acc_finish(a.cand2 + F.base[s], F.cnt[s], F.pf[t], L.shift - kSelBits, F.rk[t], F.cnt[s], sh);
+    if (L.pf[t] != ~0ull) {
+      if (direct) {
+        for (int i = tid; i < kSelBins; i += kAccBlock) sh[i] = __ldcg(a.hist2 + L.slot[t] * kSelBins + i);
+        __syncthreads();
+        if (wid == 0) {
+          int bin;
+          int64_t below, c2;
+          acc_pick1(sh, L.rk[t], bin, below, c2);
+          if (lane == 0) {
+            F.pf[t] = (L.pf[t] << kSelBits) | (uint64_t)bin;
+            F.rk[t] = L.rk[t] - below;
+            F.cnt[t] = c2;
+          }
+        }
+        __syncthreads();
+        r = acc_finish(a.cand + L.base[t], L.cnt[t], F.pf[t], L.shift - kSelBits, F.rk[t], F.cnt[t], sh);
+      } else {
+        const int s = F.slot[t];
+        r = acc_finish(a.cand2 + F.base[s], F.cnt[s], F.pf[t], L.shift - kSelBits, F.rk[t], F.cnt[s], sh);
+      }
     }
     if (tid == 0) pct[t] = r;
     __syncthreads();
