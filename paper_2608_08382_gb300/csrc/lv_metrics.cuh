@@ -558,6 +558,7 @@ __device__ __forceinline__ int acc_key1(uint64_t rb, const AccKey &K) {
 // from the same global data in the same order).
 struct AccSel {
   uint64_t pf[kAccTargets];   // prefix after the first digit; ~0 once a target is settled at 0
+  int bin[kAccTargets];       // its first-digit bin
   int64_t rk[kAccTargets];    // rank still to find below it
   int64_t cnt[kAccTargets];   // samples in its first-digit bin (its list's length)
   int64_t base[kAccTargets];  // list offset of its slot
@@ -566,35 +567,80 @@ struct AccSel {
   int64_t m;                  // samples
 };
 
-// Exact pass over this block's share of y and T on the narrow or wide grid:
-// the sums into w, rel's patterns into relbits, rel's first digit into the
-// block histogram h1 and rel into srel (fp64, in the thread's fixed order);
-// `lost` when a value is off the wide grid.
+// Exact pass over the block's range [lo, hi) of y and T on the narrow or
+// wide grid: the sums into w, rel's patterns into relbits, rel's first digit
+// into the block histogram h1 and rel into srel (fp64, in the thread's fixed
+// order); `lost` when a value is off the wide grid.
 template <bool kNarrow>
-__device__ __forceinline__ void acc_exact_loop(const double *__restrict__ y, const double *__restrict__ T, int64_t n,
-                                               int S, uint64_t *__restrict__ relbits, uint64_t *w, unsigned int *h1,
-                                               const AccKey &K, double &srel, bool &lost) {
-  const int64_t stride = (int64_t)gridDim.x * kAccBlock;
-  for (int64_t i0 = blockIdx.x * (int64_t)kAccBlock + threadIdx.x; i0 < n; i0 += 2 * stride) {
+__device__ __forceinline__ void acc_exact_loop(const double *__restrict__ y, const double *__restrict__ T, int64_t lo,
+                                               int64_t hi, int S, uint64_t *__restrict__ relbits, uint64_t *w,
+                                               unsigned int *h1, const AccKey &K, double &srel, bool &lost) {
+  for (int64_t i0 = lo + threadIdx.x; i0 < hi; i0 += 2 * kAccBlock) {
     uint64_t yb[2], tb[2];  // two elements' loads in flight (a pattern of 0 is not a sample)
 #pragma unroll
     for (int k = 0; k < 2; ++k) {
-      const int64_t i = i0 + k * stride;
-      yb[k] = i < n ? (uint64_t)__double_as_longlong(__ldg(y + i)) : 0ull;
-      tb[k] = i < n ? (uint64_t)__double_as_longlong(__ldg(T + i)) : 0ull;
+      const int64_t i = i0 + k * kAccBlock;
+      yb[k] = i < hi ? (uint64_t)__double_as_longlong(__ldg(y + i)) : 0ull;
+      tb[k] = i < hi ? (uint64_t)__double_as_longlong(__ldg(T + i)) : 0ull;
     }
 #pragma unroll
     for (int k = 0; k < 2; ++k) {
-      const int64_t i = i0 + k * stride;
+      const int64_t i = i0 + k * kAccBlock;
       uint64_t rb = ~0ull;  // not a sample
       if (acc_is_sample(yb[k])) {
         rb = kNarrow ? acc_exact_sample64(yb[k], tb[k], S, w) : acc_exact_sample(yb[k], tb[k], S, w, lost);
         atomicAdd(&h1[acc_key1(rb, K)], 1u);
         srel += __longlong_as_double((long long)rb);
       }
-      if (i < n) relbits[i] = rb;
+      if (i < hi) relbits[i] = rb;
     }
   }
+}
+
+// Counting sort of the block's samples by first digit: off = exclusive prefix
+// sums of the block histogram h1, then each sample of relbits[lo, hi) goes to
+// sorted[lo + off[key] + (its place among the block's samples of that key)]
+// (`cur`: kSelBins cursors of scratch).  Afterwards the samples of bin k lie
+// at sorted[lo + off[k], lo + off[k] + h1[k]).
+__device__ __forceinline__ void acc_block_sort(const uint64_t *__restrict__ relbits, uint64_t *__restrict__ sorted,
+                                               int64_t lo, int64_t hi, const unsigned int *h1, unsigned int *off,
+                                               unsigned int *cur, const AccKey &K) {
+  __shared__ unsigned int wsum[kAccBlock / 32];
+  constexpr int kPer = kSelBins / kAccBlock;  // bins per thread
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  unsigned int c[kPer], s = 0u;
+#pragma unroll
+  for (int j = 0; j < kPer; ++j) {
+    c[j] = h1[threadIdx.x * kPer + j];
+    s += c[j];
+  }
+  unsigned int inc = s;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const unsigned int o = __shfl_up_sync(0xffffffffu, inc, d);
+    if (lane >= d) inc += o;
+  }
+  if (lane == 31) wsum[wid] = inc;
+  __syncthreads();
+  unsigned int wb = 0u;
+  for (int v = 0; v < wid; ++v) wb += wsum[v];
+  unsigned int run = wb + inc - s;
+#pragma unroll
+  for (int j = 0; j < kPer; ++j) {
+    off[threadIdx.x * kPer + j] = run;
+    cur[threadIdx.x * kPer + j] = run;
+    run += c[j];
+  }
+  __syncthreads();
+  for (int64_t i0 = lo + threadIdx.x; i0 < hi; i0 += 4 * kAccBlock) {
+    uint64_t v[4];  // four loads in flight
+#pragma unroll
+    for (int k = 0; k < 4; ++k) v[k] = i0 + k * kAccBlock < hi ? __ldcg(relbits + i0 + k * kAccBlock) : ~0ull;
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (v[k] != ~0ull) sorted[lo + atomicAdd(&cur[acc_key1(v[k], K)], 1u)] = v[k];
+  }
+  __syncthreads();
 }
 
 // Visit this block's share of the rel patterns in warp tiles of 256 (load k
@@ -790,32 +836,49 @@ __device__ __forceinline__ void acc_exact_totals(const AccArgs &a, uint64_t *red
   if (q == 0) a.res[0] = (double)m;
 }
 
+// The samples of the block's segment for first-digit bin `bin` (the block's
+// sorted range), visited by the whole block with eight loads in flight per
+// thread.
+template <class F>
+__device__ __forceinline__ void acc_for_segment(const uint64_t *__restrict__ seg, int cnt, F &&visit) {
+  for (int i0 = threadIdx.x; i0 < cnt; i0 += 8 * kAccBlock) {
+    uint64_t v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = i0 + k * kAccBlock < cnt ? __ldcg(seg + i0 + k * kAccBlock) : ~0ull;
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (i0 + k * kAccBlock < cnt) visit(v[k]);
+  }
+}
+
 // The whole accuracy computation of one call; a cooperative launch of at
-// most as many blocks as fit at once.
+// most as many blocks as fit at once.  Block b owns the elements [lo, hi).
 __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
   __shared__ __align__(16) unsigned int sh[kAccTargets * kSelBins];  // per-phase scratch
+  __shared__ unsigned int bh1[kSelBins], bof1[kSelBins];  // the block's first-digit counts and offsets
   __shared__ unsigned long long red2[kAccBlock / 32 * 2];
   __shared__ double redd[kAccBlock / 32];
   __shared__ uint64_t redw[kAccBlock / 32 * kAccWords];
   __shared__ AccSel L, F;  // after the first digit; after the second
   __shared__ AccKey K;
-  __shared__ int bcnt[kAccTargets];
-  __shared__ unsigned long long bbase[kAccTargets];
   __shared__ int path[3];  // exact, narrow, S
   __shared__ double mean[2];
   int *err = reinterpret_cast<int *>(a.err);
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, nb = gridDim.x;
   const int64_t n = a.n, stride = (int64_t)nb * kAccBlock, g0 = blockIdx.x * (int64_t)kAccBlock + tid;
+  const int64_t chunk = (n + nb - 1) / nb, lo = min(n, chunk * blockIdx.x), hi = min(n, lo + chunk);
   uint64_t *mine = a.part + (int64_t)blockIdx.x * kAccPartW;
   const uint64_t *all = a.part;
+  uint64_t *sorted = a.cand;  // each block's samples, sorted by first digit within its range
 
   // ---- range: the largest magnitude (high word of the largest sample y or
   // |T|) and smallest exponent over the samples' y and non-zero T.  (A NaN y
   // counts here, sending the call to the fp64 phases, which leave it out.)
-  // The histograms and list cursors of the previous call are cleared here.
+  // The second-digit histograms, the first-digit totals and the list cursors
+  // of the previous call are cleared here.
   for (int64_t i = g0; i < 2 * kSelBins; i += stride) a.hist1[i] = 0u;
   for (int64_t i = g0; i < kAccTargets * kSelBins; i += stride) a.hist2[i] = 0u;
-  if (g0 < 2 * kAccTargets) a.ccur[g0] = 0ull;
+  if (g0 < kAccTargets) a.ccur[g0] = 0ull;
   {
     unsigned int top = 0u, nmin = 0u;  // nmin: max of 2047 - biased exponent
     for (int64_t i0 = g0; i0 < n; i0 += 4 * stride) {
@@ -867,11 +930,12 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
       K.kbits = path[1] ? 4 : 3;
       K.elo = path[1] ? -63 : -79;
     }
-    for (int i = tid; i < kSelBins; i += kAccBlock) sh[i] = 0u;
+    for (int i = tid; i < kSelBins; i += kAccBlock) bh1[i] = 0u;
     __syncthreads();
   }
 
-  // ---- exact: sums, rel and its first digit on the grid
+  // ---- exact: sums, rel and its first digit on the grid; the block's
+  // samples sorted by first digit
   bool fp64 = path[0] == 0;
   if (!fp64) {
     uint64_t w[kAccWords];
@@ -880,12 +944,13 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
     double srel = 0.0;
     bool lost = false;
     if (path[1])
-      acc_exact_loop<true>(a.y, a.T, n, path[2], a.relbits, w, sh, K, srel, lost);
+      acc_exact_loop<true>(a.y, a.T, lo, hi, path[2], a.relbits, w, bh1, K, srel, lost);
     else
-      acc_exact_loop<false>(a.y, a.T, n, path[2], a.relbits, w, sh, K, srel, lost);
+      acc_exact_loop<false>(a.y, a.T, lo, hi, path[2], a.relbits, w, bh1, K, srel, lost);
     const int anylost = __syncthreads_or(lost);
+    acc_block_sort(a.relbits, sorted, lo, hi, bh1, bof1, sh, K);
     for (int i = tid; i < kSelBins; i += kAccBlock) {
-      const unsigned int c = sh[i];
+      const unsigned int c = bh1[i];
       if (c) atomicAdd(a.hist1 + i, c);
     }
     srel = block_sum_fixed(srel, redd);
@@ -903,19 +968,19 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
     fp64 = __syncthreads_or(off) != 0;  // a value off the wide grid: redo the call in fp64
   }
 
-  // ---- fp64: rel and its first digit, means, then centred moments, each in
-  // a fixed order
+  // ---- fp64: rel and its first digit, the block's samples sorted by it,
+  // means, then centred moments, each in a fixed order
   if (fp64) {
     if (tid == 0) {
       K.exact = 0;
       K.kbits = 0;
       K.elo = 0;
     }
-    for (int i = tid; i < kSelBins; i += kAccBlock) sh[i] = 0u;
+    for (int i = tid; i < kSelBins; i += kAccBlock) bh1[i] = 0u;
     __syncthreads();
     double c = 0.0, sy = 0.0, st = 0.0, srel = 0.0;
     uint64_t cnt = 0;
-    for (int64_t i = g0; i < n; i += stride) {
+    for (int64_t i = lo + tid; i < hi; i += kAccBlock) {
       const double yv = a.y[i], tv = a.T[i];
       uint64_t bits = ~0ull;
       if (yv > 0.0) {
@@ -924,14 +989,15 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
         sy += yv;
         st += tv;
         bits = (uint64_t)__double_as_longlong(__ddiv_rn(fabs(__dsub_rn(tv, yv)), yv));
-        atomicAdd(&sh[(int)(bits >> 52)], 1u);
+        atomicAdd(&bh1[(int)(bits >> 52)], 1u);
         srel += __longlong_as_double((long long)bits);
       }
       a.relbits[i] = bits;
     }
     __syncthreads();
+    acc_block_sort(a.relbits, sorted, lo, hi, bh1, bof1, sh, K);
     for (int i = tid; i < kSelBins; i += kAccBlock) {
-      const unsigned int h = sh[i];
+      const unsigned int h = bh1[i];
       if (h) atomicAdd(a.hist1 + kSelBins + i, h);
     }
     const double A = block_sum_fixed(c, redd), B = block_sum_fixed(sy, redd), C = block_sum_fixed(st, redd);
@@ -961,7 +1027,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
     __syncthreads();
     const double my = mean[0], mt = mean[1];
     double sxx = 0.0, syy = 0.0, sxy = 0.0, ssr = 0.0;
-    for (int64_t i = g0; i < n; i += stride) {
+    for (int64_t i = lo + tid; i < hi; i += kAccBlock) {
       const double yv = a.y[i], tv = a.T[i];
       if (yv > 0.0) {
         const double dy = yv - my, dt = tv - mt, e = yv - tv;
@@ -1009,6 +1075,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
     int64_t below = 0, c1 = 0;
     if (wid < kAccTargets && L.m > 0) acc_pick1(sh, L.rk[wid], bin, below, c1);
     if (wid < kAccTargets && lane == 0) {
+      L.bin[wid] = bin;
       if (L.m == 0 || (K.exact && bin == 0)) {
         L.pf[wid] = ~0ull;  // settled: rel = 0 (or no sample)
         L.cnt[wid] = 0;
@@ -1019,86 +1086,35 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
       }
     }
     __syncthreads();
-    if (tid == 0) {
-      // candidate lists: targets in the same bin share one, of that bin's count
-      int64_t base = 0;
-      for (int t = 0; t < kAccTargets; ++t) {
+    if (tid == 0)
+      for (int t = 0; t < kAccTargets; ++t) {  // targets in the same bin share one second-digit histogram
         int s = t;
         for (int u = t - 1; u >= 0; --u)
           if (L.pf[u] == L.pf[t]) s = L.slot[u];
         L.slot[t] = s;
-        L.base[t] = s == t ? base : L.base[s];
-        if (s == t) base += L.cnt[t];
       }
-    }
     __syncthreads();
   }
 
-  // ---- second digit and candidate lists: each sample in a target's bin adds
-  // one to that bin's histogram of its next 11 bits and joins the bin's list
-  // (a sample joins at most one).  A block gathers its samples per list in
-  // shared memory and reserves each list's range with one atomic; samples
-  // beyond a buffer's capacity are appended one warp's worth at a time.
+  // ---- second digit: each block histograms the next 11 bits of its samples
+  // in the targets' first-digit bins (its sorted segments)
   {
-    const int shift = L.shift, lo = shift - kSelBits;
-    const uint64_t pf0 = L.pf[0], pf1 = L.pf[1], pf2 = L.pf[2];
-    uint64_t *buf = reinterpret_cast<uint64_t *>(sh);  // kAccTargets lists of kAccBuf patterns
-    if (tid < kAccTargets) bcnt[tid] = 0;
-    __syncthreads();
-    const unsigned below_me = (1u << lane) - 1u;
-    auto spill = [&](uint64_t v, int s) {  // every lane of the warp calls it together
-#pragma unroll
-      for (int j = 0; j < kAccTargets; ++j) {
-        const unsigned mk = __ballot_sync(0xffffffffu, s == j);
-        if (mk == 0u) continue;
-        const int leader = __ffs(mk) - 1;
-        unsigned long long b = 0ull;
-        if (lane == leader) b = atomicAdd(a.ccur + j, (unsigned long long)__popc(mk));
-        b = __shfl_sync(0xffffffffu, b, leader);
-        const int64_t pos = (int64_t)b + __popc(mk & below_me);
-        if (s == j && pos < L.cnt[j]) a.cand[L.base[j] + pos] = v;
-      }
-    };
-    acc_for_rel(a.relbits, n, [&](uint64_t v) {
-      int s = -1;
-      if (v != ~0ull) {
-        const uint64_t key = v >> shift;
-        s = key == pf0 ? 0 : key == pf1 ? 1 : key == pf2 ? 2 : -1;
-      }
-      int over = -1;
-      if (s >= 0) {
-        atomicAdd(a.hist2 + s * kSelBins + (int)((v >> lo) & (uint64_t)(kSelBins - 1)), 1u);
-        const int p = atomicAdd(&bcnt[s], 1);
-        if (p < kAccBuf)
-          buf[s * kAccBuf + p] = v;
-        else
-          over = s;
-      }
-      if (__any_sync(0xffffffffu, over >= 0)) spill(v, over);
-    });
-    __syncthreads();
-    if (tid < kAccTargets) {
-      const int k = min(bcnt[tid], kAccBuf);
-      bbase[tid] = k ? atomicAdd(a.ccur + tid, (unsigned long long)k) : 0ull;
-    }
-    __syncthreads();
-    for (int j = 0; j < kAccTargets; ++j) {
-      const int k = min(bcnt[j], kAccBuf);
-      for (int i = tid; i < k; i += kAccBlock) {
-        const int64_t pos = (int64_t)bbase[j] + i;
-        if (pos < L.cnt[j]) a.cand[L.base[j] + pos] = buf[j * kAccBuf + i];
-      }
+    const int lo2 = L.shift - kSelBits;
+    for (int t = 0; t < kAccTargets; ++t) {
+      if (L.slot[t] != t || L.pf[t] == ~0ull) continue;  // the same in every block
+      const int b = L.bin[t];
+      unsigned int *h2 = a.hist2 + t * kSelBins;
+      acc_for_segment(sorted + lo + bof1[b], (int)bh1[b], [&](uint64_t v) {
+        atomicAdd(h2 + (int)((v >> lo2) & (uint64_t)(kSelBins - 1)), 1u);
+      });
     }
   }
   if (!grid_barrier(a.bar, err)) return acc_left(a);
 
   // ---- each target's second digit (every block), then every block copies
-  // its slice of each list's samples in the chosen bin to the target's final
-  // list (targets whose prefixes coincide share one).  Skipped when every
-  // first-digit list is short: the finishing blocks then filter their lists
-  // themselves.
-  const bool direct = max(L.cnt[0], max(L.cnt[1], L.cnt[2])) <= kAccDirect;
-  if (!direct) {
+  // its samples in the chosen bin to the target's final list (targets whose
+  // prefixes coincide share one)
+  {
     for (int i = tid; i < kAccTargets * kSelBins; i += kAccBlock) sh[i] = __ldcg(a.hist2 + i);
     __syncthreads();
     int bin = 0;
@@ -1128,53 +1144,35 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
     const int cur = L.shift - kSelBits;
     const unsigned below_me = (1u << lane) - 1u;
     for (int t = 0; t < kAccTargets; ++t) {
-      if (F.slot[t] != t || F.pf[t] == ~0ull) continue;  // the same list for every block
-      const uint64_t *list = a.cand + L.base[t];
-      const int64_t c = L.cnt[t], per = (c + nb - 1) / nb, lo = per * blockIdx.x, hi = min(c, lo + per);
+      if (F.slot[t] != t || F.pf[t] == ~0ull) continue;  // the same in every block
+      const int b = L.bin[t], cnt = (int)bh1[b];
+      const uint64_t *seg = sorted + lo + bof1[b];
       const uint64_t want = F.pf[t];
-      for (int64_t i0 = lo; i0 < hi; i0 += kAccBlock) {  // the same trip count in every thread
-        const int64_t i = i0 + tid;
-        const uint64_t v = i < hi ? __ldcg(list + i) : ~0ull;
-        const bool hit = i < hi && (v >> cur) == want;
+      for (int i0 = 0; i0 < cnt; i0 += kAccBlock) {  // the same trip count in every thread
+        const int i = i0 + tid;
+        const uint64_t v = i < cnt ? __ldcg(seg + i) : ~0ull;
+        const bool hit = i < cnt && (v >> cur) == want;
         const unsigned mk = __ballot_sync(0xffffffffu, hit);
         if (mk == 0u) continue;
         const int leader = __ffs(mk) - 1;
-        unsigned long long b = 0ull;
-        if (lane == leader) b = atomicAdd(a.ccur + kAccTargets + t, (unsigned long long)__popc(mk));
-        b = __shfl_sync(0xffffffffu, b, leader);
-        const int64_t pos = (int64_t)b + __popc(mk & below_me);
+        unsigned long long bb = 0ull;
+        if (lane == leader) bb = atomicAdd(a.ccur + t, (unsigned long long)__popc(mk));
+        bb = __shfl_sync(0xffffffffu, bb, leader);
+        const int64_t pos = (int64_t)bb + __popc(mk & below_me);
         if (hit && pos < F.cnt[t]) a.cand2[F.base[t] + pos] = v;
       }
     }
-    if (!grid_barrier(a.bar, err)) return acc_left(a);
   }
+  if (!grid_barrier(a.bar, err)) return acc_left(a);
 
-  // ---- finish: block t ranks target t among its list's samples in the
-  // chosen second-digit bin (its final list, or its first-digit list filtered
-  // here); other blocks form the totals
+  // ---- finish: block t ranks target t's final list; other blocks form the
+  // totals
   uint64_t *pct = reinterpret_cast<uint64_t *>(a.res + 8);
   for (int t = blockIdx.x; t < kAccTargets; t += nb) {
     uint64_t r = 0ull;
-    if (L.pf[t] != ~0ull) {
-      if (direct) {
-        for (int i = tid; i < kSelBins; i += kAccBlock) sh[i] = __ldcg(a.hist2 + L.slot[t] * kSelBins + i);
-        __syncthreads();
-        if (wid == 0) {
-          int bin;
-          int64_t below, c2;
-          acc_pick1(sh, L.rk[t], bin, below, c2);
-          if (lane == 0) {
-            F.pf[t] = (L.pf[t] << kSelBits) | (uint64_t)bin;
-            F.rk[t] = L.rk[t] - below;
-            F.cnt[t] = c2;
-          }
-        }
-        __syncthreads();
-        r = acc_finish(a.cand + L.base[t], L.cnt[t], F.pf[t], L.shift - kSelBits, F.rk[t], F.cnt[t], sh);
-      } else {
-        const int s = F.slot[t];
-        r = acc_finish(a.cand2 + F.base[s], F.cnt[s], F.pf[t], L.shift - kSelBits, F.rk[t], F.cnt[s], sh);
-      }
+    if (F.pf[t] != ~0ull) {
+      const int s = F.slot[t];
+      r = acc_finish(a.cand2 + F.base[s], F.cnt[s], F.pf[t], L.shift - kSelBits, F.rk[t], F.cnt[s], sh);
     }
     if (tid == 0) pct[t] = r;
     __syncthreads();
