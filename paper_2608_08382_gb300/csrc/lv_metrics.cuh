@@ -93,31 +93,34 @@ __device__ __forceinline__ bool acc_is_sample(uint64_t b) {
 }
 
 // Grid-wide barrier of a cooperative launch (every block resident).  Thread 0
-// of each block arrives on bar[0]; the last arrival resets it and advances
-// the generation bar[1]; the others wait for the generation to move, for at
-// most about a second, after which they set the error word and go on.
-// Returns false once the error word is set (every block then leaves).
+// of each block arrives on bar[0] with release ordering (the block's earlier
+// writes become visible with it); the last arrival resets the count and
+// advances the generation bar[1]; the others wait, with acquire ordering, for
+// the generation to move, for at most about a second, after which they set
+// the error word and go on.  Returns false once the error word is set (every
+// block then leaves).
 __device__ __forceinline__ bool grid_barrier(unsigned int *bar, int *err) {
   __shared__ int ok;
   __syncthreads();
   if (threadIdx.x == 0) {
-    volatile unsigned int *gen = bar + 1;
-    const unsigned int g = *gen;  // read before arriving: it cannot move until this block arrives
-    __threadfence();
-    if (atomicAdd(bar, 1u) == gridDim.x - 1) {
-      atomicExch(bar, 0u);
-      __threadfence();
-      atomicAdd(bar + 1, 1u);
+    unsigned int g, old;
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(g) : "l"(bar + 1) : "memory");
+    asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], 1;" : "=r"(old) : "l"(bar) : "memory");
+    if (old == gridDim.x - 1) {
+      asm volatile("st.relaxed.gpu.global.u32 [%0], 0;" ::"l"(bar) : "memory");
+      asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(bar + 1) : "memory");
     } else {
-      for (long long k = 0; *gen == g; ++k) {
+      unsigned int now;
+      for (long long k = 0;; ++k) {
+        asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(now) : "l"(bar + 1) : "memory");
+        if (now != g) break;
         if (k > (1ll << 24)) {
           atomicExch(err, 1);
           break;
         }
-        __nanosleep(32);
+        __nanosleep(20);
       }
     }
-    __threadfence();
     ok = *(volatile int *)err == 0;
   }
   __syncthreads();
