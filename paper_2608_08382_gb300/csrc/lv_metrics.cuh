@@ -578,16 +578,16 @@ template <bool kNarrow>
 __device__ __forceinline__ void acc_exact_loop(const double *__restrict__ y, const double *__restrict__ T, int64_t lo,
                                                int64_t hi, int S, uint64_t *__restrict__ relbits, uint64_t *w,
                                                unsigned int *h1, const AccKey &K, double &srel, bool &lost) {
-  for (int64_t i0 = lo + threadIdx.x; i0 < hi; i0 += 2 * kAccBlock) {
-    uint64_t yb[2], tb[2];  // two elements' loads in flight (a pattern of 0 is not a sample)
+  for (int64_t i0 = lo + threadIdx.x; i0 < hi; i0 += 4 * kAccBlock) {
+    uint64_t yb[4], tb[4];  // four elements' loads in flight (a pattern of 0 is not a sample)
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
+    for (int k = 0; k < 4; ++k) {
       const int64_t i = i0 + k * kAccBlock;
       yb[k] = i < hi ? (uint64_t)__double_as_longlong(__ldg(y + i)) : 0ull;
       tb[k] = i < hi ? (uint64_t)__double_as_longlong(__ldg(T + i)) : 0ull;
     }
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
+    for (int k = 0; k < 4; ++k) {
       const int64_t i = i0 + k * kAccBlock;
       uint64_t rb = ~0ull;  // not a sample
       if (acc_is_sample(yb[k])) {
@@ -884,16 +884,16 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
   if (g0 < kAccTargets) a.ccur[g0] = 0ull;
   {
     unsigned int top = 0u, nmin = 0u;  // nmin: max of 2047 - biased exponent
-    for (int64_t i0 = g0; i0 < n; i0 += 4 * stride) {
-      uint2 yv[4], tv[4];  // four elements' loads in flight (a pattern of 0 is not a sample)
+    for (int64_t i0 = g0; i0 < n; i0 += 8 * stride) {
+      uint2 yv[8], tv[8];  // eight elements' loads in flight (a pattern of 0 is not a sample)
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
+      for (int k = 0; k < 8; ++k) {
         const int64_t i = i0 + k * stride;
         yv[k] = i < n ? __ldg(reinterpret_cast<const uint2 *>(a.y) + i) : make_uint2(0u, 0u);
         tv[k] = i < n ? __ldg(reinterpret_cast<const uint2 *>(a.T) + i) : make_uint2(0u, 0u);
       }
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
+      for (int k = 0; k < 8; ++k) {
         const unsigned int yh = yv[k].y, th = tv[k].y & 0x7FFFFFFFu;
         if ((int)yh > 0 || (yh == 0u && yv[k].x != 0u)) {
           top = max(top, max(yh, th));
