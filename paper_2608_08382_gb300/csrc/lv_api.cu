@@ -1041,8 +1041,10 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
     ctx->h_acc = static_cast<double *>(h);
     ctx->hd_acc = static_cast<double *>(d);
   }
+  constexpr size_t acc_dyn = kAccStage * sizeof(uint64_t);
   if (ctx->acc_occ == 0) {
-    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ, k_acc, kAccBlock, 0));
+    LV_CUDA(cudaFuncSetAttribute(k_acc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)acc_dyn));
+    LV_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ctx->acc_occ, k_acc, kAccBlock, acc_dyn));
     if (ctx->acc_occ <= 0) return LV_ECUDA;
   }
   // a cooperative launch: at most the blocks that fit at once, each looping over its share
@@ -1087,8 +1089,8 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   volatile double *h = ctx->h_acc;  // eight sums, three percentile bit patterns, error word
   *reinterpret_cast<volatile int *>(ctx->h_acc + 11) = 0;
   void *args[] = {&a};
-  LV_CUDA(cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(k_acc), dim3(blocks), dim3(kAccBlock), args, 0,
-                                      stream));
+  LV_CUDA(cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(k_acc), dim3(blocks), dim3(kAccBlock), args,
+                                      acc_dyn, stream));
   LV_CUDA(cudaStreamSynchronize(stream));
   if (*reinterpret_cast<volatile int *>(ctx->h_acc + 11)) {
     // a block waited out a barrier: reset the barrier and its error word for the next call

@@ -53,7 +53,7 @@ constexpr int kAccWords = 14;   // the exact sums of one block
 constexpr int kSelBits = 11;    // radix digit
 constexpr int kSelBins = 1 << kSelBits;
 constexpr int kAccBuf = kSelBins / 2;  // a block's buffered candidates per list
-constexpr int64_t kAccDirect = 1 << 15;  // first-digit lists a finishing block filters itself
+constexpr int kAccStage = 8192;  // a block's rel values kept in shared memory when its range fits
 constexpr int kAccGrid = 78;  // wide grid: S = kAccGrid - Emax puts every |v 2^S| below 2^79
 // Range of Emax for the exact path: within it the definition's own fp64
 // arithmetic (squared deviations, their products in r2_corr) neither overflows
@@ -571,13 +571,15 @@ struct AccSel {
 };
 
 // Exact pass over the block's range [lo, hi) of y and T on the narrow or
-// wide grid: the sums into w, rel's patterns into relbits, rel's first digit
+// wide grid: the sums into w, rel's patterns into `stage` (shared memory,
+// when the range fits there) or relbits, rel's first digit
 // into the block histogram h1 and rel into srel (fp64, in the thread's fixed
 // order); `lost` when a value is off the wide grid.
 template <bool kNarrow>
 __device__ __forceinline__ void acc_exact_loop(const double *__restrict__ y, const double *__restrict__ T, int64_t lo,
-                                               int64_t hi, int S, uint64_t *__restrict__ relbits, uint64_t *w,
-                                               unsigned int *h1, const AccKey &K, double &srel, bool &lost) {
+                                               int64_t hi, int S, uint64_t *__restrict__ relbits, uint64_t *stage,
+                                               uint64_t *w, unsigned int *h1, const AccKey &K, double &srel,
+                                               bool &lost) {
   for (int64_t i0 = lo + threadIdx.x; i0 < hi; i0 += 4 * kAccBlock) {
     uint64_t yb[4], tb[4];  // four elements' loads in flight (a pattern of 0 is not a sample)
 #pragma unroll
@@ -595,19 +597,26 @@ __device__ __forceinline__ void acc_exact_loop(const double *__restrict__ y, con
         atomicAdd(&h1[acc_key1(rb, K)], 1u);
         srel += __longlong_as_double((long long)rb);
       }
-      if (i < hi) relbits[i] = rb;
+      if (i < hi) {
+        if (stage)
+          stage[i - lo] = rb;
+        else
+          relbits[i] = rb;
+      }
     }
   }
 }
 
 // Counting sort of the block's samples by first digit: off = exclusive prefix
-// sums of the block histogram h1, then each sample of relbits[lo, hi) goes to
+// sums of the block histogram h1, then each sample of the block's range (from
+// `stage` when given, else relbits[lo, hi)) goes to
 // sorted[lo + off[key] + (its place among the block's samples of that key)]
 // (`cur`: kSelBins cursors of scratch).  Afterwards the samples of bin k lie
 // at sorted[lo + off[k], lo + off[k] + h1[k]).
-__device__ __forceinline__ void acc_block_sort(const uint64_t *__restrict__ relbits, uint64_t *__restrict__ sorted,
-                                               int64_t lo, int64_t hi, const unsigned int *h1, unsigned int *off,
-                                               unsigned int *cur, const AccKey &K) {
+__device__ __forceinline__ void acc_block_sort(const uint64_t *__restrict__ relbits, const uint64_t *stage,
+                                               uint64_t *__restrict__ sorted, int64_t lo, int64_t hi,
+                                               const unsigned int *h1, unsigned int *off, unsigned int *cur,
+                                               const AccKey &K) {
   __shared__ unsigned int wsum[kAccBlock / 32];
   constexpr int kPer = kSelBins / kAccBlock;  // bins per thread
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
@@ -635,13 +644,20 @@ __device__ __forceinline__ void acc_block_sort(const uint64_t *__restrict__ relb
     run += c[j];
   }
   __syncthreads();
-  for (int64_t i0 = lo + threadIdx.x; i0 < hi; i0 += 4 * kAccBlock) {
-    uint64_t v[4];  // four loads in flight
+  if (stage) {
+    for (int i = threadIdx.x; i < (int)(hi - lo); i += kAccBlock) {
+      const uint64_t v = stage[i];
+      if (v != ~0ull) sorted[lo + atomicAdd(&cur[acc_key1(v, K)], 1u)] = v;
+    }
+  } else {
+    for (int64_t i0 = lo + threadIdx.x; i0 < hi; i0 += 4 * kAccBlock) {
+      uint64_t v[4];  // four loads in flight
 #pragma unroll
-    for (int k = 0; k < 4; ++k) v[k] = i0 + k * kAccBlock < hi ? __ldcg(relbits + i0 + k * kAccBlock) : ~0ull;
+      for (int k = 0; k < 4; ++k) v[k] = i0 + k * kAccBlock < hi ? __ldcg(relbits + i0 + k * kAccBlock) : ~0ull;
 #pragma unroll
-    for (int k = 0; k < 4; ++k)
-      if (v[k] != ~0ull) sorted[lo + atomicAdd(&cur[acc_key1(v[k], K)], 1u)] = v[k];
+      for (int k = 0; k < 4; ++k)
+        if (v[k] != ~0ull) sorted[lo + atomicAdd(&cur[acc_key1(v[k], K)], 1u)] = v[k];
+    }
   }
   __syncthreads();
 }
@@ -857,6 +873,7 @@ __device__ __forceinline__ void acc_for_segment(const uint64_t *__restrict__ seg
 // The whole accuracy computation of one call; a cooperative launch of at
 // most as many blocks as fit at once.  Block b owns the elements [lo, hi).
 __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
+  extern __shared__ uint64_t stage_mem[];  // kAccStage patterns (dynamic): the block's rel values
   __shared__ __align__(16) unsigned int sh[kAccTargets * kSelBins];  // per-phase scratch
   __shared__ unsigned int bh1[kSelBins], bof1[kSelBins];  // the block's first-digit counts and offsets
   __shared__ unsigned long long red2[kAccBlock / 32 * 2];
@@ -946,12 +963,13 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
     for (int j = 0; j < kAccWords; ++j) w[j] = 0ull;
     double srel = 0.0;
     bool lost = false;
+    uint64_t *stage = hi - lo <= kAccStage ? stage_mem : nullptr;
     if (path[1])
-      acc_exact_loop<true>(a.y, a.T, lo, hi, path[2], a.relbits, w, bh1, K, srel, lost);
+      acc_exact_loop<true>(a.y, a.T, lo, hi, path[2], a.relbits, stage, w, bh1, K, srel, lost);
     else
-      acc_exact_loop<false>(a.y, a.T, lo, hi, path[2], a.relbits, w, bh1, K, srel, lost);
+      acc_exact_loop<false>(a.y, a.T, lo, hi, path[2], a.relbits, stage, w, bh1, K, srel, lost);
     const int anylost = __syncthreads_or(lost);
-    acc_block_sort(a.relbits, sorted, lo, hi, bh1, bof1, sh, K);
+    acc_block_sort(a.relbits, stage, sorted, lo, hi, bh1, bof1, sh, K);
     for (int i = tid; i < kSelBins; i += kAccBlock) {
       const unsigned int c = bh1[i];
       if (c) atomicAdd(a.hist1 + i, c);
@@ -998,7 +1016,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
       a.relbits[i] = bits;
     }
     __syncthreads();
-    acc_block_sort(a.relbits, sorted, lo, hi, bh1, bof1, sh, K);
+    acc_block_sort(a.relbits, nullptr, sorted, lo, hi, bh1, bof1, sh, K);
     for (int i = tid; i < kSelBins; i += kAccBlock) {
       const unsigned int h = bh1[i];
       if (h) atomicAdd(a.hist1 + kSelBins + i, h);

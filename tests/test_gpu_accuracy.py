@@ -225,3 +225,15 @@ def test_accuracy_select_list_sizes(lv, ctx, n):
     rel = np.where(first, 0.5 + rng.uniform(0.0, 2.0 ** -14, n), rng.uniform(0.52, 0.53, n))
     T = y * (1.0 + rel)
     _check_accuracy(lv.lv_accuracy(ctx, _dev(y), _dev(T)), oracle.accuracy(y, T))
+
+
+def test_accuracy_large_block_ranges(lv, ctx):
+    """3.2 million batches: each block's share of the exact pass is then more
+    than its shared-memory stage holds, so its relative errors go through
+    device memory on their way to the block's first-digit sort."""
+    rng = np.random.default_rng(77)
+    n = 3_200_000
+    T = rng.lognormal(-3.0, 0.6, n)
+    y = T * rng.lognormal(0.0, 0.1, n)
+    y[rng.random(n) < 0.02] = 0.0
+    _check_accuracy(lv.lv_accuracy(ctx, _dev(y), _dev(T)), oracle.accuracy(y, T))
