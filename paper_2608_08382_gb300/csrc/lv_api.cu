@@ -1060,7 +1060,8 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
                     o_out + 12 * sizeof(double) <= o_hist1 && o_hist2 + 4 * kAccTargets * kSelBins <= o_rel,
                 "accuracy scratch head");
   const size_t rel_bytes = ((size_t)n * sizeof(uint64_t) + 255) & ~(size_t)255;
-  const size_t o_cand = o_rel + rel_bytes, o_cand2 = o_cand + rel_bytes, o_part = o_cand2 + rel_bytes;
+  const size_t o_cand = o_rel + rel_bytes, o_cand2 = o_cand + rel_bytes, o_bucket = o_cand2 + rel_bytes;
+  const size_t o_part = o_bucket + sizeof(uint64_t) * kAccTargets * kSelBins * kAccBucket;
   const size_t need = o_part + sizeof(uint64_t) * kAccPartW * (size_t)blocks;
   if (need > ctx->acc_cap) {
     LV_CUDA(cudaDeviceSynchronize());
@@ -1079,6 +1080,7 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   a.relbits = reinterpret_cast<uint64_t *>(base + o_rel);
   a.cand = reinterpret_cast<uint64_t *>(base + o_cand);
   a.cand2 = reinterpret_cast<uint64_t *>(base + o_cand2);
+  a.bucket = reinterpret_cast<uint64_t *>(base + o_bucket);
   a.part = reinterpret_cast<uint64_t *>(base + o_part);
   a.res = ctx->hd_acc;
   a.err = reinterpret_cast<int *>(base + o_out);

@@ -54,6 +54,7 @@ constexpr int kSelBits = 11;    // radix digit
 constexpr int kSelBins = 1 << kSelBits;
 constexpr int kAccBuf = kSelBins / 2;  // a block's buffered candidates per list
 constexpr int kAccStage = 8192;  // a block's rel values kept in shared memory when its range fits
+constexpr int kAccBucket = 64;   // samples kept per second-digit bin
 constexpr int kAccGrid = 78;  // wide grid: S = kAccGrid - Emax puts every |v 2^S| below 2^79
 // Range of Emax for the exact path: within it the definition's own fp64
 // arithmetic (squared deviations, their products in r2_corr) neither overflows
@@ -78,6 +79,7 @@ struct AccArgs {
   uint64_t *relbits;          // n rel bit patterns (all ones: not a sample)
   uint64_t *cand;             // first-digit candidate lists, n patterns
   uint64_t *cand2;            // final candidate lists, n patterns
+  uint64_t *bucket;           // kAccTargets * kSelBins buckets of kAccBucket patterns
   uint64_t *part;             // kAccPartW words per block
   double *res;                // results (host memory, mapped): 8 sums, 3 patterns, error word
   int *err;                   // the barrier's error word (device memory)
@@ -1118,23 +1120,28 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
   }
 
   // ---- second digit: each block histograms the next 11 bits of its samples
-  // in the targets' first-digit bins (its sorted segments)
+  // in the targets' first-digit bins (its sorted segments), keeping each
+  // bin's first kAccBucket samples in a bucket
   {
     const int lo2 = L.shift - kSelBits;
     for (int t = 0; t < kAccTargets; ++t) {
       if (L.slot[t] != t || L.pf[t] == ~0ull) continue;  // the same in every block
       const int b = L.bin[t];
       unsigned int *h2 = a.hist2 + t * kSelBins;
+      uint64_t *bk = a.bucket + (int64_t)t * kSelBins * kAccBucket;
       acc_for_segment(sorted + lo + bof1[b], (int)bh1[b], [&](uint64_t v) {
-        atomicAdd(h2 + (int)((v >> lo2) & (uint64_t)(kSelBins - 1)), 1u);
+        const int d = (int)((v >> lo2) & (uint64_t)(kSelBins - 1));
+        const unsigned int p = atomicAdd(h2 + d, 1u);
+        if (p < kAccBucket) bk[d * kAccBucket + p] = v;  // the bin's first samples, kept for the finish
       });
     }
   }
   if (!grid_barrier(a.bar, err)) return acc_left(a);
 
-  // ---- each target's second digit (every block), then every block copies
-  // its samples in the chosen bin to the target's final list (targets whose
-  // prefixes coincide share one)
+  // ---- each target's second digit (every block); when a chosen bin holds
+  // more samples than its bucket kept, every block copies its samples in that
+  // bin to the target's final list (targets whose prefixes coincide share one)
+  bool gather = false;
   {
     for (int i = tid; i < kAccTargets * kSelBins; i += kAccBlock) sh[i] = __ldcg(a.hist2 + i);
     __syncthreads();
@@ -1162,6 +1169,9 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
       }
     }
     __syncthreads();
+    for (int t = 0; t < kAccTargets; ++t) gather |= F.pf[t] != ~0ull && F.cnt[t] > kAccBucket;
+  }
+  if (gather) {
     const int cur = L.shift - kSelBits;
     const unsigned below_me = (1u << lane) - 1u;
     for (int t = 0; t < kAccTargets; ++t) {
@@ -1183,8 +1193,8 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
         if (hit && pos < F.cnt[t]) a.cand2[F.base[t] + pos] = v;
       }
     }
+    if (!grid_barrier(a.bar, err)) return acc_left(a);
   }
-  if (!grid_barrier(a.bar, err)) return acc_left(a);
 
   // ---- finish: block t ranks target t's final list; other blocks form the
   // totals
@@ -1193,7 +1203,10 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
     uint64_t r = 0ull;
     if (F.pf[t] != ~0ull) {
       const int s = F.slot[t];
-      r = acc_finish(a.cand2 + F.base[s], F.cnt[s], F.pf[t], L.shift - kSelBits, F.rk[t], F.cnt[s], sh);
+      const uint64_t *list =
+          gather ? a.cand2 + F.base[s]
+                 : a.bucket + ((int64_t)L.slot[t] * kSelBins + (int64_t)(F.pf[t] & (kSelBins - 1))) * kAccBucket;
+      r = acc_finish(list, F.cnt[s], F.pf[t], L.shift - kSelBits, F.rk[t], F.cnt[s], sh);
     }
     if (tid == 0) pct[t] = r;
     __syncthreads();
