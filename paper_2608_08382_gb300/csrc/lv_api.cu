@@ -1054,14 +1054,13 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   // once at allocation, and every call leaves the barrier, cursors and
   // histograms at zero), then the relative errors' bit patterns, the
   // candidate lists and the block partials
-  constexpr size_t o_bar = 0, o_ccur = 64, o_out = 128, o_hist1 = 256, o_hist2 = o_hist1 + 8 * kSelBins,
+  constexpr size_t o_bar = 0, o_err = 64, o_lost = 68, o_hist1 = 256, o_hist2 = o_hist1 + 8 * kSelBins,
                    o_rel = 45056;
-  static_assert(o_ccur + 2 * kAccTargets * sizeof(unsigned long long) <= o_out &&
-                    o_out + 12 * sizeof(double) <= o_hist1 && o_hist2 + 4 * kAccTargets * kSelBins <= o_rel,
-                "accuracy scratch head");
+  static_assert(o_hist2 + 4 * kAccTargets * kSelBins <= o_rel, "accuracy scratch head");
   const size_t rel_bytes = ((size_t)n * sizeof(uint64_t) + 255) & ~(size_t)255;
-  const size_t o_cand = o_rel + rel_bytes, o_cand2 = o_cand + rel_bytes, o_bucket = o_cand2 + rel_bytes;
-  const size_t o_part = o_bucket + sizeof(uint64_t) * kAccTargets * kSelBins * kAccBucket;
+  const size_t o_sorted = o_rel + rel_bytes, o_bucket = o_sorted + rel_bytes;
+  const size_t o_segs = o_bucket + sizeof(uint64_t) * kAccTargets * kSelBins * kAccBucket;
+  const size_t o_part = o_segs + ((sizeof(uint64_t) * 2 * kAccTargets * (size_t)blocks + 255) & ~(size_t)255);
   const size_t need = o_part + sizeof(uint64_t) * kAccPartW * (size_t)blocks;
   if (need > ctx->acc_cap) {
     LV_CUDA(cudaDeviceSynchronize());
@@ -1078,15 +1077,15 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   a.T = T;
   a.n = n;
   a.relbits = reinterpret_cast<uint64_t *>(base + o_rel);
-  a.cand = reinterpret_cast<uint64_t *>(base + o_cand);
-  a.cand2 = reinterpret_cast<uint64_t *>(base + o_cand2);
+  a.cand = reinterpret_cast<uint64_t *>(base + o_sorted);
   a.bucket = reinterpret_cast<uint64_t *>(base + o_bucket);
+  a.segs = reinterpret_cast<uint64_t *>(base + o_segs);
   a.part = reinterpret_cast<uint64_t *>(base + o_part);
   a.res = ctx->hd_acc;
-  a.err = reinterpret_cast<int *>(base + o_out);
+  a.err = reinterpret_cast<int *>(base + o_err);
+  a.lost = reinterpret_cast<int *>(base + o_lost);
   a.hist1 = reinterpret_cast<unsigned int *>(base + o_hist1);
   a.hist2 = reinterpret_cast<unsigned int *>(base + o_hist2);
-  a.ccur = reinterpret_cast<unsigned long long *>(base + o_ccur);
   a.bar = reinterpret_cast<unsigned int *>(base + o_bar);
   volatile double *h = ctx->h_acc;  // eight sums, three percentile bit patterns, error word
   *reinterpret_cast<volatile int *>(ctx->h_acc + 11) = 0;
@@ -1097,7 +1096,7 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   if (*reinterpret_cast<volatile int *>(ctx->h_acc + 11)) {
     // a block waited out a barrier: reset the barrier and its error word for the next call
     LV_CUDA(cudaMemset(base + o_bar, 0, 8));
-    LV_CUDA(cudaMemset(base + o_out, 0, sizeof(int)));
+    LV_CUDA(cudaMemset(base + o_err, 0, sizeof(int)));
     return LV_ETIMEOUT;
   }
   const double m = h[0];

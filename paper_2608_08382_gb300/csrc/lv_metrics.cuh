@@ -63,11 +63,11 @@ constexpr int kAccGrid = 78;  // wide grid: S = kAccGrid - Emax puts every |v 2^
 constexpr int kAccEmaxLo = -160, kAccEmaxHi = 224;
 constexpr uint64_t kFracMask = (1ull << 52) - 1, kHiddenBit = 1ull << 52;
 
-// One block's partial, kAccPartW words: sample count, off-grid flag, rel sum
-// (fp64), the range maxima, the exact sums, the fp64 sums (count, sum y,
-// sum T) and the fp64 centred moments.
+// One block's partial, kAccPartW words: sample count, rel sum (fp64), the
+// range maxima, the exact sums, the fp64 sums (count, sum y, sum T) and the
+// fp64 centred moments.
 constexpr int kAccPartW = 32;
-constexpr int kPC = 0, kPL = 1, kPQ = 2, kPR = 4, kPX = 8, kPS = 22, kPM = 25;
+constexpr int kPC = 0, kPQ = 2, kPR = 4, kPX = 8, kPS = 22, kPM = 25;
 static_assert(kPX + kAccWords <= kPS && kPS + 3 <= kPM && kPM + 4 <= kAccPartW, "partial layout");
 
 // Device arguments of one call.  `res` receives the eight sums (m, -, -,
@@ -77,15 +77,15 @@ struct AccArgs {
   const double *y, *T;
   int64_t n;
   uint64_t *relbits;          // n rel bit patterns (all ones: not a sample)
-  uint64_t *cand;             // first-digit candidate lists, n patterns
-  uint64_t *cand2;            // final candidate lists, n patterns
+  uint64_t *cand;             // each block's samples sorted by first digit within its range, n patterns
+  uint64_t *segs;             // per block and first-digit slot: offset and length of its segment
   uint64_t *bucket;           // kAccTargets * kSelBins buckets of kAccBucket patterns
   uint64_t *part;             // kAccPartW words per block
   double *res;                // results (host memory, mapped): 8 sums, 3 patterns, error word
   int *err;                   // the barrier's error word (device memory)
+  int *lost;                  // set when a value is off the wide grid (device memory)
   unsigned int *hist1;        // 2 * kSelBins: first digit, exact pass then fp64 pass
   unsigned int *hist2;        // kAccTargets * kSelBins: the second digit
-  unsigned long long *ccur;   // 2 * kAccTargets list cursors (first-digit lists, final lists)
   unsigned int *bar;          // grid barrier: arrivals, generation (zero between calls)
 };
 
@@ -782,6 +782,81 @@ __device__ __forceinline__ double acc_fold_double(const uint64_t *part, int off,
   return block_sum_fixed(s, redd);
 }
 
+// The r-th smallest (1-based) of the samples whose bits above `cur` equal
+// `prefix`, c of them, found in the blocks' published segments of first-digit
+// slot s (segs: nb x kAccTargets pairs of offset into `sorted` and length).
+// By one block: at most kShort of them are gathered into shared memory and
+// ranked directly, more are settled digit by digit over the segments.
+__device__ uint64_t acc_finish_segs(const uint64_t *segs, const uint64_t *__restrict__ sorted, int nb, int s,
+                                    uint64_t prefix, int cur, int64_t r, int64_t c, unsigned int *sh) {
+  __shared__ uint64_t res;
+  __shared__ int nsel;
+  __shared__ int64_t pick[2];
+  constexpr int kShort = kAccTargets * kSelBins / 2;
+  auto each = [&](auto &&f) {  // every sample of the slot's segments, by the whole block
+    for (int b = 0; b < nb; ++b) {
+      const int64_t off = (int64_t)__ldcg(segs + 2 * (b * kAccTargets + s));
+      const int64_t cnt = (int64_t)__ldcg(segs + 2 * (b * kAccTargets + s) + 1);
+      for (int64_t i = threadIdx.x; i < cnt; i += kAccBlock) f(__ldcg(sorted + off + i));
+    }
+  };
+  if (c <= kShort) {
+    uint64_t *ls = reinterpret_cast<uint64_t *>(sh);
+    if (threadIdx.x == 0) {
+      nsel = 0;
+      res = 0ull;
+    }
+    __syncthreads();
+    each([&](uint64_t v) {
+      if ((v >> cur) == prefix) {
+        const int p = atomicAdd(&nsel, 1);
+        if (p < kShort) ls[p] = v;
+      }
+    });
+    __syncthreads();
+    const int k = min(nsel, kShort);
+    for (int i = threadIdx.x; i < k; i += kAccBlock) {
+      const uint64_t v = ls[i];
+      int64_t less = 0, leq = 0;
+      for (int j = 0; j < k; ++j) {
+        const uint64_t u = ls[j];
+        less += u < v ? 1 : 0;
+        leq += u <= v ? 1 : 0;
+      }
+      if (less < r && r <= leq) res = v;  // every finder holds the same value
+    }
+    __syncthreads();
+    const uint64_t out = res;
+    __syncthreads();
+    return out;
+  }
+  while (cur > 0) {
+    const int w = min(kSelBits, cur), lo = cur - w;
+    const uint64_t dmask = (1ull << w) - 1;
+    for (int i = threadIdx.x; i < kSelBins; i += kAccBlock) sh[i] = 0u;
+    __syncthreads();
+    each([&](uint64_t v) {
+      if ((v >> cur) == prefix) atomicAdd(&sh[(int)((v >> lo) & dmask)], 1u);
+    });
+    __syncthreads();
+    if (threadIdx.x < 32) {
+      int bin;
+      int64_t below, cnt;
+      acc_scan_pick<false>(sh, r, bin, below, cnt);
+      if (threadIdx.x == 0) {
+        pick[0] = bin;
+        pick[1] = below;
+      }
+    }
+    __syncthreads();
+    r -= pick[1];
+    prefix = (prefix << w) | (uint64_t)pick[0];
+    cur = lo;
+    __syncthreads();
+  }
+  return prefix;
+}
+
 // Exact totals to sums: fold the blocks' exact partials and write res[0] = m
 // and, scaled by m 2^(2S), res[3..6] = sxx, syy, sxy, ssr (one each on
 // threads 0..3).  One block.
@@ -881,7 +956,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
   __shared__ unsigned long long red2[kAccBlock / 32 * 2];
   __shared__ double redd[kAccBlock / 32];
   __shared__ uint64_t redw[kAccBlock / 32 * kAccWords];
-  __shared__ AccSel L, F;  // after the first digit; after the second
+  __shared__ AccSel L, F;  // after the first digit; after the second (finishing blocks)
   __shared__ AccKey K;
   __shared__ int path[3];  // exact, narrow, S
   __shared__ double mean[2];
@@ -900,7 +975,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
   // of the previous call are cleared here.
   for (int64_t i = g0; i < 2 * kSelBins; i += stride) a.hist1[i] = 0u;
   for (int64_t i = g0; i < kAccTargets * kSelBins; i += stride) a.hist2[i] = 0u;
-  if (g0 < kAccTargets) a.ccur[g0] = 0ull;
+  if (g0 == 0) *a.lost = 0;
   {
     unsigned int top = 0u, nmin = 0u;  // nmin: max of 2047 - biased exponent
     for (int64_t i0 = g0; i0 < n; i0 += 8 * stride) {
@@ -970,7 +1045,7 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
       acc_exact_loop<true>(a.y, a.T, lo, hi, path[2], a.relbits, stage, w, bh1, K, srel, lost);
     else
       acc_exact_loop<false>(a.y, a.T, lo, hi, path[2], a.relbits, stage, w, bh1, K, srel, lost);
-    const int anylost = __syncthreads_or(lost);
+    if (__syncthreads_or(lost) && tid == 0) atomicOr(a.lost, 1);
     acc_block_sort(a.relbits, stage, sorted, lo, hi, bh1, bof1, sh, K);
     for (int i = tid; i < kSelBins; i += kAccBlock) {
       const unsigned int c = bh1[i];
@@ -980,15 +1055,12 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
     acc_block_combine(w, redw);
     if (tid == 0) {
       mine[kPC] = w[0];
-      mine[kPL] = (uint64_t)anylost;
       mine[kPQ] = (uint64_t)__double_as_longlong(srel);
 #pragma unroll
       for (int j = 0; j < kAccWords; ++j) mine[kPX + j] = w[j];
     }
     if (!grid_barrier(a.bar, err)) return acc_left(a);
-    int off = 0;
-    for (int b = tid; b < nb; b += kAccBlock) off |= (int)__ldcg(all + (int64_t)b * kAccPartW + kPL);
-    fp64 = __syncthreads_or(off) != 0;  // a value off the wide grid: redo the call in fp64
+    fp64 = __ldcg(a.lost) != 0;  // a value off the wide grid: redo the call in fp64
   }
 
   // ---- fp64: rel and its first digit, the block's samples sorted by it,
@@ -1072,25 +1144,25 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
     if (!grid_barrier(a.bar, err)) return acc_left(a);
   }
 
-  // ---- first digit: sample count, then each target's bin (every block)
+  // ---- first digit: the sample count (the histogram's total), then each
+  // target's bin (every block)
   {
-    unsigned long long cnt = 0ull;
-    for (int b = tid; b < nb; b += kAccBlock) cnt += __ldcg(all + (int64_t)b * kAccPartW + kPC);
-#pragma unroll
-    for (int d = 16; d; d >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, d);
     const unsigned int *h1 = a.hist1 + (fp64 ? kSelBins : 0);
     for (int i = tid; i < kSelBins; i += kAccBlock) sh[i] = __ldcg(h1 + i);
     __syncthreads();
-    if (lane == 0) redw[wid] = cnt;
-    __syncthreads();
-    if (tid == 0) {
-      int64_t m = 0;
-      for (int v = 0; v < kAccBlock / 32; ++v) m += (int64_t)redw[v];
-      L.m = m;
-      L.shift = 52 - K.kbits;
-      for (int t = 0; t < kAccTargets; ++t) {
-        const int64_t q = t == 0 ? 50 : t == 1 ? 90 : 99;
-        L.rk[t] = (q * m + 99) / 100;
+    if (wid == 0) {
+      unsigned long long c = 0ull;
+      for (int i = lane; i < kSelBins; i += 32) c += sh[i];
+#pragma unroll
+      for (int d = 16; d; d >>= 1) c += __shfl_xor_sync(0xffffffffu, c, d);
+      if (lane == 0) {
+        const int64_t m = (int64_t)c;
+        L.m = m;
+        L.shift = 52 - K.kbits;
+        for (int t = 0; t < kAccTargets; ++t) {
+          const int64_t q = t == 0 ? 50 : t == 1 ? 90 : 99;
+          L.rk[t] = (q * m + 99) / 100;
+        }
       }
     }
     __syncthreads();
@@ -1121,7 +1193,8 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
 
   // ---- second digit: each block histograms the next 11 bits of its samples
   // in the targets' first-digit bins (its sorted segments), keeping each
-  // bin's first kAccBucket samples in a bucket
+  // bin's first kAccBucket samples in a bucket and publishing where its
+  // segments lie
   {
     const int lo2 = L.shift - kSelBits;
     for (int t = 0; t < kAccTargets; ++t) {
@@ -1134,79 +1207,41 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
         const unsigned int p = atomicAdd(h2 + d, 1u);
         if (p < kAccBucket) bk[d * kAccBucket + p] = v;  // the bin's first samples, kept for the finish
       });
+      if (tid == 0) {
+        a.segs[2 * (blockIdx.x * kAccTargets + t)] = (uint64_t)(lo + bof1[b]);
+        a.segs[2 * (blockIdx.x * kAccTargets + t) + 1] = bh1[b];
+      }
     }
   }
   if (!grid_barrier(a.bar, err)) return acc_left(a);
 
-  // ---- each target's second digit (every block); when a chosen bin holds
-  // more samples than its bucket kept, every block copies its samples in that
-  // bin to the target's final list (targets whose prefixes coincide share one)
-  bool gather = false;
-  {
-    for (int i = tid; i < kAccTargets * kSelBins; i += kAccBlock) sh[i] = __ldcg(a.hist2 + i);
-    __syncthreads();
-    int bin = 0;
-    int64_t below = 0, c2 = 0;
-    if (wid < kAccTargets && L.pf[wid] != ~0ull) acc_pick1(sh + L.slot[wid] * kSelBins, L.rk[wid], bin, below, c2);
-    if (wid < kAccTargets && lane == 0 && L.pf[wid] != ~0ull) {
-      F.pf[wid] = (L.pf[wid] << kSelBits) | (uint64_t)bin;
-      F.rk[wid] = L.rk[wid] - below;
-      F.cnt[wid] = c2;
-    }
-    __syncthreads();
-    if (tid == 0) {
-      int64_t base = 0;
-      for (int t = 0; t < kAccTargets; ++t) {
-        F.slot[t] = t;
-        if (L.pf[t] == ~0ull) {
-          F.pf[t] = ~0ull;
-          F.cnt[t] = 0;
-        }
-        for (int u = t - 1; u >= 0; --u)
-          if (F.pf[u] == F.pf[t]) F.slot[t] = F.slot[u];
-        F.base[t] = F.slot[t] == t ? base : F.base[F.slot[t]];
-        if (F.slot[t] == t) base += F.cnt[t];
-      }
-    }
-    __syncthreads();
-    for (int t = 0; t < kAccTargets; ++t) gather |= F.pf[t] != ~0ull && F.cnt[t] > kAccBucket;
-  }
-  if (gather) {
-    const int cur = L.shift - kSelBits;
-    const unsigned below_me = (1u << lane) - 1u;
-    for (int t = 0; t < kAccTargets; ++t) {
-      if (F.slot[t] != t || F.pf[t] == ~0ull) continue;  // the same in every block
-      const int b = L.bin[t], cnt = (int)bh1[b];
-      const uint64_t *seg = sorted + lo + bof1[b];
-      const uint64_t want = F.pf[t];
-      for (int i0 = 0; i0 < cnt; i0 += kAccBlock) {  // the same trip count in every thread
-        const int i = i0 + tid;
-        const uint64_t v = i < cnt ? __ldcg(seg + i) : ~0ull;
-        const bool hit = i < cnt && (v >> cur) == want;
-        const unsigned mk = __ballot_sync(0xffffffffu, hit);
-        if (mk == 0u) continue;
-        const int leader = __ffs(mk) - 1;
-        unsigned long long bb = 0ull;
-        if (lane == leader) bb = atomicAdd(a.ccur + t, (unsigned long long)__popc(mk));
-        bb = __shfl_sync(0xffffffffu, bb, leader);
-        const int64_t pos = (int64_t)bb + __popc(mk & below_me);
-        if (hit && pos < F.cnt[t]) a.cand2[F.base[t] + pos] = v;
-      }
-    }
-    if (!grid_barrier(a.bar, err)) return acc_left(a);
-  }
-
-  // ---- finish: block t ranks target t's final list; other blocks form the
-  // totals
+  // ---- finish: block t picks target t's second digit and ranks its
+  // candidates (from the bin's bucket, or from every block's segment when
+  // the bin outgrew its bucket); other blocks form the totals
   uint64_t *pct = reinterpret_cast<uint64_t *>(a.res + 8);
   for (int t = blockIdx.x; t < kAccTargets; t += nb) {
     uint64_t r = 0ull;
-    if (F.pf[t] != ~0ull) {
-      const int s = F.slot[t];
-      const uint64_t *list =
-          gather ? a.cand2 + F.base[s]
-                 : a.bucket + ((int64_t)L.slot[t] * kSelBins + (int64_t)(F.pf[t] & (kSelBins - 1))) * kAccBucket;
-      r = acc_finish(list, F.cnt[s], F.pf[t], L.shift - kSelBits, F.rk[t], F.cnt[s], sh);
+    if (L.pf[t] != ~0ull) {
+      const int s = L.slot[t];
+      for (int i = tid; i < kSelBins; i += kAccBlock) sh[i] = __ldcg(a.hist2 + s * kSelBins + i);
+      __syncthreads();
+      if (wid == 0) {
+        int bin;
+        int64_t below, c2;
+        acc_pick1(sh, L.rk[t], bin, below, c2);
+        if (lane == 0) {
+          F.pf[t] = (L.pf[t] << kSelBits) | (uint64_t)bin;
+          F.rk[t] = L.rk[t] - below;
+          F.cnt[t] = c2;
+        }
+      }
+      __syncthreads();
+      const int cur = L.shift - kSelBits;
+      if (F.cnt[t] <= kAccBucket)
+        r = acc_finish(a.bucket + ((int64_t)s * kSelBins + (int64_t)(F.pf[t] & (kSelBins - 1))) * kAccBucket,
+                       F.cnt[t], F.pf[t], cur, F.rk[t], F.cnt[t], sh);
+      else
+        r = acc_finish_segs(a.segs, sorted, nb, s, F.pf[t], cur, F.rk[t], F.cnt[t], sh);
     }
     if (tid == 0) pct[t] = r;
     __syncthreads();
