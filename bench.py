@@ -396,12 +396,15 @@ def _setup_acc(lv, ctx, w, stream):
         step()
 
     return dict(step=step, e2e_step=e2e_step, units=w.n_batch, unit="batches/s", metric=METRIC_ACC,
-                h2d=3 * 8 * w.n_batch, d2h=2 * 88, launches_per_step=2 * 10, kernel="accuracy", time_mask=0,
+                h2d=3 * 8 * w.n_batch, d2h=2 * 88, launches_per_step=2, kernel="k_acc", time_mask=0,
                 whole_step=True, timed="the whole step (two synchronous lv_accuracy calls), CUDA events",
                 bytes_per_launch=2 * 16.0 * w.n_batch, flush=True,
-                bytes_rule="16 B/batch (y, T) read once per model; the range pass's second read of y and T, the "
-                           "8 B/batch of relative-error bits written, and their re-reads by the select passes "
-                           "(11-bit digits, up to 6) are counted as overhead",
+                bytes_rule="16 B/batch (y, T) read once per model; the second read of y and T, the relative "
+                           "errors staged in shared memory, their per-block sort and the select's reads of the "
+                           "target bins are counted as overhead",
+                bound_note=("one cooperative kernel per call; its exact-sum phase is bound by the integer pipes "
+                            "(64- and 128-bit fixed-point products and an integer division per batch), not by "
+                            "HBM, so the fraction of the copy rate is reported for reference only"),
                 config={"n_batch": w.n_batch, "seed": w.seed,
                         "l2": "working set below L2 size: a 512 MB buffer is overwritten before every timed step, "
                               "outside the step's events",

@@ -7,9 +7,10 @@
 //             double, as fp64 arithmetic gives them), its mean and its
 //             nearest-rank p50, p90, p99 (the ceil(q m / 100)-th smallest).
 //
-// One cooperative kernel computes all of it; its phases are separated by a
-// grid-wide barrier, and after each barrier every block folds the small
-// per-block partials it needs itself (in a fixed order, so all blocks agree):
+// One cooperative kernel computes all of it.  Its phases are separated by a
+// grid-wide barrier; after one, every block derives what it needs from small
+// shared results itself (in the same order, so all blocks agree).  Block b
+// owns one contiguous range of the batches.
 //   range   the largest and smallest binary exponents Emax, Emin among the
 //           samples' y and non-zero T.  GB300 issues fp64 at 1/64 of the fp32
 //           rate, so when Emax is finite and moderate the sums are formed
@@ -22,21 +23,23 @@
 //             2 m sxy = m (sum Y^2 + sum T^2 - sum D^2) - 2 sum Y sum T,
 //             m ssr = m sum D^2
 //           follow exactly (all on the grid 2^(-2S), which both R^2 cancel);
-//           and rel by exact integer division.  A value off the wide grid
-//           sends the call to the fp64 phases.
+//           rel by exact integer division; the mean of rel as an fp64 sum in
+//           a fixed order.  A value off the wide grid sends the call to the
+//           fp64 phases.
 //   fp64    otherwise (a non-finite sample value, extreme magnitudes, a value
-//           off the grid): the same quantities in fp64, means first, then
-//           centred moments, each in a fixed order.
+//           off the grid): rel, means, then centred moments, each in a fixed
+//           order.
 //   select  the percentiles, exact: rel is a non-negative double, so its bit
 //           pattern orders like its value, and a most-significant-digit radix
 //           select finds the bit pattern of the element of each target rank.
-//           The first digit (the pattern's exponent and top mantissa bits) is
-//           histogrammed by the pass that forms rel; a second pass takes the
-//           next 11 bits of the samples in a target's first-digit bin
-//           (typically a small fraction) and copies those samples into a
-//           candidate list per target; one block per target then picks the
-//           second digit and finds the rank among the list's matching samples.
-//           The mean of rel is an fp64 sum in a fixed order.
+//           The pass that forms rel also histograms its first digit (exponent
+//           and top mantissa bits) and sorts each block's samples by it, so a
+//           target's first-digit bin is one short segment per block (typically
+//           well under 1% of the samples in all).  The next phase histograms
+//           the next 11 bits of those segments, keeping each second-digit bin's
+//           first samples in a bucket; the block of each target then picks its
+//           second digit and ranks the bin's samples (from the bucket, or the
+//           blocks' segments when the bin outgrew it).
 #pragma once
 
 #include <cstdint>
@@ -52,7 +55,6 @@ constexpr int kAccTargets = 3;  // p50, p90, p99
 constexpr int kAccWords = 14;   // the exact sums of one block
 constexpr int kSelBits = 11;    // radix digit
 constexpr int kSelBins = 1 << kSelBits;
-constexpr int kAccBuf = kSelBins / 2;  // a block's buffered candidates per list
 constexpr int kAccStage = 8192;  // a block's rel values kept in shared memory when its range fits
 constexpr int kAccBucket = 64;   // samples kept per second-digit bin
 constexpr int kAccGrid = 78;  // wide grid: S = kAccGrid - Emax puts every |v 2^S| below 2^79
@@ -170,12 +172,6 @@ __device__ __forceinline__ void block_max2(unsigned long long &a, unsigned long 
       a = max(a, red[2 * w]);
       b = max(b, red[2 * w + 1]);
     }
-}
-
-// Largest rel and largest ~rel (so zero is the identity of both).
-__device__ __forceinline__ void acc_note_rel(uint64_t rb, unsigned long long &rmax, unsigned long long &rnmax) {
-  rmax = max(rmax, (unsigned long long)rb);
-  rnmax = max(rnmax, (unsigned long long)~rb);
 }
 
 // ---------------------------------------------------------------- exact path
@@ -483,23 +479,10 @@ __device__ __forceinline__ double acc_i256_to_double(const uint64_t *wi, int e2,
 
 // ---------------------------------------------------------------- select helpers
 
-// rel (bit pattern v, finite, non-negative) on the grid 2^(bemax - 1123),
-// bemax the largest rel's biased exponent: below 2^101, truncated under the
-// grid (at most 2^-100 of the largest rel per term).
-__device__ __forceinline__ u128 acc_rel_fixed(uint64_t v, int bemax) {
-  const int be = (int)(v >> 52);
-  const uint64_t M = (v & kFracMask) | (be ? kHiddenBit : 0ull);
-  const int sv = (be ? be : 1) - bemax + 48;
-  return sv >= 0 ? (u128)M << sv : sv > -64 ? (u128)(M >> -sv) : (u128)0;
-}
-
-
-// One warp: the bin of a kSelBins-bin histogram that holds rank r (1-based),
-// the count below that bin and the bin's own count, valid in every lane.  Lane
-// l sums bins [64 l, 64 l + 64), a warp scan finds the lane whose range holds
-// r, then the same over that lane's bins two at a time.  kGlobal: the
-// histogram is in global memory, written by other blocks' atomics.
-template <bool kGlobal>
+// One warp: the bin of a kSelBins-bin histogram in shared memory that holds
+// rank r (1-based), the count below that bin and the bin's own count, valid in
+// every lane.  Lane l sums bins [64 l, 64 l + 64), a warp scan finds the lane
+// whose range holds r, then the same over that lane's bins two at a time.
 __device__ __forceinline__ void acc_scan_pick(const unsigned int *h, int64_t r, int &bin, int64_t &below,
                                               int64_t &cnt) {
   static_assert(kSelBins == 64 * 32, "64 bins per lane");
@@ -508,7 +491,7 @@ __device__ __forceinline__ void acc_scan_pick(const unsigned int *h, int64_t r, 
 #pragma unroll
   for (int j = 0; j < 16; ++j) {
     const uint4 *p = reinterpret_cast<const uint4 *>(h + 64 * lane + 4 * j);
-    const uint4 q = kGlobal ? __ldcg(p) : *p;
+    const uint4 q = *p;
     s += (int64_t)q.x + q.y + q.z + q.w;
   }
   int64_t inc = s;
@@ -521,7 +504,7 @@ __device__ __forceinline__ void acc_scan_pick(const unsigned int *h, int64_t r, 
   const int L = ball ? __ffs(ball) - 1 : 31;
   const int64_t bl = __shfl_sync(0xffffffffu, inc - s, L);
   const uint2 *p2 = reinterpret_cast<const uint2 *>(h + 64 * L + 2 * lane);
-  const uint2 pr = kGlobal ? __ldcg(p2) : *p2;
+  const uint2 pr = *p2;
   const int64_t ps = (int64_t)pr.x + pr.y;
   int64_t inc2 = ps;
 #pragma unroll
@@ -565,9 +548,8 @@ struct AccSel {
   uint64_t pf[kAccTargets];   // prefix after the first digit; ~0 once a target is settled at 0
   int bin[kAccTargets];       // its first-digit bin
   int64_t rk[kAccTargets];    // rank still to find below it
-  int64_t cnt[kAccTargets];   // samples in its first-digit bin (its list's length)
-  int64_t base[kAccTargets];  // list offset of its slot
-  int slot[kAccTargets];      // list shared by targets whose prefixes coincide
+  int64_t cnt[kAccTargets];   // samples in its bin
+  int slot[kAccTargets];      // histogram shared by targets whose prefixes coincide
   int shift;                  // bits below the first digit
   int64_t m;                  // samples
 };
@@ -664,37 +646,10 @@ __device__ __forceinline__ void acc_block_sort(const uint64_t *__restrict__ relb
   __syncthreads();
 }
 
-// Visit this block's share of the rel patterns in warp tiles of 256 (load k
-// of a warp reads 512 contiguous bytes; four loads in flight), then the tail.
-// Every lane of a warp runs the same number of iterations and visits, so the
-// visitor may use warp collectives.
-template <class F>
-__device__ __forceinline__ void acc_for_rel(const uint64_t *__restrict__ relbits, int64_t n, F &&visit) {
-  const int lane = threadIdx.x & 31;
-  const int64_t tiles = n >> 8, gw = blockIdx.x * (int64_t)(kAccBlock / 32) + (threadIdx.x >> 5);
-  const int64_t wstride = (int64_t)gridDim.x * (kAccBlock / 32);
-  const ulonglong2 *r2 = reinterpret_cast<const ulonglong2 *>(relbits);
-  for (int64_t t = gw; t < tiles; t += wstride) {
-    ulonglong2 q[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k) q[k] = __ldcg(r2 + 128 * t + 32 * k + lane);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      visit(q[k].x);
-      visit(q[k].y);
-    }
-  }
-  // the tail (fewer than 256): the first warp of each block takes a slice
-  const int64_t rest = n - 256 * tiles;
-  if (threadIdx.x < 32)
-    for (int64_t i = blockIdx.x * 32; i < rest; i += (int64_t)gridDim.x * 32)
-      visit(i + lane < rest ? __ldcg(relbits + 256 * tiles + i + lane) : ~0ull);
-}
-
 // Pick the digit of a histogram in shared memory (kSelBins bins) that holds
 // rank r: bin, count below it, its count.  One warp; valid in every lane.
 __device__ __forceinline__ void acc_pick1(const unsigned int *h, int64_t r, int &bin, int64_t &below, int64_t &cnt) {
-  acc_scan_pick<false>(h, r, bin, below, cnt);
+  acc_scan_pick(h, r, bin, below, cnt);
 }
 
 // The r-th smallest (1-based) of the samples in `list` (c patterns) whose
@@ -757,7 +712,7 @@ __device__ uint64_t acc_finish(const uint64_t *__restrict__ list, int64_t c, uin
     if (threadIdx.x < 32) {
       int bin;
       int64_t below, cnt;
-      acc_scan_pick<false>(sh, r, bin, below, cnt);
+      acc_scan_pick(sh, r, bin, below, cnt);
       if (threadIdx.x == 0) {
         pick[0] = bin;
         pick[1] = below;
@@ -842,7 +797,7 @@ __device__ uint64_t acc_finish_segs(const uint64_t *segs, const uint64_t *__rest
     if (threadIdx.x < 32) {
       int bin;
       int64_t below, cnt;
-      acc_scan_pick<false>(sh, r, bin, below, cnt);
+      acc_scan_pick(sh, r, bin, below, cnt);
       if (threadIdx.x == 0) {
         pick[0] = bin;
         pick[1] = below;
