@@ -153,6 +153,13 @@ const char *lv_status_string(lv_status s);
 #define LV_TIME_PAIRS 2
 lv_status lv_ctx_set_timing(lv_ctx *ctx, int32_t mask);
 lv_status lv_ctx_kernel_time(lv_ctx *ctx, double *ms, int64_t *launches);
+/* Failure-detection support (no counterpart in the paper): runs the grid-wide
+ * barrier that lv_accuracy's kernel uses in a cooperative launch of two blocks,
+ * one of which leaves without arriving, so that the other's bounded wait runs
+ * out.  Returns LV_ETIMEOUT after a few seconds when the bound works as
+ * designed (LV_OK would mean the barrier let a block through alone), with the
+ * context left usable.  Synchronises `stream`. */
+lv_status lv_ctx_selftest_barrier(lv_ctx *ctx, void *stream);
 
 /* Architecture constants (Section 2.1: features proportional to FLOPs and to
  * memory I/O).  With P_layer = d*hq*hd + 2*d*hkv*hd + hq*hd*d + 3*d*F:
@@ -269,7 +276,7 @@ lv_status lv_fit_vtc(lv_ctx *ctx, const lv_batches *b, const double *y, int32_t 
  * extreme) they are fp64 in a fixed order.  The mean relative error is an
  * fp64 sum in a fixed order.  Either way results repeat bit for bit.  n < 2^32
  * (LV_EINVAL otherwise).  One cooperative kernel launch: its blocks meet at
- * grid-wide barriers whose waits are bounded (about a second), after which the
+ * grid-wide barriers whose waits are bounded (a few seconds), after which the
  * call returns LV_ETIMEOUT.  rep: host.  With no sample every value is NaN and
  * n = 0; an R^2 whose denominator is 0 is NaN.  Synchronous. */
 lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, lv_accuracy_report *rep,

@@ -26,7 +26,7 @@ LV_TIME_TILES, LV_TIME_PAIRS = 1, 2
 
 EXPORTED = [
     "lv_status_string", "lv_arch_constants", "lv_ctx_create", "lv_ctx_destroy", "lv_ctx_set_arith", "lv_ctx_status",
-    "lv_ctx_set_timing", "lv_ctx_kernel_time",
+    "lv_ctx_set_timing", "lv_ctx_kernel_time", "lv_ctx_selftest_barrier",
     "lv_features", "lv_batch_latency", "lv_attribute", "lv_attribute_f32", "lv_tenant_acc_create", "lv_tenant_acc_destroy",
     "lv_tenant_acc_reset", "lv_tenant_accumulate", "lv_tenant_totals", "lv_tenant_acc_state_bytes",
     "lv_tenant_acc_export", "lv_tenant_acc_import", "lv_fit", "lv_fit_vtc", "lv_accuracy", "lv_whatif",
@@ -85,6 +85,7 @@ def _load():
         "lv_ctx_status": ([P, P], I32),
         "lv_ctx_set_timing": ([P, I32], I32),
         "lv_ctx_kernel_time": ([P, P, P], I32),
+        "lv_ctx_selftest_barrier": ([P, P], I32),
         "lv_features": ([P, P, P, P, P, P, P, P], I32),
         "lv_batch_latency": ([P, P, P, P, I64, P, P], I32),
         "lv_attribute": ([P, P, P, P, P, P, P], I32),
@@ -224,6 +225,10 @@ class Context:
         ms, n = ctypes.c_double(), ctypes.c_int64()
         _check(_lib.lv_ctx_kernel_time(self.h, ctypes.byref(ms), ctypes.byref(n)), "lv_ctx_kernel_time")
         return float(ms.value), int(n.value)
+
+    def selftest_barrier(self, stream=None) -> int:
+        """Status of the grid-barrier self-test: LV_ETIMEOUT when the bounded wait works."""
+        return int(_lib.lv_ctx_selftest_barrier(self.h, _stream(stream)))
 
     def status(self, stream=None) -> int:
         return int(_lib.lv_ctx_status(self.h, _stream(stream)))

@@ -49,6 +49,7 @@ struct lv_ctx {
   int acc_occ = 0;            // CTAs per SM of the accuracy kernel (0: not yet queried)
   double *h_acc = nullptr;    // accuracy results: pinned host memory the kernel writes (mapped)
   double *hd_acc = nullptr;   // its device address
+  void *d_probe = nullptr;    // barrier self-test: arrivals, generation, error word
   int timing = 0;  // LV_TIME_* mask
   std::vector<cudaEvent_t> tev;  // start/stop pairs
   size_t tev_used = 0;
@@ -665,6 +666,7 @@ void lv_ctx_destroy(lv_ctx *ctx) {
   if (ctx->d_wi) cudaFree(ctx->d_wi);
   if (ctx->d_acc) cudaFree(ctx->d_acc);
   if (ctx->h_acc) cudaFreeHost(ctx->h_acc);
+  if (ctx->d_probe) cudaFree(ctx->d_probe);
   if (ctx->ev_built) cudaEventDestroy(ctx->ev_built);
   if (ctx->ev_used) cudaEventDestroy(ctx->ev_used);
   for (cudaEvent_t e : ctx->tev) cudaEventDestroy(e);
@@ -1112,6 +1114,22 @@ lv_status lv_accuracy(lv_ctx *ctx, const double *y, const double *T, int64_t n, 
   rep->p90 = h[9];
   rep->p99 = h[10];
   return LV_OK;
+}
+
+lv_status lv_ctx_selftest_barrier(lv_ctx *ctx, void *stream_) {
+  if (!ctx) return LV_EINVAL;
+  cudaStream_t stream = (cudaStream_t)stream_;
+  if (!ctx->d_probe && cudaMalloc(&ctx->d_probe, 16) != cudaSuccess) return LV_ENOMEM;
+  LV_CUDA(cudaMemsetAsync(ctx->d_probe, 0, 16, stream));
+  unsigned int *bar = static_cast<unsigned int *>(ctx->d_probe);
+  int *err = reinterpret_cast<int *>(bar + 2);
+  void *args[] = {&bar, &err};
+  LV_CUDA(cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(k_barrier_probe), dim3(2), dim3(32), args, 0,
+                                      stream));
+  int h = 0;
+  LV_CUDA(cudaMemcpyAsync(&h, err, sizeof(int), cudaMemcpyDeviceToHost, stream));
+  LV_CUDA(cudaStreamSynchronize(stream));
+  return h ? LV_ETIMEOUT : LV_OK;
 }
 
 lv_status lv_whatif(lv_ctx *ctx, const lv_model *model, const lv_batches *cand, const int32_t *p_new,

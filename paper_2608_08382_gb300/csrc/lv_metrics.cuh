@@ -1220,6 +1220,13 @@ __global__ void __launch_bounds__(kAccBlock) k_acc(AccArgs a) {
   }
 }
 
+// Barrier self-test: the last block leaves without arriving, so the others'
+// wait at the barrier runs out and sets the error word.
+__global__ void k_barrier_probe(unsigned int *bar, int *err) {
+  if (blockIdx.x == gridDim.x - 1) return;
+  grid_barrier(bar, err);
+}
+
 // ---------------------------------------------------------------- token-count baseline
 //
 // The token-count baseline (VTC, compared against in Tables 1-2): one line

@@ -237,3 +237,16 @@ def test_accuracy_large_block_ranges(lv, ctx):
     y = T * rng.lognormal(0.0, 0.1, n)
     y[rng.random(n) < 0.02] = 0.0
     _check_accuracy(lv.lv_accuracy(ctx, _dev(y), _dev(T)), oracle.accuracy(y, T))
+
+
+def test_barrier_wait_is_bounded(lv, ctx):
+    """Failure detection without a fault: the accuracy kernel's grid barrier,
+    run with one block that never arrives, gives up after a few seconds and
+    reports LV_ETIMEOUT; the context stays usable."""
+    import time
+    t = time.perf_counter()
+    assert ctx.selftest_barrier() == lv.LV_ETIMEOUT
+    assert time.perf_counter() - t < 30.0
+    y = np.array([1.0, 2.0, 4.0])
+    T = np.array([1.5, 2.0, 3.0])
+    _check_accuracy(lv.lv_accuracy(ctx, _dev(y), _dev(T)), oracle.accuracy(y, T))
