@@ -100,7 +100,7 @@ __device__ __forceinline__ bool acc_is_sample(uint64_t b) {
 // of each block arrives on bar[0] with release ordering (the block's earlier
 // writes become visible with it); the last arrival resets the count and
 // advances the generation bar[1]; the others wait, with acquire ordering, for
-// the generation to move, for at most about a second, after which they set
+// the generation to move, for at most a few seconds, after which they set
 // the error word and go on.  Returns false once the error word is set (every
 // block then leaves).
 __device__ __forceinline__ bool grid_barrier(unsigned int *bar, int *err) {
