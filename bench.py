@@ -307,8 +307,8 @@ def _setup_attr(lv, ctx, w, stream, f32=False):
 
 
 def _setup_step(lv, ctx, w, stream):
-    """Step: one serving batch through a CUDA graph of lv_tenant_acc_reset + lv_attribute (T, shares, tenant
-    pass) + lv_tenant_totals, captured once on a side stream (after eager warm-up there) and replayed."""
+    """Step: one serving batch through a CUDA graph of lv_attribute_step (accumulator reset, T, shares, tenant
+    add, tenant totals), captured once on a side stream (after eager warm-up there) and replayed."""
     import torch
     b = lv.batches_to_device(w.p, w.c, w.phase, w.offsets, w.tenant, w.n_tenants)
     model = lv.make_model(w.coef, w.split)
@@ -318,9 +318,7 @@ def _setup_step(lv, ctx, w, stream):
     acc = lv.TenantAcc(ctx, w.n_tenants)
 
     def eager(st):
-        acc.reset(stream=st)
-        lv.lv_attribute(ctx, model, b, T, share, acc, stream=st)
-        lv.lv_tenant_totals(ctx, acc, L, stream=st)
+        lv.lv_attribute_step(ctx, model, b, T, share, acc, L, reset=True, stream=st)
 
     cs = torch.cuda.Stream()
     cs.wait_stream(torch.cuda.current_stream())
@@ -352,17 +350,18 @@ def _setup_step(lv, ctx, w, stream):
 
     return dict(step=step, e2e_step=e2e_step, units=w.n_req, unit="requests/s", metric=METRIC_STEP,
                 h2d=sum(int(t.numel() * t.element_size()) for t in hp.values()),
-                d2h=8 * (w.n_req + w.n_batch + w.n_tenants), launches_per_step=5,
+                d2h=8 * (w.n_req + w.n_batch + w.n_tenants), launches_per_step=1,
                 kernel="graph", time_mask=0, graph=True, whole_step=True, flush=True,
                 timed="the whole CUDA-graph replay, CUDA events on the launching stream",
                 bytes_per_launch=24.0 * w.n_req + 16.0 * w.n_batch,
-                bytes_rule="24 B/request + 16 B/batch over the whole replay (memsets, k_partition, k_warps, k_jumbo, "
-                           "k_tenant_fold, k_tenant_totals): a single batch is bound by launch latency, not HBM",
+                bytes_rule="24 B/request + 16 B/batch over the whole replay (one k_step launch: reads p, c, phase, "
+                            "tenant, writes the share; tenant state and totals are 40 B/tenant more): a single "
+                            "batch is bound by launch latency, not HBM",
                 config={"n_batch": w.n_batch, "n_req": w.n_req, "n_tenants": w.n_tenants, "seed": w.seed,
                         "l2": "working set below L2 size: a 512 MB buffer is overwritten before every timed step, "
                               "outside the step's events",
-                        "step": "CUDA-graph replay of lv_tenant_acc_reset + lv_attribute(T, shares, tenant pass) + "
-                                "lv_tenant_totals"})
+                        "step": "CUDA-graph replay of lv_attribute_step(T, shares, tenant pass, totals; "
+                                "accumulator reset)"})
 
 
 def _setup_acc(lv, ctx, w, stream):

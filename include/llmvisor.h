@@ -38,7 +38,8 @@
  *    fp64 outputs 8-byte aligned; otherwise LV_EINVAL.
  *  - One lv_ctx must not be used from two host threads at once.
  *  - CUDA graphs: lv_features, lv_batch_latency, lv_attribute,
- *    lv_tenant_acc_reset, lv_tenant_accumulate, lv_tenant_totals, lv_whatif
+ *    lv_attribute_step, lv_tenant_acc_reset, lv_tenant_accumulate,
+ *    lv_tenant_totals, lv_whatif
  *    and lv_whatif_admit may be captured into a CUDA graph once an uncaptured call with
  *    the same context, model and sizes has run (it creates the context's
  *    buffers and caches the kernel configuration; a capture never allocates).
@@ -226,6 +227,19 @@ lv_status lv_tenant_accumulate(lv_ctx *ctx, lv_tenant_acc *acc, const double *sh
                                int64_t n_req, void *stream);
 /* L double[n_tenants] (device): the current totals. */
 lv_status lv_tenant_totals(lv_ctx *ctx, lv_tenant_acc *acc, double *L, void *stream);
+/* One serving step (Section 2.1: attribution runs inside the scheduler, once
+ * per engine step): lv_attribute of the step's batches, then, with acc, the
+ * per-tenant totals, as lv_attribute followed by lv_tenant_totals would give
+ * them.  flags: 0 or LV_STEP_RESET, which starts acc from zero before the
+ * step's shares are added (the totals are then this step's alone).  L is
+ * double[n_tenants] (device) or NULL; L and LV_STEP_RESET need acc.  T, share,
+ * acc and the errors are as for lv_attribute; results are bit-identical to the
+ * separate calls.  A step of at most 4,096 requests in at most 16 batches,
+ * with at most 512 tenants, is one kernel launch (one thread-block cluster);
+ * larger inputs run the separate calls' kernels. */
+#define LV_STEP_RESET 1
+lv_status lv_attribute_step(lv_ctx *ctx, const lv_model *model, const lv_batches *b, double *T, double *share,
+                            lv_tenant_acc *acc, double *L, int32_t flags, void *stream);
 /* Checkpoint / resume: the exact state is n_tenants * 16 bytes (host buffer).
  * export synchronises the stream. */
 int64_t lv_tenant_acc_state_bytes(const lv_tenant_acc *acc);

@@ -23,11 +23,13 @@ LV_OK, LV_EINVAL, LV_EOVERFLOW, LV_ENODATA, LV_ESINGULAR, LV_ECUDA, LV_EDATA, LV
     0, -1, -2, -3, -4, -5, -6, -7, -8)
 LV_ARITH_AUTO, LV_ARITH_FP64 = 0, 1
 LV_TIME_TILES, LV_TIME_PAIRS = 1, 2
+LV_STEP_RESET = 1
 
 EXPORTED = [
     "lv_status_string", "lv_arch_constants", "lv_ctx_create", "lv_ctx_destroy", "lv_ctx_set_arith", "lv_ctx_status",
     "lv_ctx_set_timing", "lv_ctx_kernel_time", "lv_ctx_selftest_barrier",
-    "lv_features", "lv_batch_latency", "lv_attribute", "lv_attribute_f32", "lv_tenant_acc_create", "lv_tenant_acc_destroy",
+    "lv_features", "lv_batch_latency", "lv_attribute", "lv_attribute_f32", "lv_attribute_step",
+    "lv_tenant_acc_create", "lv_tenant_acc_destroy",
     "lv_tenant_acc_reset", "lv_tenant_accumulate", "lv_tenant_totals", "lv_tenant_acc_state_bytes",
     "lv_tenant_acc_export", "lv_tenant_acc_import", "lv_fit", "lv_fit_vtc", "lv_accuracy", "lv_whatif",
     "lv_whatif_admit", "lv_attribute_noalloc",
@@ -90,6 +92,7 @@ def _load():
         "lv_batch_latency": ([P, P, P, P, I64, P, P], I32),
         "lv_attribute": ([P, P, P, P, P, P, P], I32),
         "lv_attribute_f32": ([P, P, P, P, P, P, P], I32),
+        "lv_attribute_step": ([P, P, P, P, P, P, P, I32, P], I32),
         "lv_tenant_acc_create": ([P, I32, P], I32),
         "lv_tenant_acc_destroy": ([P], None),
         "lv_tenant_acc_reset": ([P, P], I32),
@@ -273,6 +276,15 @@ def lv_attribute(ctx: Context, model: lv_model, b: Batches, T=None, share=None, 
     bs = b.struct()
     _check(_lib.lv_attribute(ctx.h, ctypes.byref(model), ctypes.byref(bs), _ptr(T), _ptr(share),
                              acc.h if acc is not None else None, _stream(stream)), "lv_attribute")
+
+
+def lv_attribute_step(ctx: Context, model: lv_model, b: Batches, T=None, share=None, acc: "TenantAcc | None" = None,
+                      L=None, reset: bool = False, stream=None):
+    """One serving step: lv_attribute, then (with acc) the tenant totals into L; reset starts acc from zero."""
+    bs = b.struct()
+    _check(_lib.lv_attribute_step(ctx.h, ctypes.byref(model), ctypes.byref(bs), _ptr(T), _ptr(share),
+                                  acc.h if acc is not None else None, _ptr(L), LV_STEP_RESET if reset else 0,
+                                  _stream(stream)), "lv_attribute_step")
 
 
 def lv_attribute_f32(ctx: Context, model: lv_model, b: "Batches", T=None, share=None, acc: "TenantAcc | None" = None,

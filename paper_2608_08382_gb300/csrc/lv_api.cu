@@ -213,7 +213,8 @@ lv_status wait_event(cudaStream_t stream, cudaEvent_t ev) {
   return LV_OK;
 }
 
-lv_status prepare_model(lv_ctx *ctx, const lv_model *m, cudaStream_t stream, ModelP *mp) {
+// Per-model launch parameters, formed on the host (no K table).
+void model_params(const lv_ctx *ctx, const lv_model *m, ModelP *mp) {
   std::memset(mp, 0, sizeof(*mp));
   for (int s = 0; s < 4; ++s) {
     const lv_coef &k = m->seg[s >> 1][s & 1];
@@ -228,6 +229,10 @@ lv_status prepare_model(lv_ctx *ctx, const lv_model *m, cudaStream_t stream, Mod
   mp->nk = kKTableN;
   mp->fixed = 0;
   if (ctx->arith == LV_ARITH_AUTO) mp->fixed = derive_fixed(m, kKTableN, mp) ? 1 : 0;
+}
+
+lv_status prepare_model(lv_ctx *ctx, const lv_model *m, cudaStream_t stream, ModelP *mp) {
+  model_params(ctx, m, mp);
   if (!ctx->d_ktab) {
     if (cudaMalloc(&ctx->d_ktab, sizeof(KEntry) * 4 * (kKTableN + 1)) != cudaSuccess) return LV_ENOMEM;
   }
@@ -418,22 +423,69 @@ lv_status run_tiles(lv_ctx *ctx, TileArgs &a, int mode, cudaStream_t stream) {
   }
 }
 
-// The single-CTA path for small inputs (k_small); state: the tenant
-// accumulator's exact state, or null.
-lv_status run_small(lv_ctx *ctx, TileArgs &a, int mode, i128 *state, cudaStream_t stream) {
-  const size_t smem = sizeof(SmallSmem) + ((mode & M_TEN) ? ten_bytes(a.H) : 0);
+// The one-cluster path for small inputs (k_step); state: the tenant
+// accumulator's exact state, or null; L: the totals after the step, or null;
+// reset: the state is taken as zero.  The kernel forms every batch constant
+// itself, so it reads no K table.
+lv_status run_step(lv_ctx *ctx, TileArgs &a, int mode, i128 *state, double *L, int reset, cudaStream_t stream) {
+  a.mp.nk = 0;
+  a.mp.ktab = nullptr;
+  const size_t smem = sizeof(StepSmem) + ((mode & M_TEN) ? ten_bytes(a.H) : 0);
   cudaEvent_t stop = nullptr;
   lv_status st = timing_begin(ctx, LV_TIME_TILES, stream, &stop);
   if (st != LV_OK) return st;
   switch (mode) {
-    case M_ATTR: k_small<M_ATTR><<<1, kSmallThreads, smem, stream>>>(a, state); break;
-    case M_ATTR | M_FIX: k_small<M_ATTR | M_FIX><<<1, kSmallThreads, smem, stream>>>(a, state); break;
-    case M_ATTR | M_TEN: k_small<M_ATTR | M_TEN><<<1, kSmallThreads, smem, stream>>>(a, state); break;
-    case M_ATTR | M_TEN | M_FIX: k_small<M_ATTR | M_TEN | M_FIX><<<1, kSmallThreads, smem, stream>>>(a, state); break;
+    case M_ATTR: k_step<M_ATTR><<<kStepCtas, kStepThreads, smem, stream>>>(a, state, L, reset); break;
+    case M_ATTR | M_FIX: k_step<M_ATTR | M_FIX><<<kStepCtas, kStepThreads, smem, stream>>>(a, state, L, reset); break;
+    case M_ATTR | M_TEN: k_step<M_ATTR | M_TEN><<<kStepCtas, kStepThreads, smem, stream>>>(a, state, L, reset); break;
+    case M_ATTR | M_TEN | M_FIX:
+      k_step<M_ATTR | M_TEN | M_FIX><<<kStepCtas, kStepThreads, smem, stream>>>(a, state, L, reset);
+      break;
     default: return LV_EINVAL;
   }
   LV_CUDA(cudaGetLastError());
   return timing_end(stop, stream);
+}
+
+// Argument checks shared by lv_attribute and lv_attribute_step.
+lv_status attr_check(lv_ctx *ctx, const lv_model *model, const lv_batches *b, const double *T, const double *share,
+                     const lv_tenant_acc *acc) {
+  if (!ctx || check_model(model) != LV_OK) return LV_EINVAL;
+  lv_status st = check_batches(b, acc != nullptr);
+  if (st != LV_OK) return st;
+  if ((T && !aligned(T, 8)) || (share && !aligned(share, 8))) return LV_EINVAL;
+  if (acc && (acc->ctx != ctx || acc->n_tenants != b->n_tenants)) return LV_EINVAL;
+  return LV_OK;
+}
+
+// Launch arguments of an fp64 attribution and its kernel mode.
+TileArgs attr_args(lv_ctx *ctx, const lv_batches *b, double *T, double *share, lv_tenant_acc *acc, const ModelP &mp,
+                   int *mode) {
+  TileArgs a{};
+  a.p = b->p;
+  a.c = b->c;
+  a.ph = b->phase;
+  a.ten = acc ? b->tenant : nullptr;
+  a.off = b->offsets;
+  a.n_req = b->n_req;
+  a.n_batch = b->n_batch;
+  a.T = T;
+  a.share = share;
+  a.status = ctx->d_status;
+  a.mp = mp;
+  *mode = M_ATTR | (mp.fixed ? M_FIX : 0);
+  if (acc) {
+    *mode |= M_TEN;
+    a.ten_pend = acc->d_pend;
+    a.n_tenants = acc->n_tenants;
+    a.H = std::min<int32_t>(acc->n_tenants, kHotMax);
+  }
+  return a;
+}
+
+// Inputs the one-cluster kernel takes: one serving step.
+bool step_sized(const lv_batches *b) {
+  return b->n_req <= kSmallMaxReq && b->n_batch <= kSmallMaxBatch && b->n_batch > 0;
 }
 
 lv_status fold_tenants(lv_ctx *ctx, lv_tenant_acc *acc, cudaStream_t stream) {
@@ -777,52 +829,55 @@ lv_status lv_batch_latency(lv_ctx *ctx, const lv_model *model, const int64_t *ba
 
 lv_status lv_attribute(lv_ctx *ctx, const lv_model *model, const lv_batches *b, double *T, double *share,
                        lv_tenant_acc *acc, void *stream_) {
-  if (!ctx || check_model(model) != LV_OK) return LV_EINVAL;
-  lv_status st = check_batches(b, acc != nullptr);
+  lv_status st = attr_check(ctx, model, b, T, share, acc);
   if (st != LV_OK) return st;
-  if (T && !aligned(T, 8)) return LV_EINVAL;
-  if (share && !aligned(share, 8)) return LV_EINVAL;
   if (b->n_batch > 0 && !T && !share && !acc) return LV_OK;
-  if (acc && (acc->ctx != ctx || acc->n_tenants != b->n_tenants)) return LV_EINVAL;
-  if (b->n_batch > 0 && b->n_req > 0 && !share && !acc && !T) return LV_OK;
   cudaStream_t stream = (cudaStream_t)stream_;
   ModelP mp;
-  st = prepare_model(ctx, model, stream, &mp);
-  if (st != LV_OK) return st;
-  TileArgs a{};
-  a.p = b->p;
-  a.c = b->c;
-  a.ph = b->phase;
-  a.ten = acc ? b->tenant : nullptr;
-  a.off = b->offsets;
-  a.n_req = b->n_req;
-  a.n_batch = b->n_batch;
-  a.T = T;
-  a.share = share;
-  a.status = ctx->d_status;
-  a.mp = mp;
-  int mode = M_ATTR | (mp.fixed ? M_FIX : 0);
-  if (acc) {
-    mode |= M_TEN;
-    a.ten_pend = acc->d_pend;
-    a.n_tenants = acc->n_tenants;
-    a.H = std::min<int32_t>(acc->n_tenants, kHotMax);
-  }
-  if (b->n_req <= kSmallMaxReq && b->n_batch <= kSmallMaxBatch && b->n_batch > 0) {
-    // one serving step: a single CTA, no partition, scheduling counters or fold
-    st = run_small(ctx, a, mode, acc ? acc->d_state : nullptr, stream);
-    if (st != LV_OK) return st;
-    st = record_event(ctx->ev_used, stream);
+  int mode = 0;
+  if (step_sized(b)) {
+    // one serving step: a single cluster, no partition, scheduling counters or K table
+    model_params(ctx, model, &mp);
+    TileArgs a = attr_args(ctx, b, T, share, acc, mp, &mode);
+    st = run_step(ctx, a, mode, acc ? acc->d_state : nullptr, nullptr, 0, stream);
     if (st != LV_OK) return st;
     if (acc && acc->n_tenants > kHotMax) return fold_tenants(ctx, acc, stream);
     return LV_OK;
   }
+  st = prepare_model(ctx, model, stream, &mp);
+  if (st != LV_OK) return st;
+  TileArgs a = attr_args(ctx, b, T, share, acc, mp, &mode);
   st = run_tiles(ctx, a, mode, stream);
   if (st != LV_OK) return st;
   st = record_event(ctx->ev_used, stream);
   if (st != LV_OK) return st;
   if (acc) return fold_tenants(ctx, acc, stream);
   return LV_OK;
+}
+
+lv_status lv_attribute_step(lv_ctx *ctx, const lv_model *model, const lv_batches *b, double *T, double *share,
+                            lv_tenant_acc *acc, double *L, int32_t flags, void *stream_) {
+  if ((flags & ~LV_STEP_RESET) != 0 || (!acc && (L || (flags & LV_STEP_RESET))) || (L && !aligned(L, 8)))
+    return LV_EINVAL;
+  lv_status st = attr_check(ctx, model, b, T, share, acc);
+  if (st != LV_OK) return st;
+  const int reset = (flags & LV_STEP_RESET) ? 1 : 0;
+  if (step_sized(b) && (!acc || acc->n_tenants <= kHotMax)) {
+    if (!T && !share && !acc) return LV_OK;
+    // the whole step in one launch: attribution, tenant add and totals
+    ModelP mp;
+    model_params(ctx, model, &mp);
+    int mode = 0;
+    TileArgs a = attr_args(ctx, b, T, share, acc, mp, &mode);
+    return run_step(ctx, a, mode, acc ? acc->d_state : nullptr, L, reset, (cudaStream_t)stream_);
+  }
+  if (reset) {
+    st = lv_tenant_acc_reset(acc, stream_);
+    if (st != LV_OK) return st;
+  }
+  st = lv_attribute(ctx, model, b, T, share, acc, stream_);
+  if (st != LV_OK) return st;
+  return L ? lv_tenant_totals(ctx, acc, L, stream_) : LV_OK;
 }
 
 lv_status lv_attribute_f32(lv_ctx *ctx, const lv_model *model, const lv_batches *b, float *T, float *share,

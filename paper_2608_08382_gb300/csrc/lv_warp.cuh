@@ -24,6 +24,8 @@
 // All sums are exact integers, so results do not depend on this schedule.
 #pragma once
 
+#include <cooperative_groups.h>
+
 #include "lv_kernels.cuh"
 
 namespace lv {
@@ -1028,114 +1030,214 @@ __global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_bas
 
 // ---------------------------------------------------------------- small inputs
 
-// A serving scheduler attributes one step's batch (a few thousand requests) at
-// a time, where launch latency, not bandwidth, bounds the call.  For such
-// inputs lv_attribute runs this single CTA instead of the partition, tile,
-// jumbo and fold kernels: it takes the batches one after another, each with a
-// block-wide reduction, forms T and every share, and adds its shared-memory
-// tenant table straight into the exact per-tenant state (tenant ids from H up
-// still go to the pending limbs, which the caller folds).
-constexpr int kSmallThreads = 1024;
-constexpr int kSmallWarps = kSmallThreads / 32;
-constexpr int64_t kSmallMaxReq = 4096;
+// A serving scheduler attributes one step's batches (a few thousand requests)
+// at a time, where launch latency, not bandwidth, bounds the call.  For such
+// inputs lv_attribute and lv_attribute_step run this kernel instead of the
+// partition, tile, jumbo, fold and totals kernels: one cluster of kStepCtas
+// CTAs with one request per thread (CTA r takes the r-th contiguous share of
+// the requests), whose CTAs meet at three cluster barriers and read one
+// another's shared memory for the batch sums and the tenant tables.
+//   1. Every global read is issued at once: the thread's request, the offsets
+//      (warp 0 clamps them into non-decreasing batch bounds with a max-scan),
+//      and the state of the tenants this CTA folds.  Each CTA zeroes its own
+//      tenant table.
+//   2. Per-batch sums of the CTA's requests: a warp whose requests share one
+//      batch (the common case) adds its warp sum with one shared atomic per
+//      word, a warp that spans a batch bound adds lane by lane.  Meanwhile
+//      4 * n_batch threads form each batch's per-request constant for all four
+//      segments (it depends only on the batch's size).
+//   3. Cluster barrier.  One thread per batch adds the CTAs' partial sums
+//      through distributed shared memory, picks the segment and the constant,
+//      and CTA 0 writes T.
+//   4. Every thread attributes its request and adds its share into the CTA's
+//      exact tenant table.
+//   5. Cluster barrier.  CTA r folds its slice of the tenants: eight lanes per
+//      tenant read the tables of the cluster's CTAs and add them exactly; the
+//      tenant's state (zero on a reset) is added, stored and, when asked,
+//      converted to the correctly rounded total.
+//   6. Cluster barrier, so that no CTA leaves while another reads its table.
+// Tenant ids from H up still go to the pending limbs, which the caller folds.
+constexpr int kStepCtas = 8;
+constexpr int kStepThreads = 512;
+constexpr int64_t kSmallMaxReq = (int64_t)kStepCtas * kStepThreads;
 constexpr int64_t kSmallMaxBatch = 16;
+static_assert(kSmallMaxBatch < 32, "warp 0 scans the offsets");
+static_assert(kStepCtas == 8, "the fold adds eight tables with three shuffle steps");
+static_assert(kStepThreads >= 8 * ((kHotMax + kStepCtas - 1) / kStepCtas), "eight lanes per tenant of a slice");
 
-struct SmallSmem {
+struct StepSmem {
   alignas(16) SegS seg[4];
-  alignas(16) Sums red[kSmallWarps];
-  alignas(16) i128 kf;  // the current batch's per-request constant
-  int s, slow;
-  alignas(16) int64_t off[kSmallMaxBatch + 1];
+  alignas(16) i128 kf[kSmallMaxBatch][4];                // per-request constant, each batch and segment
+  alignas(16) i128 bk[kSmallMaxBatch];                   // the chosen segment's constant
+  alignas(16) unsigned long long sum[kSmallMaxBatch][4];  // this CTA's s1, s2, s3 and prefill count
+  alignas(16) int64_t cb[kSmallMaxBatch + 1];            // clamped batch bounds
+  int kslow[kSmallMaxBatch][4];
+  int bs[kSmallMaxBatch], bslow[kSmallMaxBatch];
+  int pad[2];
 };
-static_assert(sizeof(SmallSmem) % 16 == 0, "tenant table follows SmallSmem");
+static_assert(sizeof(StepSmem) % 16 == 0, "tenant table follows StepSmem");
 
-template <int MODE>
-__global__ void __launch_bounds__(kSmallThreads) k_small(const TileArgs a, i128 *state) {
-  extern __shared__ __align__(128) unsigned char smem_raw[];
-  SmallSmem &ss = *reinterpret_cast<SmallSmem *>(smem_raw);
-  uint32_t *tt = reinterpret_cast<uint32_t *>(smem_raw + sizeof(SmallSmem));
-  constexpr bool kTen = (MODE & M_TEN) != 0;
-  constexpr int kPer = (int)(kSmallMaxReq / kSmallThreads);  // requests per thread
-  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-  int bad = 0;
-  // every global read up front, independent of one another: this thread's
-  // requests (i = tid + k * kSmallThreads; every request lies in some batch of
-  // valid offsets), the offsets, and the state of the tenants it will fold
-  int32_t p[kPer], c[kPer], ph[kPer], u[kPer];
-#pragma unroll
-  for (int k = 0; k < kPer; ++k) {
-    const int64_t i = tid + (int64_t)k * kSmallThreads;
-    const bool in = i < a.n_req;
-    p[k] = in ? a.p[i] : 0;
-    c[k] = in ? a.c[i] : 0;
-    ph[k] = in ? a.ph[i] : 0;
-    u[k] = (kTen && in) ? a.ten[i] : 0;
+// Adds one request's fields into the shared per-batch sums: one atomic per
+// word from lane 0 when every active lane of the warp is in the same batch,
+// else one per lane.
+__device__ __forceinline__ void step_sums(StepSmem &ss, bool at, int b, int32_t p, int32_t c, int32_t ph, int lane) {
+  const unsigned am = __ballot_sync(kFull, at);
+  if (!am) return;
+  const int b0 = __shfl_sync(kFull, b, __ffs(am) - 1);
+  if (__all_sync(kFull, !at || b == b0)) {
+    Sums s{at ? p : 0, at ? c : 0, at ? (int64_t)p * p : 0, at ? ph : 0};
+    s = warp_sum(s);
+    if (lane == 0) {
+      atomicAdd(&ss.sum[b0][0], (unsigned long long)s.s1);
+      atomicAdd(&ss.sum[b0][1], (unsigned long long)s.s2);
+      atomicAdd(&ss.sum[b0][2], (unsigned long long)s.s3);
+      atomicAdd(&ss.sum[b0][3], (unsigned long long)s.ph);
+    }
+  } else if (at) {
+    atomicAdd(&ss.sum[b][0], (unsigned long long)p);
+    atomicAdd(&ss.sum[b][1], (unsigned long long)c);
+    atomicAdd(&ss.sum[b][2], (unsigned long long)((int64_t)p * p));
+    atomicAdd(&ss.sum[b][3], (unsigned long long)ph);
   }
-  if (tid <= a.n_batch) ss.off[tid] = a.off[tid];
+}
+
+// state: the tenant accumulator's exact state (with M_TEN); L: the tenants'
+// totals after this step, or null (then tenant ids may exceed H); reset: the
+// state is taken as zero.
+template <int MODE>
+__global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepThreads)
+    k_step(const TileArgs a, i128 *state, double *L, int reset) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  StepSmem &ss = *reinterpret_cast<StepSmem *>(smem_raw);
+  uint32_t *tt = reinterpret_cast<uint32_t *>(smem_raw + sizeof(StepSmem));
+  namespace cg = cooperative_groups;
+  cg::cluster_group cl = cg::this_cluster();
+  constexpr bool kTen = (MODE & M_TEN) != 0;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const int r = (int)cl.block_rank();
+  const int64_t nr = a.n_req, nb = a.n_batch;
+  int bad = 0;
+
+  // 1. reads
+  const int64_t chunk = (nr + kStepCtas - 1) / kStepCtas;
+  const int64_t i = r * chunk + tid;
+  const bool in = tid < chunk && i < nr;
+  int32_t p = 0, c = 0, ph = 0, u = 0;
+  if (in) {
+    p = a.p[i];
+    c = a.c[i];
+    ph = a.ph[i];
+    if (kTen) u = a.ten[i];
+  }
+  int64_t ob = 0;
+  if (wid == 0 && lane <= nb) ob = a.off[lane];
+  // the fold: lane q of tenant v of this CTA's slice reads CTA q's table
+  const int TS = kTen ? (a.H + kStepCtas - 1) / kStepCtas : 0;
+  const int v = r * TS + (tid >> 3), q = tid & 7;
+  const bool fv = kTen && (tid >> 3) < TS && v < a.H;
   i128 st0 = mk128(0, 0);
-  if (kTen && tid < a.H) st0 = state[tid];
+  if (fv && q == 0 && !reset) st0 = state[v];
   if (kTen)
-    for (int i = tid; i < 4 * ten_plane(a.H); i += kSmallThreads) tt[i] = 0;
+    for (int k = tid; k < 4 * ten_plane(a.H); k += kStepThreads) tt[k] = 0;
+  if (tid < 4 * kSmallMaxBatch) (&ss.sum[0][0])[tid] = 0ull;
   init_segs<MODE>(a, ss.seg);
+  if (in) check_req(p, c, ph, &bad);
+  if (wid == 0) {
+    // bound k = min(n_req, max(0, off[0..k])): batch b takes requests
+    // [cb[b], cb[b + 1]); valid offsets are their own bounds
+    int64_t m = lane <= nb ? max(ob, (int64_t)0) : 0;
 #pragma unroll
-  for (int k = 0; k < kPer; ++k) check_req(p[k], c[k], ph[k], &bad);
+    for (int d = 1; d < 32; d <<= 1) {
+      const int64_t o = __shfl_up_sync(kFull, m, d);
+      if (lane >= d) m = max(m, o);
+    }
+    m = min(m, nr);
+    if (lane <= nb) {
+      ss.cb[lane] = m;
+      if (r == 0 && (m != ob || (lane == 0 && ob != 0) || (lane == nb && ob != nr))) bad = 1;
+    }
+  }
   __syncthreads();
-  int64_t prev = 0;
-  for (int64_t b = 0; b < a.n_batch; ++b) {
-    const int64_t o0 = ss.off[b], o1 = ss.off[b + 1];
-    const int64_t r0 = clampi(o0, prev, a.n_req), r1 = clampi(o1, r0, a.n_req);
-    if (r0 != o0 || r1 != o1 || (b == 0 && o0 != 0) || (b == a.n_batch - 1 && o1 != a.n_req)) bad = 1;
-    prev = r1;
-    Sums acc{0, 0, 0, 0};
+
+  // 2. per-batch sums; each batch's constant for every segment
+  int b = 0;
+  for (int k = 1; k < nb; ++k) b += ss.cb[k] <= i ? 1 : 0;
+  const bool at = in && i >= ss.cb[0] && i < ss.cb[nb];
+  step_sums(ss, at, b, p, c, ph, lane);
+  if (tid < 4 * nb) {
+    const int kb = tid >> 2, s = tid & 3;
+    const int64_t n = ss.cb[kb + 1] - ss.cb[kb];
+    bool slow = false;
+    ss.kf[kb][s] = n > 0 ? batch_const_w<MODE>(a, nullptr, s, n, &slow) : mk128(0, 0);
+    ss.kslow[kb][s] = slow ? 1 : 0;
+  }
+
+  // 3. the batches' totals, segment, T and constant
+  cl.sync();
+  if (tid < nb) {
+    unsigned long long t[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-      const int64_t i = tid + (int64_t)k * kSmallThreads;
-      if (i >= r0 && i < r1) {
-        acc.s1 += p[k];
-        acc.s2 += c[k];
-        acc.s3 += (int64_t)p[k] * p[k];
-        acc.ph += ph[k];
+    for (int qq = 0; qq < kStepCtas; ++qq) {
+      const unsigned long long *rs = cl.map_shared_rank(&ss.sum[tid][0], qq);
+#pragma unroll
+      for (int w = 0; w < 4; ++w) t[w] += rs[w];
+    }
+    const BatchAgg g{(int64_t)t[0], (int64_t)t[1], (int64_t)t[2], ss.cb[tid + 1] - ss.cb[tid], t[3] > 0};
+    const int s = segment_of(a.mp, g);
+    if (r == 0) emit_batch<MODE>(a, tid, g, s, a.mp.fx);
+    ss.bs[tid] = s;
+    ss.bk[tid] = ss.kf[tid][s];
+    ss.bslow[tid] = ss.kslow[tid][s];
+  }
+  __syncthreads();
+
+  // 4. this thread's request
+  if (at) {
+    const int s = ss.bs[b];
+    const bool slow = ss.bslow[b] != 0;
+    const i128 kf = ss.bk[b];
+    const SegS sg = ss.seg[s];
+    bool done = false;
+    if ((MODE & M_FIX) && !slow && sg.a2_narrow && p == 1) {
+      // a decode request: the same exact steps as the warp-tile fast path
+      const i128 K13 = add128(kf, sg.A13);
+      uint32_t v0, v1, v2, v3;
+      mad_k13((uint32_t)K13.lo, (uint32_t)(K13.lo >> 32), (uint32_t)K13.hi, (uint32_t)(K13.hi >> 32),
+              (uint32_t)sg.A2.lo, (uint32_t)(sg.A2.lo >> 32), (uint32_t)c, v0, v1, v2, v3);
+      if (v3 == 0u && v2 != 0u) {
+        uint64_t m;
+        int ex2;
+        const double d = round96(v0, v1, v2, sg.E, m, ex2);
+        if (!kTen || tenant_fast(a, tt, u, m, ex2)) {
+          if (a.share) __stcs(a.share + i, d);
+          done = true;
+        }
       }
     }
-    acc = warp_sum(acc);
-    if (lane == 0) ss.red[wid] = acc;
-    __syncthreads();
-    if (tid == 0) {
-      // the batch's sums, segment, T and per-request constant, formed once
-      Sums t{0, 0, 0, 0};
-      for (int w = 0; w < kSmallWarps; ++w) t = add_sums(t, ss.red[w]);
-      const BatchAgg g{t.s1, t.s2, t.s3, r1 - r0, t.ph > 0};
-      const int s = segment_of(a.mp, g);
-      emit_batch<MODE>(a, b, g, s, a.mp.fx);
-      bool slow = false;
-      ss.kf = r1 > r0 ? batch_const_w<MODE>(a, nullptr, s, g.n, &slow) : mk128(0, 0);
-      ss.s = s;
-      ss.slow = slow ? 1 : 0;
-    }
-    __syncthreads();
-    const int s = ss.s;
-    const bool slow = ss.slow != 0;
-    const i128 kf = ss.kf;
-    const SegS sg = ss.seg[s];
-#pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-      const int64_t i = tid + (int64_t)k * kSmallThreads;
-      if (i >= r0 && i < r1) attribute_one<MODE>(a, tt, sg, s, slow, kf, r1 - r0, i, p[k], c[k], u[k], &bad);
-    }
-    __syncthreads();  // ss is rewritten for the next batch
+    if (!done) attribute_one<MODE>(a, tt, sg, s, slow, kf, ss.cb[b + 1] - ss.cb[b], i, p, c, u, &bad);
   }
   if (bad) flag(a.status, kStatusData);
+
+  // 5. the tenant tables into the exact state
   if (kTen) {
-    // the table into the exact state (this CTA is the only writer here)
-    for (int v0 = tid; v0 < a.H; v0 += kSmallThreads) {
-      const i128 v = hot_value(tt, a.H, v0);
-      if (!(v.lo | v.hi)) continue;
-      const i128 old = v0 == tid ? st0 : state[v0];
-      const i128 nw = add128(old, v);
-      if (is_neg128(old) == is_neg128(v) && is_neg128(nw) != is_neg128(old)) flag(a.status, kStatusData);
-      state[v0] = nw;
+    cl.sync();
+    i128 tv = mk128(0, 0);
+    if (fv) tv = hot_value(cl.map_shared_rank(tt, q), a.H, v);
+#pragma unroll
+    for (int d = 1; d < 8; d <<= 1) {
+      const uint64_t lo = __shfl_xor_sync(kFull, tv.lo, d), hi = __shfl_xor_sync(kFull, tv.hi, d);
+      tv = add128(tv, mk128(lo, hi));
+    }
+    if (fv && q == 0) {
+      const i128 nw = add128(st0, tv);
+      // overflow of the signed 128-bit total (|total| >= 2^127 * 2^-72 s)
+      if (is_neg128(st0) == is_neg128(tv) && is_neg128(nw) != is_neg128(st0)) flag(a.status, kStatusData);
+      if (reset || (tv.lo | tv.hi)) state[v] = nw;
+      if (L) L[v] = fix_to_double(nw, kTenLsb).d;
     }
   }
+  // 6. no CTA leaves while another may still read its shared memory
+  cl.sync();
 }
 
 }  // namespace lv
