@@ -66,7 +66,7 @@ typedef int32_t lv_status;
 #define LV_ECUDA (-5)      /* a CUDA runtime call failed */
 #define LV_EDATA (-6)      /* invalid input data seen on the device (sticky) */
 #define LV_ENOMEM (-7)     /* device allocation failed */
-#define LV_ETIMEOUT (-8)   /* a grid-wide barrier inside a kernel waited out its bound (lv_accuracy) */
+#define LV_ETIMEOUT (-8)   /* a bounded wait inside a kernel ran out (lv_accuracy, or lv_ctx_status after a serving-step launch) */
 
 /* Model architecture; integers only.  tp is the modelled tensor-parallel degree
  * (an arithmetic input: constants are per rank).  kv_bytes is the KV-cache

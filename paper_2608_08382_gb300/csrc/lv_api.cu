@@ -430,16 +430,19 @@ lv_status run_tiles(lv_ctx *ctx, TileArgs &a, int mode, cudaStream_t stream) {
 lv_status run_step(lv_ctx *ctx, TileArgs &a, int mode, i128 *state, double *L, int reset, cudaStream_t stream) {
   a.mp.nk = 0;
   a.mp.ktab = nullptr;
-  const size_t smem = sizeof(StepSmem) + ((mode & M_TEN) ? ten_bytes(a.H) : 0);
+  // shared memory: the kernel's fixed part, the tenant table and the received slice entries
+  const int slice = (a.H + kStepCtas - 1) / kStepCtas;
+  const size_t smem =
+      sizeof(StepSmem) + ((mode & M_TEN) ? ten_bytes(a.H) + sizeof(i128) * kStepCtas * (size_t)slice : 0);
   cudaEvent_t stop = nullptr;
   lv_status st = timing_begin(ctx, LV_TIME_TILES, stream, &stop);
   if (st != LV_OK) return st;
   switch (mode) {
-    case M_ATTR: k_step<M_ATTR><<<kStepCtas, kStepThreads, smem, stream>>>(a, state, L, reset); break;
-    case M_ATTR | M_FIX: k_step<M_ATTR | M_FIX><<<kStepCtas, kStepThreads, smem, stream>>>(a, state, L, reset); break;
-    case M_ATTR | M_TEN: k_step<M_ATTR | M_TEN><<<kStepCtas, kStepThreads, smem, stream>>>(a, state, L, reset); break;
+    case M_ATTR: k_step<M_ATTR><<<kStepCtas, kStepBlock, smem, stream>>>(a, state, L, reset); break;
+    case M_ATTR | M_FIX: k_step<M_ATTR | M_FIX><<<kStepCtas, kStepBlock, smem, stream>>>(a, state, L, reset); break;
+    case M_ATTR | M_TEN: k_step<M_ATTR | M_TEN><<<kStepCtas, kStepBlock, smem, stream>>>(a, state, L, reset); break;
     case M_ATTR | M_TEN | M_FIX:
-      k_step<M_ATTR | M_TEN | M_FIX><<<kStepCtas, kStepThreads, smem, stream>>>(a, state, L, reset);
+      k_step<M_ATTR | M_TEN | M_FIX><<<kStepCtas, kStepBlock, smem, stream>>>(a, state, L, reset);
       break;
     default: return LV_EINVAL;
   }
@@ -759,6 +762,7 @@ lv_status lv_ctx_status(lv_ctx *ctx, void *stream) {
   int h = 0;
   LV_CUDA(cudaMemcpy(&h, ctx->d_status, sizeof(int), cudaMemcpyDeviceToHost));
   LV_CUDA(cudaMemset(ctx->d_status, 0, sizeof(int)));
+  if (h & kStatusTimeout) return LV_ETIMEOUT;
   if (h & kStatusData) return LV_EDATA;
   return LV_OK;
 }

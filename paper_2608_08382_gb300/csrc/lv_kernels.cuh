@@ -21,6 +21,7 @@ constexpr int kTenLsb = -72;                       // tenant totals: shares roun
 // the exact range (bit 2 is reserved).
 constexpr int kStatusData = 1;
 constexpr int kStatusOverflow = 4;
+constexpr int kStatusTimeout = 8;  // a bounded wait inside a kernel ran out
 
 struct SegFix {
   i128 A1, A2, A3;   // exact a_k * 2^-E

@@ -1035,47 +1035,105 @@ __global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_bas
 // inputs lv_attribute and lv_attribute_step run this kernel instead of the
 // partition, tile, jumbo, fold and totals kernels: one cluster of kStepCtas
 // CTAs with one request per thread (CTA r takes the r-th contiguous share of
-// the requests), whose CTAs meet at three cluster barriers and read one
-// another's shared memory for the batch sums and the tenant tables.
-//   1. Every global read is issued at once: the thread's request, the offsets
-//      (warp 0 clamps them into non-decreasing batch bounds with a max-scan),
-//      and the state of the tenants this CTA folds.  Each CTA zeroes its own
-//      tenant table.
+// the requests) and one more warp per CTA for the batch constant.  The CTAs
+// exchange partial results by asynchronous stores into one another's shared
+// memory, each completing bytes on the receiver's transaction barrier, so no
+// step waits at a cluster-wide barrier.
+//   1. Thread 0 sets up the two receive barriers (the batch sums, the tenant
+//      slice), and the cluster's threads arrive once on the cluster barrier,
+//      which they wait for only before their first remote store.  Every global
+//      read is issued at once: the thread's request, the offsets (warp 0
+//      clamps them into non-decreasing batch bounds with a max-scan), and the
+//      state of the tenants this CTA folds; each CTA zeroes its tenant table.
+//      The constant warp meanwhile forms the per-request constant of a batch
+//      of n_req requests for all four segments (the single-batch step's).
 //   2. Per-batch sums of the CTA's requests: a warp whose requests share one
 //      batch (the common case) adds its warp sum with one shared atomic per
-//      word, a warp that spans a batch bound adds lane by lane.  Meanwhile
-//      4 * n_batch threads form each batch's per-request constant for all four
-//      segments (it depends only on the batch's size).
-//   3. Cluster barrier.  One thread per batch adds the CTAs' partial sums
-//      through distributed shared memory, picks the segment and the constant,
-//      and CTA 0 writes T.
+//      word, a warp that spans a batch bound adds lane by lane.  The sums go
+//      to every CTA of the cluster.
+//   3. One thread per batch adds the CTAs' partial sums as they arrive, picks
+//      the segment and the constant, and CTA 0 writes T.
 //   4. Every thread attributes its request and adds its share into the CTA's
 //      exact tenant table.
-//   5. Cluster barrier.  CTA r folds its slice of the tenants: eight lanes per
-//      tenant read the tables of the cluster's CTAs and add them exactly; the
-//      tenant's state (zero on a reset) is added, stored and, when asked,
-//      converted to the correctly rounded total.
-//   6. Cluster barrier, so that no CTA leaves while another reads its table.
-// Tenant ids from H up still go to the pending limbs, which the caller folds.
+//   5. Tenant u's table entry goes to the CTA that owns u's slice; there eight
+//      lanes per tenant add the cluster's entries exactly, and the tenant's
+//      state (zero on a reset) is added, stored and, when asked, converted to
+//      the correctly rounded total.
+// A CTA leaves only after every byte addressed to it has arrived.  Each wait
+// on a receive barrier is bounded (a few seconds); one that runs out records
+// a timeout in the status word.  Tenant ids from H up still go to the pending
+// limbs, which the caller folds.
 constexpr int kStepCtas = 8;
-constexpr int kStepThreads = 512;
+constexpr int kStepThreads = 512;                 // request threads
+constexpr int kStepBlock = kStepThreads + 32;     // and the constant warp
 constexpr int64_t kSmallMaxReq = (int64_t)kStepCtas * kStepThreads;
 constexpr int64_t kSmallMaxBatch = 16;
+constexpr int kStepSlice = (kHotMax + kStepCtas - 1) / kStepCtas;  // tenants a CTA folds, at most
 static_assert(kSmallMaxBatch < 32, "warp 0 scans the offsets");
-static_assert(kStepCtas == 8, "the fold adds eight tables with three shuffle steps");
-static_assert(kStepThreads >= 8 * ((kHotMax + kStepCtas - 1) / kStepCtas), "eight lanes per tenant of a slice");
+static_assert(kStepCtas == 8, "the fold adds eight entries with three shuffle steps");
+static_assert(kStepThreads >= 8 * kStepSlice, "eight lanes per tenant of a slice");
+static_assert(kStepThreads >= kStepCtas * kSmallMaxBatch * 4, "one remote store per thread sends the sums");
+static_assert(kStepThreads >= kHotMax, "one thread per tenant sends the table");
 
 struct StepSmem {
   alignas(16) SegS seg[4];
-  alignas(16) i128 kf[kSmallMaxBatch][4];                // per-request constant, each batch and segment
-  alignas(16) i128 bk[kSmallMaxBatch];                   // the chosen segment's constant
-  alignas(16) unsigned long long sum[kSmallMaxBatch][4];  // this CTA's s1, s2, s3 and prefill count
-  alignas(16) int64_t cb[kSmallMaxBatch + 1];            // clamped batch bounds
-  int kslow[kSmallMaxBatch][4];
+  alignas(16) i128 kspec[4];                                // constant of a batch of n_req requests, per segment
+  alignas(16) i128 bk[kSmallMaxBatch];                      // each batch's constant
+  alignas(16) unsigned long long sum[kSmallMaxBatch][4];     // this CTA's s1, s2, s3 and prefill count
+  alignas(16) unsigned long long rsum[kStepCtas][kSmallMaxBatch][4];  // every CTA's, as received
+  alignas(16) int64_t cb[kSmallMaxBatch + 1];               // clamped batch bounds
+  alignas(8) unsigned long long mbar[2];                    // receive barriers: sums, tenant slice
+  int kspec_slow[4];
   int bs[kSmallMaxBatch], bslow[kSmallMaxBatch];
-  int pad[2];
 };
-static_assert(sizeof(StepSmem) % 16 == 0, "tenant table follows StepSmem");
+static_assert(sizeof(StepSmem) % 16 == 0, "the tenant table follows StepSmem");
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+// The address of shared-memory address `a` in the CTA of cluster rank `rank`.
+__device__ __forceinline__ uint32_t peer_addr(uint32_t a, int rank) {
+  uint32_t d;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(rank));
+  return d;
+}
+
+// A receive barrier of one phase: one arrival (here) and `bytes` to come.
+__device__ __forceinline__ void rx_init(uint32_t mb, uint32_t bytes) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(mb) : "memory");
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(mb), "r"(bytes) : "memory");
+}
+
+// 8 or 16 bytes into a peer's shared memory, completing as many bytes on the
+// peer's barrier `rmb`.
+__device__ __forceinline__ void rx_put64(uint32_t raddr, uint64_t v, uint32_t rmb) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b64 [%0], %1, [%2];" ::"r"(raddr), "l"(v),
+               "r"(rmb)
+               : "memory");
+}
+__device__ __forceinline__ void rx_put128(uint32_t raddr, i128 v, uint32_t rmb) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+                   raddr),
+               "r"((uint32_t)v.lo), "r"((uint32_t)(v.lo >> 32)), "r"((uint32_t)v.hi), "r"((uint32_t)(v.hi >> 32)),
+               "r"(rmb)
+               : "memory");
+}
+
+// Waits for the receive barrier's first phase (bounded: false when it ran
+// out); what arrived is then visible to this thread.
+__device__ __forceinline__ bool rx_wait(uint32_t mb) {
+  for (long long k = 0; k < (1ll << 24); ++k) {
+    uint32_t done;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], 0;\n"
+        " selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(done)
+        : "r"(mb)
+        : "memory");
+    if (done) return true;
+    if (k > 64) __nanosleep(32);
+  }
+  return false;
+}
 
 // Adds one request's fields into the shared per-batch sums: one atomic per
 // word from lane 0 when every active lane of the warp is in the same batch,
@@ -1101,27 +1159,39 @@ __device__ __forceinline__ void step_sums(StepSmem &ss, bool at, int b, int32_t 
   }
 }
 
+// Barrier of the request threads alone (the constant warp does not wait).
+__device__ __forceinline__ void sync_requests() { asm volatile("bar.sync 1, %0;" ::"n"(kStepThreads) : "memory"); }
+
 // state: the tenant accumulator's exact state (with M_TEN); L: the tenants'
 // totals after this step, or null (then tenant ids may exceed H); reset: the
 // state is taken as zero.
 template <int MODE>
-__global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepThreads)
+__global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepBlock)
     k_step(const TileArgs a, i128 *state, double *L, int reset) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   StepSmem &ss = *reinterpret_cast<StepSmem *>(smem_raw);
   uint32_t *tt = reinterpret_cast<uint32_t *>(smem_raw + sizeof(StepSmem));
-  namespace cg = cooperative_groups;
-  cg::cluster_group cl = cg::this_cluster();
   constexpr bool kTen = (MODE & M_TEN) != 0;
+  const int TS = kTen ? (a.H + kStepCtas - 1) / kStepCtas : 0;  // tenants per slice
+  i128 *rt = reinterpret_cast<i128 *>(smem_raw + sizeof(StepSmem) + (kTen ? ten_bytes(a.H) : 0));  // [src][TS]
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-  const int r = (int)cl.block_rank();
+  const int r = (int)cooperative_groups::this_cluster().block_rank();
   const int64_t nr = a.n_req, nb = a.n_batch;
+  const bool req = tid < kStepThreads;
+  const uint32_t mb0 = smem_u32(&ss.mbar[0]), mb1 = smem_u32(&ss.mbar[1]);
   int bad = 0;
 
-  // 1. reads
+  // 1. receive barriers, reads, the single-batch constant
+  const int own = kTen ? max(0, min(TS, a.H - r * TS)) : 0;  // tenants of this CTA's slice
+  if (tid == 0) {
+    rx_init(mb0, (uint32_t)(kStepCtas * 32 * nb));
+    rx_init(mb1, (uint32_t)(kStepCtas * 16 * own));
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory");
   const int64_t chunk = (nr + kStepCtas - 1) / kStepCtas;
   const int64_t i = r * chunk + tid;
-  const bool in = tid < chunk && i < nr;
+  const bool in = req && tid < chunk && i < nr;
   int32_t p = 0, c = 0, ph = 0, u = 0;
   if (in) {
     p = a.p[i];
@@ -1131,68 +1201,85 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepThreads
   }
   int64_t ob = 0;
   if (wid == 0 && lane <= nb) ob = a.off[lane];
-  // the fold: lane q of tenant v of this CTA's slice reads CTA q's table
-  const int TS = kTen ? (a.H + kStepCtas - 1) / kStepCtas : 0;
-  const int v = r * TS + (tid >> 3), q = tid & 7;
-  const bool fv = kTen && (tid >> 3) < TS && v < a.H;
+  // the fold: lane q of tenant v of this CTA's slice takes CTA q's entry
+  const int jv = tid >> 3, q = tid & 7, v = r * TS + jv;
+  const bool fv = req && jv < own;
   i128 st0 = mk128(0, 0);
   if (fv && q == 0 && !reset) st0 = state[v];
-  if (kTen)
-    for (int k = tid; k < 4 * ten_plane(a.H); k += kStepThreads) tt[k] = 0;
-  if (tid < 4 * kSmallMaxBatch) (&ss.sum[0][0])[tid] = 0ull;
-  init_segs<MODE>(a, ss.seg);
-  if (in) check_req(p, c, ph, &bad);
-  if (wid == 0) {
-    // bound k = min(n_req, max(0, off[0..k])): batch b takes requests
-    // [cb[b], cb[b + 1]); valid offsets are their own bounds
-    int64_t m = lane <= nb ? max(ob, (int64_t)0) : 0;
+  if (!req) {
+    if (lane < 4) {
+      bool slow = false;
+      ss.kspec[lane] = nr > 0 ? batch_const_w<MODE>(a, nullptr, lane, nr, &slow) : mk128(0, 0);
+      ss.kspec_slow[lane] = slow ? 1 : 0;
+    }
+  } else {
+    if (kTen)
+      for (int k = tid; k < 4 * ten_plane(a.H); k += kStepThreads) tt[k] = 0;
+    if (tid < 4 * kSmallMaxBatch) (&ss.sum[0][0])[tid] = 0ull;
+    init_segs<MODE>(a, ss.seg);
+    if (in) check_req(p, c, ph, &bad);
+    if (wid == 0) {
+      // bound k = min(n_req, max(0, off[0..k])): batch b takes requests
+      // [cb[b], cb[b + 1]); valid offsets are their own bounds
+      int64_t m = lane <= nb ? max(ob, (int64_t)0) : 0;
 #pragma unroll
-    for (int d = 1; d < 32; d <<= 1) {
-      const int64_t o = __shfl_up_sync(kFull, m, d);
-      if (lane >= d) m = max(m, o);
+      for (int d = 1; d < 32; d <<= 1) {
+        const int64_t o = __shfl_up_sync(kFull, m, d);
+        if (lane >= d) m = max(m, o);
+      }
+      m = min(m, nr);
+      if (lane <= nb) {
+        ss.cb[lane] = m;
+        if (r == 0 && (m != ob || (lane == 0 && ob != 0) || (lane == nb && ob != nr))) bad = 1;
+      }
     }
-    m = min(m, nr);
-    if (lane <= nb) {
-      ss.cb[lane] = m;
-      if (r == 0 && (m != ob || (lane == 0 && ob != 0) || (lane == nb && ob != nr))) bad = 1;
+    sync_requests();
+
+    // 2. per-batch sums, sent to every CTA of the cluster
+    int b = 0;
+    for (int k = 1; k < nb; ++k) b += ss.cb[k] <= i ? 1 : 0;
+    const bool at = in && i >= ss.cb[0] && i < ss.cb[nb];
+    step_sums(ss, at, b, p, c, ph, lane);
+    sync_requests();
+    asm volatile("barrier.cluster.wait;" ::: "memory");  // the peers' receive barriers are set up
+    if (tid < kStepCtas * 4 * nb) {
+      const int dst = tid / (4 * (int)nb), k = tid % (4 * (int)nb);
+      rx_put64(peer_addr(smem_u32(&ss.rsum[r][k >> 2][k & 3]), dst), (&ss.sum[0][0])[k], peer_addr(mb0, dst));
     }
+    // each request thread keeps its batch index in p's place until step 4
+    ph = at ? b : -1;
   }
   __syncthreads();
 
-  // 2. per-batch sums; each batch's constant for every segment
-  int b = 0;
-  for (int k = 1; k < nb; ++k) b += ss.cb[k] <= i ? 1 : 0;
-  const bool at = in && i >= ss.cb[0] && i < ss.cb[nb];
-  step_sums(ss, at, b, p, c, ph, lane);
-  if (tid < 4 * nb) {
-    const int kb = tid >> 2, s = tid & 3;
-    const int64_t n = ss.cb[kb + 1] - ss.cb[kb];
-    bool slow = false;
-    ss.kf[kb][s] = n > 0 ? batch_const_w<MODE>(a, nullptr, s, n, &slow) : mk128(0, 0);
-    ss.kslow[kb][s] = slow ? 1 : 0;
-  }
-
   // 3. the batches' totals, segment, T and constant
-  cl.sync();
   if (tid < nb) {
+    if (!rx_wait(mb0)) flag(a.status, kStatusTimeout);
     unsigned long long t[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-    for (int qq = 0; qq < kStepCtas; ++qq) {
-      const unsigned long long *rs = cl.map_shared_rank(&ss.sum[tid][0], qq);
+    for (int src = 0; src < kStepCtas; ++src)
 #pragma unroll
-      for (int w = 0; w < 4; ++w) t[w] += rs[w];
-    }
-    const BatchAgg g{(int64_t)t[0], (int64_t)t[1], (int64_t)t[2], ss.cb[tid + 1] - ss.cb[tid], t[3] > 0};
+      for (int w = 0; w < 4; ++w) t[w] += ss.rsum[src][tid][w];
+    const int64_t n = ss.cb[tid + 1] - ss.cb[tid];
+    const BatchAgg g{(int64_t)t[0], (int64_t)t[1], (int64_t)t[2], n, t[3] > 0};
     const int s = segment_of(a.mp, g);
     if (r == 0) emit_batch<MODE>(a, tid, g, s, a.mp.fx);
+    bool slow = false;
+    i128 kf = mk128(0, 0);
+    if (n == nr) {
+      kf = ss.kspec[s];
+      slow = ss.kspec_slow[s] != 0;
+    } else if (n > 0) {
+      kf = batch_const_w<MODE>(a, nullptr, s, n, &slow);
+    }
     ss.bs[tid] = s;
-    ss.bk[tid] = ss.kf[tid][s];
-    ss.bslow[tid] = ss.kslow[tid][s];
+    ss.bk[tid] = kf;
+    ss.bslow[tid] = slow ? 1 : 0;
   }
   __syncthreads();
 
   // 4. this thread's request
-  if (at) {
+  if (req && ph >= 0) {
+    const int b = ph;
     const int s = ss.bs[b];
     const bool slow = ss.bslow[b] != 0;
     const i128 kf = ss.bk[b];
@@ -1218,11 +1305,19 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepThreads
   }
   if (bad) flag(a.status, kStatusData);
 
-  // 5. the tenant tables into the exact state
-  if (kTen) {
-    cl.sync();
+  // 5. each tenant's table entry to the CTA of its slice, then the fold there
+  if constexpr (kTen) {
+    __syncthreads();
+    if (tid < a.H) {
+      const int dst = tid / TS;
+      rx_put128(peer_addr(smem_u32(&rt[r * TS + (tid - dst * TS)]), dst), hot_value(tt, a.H, tid),
+                peer_addr(mb1, dst));
+    }
     i128 tv = mk128(0, 0);
-    if (fv) tv = hot_value(cl.map_shared_rank(tt, q), a.H, v);
+    if (fv) {
+      if (!rx_wait(mb1)) flag(a.status, kStatusTimeout);
+      tv = rt[q * TS + jv];
+    }
 #pragma unroll
     for (int d = 1; d < 8; d <<= 1) {
       const uint64_t lo = __shfl_xor_sync(kFull, tv.lo, d), hi = __shfl_xor_sync(kFull, tv.hi, d);
@@ -1236,8 +1331,6 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepThreads
       if (L) L[v] = fix_to_double(nw, kTenLsb).d;
     }
   }
-  // 6. no CTA leaves while another may still read its shared memory
-  cl.sync();
 }
 
 }  // namespace lv
