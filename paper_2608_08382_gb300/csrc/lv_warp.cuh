@@ -1048,15 +1048,15 @@ __global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_bas
 //      The constant warp meanwhile forms the per-request constant of a batch
 //      of n_req requests for all four segments (the single-batch step's).
 //   2. Per-batch sums of the CTA's requests: a warp whose requests share one
-//      batch (the common case) adds its warp sum with one shared atomic per
-//      word, a warp that spans a batch bound adds lane by lane.  The sums go
-//      to every CTA of the cluster.
-//   3. One thread per batch adds the CTAs' partial sums as they arrive, picks
-//      the segment and the constant, and CTA 0 writes T.
+//      batch (the common case) keeps its warp sums (hardware reductions when
+//      they fit 31 bits), a warp that spans a batch bound adds lane by lane
+//      with shared atomics.  The CTA's sums go to every CTA of the cluster.
+//   3. One thread per batch adds the CTAs' partial sums as they arrive and
+//      picks the segment and the constant.
 //   4. Every thread attributes its request and adds its share into the CTA's
-//      exact tenant table.
-//   5. Tenant u's table entry goes to the CTA that owns u's slice; there eight
-//      lanes per tenant add the cluster's entries exactly, and the tenant's
+//      exact tenant table; the constant warp of CTA 0 writes T.
+//   5. Tenant u's table entry goes to the CTA that owns u's slice; there one
+//      thread per tenant adds the cluster's entries exactly, and the tenant's
 //      state (zero on a reset) is added, stored and, when asked, converted to
 //      the correctly rounded total.
 // A CTA leaves only after every byte addressed to it has arrived.  Each wait
@@ -1070,8 +1070,7 @@ constexpr int64_t kSmallMaxReq = (int64_t)kStepCtas * kStepThreads;
 constexpr int64_t kSmallMaxBatch = 16;
 constexpr int kStepSlice = (kHotMax + kStepCtas - 1) / kStepCtas;  // tenants a CTA folds, at most
 static_assert(kSmallMaxBatch < 32, "warp 0 scans the offsets");
-static_assert(kStepCtas == 8, "the fold adds eight entries with three shuffle steps");
-static_assert(kStepThreads >= 8 * kStepSlice, "eight lanes per tenant of a slice");
+static_assert(kStepThreads >= kStepSlice, "one thread per tenant of a slice");
 static_assert(kStepThreads >= kStepCtas * kSmallMaxBatch * 4, "one remote store per thread sends the sums");
 static_assert(kStepThreads >= kHotMax, "one thread per tenant sends the table");
 
@@ -1079,12 +1078,16 @@ struct StepSmem {
   alignas(16) SegS seg[4];
   alignas(16) i128 kspec[4];                                // constant of a batch of n_req requests, per segment
   alignas(16) i128 bk[kSmallMaxBatch];                      // each batch's constant
-  alignas(16) unsigned long long sum[kSmallMaxBatch][4];     // this CTA's s1, s2, s3 and prefill count
+  alignas(16) unsigned long long sum[kSmallMaxBatch][4];     // requests of warps that span a batch bound
+  alignas(16) unsigned long long wsum[kStepThreads / 32][4];  // each warp's sums (warps within one batch)
   alignas(16) unsigned long long rsum[kStepCtas][kSmallMaxBatch][4];  // every CTA's, as received
   alignas(16) int64_t cb[kSmallMaxBatch + 1];               // clamped batch bounds
   alignas(8) unsigned long long mbar[2];                    // receive barriers: sums, tenant slice
+  alignas(16) BatchAgg agg[kSmallMaxBatch];                 // each batch's totals
   int kspec_slow[4];
   int bs[kSmallMaxBatch], bslow[kSmallMaxBatch];
+  int wb[kStepThreads / 32];                                // batch of warp wsum[w], or -1
+  int pad[3];
 };
 static_assert(sizeof(StepSmem) % 16 == 0, "the tenant table follows StepSmem");
 
@@ -1135,27 +1138,42 @@ __device__ __forceinline__ bool rx_wait(uint32_t mb) {
   return false;
 }
 
-// Adds one request's fields into the shared per-batch sums: one atomic per
-// word from lane 0 when every active lane of the warp is in the same batch,
-// else one per lane.
-__device__ __forceinline__ void step_sums(StepSmem &ss, bool at, int b, int32_t p, int32_t c, int32_t ph, int lane) {
+// This warp's contribution to the per-batch sums: when every active lane is
+// in one batch (the common case), the warp's sums go to wsum[warp] (four
+// hardware reductions when every sum fits 31 bits); otherwise each lane adds
+// its fields to sum[its batch] with shared atomics.
+__device__ __forceinline__ void step_sums(StepSmem &ss, bool at, int b, int32_t p, int32_t c, int32_t ph, int lane,
+                                          int wid) {
   const unsigned am = __ballot_sync(kFull, at);
-  if (!am) return;
-  const int b0 = __shfl_sync(kFull, b, __ffs(am) - 1);
+  const int b0 = am ? __shfl_sync(kFull, b, __ffs(am) - 1) : -1;
   if (__all_sync(kFull, !at || b == b0)) {
-    Sums s{at ? p : 0, at ? c : 0, at ? (int64_t)p * p : 0, at ? ph : 0};
-    s = warp_sum(s);
-    if (lane == 0) {
-      atomicAdd(&ss.sum[b0][0], (unsigned long long)s.s1);
-      atomicAdd(&ss.sum[b0][1], (unsigned long long)s.s2);
-      atomicAdd(&ss.sum[b0][2], (unsigned long long)s.s3);
-      atomicAdd(&ss.sum[b0][3], (unsigned long long)s.ph);
+    unsigned long long w[4];
+    if (__all_sync(kFull, (uint32_t)p < (1u << 13) && (uint32_t)c < (1u << 26))) {
+      w[0] = __reduce_add_sync(kFull, at ? (uint32_t)p : 0u);
+      w[1] = __reduce_add_sync(kFull, at ? (uint32_t)c : 0u);
+      w[2] = __reduce_add_sync(kFull, at ? (uint32_t)(p * p) : 0u);
+      w[3] = __reduce_add_sync(kFull, at ? (uint32_t)ph : 0u);
+    } else {
+      Sums v{at ? p : 0, at ? c : 0, at ? (int64_t)p * p : 0, at ? ph : 0};
+      v = warp_sum(v);
+      w[0] = (unsigned long long)v.s1;
+      w[1] = (unsigned long long)v.s2;
+      w[2] = (unsigned long long)v.s3;
+      w[3] = (unsigned long long)v.ph;
     }
-  } else if (at) {
-    atomicAdd(&ss.sum[b][0], (unsigned long long)p);
-    atomicAdd(&ss.sum[b][1], (unsigned long long)c);
-    atomicAdd(&ss.sum[b][2], (unsigned long long)((int64_t)p * p));
-    atomicAdd(&ss.sum[b][3], (unsigned long long)ph);
+    if (lane == 0) {
+      ss.wb[wid] = b0;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) ss.wsum[wid][k] = w[k];
+    }
+  } else {
+    if (lane == 0) ss.wb[wid] = -1;
+    if (at) {
+      atomicAdd(&ss.sum[b][0], (unsigned long long)p);
+      atomicAdd(&ss.sum[b][1], (unsigned long long)c);
+      atomicAdd(&ss.sum[b][2], (unsigned long long)((int64_t)p * p));
+      atomicAdd(&ss.sum[b][3], (unsigned long long)ph);
+    }
   }
 }
 
@@ -1201,11 +1219,11 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepBlock)
   }
   int64_t ob = 0;
   if (wid == 0 && lane <= nb) ob = a.off[lane];
-  // the fold: lane q of tenant v of this CTA's slice takes CTA q's entry
-  const int jv = tid >> 3, q = tid & 7, v = r * TS + jv;
-  const bool fv = req && jv < own;
+  // the fold: thread j takes tenant r * TS + j of this CTA's slice
+  const int v = r * TS + tid;
+  const bool fv = tid < own;
   i128 st0 = mk128(0, 0);
-  if (fv && q == 0 && !reset) st0 = state[v];
+  if (fv && !reset) st0 = state[v];
   if (!req) {
     if (lane < 4) {
       bool slow = false;
@@ -1239,12 +1257,16 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepBlock)
     int b = 0;
     for (int k = 1; k < nb; ++k) b += ss.cb[k] <= i ? 1 : 0;
     const bool at = in && i >= ss.cb[0] && i < ss.cb[nb];
-    step_sums(ss, at, b, p, c, ph, lane);
+    step_sums(ss, at, b, p, c, ph, lane, wid);
     sync_requests();
     asm volatile("barrier.cluster.wait;" ::: "memory");  // the peers' receive barriers are set up
     if (tid < kStepCtas * 4 * nb) {
-      const int dst = tid / (4 * (int)nb), k = tid % (4 * (int)nb);
-      rx_put64(peer_addr(smem_u32(&ss.rsum[r][k >> 2][k & 3]), dst), (&ss.sum[0][0])[k], peer_addr(mb0, dst));
+      // word k of the CTA's batch sums (batch k / 4), to CTA dst
+      const int dst = tid / (4 * (int)nb), k = tid % (4 * (int)nb), kb = k >> 2, kw = k & 3;
+      unsigned long long x = ss.sum[kb][kw];
+#pragma unroll
+      for (int j = 0; j < kStepThreads / 32; ++j) x += ss.wb[j] == kb ? ss.wsum[j][kw] : 0ull;
+      rx_put64(peer_addr(smem_u32(&ss.rsum[r][kb][kw]), dst), x, peer_addr(mb0, dst));
     }
     // each request thread keeps its batch index in p's place until step 4
     ph = at ? b : -1;
@@ -1262,7 +1284,7 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepBlock)
     const int64_t n = ss.cb[tid + 1] - ss.cb[tid];
     const BatchAgg g{(int64_t)t[0], (int64_t)t[1], (int64_t)t[2], n, t[3] > 0};
     const int s = segment_of(a.mp, g);
-    if (r == 0) emit_batch<MODE>(a, tid, g, s, a.mp.fx);
+    ss.agg[tid] = g;
     bool slow = false;
     i128 kf = mk128(0, 0);
     if (n == nr) {
@@ -1277,8 +1299,10 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepBlock)
   }
   __syncthreads();
 
-  // 4. this thread's request
-  if (req && ph >= 0) {
+  // 4. this thread's request; T from the constant warp of CTA 0
+  if (!req) {
+    if (r == 0 && lane < nb) emit_batch<MODE>(a, lane, ss.agg[lane], ss.bs[lane], a.mp.fx);
+  } else if (ph >= 0) {
     const int b = ph;
     const int s = ss.bs[b];
     const bool slow = ss.bslow[b] != 0;
@@ -1313,17 +1337,11 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepBlock)
       rx_put128(peer_addr(smem_u32(&rt[r * TS + (tid - dst * TS)]), dst), hot_value(tt, a.H, tid),
                 peer_addr(mb1, dst));
     }
-    i128 tv = mk128(0, 0);
     if (fv) {
       if (!rx_wait(mb1)) flag(a.status, kStatusTimeout);
-      tv = rt[q * TS + jv];
-    }
+      i128 tv = rt[tid];
 #pragma unroll
-    for (int d = 1; d < 8; d <<= 1) {
-      const uint64_t lo = __shfl_xor_sync(kFull, tv.lo, d), hi = __shfl_xor_sync(kFull, tv.hi, d);
-      tv = add128(tv, mk128(lo, hi));
-    }
-    if (fv && q == 0) {
+      for (int src = 1; src < kStepCtas; ++src) tv = add128(tv, rt[src * TS + tid]);
       const i128 nw = add128(st0, tv);
       // overflow of the signed 128-bit total (|total| >= 2^127 * 2^-72 s)
       if (is_neg128(st0) == is_neg128(tv) && is_neg128(nw) != is_neg128(st0)) flag(a.status, kStatusData);
