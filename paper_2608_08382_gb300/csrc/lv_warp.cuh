@@ -1034,47 +1034,44 @@ __global__ void __launch_bounds__(kJBlock) k_jumbo(const TileArgs a, int fit_bas
 // at a time, where launch latency, not bandwidth, bounds the call.  For such
 // inputs lv_attribute and lv_attribute_step run this kernel instead of the
 // partition, tile, jumbo, fold and totals kernels: one cluster of kStepCtas
-// CTAs.  Every CTA forms the batches' sums over all requests itself (the
-// inputs are a few tens of kilobytes), so the batch constants need no
-// exchange; CTA r attributes the r-th contiguous share of the requests, one
-// per thread, and the CTAs exchange tenant table entries by asynchronous
-// stores into one another's shared memory, each completing bytes on the
-// receiver's transaction barrier.
-//   1. Thread 0 sets up the receive barrier; the cluster's threads arrive
-//      once on the cluster barrier, which they wait for only before their
-//      remote stores.  Every global read is issued at once: each thread's
-//      (up to) eight requests for the sums, in 16-byte loads, its own request
-//      to attribute, the offsets (warp 0 clamps them into non-decreasing batch
-//      bounds with a max-scan), and the state of the tenants this CTA folds;
-//      each CTA zeroes its tenant table.  A ninth warp meanwhile forms the
-//      per-request constant of a batch of n_req requests for all four
-//      segments (the single-batch step's).
-//   2. Per-batch sums: a warp whose requests all lie in one batch (the common
-//      case) keeps its warp sums (hardware reductions when they fit 31 bits);
-//      otherwise each request is added to its batch's sums with shared
-//      atomics.
-//   3. One thread per batch adds them up and picks the segment and constant.
+// CTAs with one request per thread (CTA r takes the r-th contiguous share of
+// the requests) and one more warp per CTA for the batch constant.  The CTAs
+// exchange partial results by asynchronous stores into one another's shared
+// memory, each completing bytes on the receiver's transaction barrier, so no
+// step waits at a cluster-wide barrier.
+//   1. Thread 0 sets up the two receive barriers (the batch sums, the tenant
+//      slice), and the cluster's threads arrive once on the cluster barrier,
+//      which they wait for only before their first remote store.  Every global
+//      read is issued at once: the thread's request, the offsets (warp 0
+//      clamps them into non-decreasing batch bounds with a max-scan), and the
+//      state of the tenants this CTA folds; each CTA zeroes its tenant table.
+//      The constant warp meanwhile forms the per-request constant of a batch
+//      of n_req requests for all four segments (the single-batch step's).
+//   2. Per-batch sums of the CTA's requests: a warp whose requests share one
+//      batch (the common case) keeps its warp sums (hardware reductions when
+//      they fit 31 bits), a warp that spans a batch bound adds lane by lane
+//      with shared atomics.  The CTA's sums go to every CTA of the cluster.
+//   3. One thread per batch adds the CTAs' partial sums as they arrive and
+//      picks the segment and the constant.
 //   4. Every thread attributes its request and adds its share into the CTA's
 //      exact tenant table; the constant warp of CTA 0 writes T.
 //   5. Tenant u's table entry goes to the CTA that owns u's slice; there one
 //      thread per tenant adds the cluster's entries exactly, and the tenant's
 //      state (zero on a reset) is added, stored and, when asked, converted to
 //      the correctly rounded total.
-// A CTA leaves only after every byte addressed to it has arrived.  The wait
-// on the receive barrier is bounded (a few seconds); one that runs out
-// records a timeout in the status word.  Tenant ids from H up still go to the
-// pending limbs, which the caller folds.
+// A CTA leaves only after every byte addressed to it has arrived.  Each wait
+// on a receive barrier is bounded (a few seconds); one that runs out records
+// a timeout in the status word.  Tenant ids from H up still go to the pending
+// limbs, which the caller folds.
 constexpr int kStepCtas = 8;
 constexpr int kStepThreads = 512;                 // request threads
 constexpr int kStepBlock = kStepThreads + 32;     // and the constant warp
-constexpr int kStepWarps = kStepThreads / 32;
-constexpr int kStepPer = 8;                       // requests per thread in the sums
 constexpr int64_t kSmallMaxReq = (int64_t)kStepCtas * kStepThreads;
 constexpr int64_t kSmallMaxBatch = 16;
 constexpr int kStepSlice = (kHotMax + kStepCtas - 1) / kStepCtas;  // tenants a CTA folds, at most
-static_assert(kSmallMaxReq == (int64_t)kStepThreads * kStepPer, "the sums cover every request");
 static_assert(kSmallMaxBatch < 32, "warp 0 scans the offsets");
 static_assert(kStepThreads >= kStepSlice, "one thread per tenant of a slice");
+static_assert(kStepThreads >= kStepCtas * kSmallMaxBatch * 4, "one remote store per thread sends the sums");
 static_assert(kStepThreads >= kHotMax, "one thread per tenant sends the table");
 
 struct StepSmem {
@@ -1082,13 +1079,15 @@ struct StepSmem {
   alignas(16) i128 kspec[4];                                // constant of a batch of n_req requests, per segment
   alignas(16) i128 bk[kSmallMaxBatch];                      // each batch's constant
   alignas(16) unsigned long long sum[kSmallMaxBatch][4];     // requests of warps that span a batch bound
-  alignas(16) unsigned long long wsum[kStepWarps][4];        // each warp's sums (warps within one batch)
+  alignas(16) unsigned long long wsum[kStepThreads / 32][4];  // each warp's sums (warps within one batch)
+  alignas(16) unsigned long long rsum[kStepCtas][kSmallMaxBatch][4];  // every CTA's, as received
   alignas(16) int64_t cb[kSmallMaxBatch + 1];               // clamped batch bounds
+  alignas(8) unsigned long long mbar[2];                    // receive barriers: sums, tenant slice
   alignas(16) BatchAgg agg[kSmallMaxBatch];                 // each batch's totals
-  alignas(8) unsigned long long mbar;                       // receive barrier of the tenant slice
   int kspec_slow[4];
   int bs[kSmallMaxBatch], bslow[kSmallMaxBatch];
-  int wb[kStepWarps];                                       // batch of warp wsum[w], or -1
+  int wb[kStepThreads / 32];                                // batch of warp wsum[w], or -1
+  int pad[3];
 };
 static_assert(sizeof(StepSmem) % 16 == 0, "the tenant table follows StepSmem");
 
@@ -1107,8 +1106,13 @@ __device__ __forceinline__ void rx_init(uint32_t mb, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(mb), "r"(bytes) : "memory");
 }
 
-// 16 bytes into a peer's shared memory, completing as many bytes on the
+// 8 or 16 bytes into a peer's shared memory, completing as many bytes on the
 // peer's barrier `rmb`.
+__device__ __forceinline__ void rx_put64(uint32_t raddr, uint64_t v, uint32_t rmb) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b64 [%0], %1, [%2];" ::"r"(raddr), "l"(v),
+               "r"(rmb)
+               : "memory");
+}
 __device__ __forceinline__ void rx_put128(uint32_t raddr, i128 v, uint32_t rmb) {
   asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
                    raddr),
@@ -1134,23 +1138,47 @@ __device__ __forceinline__ bool rx_wait(uint32_t mb) {
   return false;
 }
 
-// Barrier of the request threads alone (the constant warp does not wait).
-__device__ __forceinline__ void sync_requests() { asm volatile("bar.sync 1, %0;" ::"n"(kStepThreads) : "memory"); }
-
-// Loads n (at most 4) consecutive int32 from x, with one 16-byte load when all
-// four are in range (x 16-byte aligned); missing ones are 0.
-__device__ __forceinline__ void load4(const int32_t *x, int n, int32_t *v) {
-  if (n >= 4) {
-    const int4 q = *reinterpret_cast<const int4 *>(x);
-    v[0] = q.x;
-    v[1] = q.y;
-    v[2] = q.z;
-    v[3] = q.w;
-  } else {
+// This warp's contribution to the per-batch sums: when every active lane is
+// in one batch (the common case), the warp's sums go to wsum[warp] (four
+// hardware reductions when every sum fits 31 bits); otherwise each lane adds
+// its fields to sum[its batch] with shared atomics.
+__device__ __forceinline__ void step_sums(StepSmem &ss, bool at, int b, int32_t p, int32_t c, int32_t ph, int lane,
+                                          int wid) {
+  const unsigned am = __ballot_sync(kFull, at);
+  const int b0 = am ? __shfl_sync(kFull, b, __ffs(am) - 1) : -1;
+  if (__all_sync(kFull, !at || b == b0)) {
+    unsigned long long w[4];
+    if (__all_sync(kFull, (uint32_t)p < (1u << 13) && (uint32_t)c < (1u << 26))) {
+      w[0] = __reduce_add_sync(kFull, at ? (uint32_t)p : 0u);
+      w[1] = __reduce_add_sync(kFull, at ? (uint32_t)c : 0u);
+      w[2] = __reduce_add_sync(kFull, at ? (uint32_t)(p * p) : 0u);
+      w[3] = __reduce_add_sync(kFull, at ? (uint32_t)ph : 0u);
+    } else {
+      Sums v{at ? p : 0, at ? c : 0, at ? (int64_t)p * p : 0, at ? ph : 0};
+      v = warp_sum(v);
+      w[0] = (unsigned long long)v.s1;
+      w[1] = (unsigned long long)v.s2;
+      w[2] = (unsigned long long)v.s3;
+      w[3] = (unsigned long long)v.ph;
+    }
+    if (lane == 0) {
+      ss.wb[wid] = b0;
 #pragma unroll
-    for (int k = 0; k < 4; ++k) v[k] = k < n ? x[k] : 0;
+      for (int k = 0; k < 4; ++k) ss.wsum[wid][k] = w[k];
+    }
+  } else {
+    if (lane == 0) ss.wb[wid] = -1;
+    if (at) {
+      atomicAdd(&ss.sum[b][0], (unsigned long long)p);
+      atomicAdd(&ss.sum[b][1], (unsigned long long)c);
+      atomicAdd(&ss.sum[b][2], (unsigned long long)((int64_t)p * p));
+      atomicAdd(&ss.sum[b][3], (unsigned long long)ph);
+    }
   }
 }
+
+// Barrier of the request threads alone (the constant warp does not wait).
+__device__ __forceinline__ void sync_requests() { asm volatile("bar.sync 1, %0;" ::"n"(kStepThreads) : "memory"); }
 
 // state: the tenant accumulator's exact state (with M_TEN); L: the tenants'
 // totals after this step, or null (then tenant ids may exceed H); reset: the
@@ -1168,41 +1196,31 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepBlock)
   const int r = (int)cooperative_groups::this_cluster().block_rank();
   const int64_t nr = a.n_req, nb = a.n_batch;
   const bool req = tid < kStepThreads;
-  const uint32_t mb = smem_u32(&ss.mbar);
+  const uint32_t mb0 = smem_u32(&ss.mbar[0]), mb1 = smem_u32(&ss.mbar[1]);
   int bad = 0;
 
-  // 1. the receive barrier, the reads, the single-batch constant
+  // 1. receive barriers, reads, the single-batch constant
   const int own = kTen ? max(0, min(TS, a.H - r * TS)) : 0;  // tenants of this CTA's slice
-  if constexpr (kTen) {
-    if (tid == 0) {
-      rx_init(mb, (uint32_t)(kStepCtas * 16 * own));
-      asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory");
+  if (tid == 0) {
+    rx_init(mb0, (uint32_t)(kStepCtas * 32 * nb));
+    rx_init(mb1, (uint32_t)(kStepCtas * 16 * own));
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory");
   const int64_t chunk = (nr + kStepCtas - 1) / kStepCtas;
-  const int64_t i = r * chunk + tid;  // the request this thread attributes
+  const int64_t i = r * chunk + tid;
   const bool in = req && tid < chunk && i < nr;
-  int32_t p = 0, c = 0, u = 0;
+  int32_t p = 0, c = 0, ph = 0, u = 0;
   if (in) {
-    p = max(a.p[i], 0);
-    c = max(a.c[i], 0);
+    p = a.p[i];
+    c = a.c[i];
+    ph = a.ph[i];
     if (kTen) u = a.ten[i];
-  }
-  int32_t sp[kStepPer], sc[kStepPer], sf[kStepPer];  // requests 4 tid + j, 2048 + 4 tid + j for the sums
-  if (req) {
-#pragma unroll
-    for (int g = 0; g < kStepPer / 4; ++g) {
-      const int64_t base = (int64_t)g * (4 * kStepThreads) + 4 * tid;
-      const int n4 = (int)max((int64_t)0, min((int64_t)4, nr - base));
-      load4(a.p + base, n4, sp + 4 * g);
-      load4(a.c + base, n4, sc + 4 * g);
-      load4(a.ph + base, n4, sf + 4 * g);
-    }
   }
   int64_t ob = 0;
   if (wid == 0 && lane <= nb) ob = a.off[lane];
-  const int v = r * TS + tid;  // the tenant this thread folds
+  // the fold: thread j takes tenant r * TS + j of this CTA's slice
+  const int v = r * TS + tid;
   const bool fv = tid < own;
   i128 st0 = mk128(0, 0);
   if (fv && !reset) st0 = state[v];
@@ -1217,6 +1235,7 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepBlock)
       for (int k = tid; k < 4 * ten_plane(a.H); k += kStepThreads) tt[k] = 0;
     if (tid < 4 * kSmallMaxBatch) (&ss.sum[0][0])[tid] = 0ull;
     init_segs<MODE>(a, ss.seg);
+    if (in) check_req(p, c, ph, &bad);
     if (wid == 0) {
       // bound k = min(n_req, max(0, off[0..k])): batch b takes requests
       // [cb[b], cb[b + 1]); valid offsets are their own bounds
@@ -1234,76 +1253,34 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepBlock)
     }
     sync_requests();
 
-    // 2. per-batch sums over every request
-    const int64_t lo = ss.cb[0], hi = ss.cb[nb];
-    uint64_t l1 = 0, l2 = 0, l3 = 0, l4 = 0;
-    int ignore = 0;
-    int bt = -2;  // the batch of every counted request of this thread; -1: several
+    // 2. per-batch sums, sent to every CTA of the cluster
+    int b = 0;
+    for (int k = 1; k < nb; ++k) b += ss.cb[k] <= i ? 1 : 0;
+    const bool at = in && i >= ss.cb[0] && i < ss.cb[nb];
+    step_sums(ss, at, b, p, c, ph, lane, wid);
+    sync_requests();
+    asm volatile("barrier.cluster.wait;" ::: "memory");  // the peers' receive barriers are set up
+    if (tid < kStepCtas * 4 * nb) {
+      // word k of the CTA's batch sums (batch k / 4), to CTA dst
+      const int dst = tid / (4 * (int)nb), k = tid % (4 * (int)nb), kb = k >> 2, kw = k & 3;
+      unsigned long long x = ss.sum[kb][kw];
 #pragma unroll
-    for (int k = 0; k < kStepPer; ++k) {
-      const int64_t q = (int64_t)(k >> 2) * (4 * kStepThreads) + 4 * tid + (k & 3);
-      check_req(sp[k], sc[k], sf[k], r == 0 ? &bad : &ignore);  // every CTA clamps, CTA 0 reports
-      if (q >= lo && q < hi) {
-        int b = 0;
-        for (int kk = 1; kk < nb; ++kk) b += ss.cb[kk] <= q ? 1 : 0;
-        bt = (bt == -2 || bt == b) ? b : -1;
-        l1 += (uint32_t)sp[k];
-        l2 += (uint32_t)sc[k];
-        l3 += (uint64_t)sp[k] * (uint64_t)sp[k];
-        l4 += (uint32_t)sf[k];
-      }
+      for (int j = 0; j < kStepThreads / 32; ++j) x += ss.wb[j] == kb ? ss.wsum[j][kw] : 0ull;
+      rx_put64(peer_addr(smem_u32(&ss.rsum[r][kb][kw]), dst), x, peer_addr(mb0, dst));
     }
-    const unsigned am = __ballot_sync(kFull, bt >= 0);
-    const int b0 = am ? __shfl_sync(kFull, bt, __ffs(am) - 1) : -1;
-    if (__all_sync(kFull, bt == -2 || (bt >= 0 && bt == b0))) {
-      unsigned long long w[4];
-      if (__all_sync(kFull, l1 < (1u << 26) && l2 < (1u << 26) && l3 < (1u << 26))) {
-        // every warp sum fits 31 bits
-        w[0] = __reduce_add_sync(kFull, (uint32_t)l1);
-        w[1] = __reduce_add_sync(kFull, (uint32_t)l2);
-        w[2] = __reduce_add_sync(kFull, (uint32_t)l3);
-        w[3] = __reduce_add_sync(kFull, (uint32_t)l4);
-      } else {
-        Sums s{(int64_t)l1, (int64_t)l2, (int64_t)l3, (int32_t)l4};
-        s = warp_sum(s);
-        w[0] = (unsigned long long)s.s1;
-        w[1] = (unsigned long long)s.s2;
-        w[2] = (unsigned long long)s.s3;
-        w[3] = (unsigned long long)s.ph;
-      }
-      if (lane == 0) {
-        ss.wb[wid] = b0;
-#pragma unroll
-        for (int k = 0; k < 4; ++k) ss.wsum[wid][k] = w[k];
-      }
-    } else {
-      if (lane == 0) ss.wb[wid] = -1;
-#pragma unroll
-      for (int k = 0; k < kStepPer; ++k) {
-        const int64_t q = (int64_t)(k >> 2) * (4 * kStepThreads) + 4 * tid + (k & 3);
-        if (q >= lo && q < hi) {
-          int b = 0;
-          for (int kk = 1; kk < nb; ++kk) b += ss.cb[kk] <= q ? 1 : 0;
-          atomicAdd(&ss.sum[b][0], (unsigned long long)(uint32_t)sp[k]);
-          atomicAdd(&ss.sum[b][1], (unsigned long long)(uint32_t)sc[k]);
-          atomicAdd(&ss.sum[b][2], (unsigned long long)((uint64_t)sp[k] * (uint64_t)sp[k]));
-          atomicAdd(&ss.sum[b][3], (unsigned long long)(uint32_t)sf[k]);
-        }
-      }
-    }
+    // each request thread keeps its batch index in p's place until step 4
+    ph = at ? b : -1;
   }
   __syncthreads();
 
-  // 3. the batches' totals, segment and constant
+  // 3. the batches' totals, segment, T and constant
   if (tid < nb) {
-    unsigned long long t[4];
+    if (!rx_wait(mb0)) flag(a.status, kStatusTimeout);
+    unsigned long long t[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-    for (int k = 0; k < 4; ++k) t[k] = ss.sum[tid][k];
+    for (int src = 0; src < kStepCtas; ++src)
 #pragma unroll
-    for (int w = 0; w < kStepWarps; ++w)
-      if (ss.wb[w] == tid)
-#pragma unroll
-        for (int k = 0; k < 4; ++k) t[k] += ss.wsum[w][k];
+      for (int w = 0; w < 4; ++w) t[w] += ss.rsum[src][tid][w];
     const int64_t n = ss.cb[tid + 1] - ss.cb[tid];
     const BatchAgg g{(int64_t)t[0], (int64_t)t[1], (int64_t)t[2], n, t[3] > 0};
     const int s = segment_of(a.mp, g);
@@ -1325,9 +1302,8 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepBlock)
   // 4. this thread's request; T from the constant warp of CTA 0
   if (!req) {
     if (r == 0 && lane < nb) emit_batch<MODE>(a, lane, ss.agg[lane], ss.bs[lane], a.mp.fx);
-  } else if (in && i >= ss.cb[0] && i < ss.cb[nb]) {
-    int b = 0;
-    for (int kk = 1; kk < nb; ++kk) b += ss.cb[kk] <= i ? 1 : 0;
+  } else if (ph >= 0) {
+    const int b = ph;
     const int s = ss.bs[b];
     const bool slow = ss.bslow[b] != 0;
     const i128 kf = ss.bk[b];
@@ -1357,13 +1333,12 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepBlock)
   if constexpr (kTen) {
     __syncthreads();
     if (tid < a.H) {
-      asm volatile("barrier.cluster.wait;" ::: "memory");  // the peers' receive barriers are set up
       const int dst = tid / TS;
       rx_put128(peer_addr(smem_u32(&rt[r * TS + (tid - dst * TS)]), dst), hot_value(tt, a.H, tid),
-                peer_addr(mb, dst));
+                peer_addr(mb1, dst));
     }
     if (fv) {
-      if (!rx_wait(mb)) flag(a.status, kStatusTimeout);
+      if (!rx_wait(mb1)) flag(a.status, kStatusTimeout);
       i128 tv = rt[tid];
 #pragma unroll
       for (int src = 1; src < kStepCtas; ++src) tv = add128(tv, rt[src * TS + tid]);
