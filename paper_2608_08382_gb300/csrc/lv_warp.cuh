@@ -1309,12 +1309,20 @@ __global__ void __cluster_dims__(kStepCtas, 1, 1) __launch_bounds__(kStepBlock)
     const i128 kf = ss.bk[b];
     const SegS sg = ss.seg[s];
     bool done = false;
-    if ((MODE & M_FIX) && !slow && sg.a2_narrow && p == 1) {
-      // a decode request: the same exact steps as the warp-tile fast path
+    if ((MODE & M_FIX) && !slow && sg.a2_narrow && (p == 1 || (sg.p_narrow && p <= kPMaxFix))) {
+      // the exact steps of the warp-tile fast path, with K + A1 + A3 for a
+      // decode request and K + p (A1 + A3 p) for a prefill (one instruction
+      // stream for both: a branch to rarely run code fetches it cold)
       const i128 K13 = add128(kf, sg.A13);
-      uint32_t v0, v1, v2, v3;
-      mad_k13((uint32_t)K13.lo, (uint32_t)(K13.lo >> 32), (uint32_t)K13.hi, (uint32_t)(K13.hi >> 32),
-              (uint32_t)sg.A2.lo, (uint32_t)(sg.A2.lo >> 32), (uint32_t)c, v0, v1, v2, v3);
+      uint32_t b0, b1, b2, b3, v0, v1, v2, v3;
+      prefill_const(sg, kf, sg.p_narrow ? (uint32_t)p : 1u, b0, b1, b2, b3);
+      if (p == 1) {
+        b0 = (uint32_t)K13.lo;
+        b1 = (uint32_t)(K13.lo >> 32);
+        b2 = (uint32_t)K13.hi;
+        b3 = (uint32_t)(K13.hi >> 32);
+      }
+      mad_k13(b0, b1, b2, b3, (uint32_t)sg.A2.lo, (uint32_t)(sg.A2.lo >> 32), (uint32_t)c, v0, v1, v2, v3);
       if (v3 == 0u && v2 != 0u) {
         uint64_t m;
         int ex2;
