@@ -1122,18 +1122,19 @@ __device__ __forceinline__ void rx_put128(uint32_t raddr, i128 v, uint32_t rmb) 
 }
 
 // Waits for the receive barrier's first phase (bounded: false when it ran
-// out); what arrived is then visible to this thread.
+// out, after a few seconds); what arrived is then visible to this thread.
+// Each try suspends the thread until the phase completes or about a
+// microsecond has passed.
 __device__ __forceinline__ bool rx_wait(uint32_t mb) {
-  for (long long k = 0; k < (1ll << 24); ++k) {
+  for (int k = 0; k < (1 << 22); ++k) {
     uint32_t done;
     asm volatile(
-        "{\n .reg .pred p;\n mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], 0;\n"
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], 0, %2;\n"
         " selp.u32 %0, 1, 0, p;\n}"
         : "=r"(done)
-        : "r"(mb)
+        : "r"(mb), "n"(1000)
         : "memory");
     if (done) return true;
-    if (k > 64) __nanosleep(32);
   }
   return false;
 }
