@@ -351,8 +351,8 @@ def _setup_step(lv, ctx, w, stream):
     return dict(step=step, e2e_step=e2e_step, units=w.n_req, unit="requests/s", metric=METRIC_STEP,
                 h2d=sum(int(t.numel() * t.element_size()) for t in hp.values()),
                 d2h=8 * (w.n_req + w.n_batch + w.n_tenants), launches_per_step=1,
-                kernel="graph", time_mask=0, graph=True, whole_step=True, flush=True,
-                timed="the whole CUDA-graph replay, CUDA events on the launching stream",
+                kernel="k_step", time_mask=0, graph=True, whole_step=True, flush=True,
+                timed="the whole CUDA-graph replay (one k_step node), CUDA events on the launching stream",
                 bytes_per_launch=24.0 * w.n_req + 16.0 * w.n_batch,
                 bytes_rule="24 B/request + 16 B/batch over the whole replay (one k_step launch: reads p, c, phase, "
                             "tenant, writes the share; tenant state and totals are 40 B/tenant more): a single "
