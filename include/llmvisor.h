@@ -137,8 +137,9 @@ void lv_ctx_destroy(lv_ctx *ctx);
 /* Select LV_ARITH_AUTO (default) or LV_ARITH_FP64. */
 lv_status lv_ctx_set_arith(lv_ctx *ctx, int32_t mode);
 /* Synchronise `stream`, then return and clear the sticky device status
- * (LV_OK, or LV_EDATA when a kernel met invalid input data since the last
- * query). */
+ * (LV_OK; LV_EDATA when a kernel met invalid input data since the last query;
+ * LV_ETIMEOUT when a bounded wait inside the serving-step kernel of
+ * lv_attribute / lv_attribute_step ran out, which takes precedence). */
 lv_status lv_ctx_status(lv_ctx *ctx, void *stream);
 /* Static description of a status code. */
 const char *lv_status_string(lv_status s);
