@@ -77,6 +77,16 @@ def test_invalid_arguments_rejected_before_launch(lv):
     assert L.lv_fit_vtc(None, None, None, 1, None, None, None, None) == lv.LV_EINVAL
     assert lv.lv_status_string(lv.LV_EDATA) == "invalid input data"
     assert L.lv_tenant_acc_state_bytes(None) == 0
+    # lv_attribute_step: unknown flags, totals or a reset without an accumulator, a misaligned L, no context
+    fake = ctypes.c_void_p(1 << 20)
+    step = L.lv_attribute_step
+    assert step(None, ctypes.byref(m), ctypes.byref(b), None, None, None, None, 2, None) == lv.LV_EINVAL
+    assert step(None, ctypes.byref(m), ctypes.byref(b), None, None, None, fake, 0, None) == lv.LV_EINVAL
+    assert step(None, ctypes.byref(m), ctypes.byref(b), None, None, None, None, lv.LV_STEP_RESET, None) == lv.LV_EINVAL
+    assert step(None, ctypes.byref(m), ctypes.byref(b), None, None, fake, ctypes.c_void_p((1 << 20) + 4), 0,
+                None) == lv.LV_EINVAL
+    assert step(None, ctypes.byref(m), ctypes.byref(b), None, None, None, None, 0, None) == lv.LV_EINVAL
+    assert L.lv_ctx_selftest_barrier(None, None) == lv.LV_EINVAL
 
 
 def test_import_fails_loudly_without_library(tmp_path):
